@@ -1,0 +1,449 @@
+"""Pins of the fp64 oracle against closed forms, special cases and
+brute force (paper Sec. 3.1-3.2, Eq. 1-6, App. A).  CPU only.
+
+Each test fixes a value that the mathematics or the paper determines, so that
+a plausible slip in the oracle (a dropped term, a sign, an index, a transposed
+operand, a wrong norm axis) fails at least one of them.
+"""
+import cmath
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_2605_27255_gb300 import synth
+
+LN3 = math.log(3.0)
+
+
+# ---------------------------------------------------------------- primitives
+
+def test_round_bf16_matches_torch_and_ties_to_even():
+    # ties: 1 + 2^-8 lies halfway between 1 and 1 + 2^-7 -> even (1.0)
+    assert O.round_bf16(1.0 + 2.0 ** -8) == 1.0
+    # 1 + 3*2^-8 lies halfway between 1+2^-7 (odd) and 1+2^-6 (even)
+    assert O.round_bf16(1.0 + 3 * 2.0 ** -8) == 1.0 + 2.0 ** -6
+    rng = np.random.default_rng(0)
+    xs = rng.standard_normal(2000).astype(np.float32) * 10.0 ** rng.integers(-3, 3, 2000)
+    ref = torch.from_numpy(xs).to(torch.bfloat16).double().numpy()
+    got = np.array([O.round_bf16(float(x)) for x in xs])
+    assert np.array_equal(got, ref)
+
+
+def test_rmsnorm_closed_forms():
+    # [3,4]: mean square 12.5 -> [3,4]/sqrt(12.5) = [3 sqrt2/5, 4 sqrt2/5]
+    y = O.rmsnorm([3.0, 4.0], [1.0, 1.0], eps=0.0)
+    assert np.allclose(y, [3 * math.sqrt(2) / 5, 4 * math.sqrt(2) / 5], rtol=0, atol=1e-15)
+    # gains multiply per element (sign included)
+    y = O.rmsnorm([3.0, 4.0], [2.0, -1.0], eps=0.0)
+    assert np.allclose(y, [6 * math.sqrt(2) / 5, -4 * math.sqrt(2) / 5], atol=1e-15)
+    # eps sits inside the root, added to the mean square: x = 1e-3 everywhere,
+    # eps = 1e-6 -> 1e-3 / sqrt(2e-6) = 1/sqrt(2)
+    y = O.rmsnorm(np.full(7, 1e-3), np.ones(7), eps=1e-6)
+    assert np.allclose(y, 1 / math.sqrt(2), atol=1e-12)
+    # zero vector stays zero (no division by zero)
+    assert np.all(O.rmsnorm(np.zeros(5), np.ones(5)) == 0)
+
+
+def test_matvec_is_row_major_out_by_in():
+    rng = np.random.default_rng(1)
+    W = rng.standard_normal((5, 9)).astype(np.float32)
+    x = rng.standard_normal(9)
+    assert np.allclose(O.matvec(W, x), W.astype(np.float64) @ x, atol=1e-12)
+
+
+def test_silu_sigmoid_closed_forms():
+    assert O.sigmoid(0.0) == 0.5
+    assert abs(O.sigmoid(LN3) - 0.75) < 1e-15          # 1/(1+1/3)
+    assert abs(O.sigmoid(-LN3) - 0.25) < 1e-15
+    assert abs(O.silu(LN3) - 0.75 * LN3) < 1e-15       # x * sigma(x)
+    assert O.silu(0.0) == 0.0
+
+
+def test_rope_is_complex_rotation_rotate_half_pairs():
+    theta = 100.0
+    d = 4
+    v = np.array([0.3, -1.2, 0.7, 2.0])
+    for pos in (0, 1, 5, 37):
+        got = O.rope(v, 1, d, pos, theta)
+        # pairs (i, i+d/2) as complex numbers v_i + 1j v_{i+d/2}, frequency theta^(-2i/d)
+        for i in range(d // 2):
+            w = complex(v[i], v[i + d // 2]) * cmath.exp(1j * pos * theta ** (-2.0 * i / d))
+            assert abs(got[i] - w.real) < 1e-12 and abs(got[i + d // 2] - w.imag) < 1e-12
+    assert np.array_equal(O.rope(v, 1, d, 0, theta), v)
+
+
+def test_rope_relative_position_and_norm():
+    rng = np.random.default_rng(2)
+    d, theta = 16, 1e4
+    q, k = rng.standard_normal(d), rng.standard_normal(d)
+    dots = [np.dot(O.rope(q, 1, d, m + s, theta), O.rope(k, 1, d, n + s, theta))
+            for (m, n, s) in ((7, 3, 0), (7, 3, 11), (7, 3, 1000))]
+    assert np.allclose(dots, dots[0], atol=1e-9)
+    assert abs(np.linalg.norm(O.rope(q, 1, d, 123, theta)) - np.linalg.norm(q)) < 1e-12
+    # two heads rotate independently and identically
+    two = O.rope(np.concatenate([q, k]), 2, d, 9, theta)
+    assert np.allclose(two[:d], O.rope(q, 1, d, 9, theta)) and np.allclose(two[d:], O.rope(k, 1, d, 9, theta))
+
+
+def test_attention_single_entry_returns_value():
+    rng = np.random.default_rng(3)
+    d, nq, nkv = 8, 4, 2
+    q = rng.standard_normal(nq * d)
+    K = rng.standard_normal((1, nkv * d))
+    V = rng.standard_normal((1, nkv * d))
+    out = O.attend(q, K, V, nq, nkv, d).reshape(nq, d)
+    # GQA: query heads 0,1 read kv head 0; heads 2,3 read kv head 1
+    for h in range(nq):
+        g = h // (nq // nkv)
+        assert np.allclose(out[h], V[0, g * d:(g + 1) * d], atol=1e-15)
+
+
+def test_attention_softmax_scale_is_inverse_sqrt_d():
+    # scores ln3 apart after scaling by 1/sqrt(d): weights 3/4 and 1/4
+    d = 16
+    q = np.zeros(d); q[0] = 1.0
+    K = np.zeros((2, d)); K[0, 0] = LN3 * math.sqrt(d); K[1, 0] = 0.0
+    V = np.zeros((2, d)); V[0, :] = 1.0; V[1, :] = -3.0
+    out = O.attend(q, K, V, 1, 1, d)
+    assert np.allclose(out, 0.75 * 1.0 + 0.25 * -3.0, atol=1e-14)
+
+
+def test_argmax_lowest_index_on_ties_and_margin():
+    i, m = O.argmax([0.1, 0.9, 0.3, 0.9, -2.0])
+    assert i == 1 and m == 0.0
+    i, m = O.argmax([0.1, 0.2, 0.7, 0.4])
+    assert i == 2 and abs(m - 0.3) < 1e-15
+
+
+# ------------------------------------------------------- model construction
+
+def small_shape(**kw):
+    base = dict(name="pin", H=8, L=1, n_q=4, n_kv=2, d_h=2, F=12, V=8,
+                compressor="linear", mtp_block=0, dtype="f32", rope_theta=1e4, tau=0.5)
+    base.update(kw)
+    return synth.ModelShape(**base)
+
+
+def zero_model(s):
+    """All projections zero and all gains one: every block is the identity."""
+    w = {}
+    for name, shape in synth.tensor_shapes(s).items():
+        w[name] = torch.ones(shape) if synth.is_gain(name) else torch.zeros(shape)
+    return w
+
+
+def onehot_model(s, perm):
+    """E = I (V = H), compressor [I I], MTP W_fc = [0 P], zero blocks,
+    confidence W2 = 0 (so c = sigma(0) = 1/2)."""
+    assert s.V == s.H
+    w = zero_model(s)
+    H = s.H
+    w["E"] = torch.eye(H)
+    w["comp.W"] = torch.cat([torch.eye(H), torch.eye(H)], 1)
+    P = torch.zeros(H, H)
+    for i, j in enumerate(perm):
+        P[j, i] = 1.0
+    w["mtp.W_fc"] = torch.cat([torch.zeros(H, H), P], 1)
+    return w
+
+
+def test_compressor_identity_pair_is_sum():
+    # Eq. 1 / App. A.1: Linear W [a;b] + b with W = [I I], b = 0 gives a + b
+    s = small_shape(V=16)
+    w = zero_model(s)
+    rng = torch.Generator().manual_seed(0)
+    w["E"] = torch.randn(s.V, s.H, generator=rng)
+    w["x_pad"] = torch.randn(s.H, generator=rng)
+    w["comp.W"] = torch.cat([torch.eye(s.H), torch.eye(s.H)], 1)
+    m = O.Model(s, w)
+    z = O.compress(m, 3, 11)
+    assert np.allclose(z, (w["E"][3] + w["E"][11]).double().numpy(), atol=1e-6)
+    # the bias is added once
+    w["comp.b"] = torch.arange(s.H, dtype=torch.float32)
+    m = O.Model(s, w)
+    assert np.allclose(O.compress(m, 3, 11), (w["E"][3] + w["E"][11] + w["comp.b"]).double().numpy(), atol=1e-6)
+    # PAD in the second slot reads x_pad
+    assert np.allclose(O.compress(m, 3, -1), (w["E"][3] + w["x_pad"] + w["comp.b"]).double().numpy(), atol=1e-6)
+    # order matters: W = [I 0] keeps the first slot
+    w["comp.W"] = torch.cat([torch.eye(s.H), torch.zeros(s.H, s.H)], 1)
+    w["comp.b"] = torch.zeros(s.H)
+    m = O.Model(s, w)
+    assert np.allclose(O.compress(m, 3, 11), w["E"][3].double().numpy(), atol=1e-7)
+
+
+def test_compressor_mlp_closed_form():
+    # MLP variant W2 SiLU(W1 [a;b]): with W1 = [I I], W2 = 2I and a + b = ln3
+    # per element, every output is 2 * ln3 * 3/4
+    s = small_shape(compressor="mlp", V=4)
+    w = zero_model(s)
+    E = torch.zeros(s.V, s.H)
+    E[1] = 0.25 * LN3
+    E[2] = 0.75 * LN3
+    w["E"] = E.to(torch.float32)
+    w["comp.W1"] = torch.cat([torch.eye(s.H), torch.eye(s.H)], 1)
+    w["comp.W2"] = 2 * torch.eye(s.H)
+    m = O.Model(s, w)
+    z = O.compress(m, 1, 2)
+    expect = 2 * (float(E[1, 0]) + float(E[2, 0])) * 0.75  # ln3 in fp32, times sigma(ln3)
+    x = float(E[1, 0]) + float(E[2, 0])
+    expect = 2 * x / (1 + math.exp(-x))
+    assert np.allclose(z, expect, atol=1e-12)
+    assert abs(expect - 1.5 * LN3) < 1e-6
+    # the nonlinearity sits between W1 and W2: a + b = 0 gives exactly 0
+    assert np.all(O.compress(m, 0, 0) == 0)
+
+
+def test_onehot_model_closed_form_tokens_and_acceptance():
+    """With E = I, a [I I] compressor and identity blocks, h_b = e_t0 + e_t1,
+    so the LM head's argmax is min(t0, t1) (a tie, lowest index wins); the MTP
+    head sees RMSNorm(E[x_b]) through W_fc = [0 P], so x_d = P(x_b); with
+    W2 = 0 the confidence is exactly 1/2 and tau = 1/2 accepts (c >= tau)."""
+    s = small_shape(L=1)
+    perm = [3, 6, 0, 7, 1, 5, 2, 4]
+    m = O.Model(s, onehot_model(s, perm))
+    st = O.State(m, 1)
+    o = st.prefill([[5, 2]], tau=0.5)
+    assert o["tokens"][0, 0] == 2 and o["tokens"][0, 1] == perm[2]
+    assert o["conf"][0] == 0.5 and o["n_acc"][0] == 1
+    assert st.seq(0) == dict(p0=2, p1=perm[2], n=1, emitted=2)
+    # next step consumes (2, 0): argmax min(2, 0) = 0, draft perm[0] = 3
+    o = st.step(tau=0.5)
+    assert list(o["tokens"][0]) == [0, perm[0]]
+    # tau just above 1/2 rejects; the pending pair then has PAD in slot 1
+    o = st.step(tau=0.5 + 1e-12)
+    assert list(o["tokens"][0]) == [min(0, 3), -1] and o["n_acc"][0] == 0
+    assert st.seq(0)["p1"] == -1
+    # PAD input: x_pad = 0, so z = e_{p0} alone and the argmax is p0
+    o = st.step(tau=0.5)
+    assert o["tokens"][0, 0] == 0
+    assert st.seq(0)["n"] == 4 and st.seq(0)["emitted"] == 2 + 2 + 1 + 2
+
+
+def test_mtp_input_order_and_block_identity():
+    # W_fc = [I 0] reads RMSNorm(h_b) (first half), not the token embedding
+    s = small_shape(L=1)
+    w = onehot_model(s, list(range(8)))
+    w["mtp.W_fc"] = torch.cat([torch.eye(s.H), torch.zeros(s.H, s.H)], 1)
+    m = O.Model(s, w)
+    st = O.State(m, 1)
+    o = st.prefill([[6, 4]])
+    # h_d = RMSNorm(e6 + e4): argmax over {4, 6} -> 4, the same as the backbone
+    assert o["x_b"][0] == 4 and o["x_d"][0] == 4
+    assert np.allclose(o["h_d"][0], O.rmsnorm(o["h_b"][0], np.ones(8)), atol=1e-12)
+
+
+def test_confidence_joint_norm_over_2H():
+    """App. A.3 normalises the concatenation [h_b; h_d] with one RMSNorm over
+    2H.  With W1 = I on the h_b half and W2 = 1, the pre-sigmoid value is
+    sum SiLU(h_b / rms([h_b; h_d])), which a per-half norm would not give."""
+    s = small_shape(H=4, V=4, n_q=2, n_kv=1, d_h=2, F=4)
+    w = zero_model(s)
+    w["conf.W1"] = torch.cat([torch.eye(4), torch.zeros(4, 4)], 1)
+    w["conf.W2"] = torch.ones(1, 4)
+    m = O.Model(s, w)
+    hb = np.array([1.0, 1.0, 1.0, 1.0])
+    hd = np.array([3.0, 3.0, 3.0, 3.0])
+    rms = math.sqrt((4 * 1 + 4 * 9) / 8 + 1e-6)
+    x = 1.0 / rms
+    expect = 1 / (1 + math.exp(-4 * x / (1 + math.exp(-x))))
+    assert abs(O.confidence(m, hb, hd) - expect) < 1e-12
+    # W2 = 0 gives exactly 1/2
+    w["conf.W2"] = torch.zeros(1, 4)
+    assert O.confidence(O.Model(s, w), hb, hd) == 0.5
+
+
+def test_block_residual_paths():
+    """A block with W_o = 0 and W_down = 0 is the identity (both residuals);
+    with only W_down = 0, h changes by W_o a where a is the attention output,
+    which at the first position is v itself (single entry)."""
+    s = small_shape(L=1, V=8, H=8)
+    w = onehot_model(s, list(range(8)))
+    m = O.Model(s, w)
+    st = O.State(m, 1)
+    o = st.prefill([[1, 2]])
+    assert np.allclose(o["h_b"][0], np.eye(8)[1] + np.eye(8)[2])
+    # now W_v = I-slice, W_o = I-slice: at position 0 a = v = W_v RMSNorm(x)
+    rng = torch.Generator().manual_seed(5)
+    w["blk.Wv"][0] = torch.randn(s.n_kv * s.d_h, s.H, generator=rng)
+    w["blk.Wo"][0] = torch.randn(s.H, s.n_q * s.d_h, generator=rng)
+    m = O.Model(s, w)
+    st = O.State(m, 1)
+    o = st.prefill([[1, 2]])
+    x = np.eye(8)[1] + np.eye(8)[2]
+    y = O.rmsnorm(x, np.ones(8))
+    v = w["blk.Wv"][0].double().numpy() @ y
+    a = np.concatenate([v[(h // 2) * 2:(h // 2) * 2 + 2] for h in range(4)])
+    assert np.allclose(o["h_b"][0], x + w["blk.Wo"][0].double().numpy() @ a, atol=1e-6)
+
+
+def test_swiglu_gate_and_up_are_not_swapped():
+    """FFN = W_down(SiLU(W_gate y) * W_up y).  With W_gate rows picking y_0,
+    W_up rows picking 2 y_0 and W_down summing, the output is
+    SiLU(y0) * 2 y0, which differs from y0 * SiLU(2 y0)."""
+    s = small_shape(L=1, V=8, H=8, F=1)
+    w = onehot_model(s, list(range(8)))
+    w["blk.Wgate"][0] = torch.zeros(1, 8); w["blk.Wgate"][0][0, 0] = 1.0
+    w["blk.Wup"][0] = torch.zeros(1, 8); w["blk.Wup"][0][0, 0] = 2.0
+    w["blk.Wdown"][0] = torch.zeros(8, 1); w["blk.Wdown"][0][7, 0] = 1.0
+    m = O.Model(s, w)
+    o = O.State(m, 1).prefill([[0, 0]])
+    x = 2 * np.eye(8)[0]
+    y0 = O.rmsnorm(x, np.ones(8))[0]
+    expect = x.copy(); expect[7] += (y0 / (1 + math.exp(-y0))) * 2 * y0
+    assert np.allclose(o["h_b"][0], expect, atol=1e-12)
+
+
+# ------------------------------------------------------ seeded small models
+
+def seeded(s, seed=0):
+    w = synth.gen_weights(s, seed=seed)
+    return w
+
+
+TINY_SMALL = synth.TINY.with_(name="t", H=32, L=2, n_q=4, n_kv=2, d_h=8, F=48, V=64)
+
+
+@pytest.mark.parametrize("comp,mtp,kvb", [("linear", 1, 0), ("mlp", 1, 1), ("mlp", 0, 0), ("linear", 0, 1)])
+def test_cached_steps_equal_bruteforce_recompute(comp, mtp, kvb):
+    s = TINY_SMALL.with_(compressor=comp, mtp_block=mtp)
+    w = seeded(s, 3)
+    w["x_pad"] = w["x_pad"] * 30  # make PAD inputs matter
+    m = O.Model(s, w, max_ctx=32, kv_bf16=bool(kvb))
+    st = O.State(m, 1)
+    prompt = synth.gen_prompts(1, 9, s.V, seed=4).numpy()  # odd: last pair has PAD
+    o = st.prefill(prompt, tau=0.5)
+    pairs = [[int(prompt[0, 2 * j]), int(prompt[0, 2 * j + 1]) if 2 * j + 1 < 9 else -1] for j in range(5)]
+    mtok = [int(prompt[0, 2 * j + 2]) for j in range(4)]
+    force = 0
+    for it in range(6):
+        bf = O.bruteforce(m, pairs, mtok, tau=0.5, force=force)
+        for k in ("logits_b", "logits_d", "h_b", "h_d", "conf"):
+            assert np.allclose(o[k][0], bf[k][0], rtol=0, atol=1e-11), (it, k)
+        assert list(o["tokens"][0]) == list(bf["tokens"][0])
+        # extend the history with what this position produced
+        mtok.append(int(o["x_b"][0]))
+        pairs.append([int(o["tokens"][0, 0]), int(o["tokens"][0, 1])])
+        force = [0, 2, 1][it % 3]
+        o = st.step(tau=0.5, force=force)
+
+
+def test_prompt_pairs_halve_the_length():
+    s = TINY_SMALL
+    m = O.Model(s, seeded(s), max_ctx=64)
+    for n_tok, n_lat in ((2, 1), (10, 5), (11, 6), (1, 1)):
+        st = O.State(m, 1)
+        st.prefill(synth.gen_prompts(1, n_tok, s.V).numpy())
+        assert st.seq(0)["n"] == n_lat
+
+
+def test_reject_all_gives_one_token_per_pair_and_accept_all_two():
+    s = TINY_SMALL
+    m = O.Model(s, seeded(s), max_ctx=64)
+    st = O.State(m, 2)
+    st.prefill(synth.gen_prompts(2, 12, s.V).numpy(), force=2)
+    for _ in range(5):
+        o = st.step(force=2)
+        assert np.all(o["n_acc"] == 0) and np.all(o["tokens"][:, 1] == -1)
+        assert all(st.seq(b)["p1"] == -1 for b in range(2))
+    assert [st.seq(b)["emitted"] for b in range(2)] == [1 + 5, 1 + 5]
+    st2 = O.State(m, 2)
+    st2.prefill(synth.gen_prompts(2, 12, s.V).numpy(), force=1)
+    for _ in range(5):
+        o = st2.step(force=1)
+        assert np.all(o["n_acc"] == 1) and np.all(o["tokens"][:, 1] == o["x_d"])
+    assert [st2.seq(b)["emitted"] for b in range(2)] == [2 + 10, 2 + 10]
+    # tau = 0 accepts every draft (c > 0), the same trajectory as forced accept
+    st3 = O.State(m, 2)
+    st3.prefill(synth.gen_prompts(2, 12, s.V).numpy(), tau=0.0)
+    st4 = O.State(m, 2)
+    st4.prefill(synth.gen_prompts(2, 12, s.V).numpy(), force=1)
+    for _ in range(3):
+        a, b = st3.step(tau=0.0), st4.step(force=1)
+        assert np.array_equal(a["tokens"], b["tokens"])
+
+
+def test_rollback_equals_never_appending():
+    s = TINY_SMALL
+    m = O.Model(s, seeded(s), max_ctx=40)
+    st = O.State(m, 2)
+    st.prefill(synth.gen_prompts(2, 14, s.V).numpy())
+    snap = [st.seq(b) for b in range(2)]
+    caches = [[st.cache(b, l, 40) for l in range(s.L + 1)] for b in range(2)]
+    ref = O.State(m, 2)
+    ref.prefill(synth.gen_prompts(2, 14, s.V).numpy())
+    for _ in range(4):
+        st.step()
+    st.rollback([snap[0]["n"], snap[1]["n"]])
+    st.set_pending([[snap[b]["p0"], snap[b]["p1"]] for b in range(2)])
+    for b in range(2):
+        assert st.seq(b)["n"] == snap[b]["n"]
+        for l in range(s.L + 1):
+            K, V = st.cache(b, l, 40)
+            assert np.array_equal(K, caches[b][l][0]) and np.array_equal(V, caches[b][l][1])
+    a, r = st.step(), ref.step()
+    assert np.array_equal(a["tokens"], r["tokens"]) and np.array_equal(a["logits_b"], r["logits_b"])
+
+
+def test_batch_equals_independent_sequences():
+    s = TINY_SMALL
+    m = O.Model(s, seeded(s), max_ctx=40)
+    prompts = synth.gen_prompts(3, 10, s.V, seed=9).numpy()
+    st = O.State(m, 3)
+    ob = [st.prefill(prompts)] + [st.step() for _ in range(3)]
+    for b in range(3):
+        one = O.State(m, 1)
+        o1 = [one.prefill(prompts[b:b + 1])] + [one.step() for _ in range(3)]
+        for x, y in zip(ob, o1):
+            assert np.array_equal(x["tokens"][b], y["tokens"][0])
+            assert np.array_equal(x["logits_d"][b], y["logits_d"][0])
+
+
+@pytest.mark.parametrize("odd", [False, True])
+def test_reprefill_of_history_reproduces_state(odd):
+    """prefill(prompt) then k steps equals prefill(prompt + the consumed pairs):
+    same caches in every layer, same next outputs (pair-level interface of
+    Sec. 3.1).  With odd=True the last consumed pair carries PAD in its second
+    slot, which a prompt of odd length expresses (PAD at the odd slot, App. B.2)."""
+    s = TINY_SMALL
+    m = O.Model(s, seeded(s, 5), max_ctx=40)
+    prompt = synth.gen_prompts(1, 8, s.V, seed=2).numpy()
+    st = O.State(m, 1)
+    st.prefill(prompt, force=1)
+    consumed = []
+    forces = [1, 1, 2, 0] if odd else [1, 1, 1, 1]
+    for f in forces:
+        consumed.append((st.seq(0)["p0"], st.seq(0)["p1"]))
+        o = st.step(force=f)
+    n_now = st.seq(0)["n"]
+    toks = list(prompt[0])
+    for i, (a, b) in enumerate(consumed):
+        toks.append(a)
+        if b >= 0:
+            toks.append(b)
+        else:
+            assert odd and i == len(consumed) - 1
+    st2 = O.State(m, 1)
+    o2 = st2.prefill(np.array([toks], np.int32), force=forces[-1])
+    assert st2.seq(0)["n"] == n_now
+    assert (st2.seq(0)["p0"], st2.seq(0)["p1"]) == (st.seq(0)["p0"], st.seq(0)["p1"])
+    assert np.array_equal(o["tokens"], o2["tokens"]) and np.array_equal(o["logits_d"], o2["logits_d"])
+    for l in range(s.L + 1):
+        K1, V1 = st.cache(0, l, n_now)
+        K2, V2 = st2.cache(0, l, n_now)
+        assert np.array_equal(K1, K2) and np.array_equal(V1, V2)
+    a, b = st.step(), st2.step()
+    assert np.array_equal(a["logits_b"], b["logits_b"]) and np.array_equal(a["tokens"], b["tokens"])
+
+
+def test_capacity_and_bad_ids_are_errors():
+    s = TINY_SMALL
+    m = O.Model(s, seeded(s), max_ctx=4)
+    st = O.State(m, 1)
+    with pytest.raises(ValueError):
+        st.prefill([[s.V, 1]])
+    st.prefill(synth.gen_prompts(1, 8, s.V).numpy())
+    with pytest.raises(ValueError):
+        st.step()

@@ -1,0 +1,335 @@
+#!/usr/bin/env python
+"""Throughput of the PIPO pair-decode step on one GB300 (one JSON line).
+
+A step is one pass of the whole hot path for every sequence of the batch:
+pair embed + compressor, L backbone blocks over the paged pair-KV cache, LM
+head + argmax, MTP head + argmax, confidence head, acceptance and the device
+bookkeeping.  Metric: accepted tokens/s over all sequences (1 + acceptance
+per sequence and step), with the pair-step latency and the HBM roofline.
+
+  python bench.py [--workload 4b-b1] [--steps K] [--warmup W] [--gpus N]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on host cores
+
+Inputs are synthetic and seeded (weights and prompts from synth.py); weights
+are streamed from HBM every step (9.3 GB/step for 4B > 129 MB L2), so no L2
+flush is needed between steps.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+# name -> model preset, batch, prompt tokens, pair-decode steps of the workload
+WORKLOADS = {
+    "tiny": dict(shape="tiny", batch=1, prompt=64, steps=32),
+    "4b-b1": dict(shape="4b", batch=1, prompt=2048, steps=512),
+    "4b-b4": dict(shape="4b", batch=4, prompt=1024, steps=256),
+    "4b-b16": dict(shape="4b", batch=16, prompt=1024, steps=256),
+    "4b-b64": dict(shape="4b", batch=64, prompt=1024, steps=256),
+    "4b-lc": dict(shape="4b", batch=4, prompt=30720, steps=1024, kv_fill=True),
+    "9b-b1": dict(shape="9b", batch=1, prompt=4096, steps=1024),
+    "9b-b8": dict(shape="9b", batch=8, prompt=4096, steps=1024),
+}
+METRIC = "accepted tokens/s/GPU (PIPO pair-decode step)"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="4b-b1", choices=sorted(WORKLOADS))
+    ap.add_argument("--impl", default="pipo", choices=["pipo", "reference"])
+    ap.add_argument("--tau", type=float, default=None)
+    ap.add_argument("--force", type=int, default=0, help="0 rule, 1 accept all, 2 reject all")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            threading.Thread(target=self._read, daemon=True).start()
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) == 8:
+                self.rows.append(parts)
+
+    def __exit__(self, *a):
+        if self.proc:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[4 + i].lower().startswith("active")})
+        pw = [float(r[2]) for r in self.rows if r[2].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.rows), "power_w_max": max(pw) if pw else None}
+
+
+# ---------------------------------------------------------------- helpers
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["hbm_gbs"], d.get("bf16_tflops"), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    return int(os.environ.get("RANK", "0")), ws, int(os.environ.get("LOCAL_RANK", "0"))
+
+
+def build_weights(shape, device):
+    from paper_2605_27255_gb300 import synth
+    return synth.gen_weights(shape, seed=0, device=device)
+
+
+def oracle_sample(shape, weights_host, batch, n_ctx, tau, force, budget_s, max_steps=None):
+    """Time the fp64 oracle on a bounded sample of the workload: decode
+    steps of `batch` sequences at context n_ctx, caches filled with seeded
+    values (the oracle's time does not depend on them)."""
+    import numpy as np
+    import torch
+
+    from oracle import oracle as O
+    from paper_2605_27255_gb300 import synth
+    model = O.Model(shape, weights_host, max_ctx=n_ctx + 64)
+    st = O.State(model, batch)
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    K, V = synth.gen_kv_fill(shape, n_ctx, seed=7, device=dev)
+    K, V = K.cpu().numpy(), V.cpu().numpy()
+    prompts = synth.gen_prompts(batch, 2, shape.V, seed=1).numpy()
+    for b in range(batch):
+        st.set_cache(b, K, V)
+    st.set_pending(np.stack([prompts[:, 0], prompts[:, 1]], 1))
+    del K, V
+    steps, toks, t0 = 0, 0, time.perf_counter()
+    while True:
+        o = st.step(tau=tau, force=force, logits=False)
+        steps += 1
+        toks += int(batch + o["n_acc"].sum())
+        el = time.perf_counter() - t0
+        if el >= budget_s or (max_steps and steps >= max_steps):
+            break
+    return dict(seconds=el, steps=steps, tokens=toks)
+
+
+# ---------------------------------------------------------------- reference arm
+
+def run_reference(args):
+    rank, ws, _ = dist_env()
+    if rank != 0:
+        return
+    import torch
+
+    from paper_2605_27255_gb300 import synth
+    wl = WORKLOADS[args.workload]
+    shape = synth.PRESETS[wl["shape"]]
+    tau = shape.tau if args.tau is None else args.tau
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    w = {k: v.cpu() for k, v in build_weights(shape, dev).items()}
+    n_ctx = (wl["prompt"] + 1) // 2
+    K = args.steps if args.steps is not None else 8
+    W = args.warmup
+    cores = os.cpu_count()
+    per_step = max(1.0, args.cpu_seconds / max(1, K + W))
+    oracle_sample(shape, w, wl["batch"], n_ctx, tau, args.force, 0.0, max_steps=max(1, W))
+    r = oracle_sample(shape, w, wl["batch"], n_ctx, tau, args.force, 1e9, max_steps=K)
+    tps = r["tokens"] / r["seconds"]
+    line = {
+        "impl": "reference", "metric": METRIC, "value": tps, "unit": "tokens/s", "n_gpus": ws, "steps": K,
+        "warmup": W, "ms_per_step": 1e3 * r["seconds"] / r["steps"], "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)",
+        "config": {"workload": args.workload, "shape": wl["shape"], "batch": wl["batch"],
+                   "context_entries": n_ctx, "tau": tau, "force_mode": args.force},
+        "cpu_baseline": {"value": tps, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{r['steps']} fp64 oracle decode steps of {wl['batch']} sequence(s) at "
+                                   f"context {n_ctx}, caches filled with seeded values"},
+        "e2e": {"value": tps, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------- GPU arm
+
+def run_pipo(args):
+    import numpy as np
+    import torch
+
+    from paper_2605_27255_gb300 import capi, roofline, synth
+
+    rank, ws, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    wl = WORKLOADS[args.workload]
+    shape = synth.PRESETS[wl["shape"]]
+    tau = shape.tau if args.tau is None else args.tau
+    B, T = wl["batch"], wl["prompt"]
+    K = args.steps if args.steps is not None else wl["steps"]
+    W = max(3, args.warmup)
+    n_pairs = (T + 1) // 2
+    max_ctx = n_pairs + W + 2 * K + 8
+
+    w = build_weights(shape, "cuda")
+    g = capi.Pipo(shape, w, max_batch=B, max_ctx=max_ctx, tau=tau, force_mode=args.force)
+    w_host = None
+    if rank == 0 and not args.no_cpu_baseline:
+        w_host = {k: v.cpu() for k, v in w.items()}
+    del w
+    torch.cuda.empty_cache()
+    stream = torch.cuda.Stream()
+    g.set_stream(stream.cuda_stream)
+
+    prompts = synth.gen_prompts(B, T if not wl.get("kv_fill") else 2, shape.V, seed=1 + rank * 1000).numpy()
+    t_pf = time.perf_counter()
+    g.prefill(prompts)
+    t_pf = time.perf_counter() - t_pf
+    if wl.get("kv_fill"):
+        Kf, Vf = synth.gen_kv_fill(shape, n_pairs, seed=7, device="cuda")
+        Kf, Vf = Kf.cpu().numpy(), Vf.cpu().numpy()
+        for b in range(B):
+            g.load_cache(b, Kf, Vf)
+        del Kf, Vf
+
+    for _ in range(W):
+        g.step_async()
+    torch.cuda.synchronize()
+    n0, e0 = g.counters()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        ev0.record(stream)
+        for _ in range(K):
+            g.step_async()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    n1, e1 = g.counters()
+    tokens = int((e1 - e0).sum())
+    ctx_avg = float(n0.mean()) + (K - 1) / 2.0
+    # end to end: the public host API, D2H of each step's outputs into pinned memory
+    tok_h = torch.empty((B, 2), dtype=torch.int32, pin_memory=True)
+    nacc_h = torch.empty((B,), dtype=torch.int32, pin_memory=True)
+    import ctypes as C
+    lib = capi.load()
+    _, e2a = g.counters()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(K):
+        rc = lib.pipo_decode_step(g.ctx, C.cast(tok_h.data_ptr(), capi._IP), C.cast(nacc_h.data_ptr(), capi._IP))
+        if rc != 0:
+            raise capi.PipoError(rc, capi.pipo_last_error(g.ctx))
+    e2e_s = time.perf_counter() - t0
+    _, e2b = g.counters()
+    e2e_tokens = int((e2b - e2a).sum())
+    launches = g.launches()
+
+    if ws > 1:
+        t = torch.tensor([ms, tokens, e2e_s, e2e_tokens], dtype=torch.float64, device="cuda")
+        mx = t.clone()
+        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+        sm = t.clone()
+        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+        ms_all, tokens_all, e2e_all, e2e_tok_all = float(mx[0]), float(sm[1]), float(mx[2]), float(sm[3])
+    else:
+        ms_all, tokens_all, e2e_all, e2e_tok_all = ms, tokens, e2e_s, e2e_tokens
+    value = tokens_all / (ms_all / 1e3)
+    hbm, tf, src = peaks()
+    step_s = ms / 1e3 / K
+    bytes_step = roofline.step_bytes(shape, B, ctx_avg)
+    achieved = bytes_step / step_s / 1e9
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline and w_host is not None:
+        r = oracle_sample(shape, w_host, B if B <= 4 else 1, n_pairs, tau, args.force, args.cpu_seconds)
+        nb = B if B <= 4 else 1
+        cpu = {"value": r["tokens"] / r["seconds"], "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"{r['steps']} fp64 oracle decode step(s) of {nb} sequence(s) at context {n_pairs}, "
+                         f"caches filled with seeded values ({r['seconds']:.1f} s)"}
+    if rank != 0:
+        if ws > 1:
+            dist.destroy_process_group()
+        return
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": K, "warmup": W,
+        "ms_per_step": ms_all / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": shape.dtype, "data": "synthetic (seeded weights and prompts)",
+        "config": {"workload": args.workload, "shape": wl["shape"], "batch": B, "prompt_tokens": T,
+                   "context_entries_avg": ctx_avg, "tau": tau, "force_mode": args.force,
+                   "acceptance": tokens / (K * B) - 1.0, "pair_step_us": 1e3 * ms / K,
+                   "prefill_s": t_pf, "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
+                   "parallelism": f"replicas x{ws}"},
+        "roofline": {"bound": "hbm", "kernel": "whole pair-decode step (graph)", "achieved": achieved,
+                     "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                     "algorithmic_bytes_per_step": bytes_step, "peak_source": src},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_tok_all / e2e_all, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": B * 12},
+        "gpu_launches": launches * K,
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    g.close()
+    if ws > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_pipo(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,197 @@
+/*
+ * pipo.h -- C ABI of the GB300 (sm_103a) PIPO pair-decode library.
+ *
+ * PIPO ("Pair-In, Pair-Out") decodes two tokens per backbone pass:
+ *   Eq. 1  z^i = f([x^{2i}; x^{2i+1}])           pair-in compressor
+ *   Eq. 2  h_b^i = Backbone(z^{<=i})              one decoder pass per pair
+ *   Eq. 3  x_b = argmax LMHead(h_b^i)             LM head tied to E (App. B.2)
+ *   Eq. 4  h_d^i = MTPHead(h_b^i, x_b)            App. A.2
+ *   Eq. 5  x_d = argmax LMHead(h_d^i)
+ *   Eq. 6  c^i = g([h_b^i; h_d^i])                confidence head, App. A.3
+ *   Sec. 3.1-3.2: the next pair is (x_b, x_d) when c >= tau, else (x_b, PAD).
+ *
+ * Conventions for every entry point:
+ *   - returns a pipo_status; never aborts the process; on failure the context
+ *     keeps its previous state and pipo_last_error() describes the failure;
+ *   - pointers named h_* or documented as "host" are host memory owned by the
+ *     caller, read or written before the call returns; "device" pointers are
+ *     device memory on the context's GPU, owned by the caller;
+ *   - token ids are int32 in [0, vocab); -1 marks the PAD slot of a pair;
+ *   - matrices are row-major [out, in] (a Linear layer's weight layout).
+ *
+ * Ownership: pipo_init copies the weights; the caller may free its buffers
+ * afterwards.  The context owns every device buffer it allocates and frees
+ * them in pipo_free.
+ */
+#ifndef PIPO_H
+#define PIPO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define PIPO_API __attribute__((visibility("default")))
+#else
+#define PIPO_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    PIPO_OK = 0,
+    PIPO_EINVAL = 1,     /* bad argument (null pointer, id out of range, shape) */
+    PIPO_ENOMEM = 2,     /* device allocation failed */
+    PIPO_ECAPACITY = 3,  /* a KV cache would exceed max_ctx entries */
+    PIPO_ECUDA = 4,      /* a CUDA runtime call failed */
+    PIPO_ESTATE = 5      /* call out of order (e.g. a step before prefill) */
+} pipo_status;
+
+typedef struct pipo_ctx pipo_ctx; /* opaque */
+
+/* Model dimensions and run-time switches. */
+typedef struct {
+    int32_t hidden;      /* H */
+    int32_t n_layers;    /* L backbone blocks */
+    int32_t n_q_heads;
+    int32_t n_kv_heads;  /* GQA: n_q_heads % n_kv_heads == 0 */
+    int32_t head_dim;    /* 64 or 128 */
+    int32_t ffn;         /* SwiGLU inner size F */
+    int32_t vocab;       /* V */
+    int32_t compressor;  /* 0: Linear W[a;b]+b;  1: MLP W2 SiLU(W1[a;b]) (App. A.1) */
+    int32_t mtp_block;   /* 1: W_fc then one decoder block (App. A.2); 0: W_fc only */
+    int32_t dtype;       /* 0: fp32 weights and KV;  1: bf16 weights and KV */
+    float rope_theta;    /* rotate-half RoPE base; position = pair index */
+    float rms_eps;       /* RMSNorm epsilon (inside the root) */
+    int32_t max_batch;   /* sequences decoded together */
+    int32_t max_ctx;     /* KV entries (pairs) per sequence, prompt included */
+    int32_t page_size;   /* entries per KV block; 64 */
+    float tau;           /* acceptance threshold tau_c (c >= tau accepts) */
+    int32_t force_mode;  /* 0: confidence rule; 1: accept every draft; 2: reject every draft */
+    int32_t debug;       /* 1: keep logits and head states for pipo_debug_dump */
+    uint32_t page_shuffle_seed; /* 0: blocks in order; else a seeded permutation of
+                                   the physical block pool (layout must not matter) */
+} pipo_config;
+
+/* Weights: one pointer per tensor, element type per pipo_config.dtype
+ * (float, or bf16 bit patterns as uint16).  Stacked tensors hold the L
+ * backbone blocks back to back.  `location`: 0 host, 1 device memory.
+ * Unused tensors (the other compressor variant, the MTP block when
+ * mtp_block == 0) may be NULL. */
+typedef struct {
+    int32_t location;
+    const void *E;          /* [V, H] token embedding, tied LM head */
+    const void *x_pad;      /* [H]    PAD embedding */
+    const void *comp_W;     /* [H, 2H] Linear compressor */
+    const void *comp_b;     /* [H] */
+    const void *comp_W1;    /* [H, 2H] MLP compressor */
+    const void *comp_W2;    /* [H, H] */
+    const void *attn_norm;  /* [L, H] */
+    const void *Wq;         /* [L, n_q*d_h, H] */
+    const void *Wk;         /* [L, n_kv*d_h, H] */
+    const void *Wv;         /* [L, n_kv*d_h, H] */
+    const void *Wo;         /* [L, H, n_q*d_h] */
+    const void *ffn_norm;   /* [L, H] */
+    const void *Wgate;      /* [L, F, H] */
+    const void *Wup;        /* [L, F, H] */
+    const void *Wdown;      /* [L, H, F] */
+    const void *final_norm; /* [H] */
+    const void *mtp_norm_h; /* [H]  norm of h_b at the MTP input */
+    const void *mtp_norm_e; /* [H]  norm of E[x_b] at the MTP input */
+    const void *mtp_W_fc;   /* [H, 2H] */
+    const void *m_attn_norm, *m_Wq, *m_Wk, *m_Wv, *m_Wo, *m_ffn_norm, *m_Wgate, *m_Wup, *m_Wdown; /* one block */
+    const void *mtp_norm_post; /* [H] norm before the LM head on h_d */
+    const void *conf_norm;  /* [2H] one RMSNorm over [h_b; h_d] */
+    const void *conf_W1;    /* [H, 2H] */
+    const void *conf_W2;    /* [1, H] */
+} pipo_weights;
+
+/* Head states of the last step (debug contexts only); host buffers. */
+typedef struct {
+    float *logits_b;   /* [B, V] backbone LM-head logits, or NULL */
+    float *logits_d;   /* [B, V] MTP LM-head logits, or NULL */
+    float *conf;       /* [B] confidence c, or NULL */
+    float *h_b;        /* [B, H] last backbone block output, or NULL */
+    float *h_d;        /* [B, H] MTP block output, or NULL */
+    int32_t *x_b;      /* [B] backbone argmax, or NULL */
+    int32_t *x_d;      /* [B] draft argmax (whether accepted or not), or NULL */
+} pipo_debug;
+
+/* Create a context on the current CUDA device: validates the config, copies
+ * the weights to device memory (fused QKV and gate|up layouts), allocates the
+ * paged KV caches (backbone layers and the MTP layer) for max_batch x max_ctx
+ * entries.  *out receives the context.  EINVAL for inconsistent shapes,
+ * ENOMEM when device memory runs out. */
+PIPO_API pipo_status pipo_init(const pipo_config *cfg, const pipo_weights *w, pipo_ctx **out);
+
+/* Prefill B sequences (B <= max_batch) from host token ids h_ids, row b at
+ * h_ids + b*stride, h_lens[b] tokens (1 <= len <= stride).  Tokens are paired
+ * (t_{2j}, t_{2j+1}); an odd length ends in (t_last, PAD) (App. B.2).  All
+ * sequences must yield the same number of pairs N (EINVAL otherwise).  Runs
+ * the backbone over the N latents, fills both caches, and runs the heads on
+ * the last latent: h_tokens[B,2] / h_n_accepted[B] (host, may be NULL) get
+ * the first pair output, which also becomes the pending pair.  Resets the
+ * emitted counters.  ECAPACITY when N > max_ctx. */
+PIPO_API pipo_status pipo_prefill(pipo_ctx *ctx, int32_t batch, const int32_t *h_ids, int32_t stride,
+                         const int32_t *h_lens, int32_t *h_tokens, int32_t *h_n_accepted);
+
+/* One pair-decode step of every prefilled sequence: compress the pending
+ * pair, one backbone pass, both heads, the confidence rule, next pair, KV
+ * append.  Host outputs (may be NULL): h_tokens[B,2] = (x_b, x_d or -1 when
+ * the draft was rejected), h_n_accepted[B] in {0,1}.  Synchronous.
+ * ESTATE before a prefill; ECAPACITY when a cache is full. */
+PIPO_API pipo_status pipo_decode_step(pipo_ctx *ctx, int32_t *h_tokens, int32_t *h_n_accepted);
+
+/* The same step, enqueued on the context stream without a host sync;
+ * d_tokens[B,2] / d_n_accepted[B] are device buffers (may be NULL).  The
+ * step is a captured CUDA graph replayed per call. */
+PIPO_API pipo_status pipo_decode_step_async(pipo_ctx *ctx, int32_t *d_tokens, int32_t *d_n_accepted);
+
+/* Truncate both KV caches of sequence b to h_n_pairs[b] entries (host,
+ * [B], each <= the current length).  Test and bookkeeping primitive: PIPO
+ * itself never caches a rejected draft (Sec. 3.1), so decoding never calls it.
+ * The pending pair is left as is (set it with pipo_set_pending). */
+PIPO_API pipo_status pipo_rollback(pipo_ctx *ctx, const int32_t *h_n_pairs);
+
+/* Acceptance threshold and force mode (0 rule, 1 accept all, 2 reject all). */
+PIPO_API pipo_status pipo_set_threshold(pipo_ctx *ctx, float tau, int32_t force_mode);
+
+/* Test hook for forced replay: overwrite the pending pairs, host [B,2]
+ * (slot 1 may be -1 = PAD). */
+PIPO_API pipo_status pipo_set_pending(pipo_ctx *ctx, const int32_t *h_pairs);
+
+/* Host copies of the per-sequence counters: kv entries [B] and tokens
+ * emitted since the prefill [B] (either may be NULL). */
+PIPO_API pipo_status pipo_get_counters(pipo_ctx *ctx, int32_t *h_kv_len, int64_t *h_emitted);
+
+/* Head states of the last step or prefill (requires cfg.debug = 1). */
+PIPO_API pipo_status pipo_debug_dump(pipo_ctx *ctx, const pipo_debug *out);
+
+/* Host fp32 copy of cache entries [0, n) of sequence b, layer l (l == L is
+ * the MTP layer): h_K, h_V [n, n_kv*d_h]. */
+PIPO_API pipo_status pipo_read_cache(pipo_ctx *ctx, int32_t b, int32_t layer, int32_t n, float *h_K, float *h_V);
+
+/* Write n entries into every cache layer of sequence b and set its length
+ * to n: host fp32 [L+1, n, n_kv*d_h] (rounded to the cache type).  For
+ * timing runs that need a long context without a long prefill. */
+PIPO_API pipo_status pipo_load_cache(pipo_ctx *ctx, int32_t b, int32_t n, const float *h_K, const float *h_V);
+
+/* Use a caller-owned CUDA stream (cudaStream_t) for all later work; NULL
+ * restores the context's own stream.  Drops the captured step graph. */
+PIPO_API pipo_status pipo_set_stream(pipo_ctx *ctx, void *stream);
+
+/* Number of kernel launches one decode step enqueues (for launch accounting). */
+PIPO_API int32_t pipo_step_launches(const pipo_ctx *ctx);
+
+/* Message of the last failure on this context (or of the last failed
+ * pipo_init when ctx is NULL); never NULL. */
+PIPO_API const char *pipo_last_error(const pipo_ctx *ctx);
+
+/* Release every device buffer and the context; NULL is a no-op. */
+PIPO_API void pipo_free(pipo_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PIPO_H */

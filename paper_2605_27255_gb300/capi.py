@@ -1,0 +1,302 @@
+"""Thin ctypes binding of the C ABI in ``include/pipo.h``.
+
+Argument marshalling only: every step of the decode path runs in the CUDA
+library (``lib/libpipo.so``).  There is no Python or CPU fallback; loading
+fails loudly when the library has not been built.  Function names mirror the
+C entry points (``pipo_init``, ``pipo_prefill``, ``pipo_decode_step`` ...);
+``Pipo`` wraps one context for convenience.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+from typing import Dict, Optional
+
+import numpy as np
+import torch
+
+from .synth import ModelShape
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "libpipo.so")
+
+PIPO_OK, PIPO_EINVAL, PIPO_ENOMEM, PIPO_ECAPACITY, PIPO_ECUDA, PIPO_ESTATE = range(6)
+_NAMES = {0: "OK", 1: "EINVAL", 2: "ENOMEM", 3: "ECAPACITY", 4: "ECUDA", 5: "ESTATE"}
+
+
+class PipoError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"PIPO_{_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+class pipo_config(C.Structure):
+    _fields_ = [(n, C.c_int32) for n in ("hidden", "n_layers", "n_q_heads", "n_kv_heads", "head_dim", "ffn",
+                                         "vocab", "compressor", "mtp_block", "dtype")] + \
+               [("rope_theta", C.c_float), ("rms_eps", C.c_float)] + \
+               [(n, C.c_int32) for n in ("max_batch", "max_ctx", "page_size")] + \
+               [("tau", C.c_float), ("force_mode", C.c_int32), ("debug", C.c_int32),
+                ("page_shuffle_seed", C.c_uint32)]
+
+
+# C field -> tensor name of synth.tensor_shapes
+WEIGHT_FIELDS = [
+    ("E", "E"), ("x_pad", "x_pad"), ("comp_W", "comp.W"), ("comp_b", "comp.b"),
+    ("comp_W1", "comp.W1"), ("comp_W2", "comp.W2"),
+    ("attn_norm", "blk.attn_norm"), ("Wq", "blk.Wq"), ("Wk", "blk.Wk"), ("Wv", "blk.Wv"),
+    ("Wo", "blk.Wo"), ("ffn_norm", "blk.ffn_norm"), ("Wgate", "blk.Wgate"), ("Wup", "blk.Wup"),
+    ("Wdown", "blk.Wdown"), ("final_norm", "final_norm"),
+    ("mtp_norm_h", "mtp.norm_h"), ("mtp_norm_e", "mtp.norm_e"), ("mtp_W_fc", "mtp.W_fc"),
+    ("m_attn_norm", "mtp.attn_norm"), ("m_Wq", "mtp.Wq"), ("m_Wk", "mtp.Wk"), ("m_Wv", "mtp.Wv"),
+    ("m_Wo", "mtp.Wo"), ("m_ffn_norm", "mtp.ffn_norm"), ("m_Wgate", "mtp.Wgate"), ("m_Wup", "mtp.Wup"),
+    ("m_Wdown", "mtp.Wdown"), ("mtp_norm_post", "mtp.norm_post"),
+    ("conf_norm", "conf.norm"), ("conf_W1", "conf.W1"), ("conf_W2", "conf.W2"),
+]
+
+
+class pipo_weights(C.Structure):
+    _fields_ = [("location", C.c_int32)] + [(f, C.c_void_p) for f, _ in WEIGHT_FIELDS]
+
+
+_FP = C.POINTER(C.c_float)
+_IP = C.POINTER(C.c_int32)
+
+
+class pipo_debug(C.Structure):
+    _fields_ = [("logits_b", _FP), ("logits_d", _FP), ("conf", _FP), ("h_b", _FP), ("h_d", _FP),
+                ("x_b", _IP), ("x_d", _IP)]
+
+
+# name -> (restype, argtypes): every entry point declared in include/pipo.h
+SIGNATURES = {
+    "pipo_init": (C.c_int, [C.POINTER(pipo_config), C.POINTER(pipo_weights), C.POINTER(C.c_void_p)]),
+    "pipo_prefill": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.c_int32, _IP, _IP, _IP]),
+    "pipo_decode_step": (C.c_int, [C.c_void_p, _IP, _IP]),
+    "pipo_decode_step_async": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "pipo_rollback": (C.c_int, [C.c_void_p, _IP]),
+    "pipo_set_threshold": (C.c_int, [C.c_void_p, C.c_float, C.c_int32]),
+    "pipo_set_pending": (C.c_int, [C.c_void_p, _IP]),
+    "pipo_get_counters": (C.c_int, [C.c_void_p, _IP, C.POINTER(C.c_int64)]),
+    "pipo_debug_dump": (C.c_int, [C.c_void_p, C.POINTER(pipo_debug)]),
+    "pipo_read_cache": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, _FP, _FP]),
+    "pipo_load_cache": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, _FP, _FP]),
+    "pipo_set_stream": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "pipo_step_launches": (C.c_int32, [C.c_void_p]),
+    "pipo_last_error": (C.c_char_p, [C.c_void_p]),
+    "pipo_free": (None, [C.c_void_p]),
+}
+
+_lib = None
+_lock = threading.Lock()
+
+
+def load(path: str = LIB_PATH):
+    """Load the CUDA library (raises if it is missing: no fallback)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(path):
+                raise RuntimeError(f"PIPO CUDA library not built: {path} (run __graft_entry__.build())")
+            L = C.CDLL(path)
+            for name, (res, args) in SIGNATURES.items():
+                fn = getattr(L, name)
+                fn.restype = res
+                fn.argtypes = args
+            _lib = L
+    return _lib
+
+
+def _check(rc: int, ctx) -> None:
+    if rc != PIPO_OK:
+        msg = load().pipo_last_error(ctx).decode()
+        raise PipoError(rc, msg)
+
+
+def _i32(a) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+
+
+def _ip(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(_IP)
+
+
+def _fp(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(_FP)
+
+
+# ---- entry points (same names as the C ABI) -----------------------------
+
+def pipo_init(cfg: pipo_config, w: pipo_weights):
+    ctx = C.c_void_p()
+    _check(load().pipo_init(C.byref(cfg), C.byref(w), C.byref(ctx)), None)
+    return ctx
+
+
+def pipo_prefill(ctx, ids: np.ndarray, lens: Optional[np.ndarray] = None):
+    ids = _i32(ids)
+    B, stride = ids.shape
+    lens = _i32(np.full(B, stride) if lens is None else lens)
+    tok = np.zeros((B, 2), np.int32)
+    nacc = np.zeros(B, np.int32)
+    _check(load().pipo_prefill(ctx, B, _ip(ids), stride, _ip(lens), _ip(tok), _ip(nacc)), ctx)
+    return tok, nacc
+
+
+def pipo_decode_step(ctx, B: int):
+    tok = np.zeros((B, 2), np.int32)
+    nacc = np.zeros(B, np.int32)
+    _check(load().pipo_decode_step(ctx, _ip(tok), _ip(nacc)), ctx)
+    return tok, nacc
+
+
+def pipo_decode_step_async(ctx, d_tokens: int = 0, d_nacc: int = 0):
+    _check(load().pipo_decode_step_async(ctx, C.c_void_p(d_tokens or None), C.c_void_p(d_nacc or None)), ctx)
+
+
+def pipo_rollback(ctx, n_pairs) -> None:
+    _check(load().pipo_rollback(ctx, _ip(_i32(n_pairs))), ctx)
+
+
+def pipo_set_threshold(ctx, tau: float, force_mode: int = 0) -> None:
+    _check(load().pipo_set_threshold(ctx, float(tau), int(force_mode)), ctx)
+
+
+def pipo_set_pending(ctx, pairs) -> None:
+    _check(load().pipo_set_pending(ctx, _ip(_i32(pairs))), ctx)
+
+
+def pipo_get_counters(ctx, B: int):
+    n = np.zeros(B, np.int32)
+    e = np.zeros(B, np.int64)
+    _check(load().pipo_get_counters(ctx, _ip(n), e.ctypes.data_as(C.POINTER(C.c_int64))), ctx)
+    return n, e
+
+
+def pipo_debug_dump(ctx, B: int, V: int, H: int) -> Dict[str, np.ndarray]:
+    o = dict(logits_b=np.zeros((B, V), np.float32), logits_d=np.zeros((B, V), np.float32),
+             conf=np.zeros(B, np.float32), h_b=np.zeros((B, H), np.float32), h_d=np.zeros((B, H), np.float32),
+             x_b=np.zeros(B, np.int32), x_d=np.zeros(B, np.int32))
+    d = pipo_debug(*[(_ip(v) if v.dtype == np.int32 else _fp(v)) for v in o.values()])
+    _check(load().pipo_debug_dump(ctx, C.byref(d)), ctx)
+    return o
+
+
+def pipo_read_cache(ctx, b: int, layer: int, n: int, kd: int):
+    K = np.zeros((n, kd), np.float32)
+    V = np.zeros((n, kd), np.float32)
+    _check(load().pipo_read_cache(ctx, b, layer, n, _fp(K), _fp(V)), ctx)
+    return K, V
+
+
+def pipo_load_cache(ctx, b: int, K: np.ndarray, V: np.ndarray) -> None:
+    K = np.ascontiguousarray(K, dtype=np.float32)
+    V = np.ascontiguousarray(V, dtype=np.float32)
+    _check(load().pipo_load_cache(ctx, b, K.shape[1], _fp(K), _fp(V)), ctx)
+
+
+def pipo_set_stream(ctx, stream: int) -> None:
+    _check(load().pipo_set_stream(ctx, C.c_void_p(stream or None)), ctx)
+
+
+def pipo_step_launches(ctx) -> int:
+    return int(load().pipo_step_launches(ctx))
+
+
+def pipo_last_error(ctx=None) -> str:
+    return load().pipo_last_error(ctx).decode()
+
+
+def pipo_free(ctx) -> None:
+    if ctx:
+        load().pipo_free(ctx)
+
+
+# ---- convenience --------------------------------------------------------
+
+def make_config(s: ModelShape, max_batch: int, max_ctx: int, *, tau: Optional[float] = None,
+                force_mode: int = 0, debug: bool = False, page_size: int = 64,
+                page_shuffle_seed: int = 0) -> pipo_config:
+    return pipo_config(s.H, s.L, s.n_q, s.n_kv, s.d_h, s.F, s.V, 0 if s.compressor == "linear" else 1,
+                       s.mtp_block, 1 if s.dtype == "bf16" else 0, s.rope_theta, s.eps, max_batch, max_ctx,
+                       page_size, s.tau if tau is None else tau, force_mode, int(debug), page_shuffle_seed)
+
+
+def make_weights(weights: Dict[str, torch.Tensor], keep: list) -> pipo_weights:
+    """pipo_weights over a dict of torch tensors (all on the CPU or all on
+    the GPU); ``keep`` receives the contiguous buffers that must outlive
+    pipo_init."""
+    w = pipo_weights()
+    loc = None
+    for field, name in WEIGHT_FIELDS:
+        t = weights.get(name)
+        if t is None:
+            continue
+        t = t.contiguous()
+        keep.append(t)
+        here = 1 if t.is_cuda else 0
+        if loc is not None and here != loc:
+            raise ValueError("weights must all be on the host or all on the device")
+        loc = here
+        setattr(w, field, t.data_ptr())
+    w.location = loc or 0
+    return w
+
+
+class Pipo:
+    """One library context: ``Pipo(shape, weights, max_batch, max_ctx)``."""
+
+    def __init__(self, shape: ModelShape, weights: Dict[str, torch.Tensor], max_batch: int, max_ctx: int, **kw):
+        self.shape = shape
+        self.cfg = make_config(shape, max_batch, max_ctx, **kw)
+        keep: list = []
+        self.ctx = pipo_init(self.cfg, make_weights(weights, keep))
+        self.B = 0
+
+    def close(self):
+        if getattr(self, "ctx", None):
+            pipo_free(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def prefill(self, ids, lens=None):
+        ids = _i32(ids)
+        self.B = ids.shape[0]
+        return pipo_prefill(self.ctx, ids, lens)
+
+    def step(self):
+        return pipo_decode_step(self.ctx, self.B)
+
+    def step_async(self, d_tokens: int = 0, d_nacc: int = 0):
+        pipo_decode_step_async(self.ctx, d_tokens, d_nacc)
+
+    def set_threshold(self, tau, force_mode=0):
+        pipo_set_threshold(self.ctx, tau, force_mode)
+
+    def set_pending(self, pairs):
+        pipo_set_pending(self.ctx, pairs)
+
+    def rollback(self, n):
+        pipo_rollback(self.ctx, n)
+
+    def counters(self):
+        return pipo_get_counters(self.ctx, self.B)
+
+    def debug(self):
+        return pipo_debug_dump(self.ctx, self.B, self.shape.V, self.shape.H)
+
+    def read_cache(self, b, layer, n):
+        return pipo_read_cache(self.ctx, b, layer, n, self.shape.n_kv * self.shape.d_h)
+
+    def load_cache(self, b, K, V):
+        pipo_load_cache(self.ctx, b, K, V)
+
+    def set_stream(self, stream: int):
+        pipo_set_stream(self.ctx, stream)
+
+    def launches(self) -> int:
+        return pipo_step_launches(self.ctx)

@@ -1,0 +1,521 @@
+// Device kernels of the PIPO pair-decode step (sm_103a).
+//
+// Every weight matrix is streamed from HBM once per step; activations stay in
+// fp32; weights, embeddings and the KV cache are bf16 (or fp32 for fp32
+// models).  The step is a chain of these kernels replayed as one CUDA graph.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace pipo {
+
+constexpr int kThreads = 256;  // GEMV block
+constexpr int kWarps = kThreads / 32;
+
+enum Epi : int {
+    EPI_STORE = 0,   // y = W x
+    EPI_BIAS = 1,    // y = W x + bias
+    EPI_SILU = 2,    // y = SiLU(W x)
+    EPI_RESADD = 3,  // y += W x            (residual stream; split-K: fixed-order sum)
+    EPI_SWIGLU = 4,  // y = SiLU(W_r x) * (W_{r+F} x)   (gate rows, then up rows)
+    EPI_ARGMAX = 5,  // packed (logit, -row) max per sequence; optional logits
+};
+
+// One input segment of a GEMV: either fp32 activations or an embedding-row
+// gather, optionally RMS-normalised (y = x / sqrt(mean(x^2) + eps) * gamma).
+struct Seg {
+    const float* src;                  // [B, ld] activations, or nullptr (gather)
+    int ld;
+    const void* table;                 // gather table [*, K] (weight type)
+    const void* pad;                   // [K] row used for token id < 0 (PAD)
+    const int32_t* tok;                // token of sequence b: tok[b * tok_ld]
+    int tok_ld;
+    const unsigned long long* tok_am;  // or: packed argmax of sequence b
+    const void* gamma;                 // [K] gain or nullptr (no norm)
+    int K;
+};
+
+struct GemvParams {
+    Seg seg[2];
+    int nseg;
+    int joint_norm;      // one RMSNorm over the concatenation (gain in seg[0].gamma, length K)
+    const void* W;       // [rows, K]
+    int N;               // output rows
+    int K;               // input length (sum of the segments)
+    int rstride;         // EPI_SWIGLU: offset of the up rows
+    int epi;
+    float* y;
+    int ldy;
+    const void* bias;
+    unsigned long long* am;  // EPI_ARGMAX target [B]
+    float* dbg;              // EPI_ARGMAX logits [B, ld_dbg] or nullptr
+    int ld_dbg;
+    int B;
+    int splitk;
+    float eps;
+    unsigned long long* zero_ptr;  // zeroed by block 0 before anything else (or nullptr)
+    int zero_n;
+    float* part;         // EPI_RESADD with splitk > 1: partials [splitk][B][N]
+    unsigned* rowcnt;    // per-row arrival counters (zero between launches)
+};
+
+// ---------------------------------------------------------------- loads
+
+__device__ __forceinline__ uint4 ldg_stream(const void* p) {
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+        : "l"(p));
+    return r;
+}
+
+__device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
+
+template <typename T> struct W8;  // 8 consecutive weights
+
+template <> struct W8<__nv_bfloat16> {
+    uint4 v;
+    __device__ __forceinline__ void load(const __nv_bfloat16* p) { v = ldg_stream(p); }
+    __device__ __forceinline__ void unpack(float (&f)[8]) const {
+        f[0] = bf_lo(v.x); f[1] = bf_hi(v.x); f[2] = bf_lo(v.y); f[3] = bf_hi(v.y);
+        f[4] = bf_lo(v.z); f[5] = bf_hi(v.z); f[6] = bf_lo(v.w); f[7] = bf_hi(v.w);
+    }
+};
+
+template <> struct W8<float> {
+    uint4 a, b;
+    __device__ __forceinline__ void load(const float* p) { a = ldg_stream(p); b = ldg_stream(p + 4); }
+    __device__ __forceinline__ void unpack(float (&f)[8]) const {
+        f[0] = __uint_as_float(a.x); f[1] = __uint_as_float(a.y); f[2] = __uint_as_float(a.z); f[3] = __uint_as_float(a.w);
+        f[4] = __uint_as_float(b.x); f[5] = __uint_as_float(b.y); f[6] = __uint_as_float(b.z); f[7] = __uint_as_float(b.w);
+    }
+};
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ float ldw(const void* p, size_t i) {
+    return to_f(static_cast<const T*>(p)[i]);
+}
+template <typename T> __device__ __forceinline__ T from_f(float v);
+template <> __device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+__device__ __forceinline__ float silu(float x) { return x / (1.0f + expf(-x)); }
+
+// Packed argmax key: higher logit first, then lower row.
+__device__ __forceinline__ unsigned long long argmax_key(float v, int row) {
+    uint32_t u = __float_as_uint(v);
+    uint32_t o = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+    return ((unsigned long long)o << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)row);
+}
+__device__ __forceinline__ int argmax_row(unsigned long long k) {
+    return (int)(0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFull));
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// ---------------------------------------------------------------- GEMV
+//
+// y[b, r] = epi( sum_k W[r, k] * xin[b, k] ),  xin = staged (gathered,
+// normalised) input in shared memory, NB sequences at a time.  A warp owns one
+// (row, K-slice) task at a time and streams its weights with 128-bit
+// non-allocating loads, kU chunks in flight per lane.
+template <typename T, int NB, bool TWO>
+__global__ void __launch_bounds__(kThreads) gemv_kernel(GemvParams p) {
+    extern __shared__ float4 smem4[];
+    float* xs = reinterpret_cast<float*>(smem4);  // [NB][K]
+    __shared__ float rstd_s[NB][2];
+    constexpr int kU = 8;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int K = p.K;
+    const T* W = static_cast<const T*>(p.W);
+
+    if (p.zero_ptr && blockIdx.x == 0)
+        for (int i = threadIdx.x; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
+
+    const int S = p.splitk;
+    const int Ks = ((K + S * 8 - 1) / (S * 8)) * 8;
+    const int tasks = p.N * S;
+
+    for (int b0 = 0; b0 < p.B; b0 += NB) {
+        const int nb = min(NB, p.B - b0);
+        __syncthreads();
+        // ---- stage inputs
+        for (int bb = 0; bb < NB; ++bb) {
+            const int b = b0 + bb;
+            int koff = 0;
+            for (int s = 0; s < p.nseg; ++s) {
+                const Seg& sg = p.seg[s];
+                int tok = 0;
+                if (!sg.src && bb < nb) tok = sg.tok_am ? argmax_row(sg.tok_am[b]) : sg.tok[(size_t)b * sg.tok_ld];
+                for (int k = threadIdx.x; k < sg.K; k += blockDim.x) {
+                    float v = 0.f;
+                    if (bb < nb) {
+                        if (sg.src) v = sg.src[(size_t)b * sg.ld + k];
+                        else v = (tok < 0) ? ldw<T>(sg.pad, k) : ldw<T>(sg.table, (size_t)tok * sg.K + k);
+                    }
+                    xs[bb * K + koff + k] = v;
+                }
+                koff += sg.K;
+            }
+        }
+        __syncthreads();
+        // ---- RMSNorm of each segment (or of the concatenation): one warp per sum
+        const bool any_norm = p.seg[0].gamma || (p.nseg > 1 && p.seg[1].gamma);
+        if (any_norm) {
+            const int ngrp = p.joint_norm ? 1 : p.nseg;
+            for (int q = warp; q < NB * ngrp; q += kWarps) {
+                const int bb = q / ngrp, s = q % ngrp;
+                const int k0 = (s == 0) ? 0 : p.seg[0].K;
+                const int len = p.joint_norm ? K : p.seg[s].K;
+                float ss = 0.f;
+                for (int k = lane; k < len; k += 32) {
+                    float v = xs[bb * K + k0 + k];
+                    ss += v * v;
+                }
+                ss = warp_sum(ss);
+                if (lane == 0) rstd_s[bb][s] = 1.0f / sqrtf(ss / (float)len + p.eps);
+            }
+            __syncthreads();
+            for (int bb = 0; bb < NB; ++bb) {
+                for (int k = threadIdx.x; k < K; k += blockDim.x) {
+                    int s = (p.joint_norm || k < p.seg[0].K) ? 0 : 1;
+                    const Seg& sg = p.seg[s];
+                    if (!sg.gamma) continue;
+                    int kk = (p.joint_norm || s == 0) ? k : k - p.seg[0].K;
+                    xs[bb * K + k] *= rstd_s[bb][s] * ldw<T>(sg.gamma, kk);
+                }
+            }
+            __syncthreads();
+        }
+
+        // ---- rows
+        float best_v[NB];
+        int best_r[NB];
+#pragma unroll
+        for (int bb = 0; bb < NB; ++bb) { best_v[bb] = -INFINITY; best_r[bb] = 0x7fffffff; }
+
+        for (int t = blockIdx.x * kWarps + warp; t < tasks; t += gridDim.x * kWarps) {
+            const int r = t / S, s = t % S;
+            const int k0 = s * Ks, k1 = min(K, k0 + Ks);
+            float acc0[NB], acc1[NB];
+#pragma unroll
+            for (int bb = 0; bb < NB; ++bb) { acc0[bb] = 0.f; acc1[bb] = 0.f; }
+            const T* w0 = W + (size_t)r * K;
+            const T* w1 = W + (size_t)(r + p.rstride) * K;
+            for (int kb = k0 + lane * 8; kb < k1; kb += 256 * kU) {
+                W8<T> wa[kU], wb[kU];
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int k = kb + u * 256;
+                    if (k < k1) {
+                        wa[u].load(w0 + k);
+                        if (TWO) wb[u].load(w1 + k);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < kU; ++u) {
+                    const int k = kb + u * 256;
+                    if (k < k1) {
+                        float fa[8], fb[8];
+                        wa[u].unpack(fa);
+                        if (TWO) wb[u].unpack(fb);
+#pragma unroll
+                        for (int bb = 0; bb < NB; ++bb) {
+                            const float4 x0 = *reinterpret_cast<const float4*>(xs + bb * K + k);
+                            const float4 x1 = *reinterpret_cast<const float4*>(xs + bb * K + k + 4);
+                            acc0[bb] += fa[0] * x0.x + fa[1] * x0.y + fa[2] * x0.z + fa[3] * x0.w +
+                                        fa[4] * x1.x + fa[5] * x1.y + fa[6] * x1.z + fa[7] * x1.w;
+                            if (TWO)
+                                acc1[bb] += fb[0] * x0.x + fb[1] * x0.y + fb[2] * x0.z + fb[3] * x0.w +
+                                            fb[4] * x1.x + fb[5] * x1.y + fb[6] * x1.z + fb[7] * x1.w;
+                        }
+                    }
+                }
+            }
+#pragma unroll
+            for (int bb = 0; bb < NB; ++bb) {
+                acc0[bb] = warp_sum(acc0[bb]);
+                if (TWO) acc1[bb] = warp_sum(acc1[bb]);
+            }
+            if (p.epi == EPI_ARGMAX) {
+#pragma unroll
+                for (int bb = 0; bb < NB; ++bb)
+                    if (acc0[bb] > best_v[bb] || (acc0[bb] == best_v[bb] && r < best_r[bb])) {
+                        best_v[bb] = acc0[bb];
+                        best_r[bb] = r;
+                    }
+                if (p.dbg && lane < nb) {
+#pragma unroll
+                    for (int bb = 0; bb < NB; ++bb)
+                        if (bb == lane) p.dbg[(size_t)(b0 + bb) * p.ld_dbg + r] = acc0[bb];
+                }
+                continue;
+            }
+            if (lane < nb) {
+#pragma unroll
+                for (int bb = 0; bb < NB; ++bb) {
+                    if (bb != lane) continue;
+                    float* yp = p.y + (size_t)(b0 + bb) * p.ldy + r;
+                    const float a = acc0[bb];
+                    switch (p.epi) {
+                        case EPI_STORE: *yp = a; break;
+                        case EPI_BIAS: *yp = a + ldw<T>(p.bias, r); break;
+                        case EPI_SILU: *yp = silu(a); break;
+                        case EPI_RESADD:
+                            if (S == 1) *yp += a;
+                            break;
+                        case EPI_SWIGLU: *yp = silu(a) * acc1[bb]; break;
+                        default: break;
+                    }
+                }
+            }
+            // split-K residual add: every slice stores its partial; the last
+            // slice of the row to arrive adds them in slice order (deterministic).
+            if (p.epi == EPI_RESADD && S > 1 && lane == 0) {
+                for (int bb = 0; bb < nb; ++bb) p.part[((size_t)s * p.B + b0 + bb) * p.N + r] = acc0[bb];
+                __threadfence();
+                const unsigned prev = atomicAdd(p.rowcnt + r, 1u);
+                if (prev == (unsigned)S - 1) {
+                    __threadfence();
+                    for (int bb = 0; bb < nb; ++bb) {
+                        float sum = 0.f;
+                        for (int ss = 0; ss < S; ++ss) sum += __ldcg(p.part + ((size_t)ss * p.B + b0 + bb) * p.N + r);
+                        p.y[(size_t)(b0 + bb) * p.ldy + r] += sum;
+                    }
+                    p.rowcnt[r] = 0u;
+                }
+            }
+        }
+        if (p.epi == EPI_ARGMAX && lane < nb) {
+#pragma unroll
+            for (int bb = 0; bb < NB; ++bb)
+                if (bb == lane && best_r[bb] != 0x7fffffff)
+                    atomicMax(p.am + b0 + bb, argmax_key(best_v[bb], best_r[bb]));
+        }
+    }
+}
+
+// ---------------------------------------------------------------- attention
+
+struct KVView {
+    void* K;                  // layer base: [blocks][n_kv][page][d_h]
+    void* V;
+    const int32_t* table;     // [B][blocks_per_seq]
+    int blocks_per_seq;
+    int page;
+    int n_kv;
+};
+
+template <typename T, int DH>
+__device__ __forceinline__ size_t kv_off(const KVView& kv, int b, int pos, int g) {
+    const int blk = kv.table[(size_t)b * kv.blocks_per_seq + pos / kv.page];
+    return (((size_t)blk * kv.n_kv + g) * kv.page + (pos % kv.page)) * DH;
+}
+
+// RoPE on q and k (rotate-half, angle = pos * theta^(-2i/d) in double), then
+// the new k and v appended at entry pos = n[b].  grid (B, n_q + 2 n_kv), DH/2 threads.
+template <typename T, int DH>
+__global__ void rope_append_kernel(const float* __restrict__ qkv, int ld_qkv, float* __restrict__ q_out,
+                                   KVView kv, const int32_t* __restrict__ n_pos, int n_q, double theta) {
+    const int b = blockIdx.x, h = blockIdx.y, i = threadIdx.x;
+    const int pos = n_pos[b];
+    const float* src = qkv + (size_t)b * ld_qkv + (size_t)h * DH;
+    const int n_kv = kv.n_kv;
+    if (h >= n_q + n_kv) {  // value head: copy into the cache
+        const int g = h - n_q - n_kv;
+        T* dst = static_cast<T*>(kv.V) + kv_off<T, DH>(kv, b, pos, g);
+        dst[i] = from_f<T>(src[i]);
+        dst[i + DH / 2] = from_f<T>(src[i + DH / 2]);
+        return;
+    }
+    double sn, cs;
+    sincos((double)pos * pow(theta, -2.0 * (double)i / (double)DH), &sn, &cs);
+    const float c = (float)cs, s = (float)sn;
+    const float a = src[i], bb = src[i + DH / 2];
+    const float ra = a * c - bb * s, rb = bb * c + a * s;
+    if (h < n_q) {
+        q_out[(size_t)b * n_q * DH + (size_t)h * DH + i] = ra;
+        q_out[(size_t)b * n_q * DH + (size_t)h * DH + i + DH / 2] = rb;
+    } else {
+        const int g = h - n_q;
+        T* dst = static_cast<T*>(kv.K) + kv_off<T, DH>(kv, b, pos, g);
+        dst[i] = from_f<T>(ra);
+        dst[i + DH / 2] = from_f<T>(rb);
+    }
+}
+
+// Split-KV flash decode.  grid (S, n_kv, B), 128 threads (4 warps).  CTA
+// (s, g, b) attends the G = n_q/n_kv query heads of group g over its slice
+// of entries [0, n[b]] and writes (m, l, o) partials; the last CTA of (b, g)
+// to finish merges the S partials (log-sum-exp) into out[b, h*DH + t].
+template <typename T, int DH, int G>
+__global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restrict__ q, KVView kv,
+                                                          const int32_t* __restrict__ n_pos, float* __restrict__ out,
+                                                          float* __restrict__ part_o, float* __restrict__ part_ml,
+                                                          unsigned int* __restrict__ counters, int S, float scale) {
+    constexpr int EPL = DH / 32;  // elements per lane
+    const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_kv = kv.n_kv, n_q = n_kv * G;
+    const int len = n_pos[b] + 1;
+    const int chunk = (len + S - 1) / S;
+    const int j0 = s * chunk, j1 = min(len, j0 + chunk);
+
+    float qr[G][EPL];
+#pragma unroll
+    for (int hh = 0; hh < G; ++hh)
+#pragma unroll
+        for (int e = 0; e < EPL; ++e)
+            qr[hh][e] = q[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + lane * EPL + e] * scale;
+
+    float m[G], l[G], o[G][EPL];
+#pragma unroll
+    for (int hh = 0; hh < G; ++hh) {
+        m[hh] = -INFINITY; l[hh] = 0.f;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) o[hh][e] = 0.f;
+    }
+    const T* Kb = static_cast<const T*>(kv.K);
+    const T* Vb = static_cast<const T*>(kv.V);
+    for (int j = j0 + warp; j < j1; j += 4) {
+        const size_t off = kv_off<T, DH>(kv, b, j, g) + lane * EPL;
+        float kk[EPL], vv[EPL];
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) { kk[e] = to_f(Kb[off + e]); vv[e] = to_f(Vb[off + e]); }
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) {
+            float d = 0.f;
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) d += qr[hh][e] * kk[e];
+            d = warp_sum(d);
+            const float mn = fmaxf(m[hh], d);
+            const float corr = expf(m[hh] - mn);
+            const float pj = expf(d - mn);
+            l[hh] = l[hh] * corr + pj;
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) o[hh][e] = o[hh][e] * corr + pj * vv[e];
+            m[hh] = mn;
+        }
+    }
+    // merge the 4 warps
+    __shared__ float sm_m[4][G], sm_l[4][G];
+    __shared__ float sm_o[4][G][DH];
+#pragma unroll
+    for (int hh = 0; hh < G; ++hh) {
+        if (lane == 0) { sm_m[warp][hh] = m[hh]; sm_l[warp][hh] = l[hh]; }
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) sm_o[warp][hh][lane * EPL + e] = o[hh][e];
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < G * DH; idx += blockDim.x) {
+        const int hh = idx / DH, t = idx % DH;
+        float M = -INFINITY;
+        for (int w = 0; w < 4; ++w) M = fmaxf(M, sm_m[w][hh]);
+        float L = 0.f, Ov = 0.f;
+        for (int w = 0; w < 4; ++w) {
+            const float f = (sm_m[w][hh] == -INFINITY) ? 0.f : expf(sm_m[w][hh] - M);
+            L += sm_l[w][hh] * f;
+            Ov += sm_o[w][hh][t] * f;
+        }
+        const int h = g * G + hh;
+        const size_t pi = ((size_t)(b * n_q + h) * S + s);
+        part_o[pi * DH + t] = Ov;
+        if (t == 0) { part_ml[pi * 2] = M; part_ml[pi * 2 + 1] = L; }
+    }
+    // last CTA of (b, g) merges the S partials
+    __shared__ bool last;
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const unsigned prev = atomicAdd(&counters[b * n_kv + g], 1u);
+        last = (prev == (unsigned)S - 1);
+    }
+    __syncthreads();
+    if (!last) return;
+    __threadfence();
+    for (int idx = threadIdx.x; idx < G * DH; idx += blockDim.x) {
+        const int hh = idx / DH, t = idx % DH;
+        const int h = g * G + hh;
+        const size_t p0 = (size_t)(b * n_q + h) * S;
+        float M = -INFINITY;
+        for (int ss = 0; ss < S; ++ss) M = fmaxf(M, __ldcg(part_ml + (p0 + ss) * 2));
+        float L = 0.f, Ov = 0.f;
+        for (int ss = 0; ss < S; ++ss) {
+            const float ms = __ldcg(part_ml + (p0 + ss) * 2);
+            const float f = (ms == -INFINITY) ? 0.f : expf(ms - M);
+            L += __ldcg(part_ml + (p0 + ss) * 2 + 1) * f;
+            Ov += __ldcg(part_o + (p0 + ss) * DH + t) * f;
+        }
+        out[(size_t)b * n_q * DH + (size_t)h * DH + t] = Ov / L;
+    }
+    if (threadIdx.x == 0) counters[b * n_kv + g] = 0u;
+}
+
+// ---------------------------------------------------------------- heads
+
+struct StepState {
+    int32_t* pending;      // [B,2]
+    int32_t* n_pos;        // [B] entries in the caches
+    long long* emitted;    // [B]
+    int32_t* out_tokens;   // [B,2]
+    int32_t* out_nacc;     // [B]
+    const unsigned long long* am_b;
+    const unsigned long long* am_d;
+    float* dbg_conf;       // [B] or nullptr
+    float* dbg_hb;         // [B,H] or nullptr
+    float* dbg_hd;
+    int32_t* dbg_xb;       // [B]
+    int32_t* dbg_xd;
+};
+
+// Confidence c = sigmoid(W2 . t) with t = SiLU(W1 RMSNorm([h_b; h_d])) computed
+// by the preceding GEMV; acceptance; next pending pair; counters.  grid B.
+template <typename T>
+__global__ void accept_kernel(const float* __restrict__ t, const void* W2, int H, float tau, int force,
+                              StepState st, const float* hb, const float* hd) {
+    const int b = blockIdx.x;
+    float acc = 0.f;
+    for (int k = threadIdx.x; k < H; k += blockDim.x) acc += ldw<T>(W2, k) * t[(size_t)b * H + k];
+    acc = warp_sum(acc);
+    __shared__ float red[32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) red[warp] = acc;
+    __syncthreads();
+    if (st.dbg_hb)
+        for (int k = threadIdx.x; k < H; k += blockDim.x) {
+            st.dbg_hb[(size_t)b * H + k] = hb[(size_t)b * H + k];
+            st.dbg_hd[(size_t)b * H + k] = hd[(size_t)b * H + k];
+        }
+    if (threadIdx.x != 0) return;
+    float s = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) s += red[w];
+    const float c = 1.0f / (1.0f + expf(-s));
+    const int accept = (force == 1) ? 1 : (force == 2) ? 0 : (c >= tau ? 1 : 0);
+    const int xb = argmax_row(st.am_b[b]), xd = argmax_row(st.am_d[b]);
+    st.out_tokens[2 * b] = xb;
+    st.out_tokens[2 * b + 1] = accept ? xd : -1;
+    st.out_nacc[b] = accept;
+    st.pending[2 * b] = xb;
+    st.pending[2 * b + 1] = accept ? xd : -1;
+    st.n_pos[b] += 1;
+    st.emitted[b] += 1 + accept;
+    if (st.dbg_conf) st.dbg_conf[b] = c;
+    if (st.dbg_xb) { st.dbg_xb[b] = xb; st.dbg_xd[b] = xd; }
+}
+
+// Prefill positions before the last: n[b] += 1.
+__global__ void advance_kernel(int32_t* n_pos, int B) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b < B) n_pos[b] += 1;
+}
+
+}  // namespace pipo

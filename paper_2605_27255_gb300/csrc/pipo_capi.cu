@@ -1,0 +1,816 @@
+// C ABI of the PIPO pair-decode library (declared in include/pipo.h).
+//
+// A context owns the model weights (fused QKV and gate|up layouts), a paged
+// KV cache per decoder block (backbone blocks + the MTP block), fp32
+// activation buffers and the per-sequence device state (pending pair, KV
+// length, emitted count).  A decode step is one captured CUDA graph: no host
+// round trip inside the step.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <numeric>
+#include <random>
+#include <string>
+#include <vector>
+
+#include "kernels.cuh"
+#include "pipo.h"
+
+using namespace pipo;
+using bf16 = __nv_bfloat16;
+
+namespace {
+
+std::string g_init_error = "no error";
+
+struct BlockW {
+    void *attn_norm = nullptr, *Wqkv = nullptr, *Wo = nullptr, *ffn_norm = nullptr, *Wgu = nullptr, *Wdown = nullptr;
+};
+
+enum Mode { DECODE = 0, PREFILL_MID = 1, PREFILL_LAST = 2 };
+
+}  // namespace
+
+struct pipo_ctx {
+    pipo_config cfg{};
+    int dev = 0, sms = 0;
+    size_t esz = 4;
+    cudaStream_t own_stream = nullptr, stream = nullptr;
+    std::vector<void*> allocs;
+
+    void *E = nullptr, *x_pad = nullptr, *comp_W = nullptr, *comp_b = nullptr, *comp_W1 = nullptr, *comp_W2 = nullptr;
+    std::vector<BlockW> blocks;
+    BlockW mtp;
+    void *final_norm = nullptr, *mtp_norm_h = nullptr, *mtp_norm_e = nullptr, *mtp_W_fc = nullptr,
+         *mtp_norm_post = nullptr, *conf_norm = nullptr, *conf_W1 = nullptr, *conf_W2 = nullptr;
+
+    // paged KV cache: n_cache_layers x [num_blocks][n_kv][page][d_h]
+    void *Kc = nullptr, *Vc = nullptr;
+    int n_cache_layers = 0, blocks_per_seq = 0, num_blocks = 0;
+    size_t layer_elems = 0;
+    int32_t* block_table = nullptr;
+
+    float *x = nullptr, *x2 = nullptr, *qkv = nullptr, *q = nullptr, *attn = nullptr, *act = nullptr, *t = nullptr;
+    float *part_o = nullptr, *part_ml = nullptr;
+    unsigned* counters = nullptr;
+    float* gemv_part = nullptr;     // split-K partials of the residual-add GEMVs
+    unsigned* gemv_rowcnt = nullptr;
+    unsigned long long* am = nullptr;  // [2][max_batch]
+
+    int32_t *pending = nullptr, *n_pos = nullptr, *out_tokens = nullptr, *out_nacc = nullptr;
+    long long* emitted = nullptr;
+    float *dbg_lb = nullptr, *dbg_ld = nullptr, *dbg_conf = nullptr, *dbg_hb = nullptr, *dbg_hd = nullptr;
+    int32_t *dbg_xb = nullptr, *dbg_xd = nullptr;
+    float* cache_tmp = nullptr;
+    size_t cache_tmp_elems = 0;
+
+    int32_t *pf_pairs = nullptr, *pf_mtp = nullptr;
+    size_t pf_cap = 0;
+
+    int B = 0;
+    bool prefilled = false;
+    std::vector<int32_t> h_len;
+    cudaGraphExec_t graph = nullptr;
+    int graph_B = -1;
+    int launches = 0;
+    std::map<long long, int> occ;
+    std::string err = "no error";
+};
+
+// ------------------------------------------------------------------ helpers
+namespace {
+
+pipo_status fail(pipo_ctx* c, pipo_status s, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (c) c->err = buf; else g_init_error = buf;
+    return s;
+}
+
+#define CK(call)                                                                                  \
+    do {                                                                                          \
+        cudaError_t e_ = (call);                                                                  \
+        if (e_ != cudaSuccess) return fail(ctx, PIPO_ECUDA, "%s: %s", #call, cudaGetErrorString(e_)); \
+    } while (0)
+
+template <typename P>
+pipo_status dalloc(pipo_ctx* ctx, P** p, size_t bytes) {
+    void* q = nullptr;
+    cudaError_t e = cudaMalloc(&q, bytes ? bytes : 16);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(ctx, PIPO_ENOMEM, "cudaMalloc(%zu bytes): %s", bytes, cudaGetErrorString(e));
+    }
+    ctx->allocs.push_back(q);
+    *p = static_cast<P*>(q);
+    return PIPO_OK;
+}
+
+#define TRY(x)                              \
+    do {                                    \
+        pipo_status s_ = (x);               \
+        if (s_ != PIPO_OK) return s_;       \
+    } while (0)
+
+// copy n elements from a host or device source (UVA) into dst + offset
+pipo_status put(pipo_ctx* ctx, void* dst, size_t off_elems, const void* src, size_t n_elems) {
+    if (!src) return fail(ctx, PIPO_EINVAL, "missing weight tensor");
+    CK(cudaMemcpy(static_cast<char*>(dst) + off_elems * ctx->esz, src, n_elems * ctx->esz, cudaMemcpyDefault));
+    return PIPO_OK;
+}
+
+pipo_status upload(pipo_ctx* ctx, void** dst, const void* src, size_t n) {
+    TRY(dalloc(ctx, reinterpret_cast<char**>(dst), n * ctx->esz));
+    return put(ctx, *dst, 0, src, n);
+}
+
+const void* at(const void* p, size_t off_elems, size_t esz) {
+    return p ? static_cast<const char*>(p) + off_elems * esz : nullptr;
+}
+
+pipo_status upload_block(pipo_ctx* ctx, BlockW& bw, int l, const void* an, const void* wq, const void* wk,
+                         const void* wv, const void* wo, const void* fn, const void* wg, const void* wu,
+                         const void* wd) {
+    const pipo_config& c = ctx->cfg;
+    const size_t H = c.hidden, qd = (size_t)c.n_q_heads * c.head_dim, kd = (size_t)c.n_kv_heads * c.head_dim,
+                 F = c.ffn, e = ctx->esz;
+    TRY(upload(ctx, &bw.attn_norm, at(an, l * H, e), H));
+    TRY(dalloc(ctx, reinterpret_cast<char**>(&bw.Wqkv), (qd + 2 * kd) * H * e));
+    TRY(put(ctx, bw.Wqkv, 0, at(wq, l * qd * H, e), qd * H));
+    TRY(put(ctx, bw.Wqkv, qd * H, at(wk, l * kd * H, e), kd * H));
+    TRY(put(ctx, bw.Wqkv, (qd + kd) * H, at(wv, l * kd * H, e), kd * H));
+    TRY(upload(ctx, &bw.Wo, at(wo, l * H * qd, e), H * qd));
+    TRY(upload(ctx, &bw.ffn_norm, at(fn, l * H, e), H));
+    TRY(dalloc(ctx, reinterpret_cast<char**>(&bw.Wgu), 2 * F * H * e));
+    TRY(put(ctx, bw.Wgu, 0, at(wg, l * F * H, e), F * H));
+    TRY(put(ctx, bw.Wgu, F * H, at(wu, l * F * H, e), F * H));
+    TRY(upload(ctx, &bw.Wdown, at(wd, l * H * F, e), H * F));
+    return PIPO_OK;
+}
+
+int next_pow2_le8(int b) {
+    int nb = 1;
+    while (nb < b && nb < 8) nb <<= 1;
+    return nb;
+}
+
+template <typename T, int NB, bool TWO>
+void* gemv_fn() { return reinterpret_cast<void*>(&gemv_kernel<T, NB, TWO>); }
+
+template <typename T>
+void* pick_gemv(int nb, bool two) {
+    switch (nb) {
+        case 1: return two ? gemv_fn<T, 1, true>() : gemv_fn<T, 1, false>();
+        case 2: return two ? gemv_fn<T, 2, true>() : gemv_fn<T, 2, false>();
+        case 4: return two ? gemv_fn<T, 4, true>() : gemv_fn<T, 4, false>();
+        default: return two ? gemv_fn<T, 8, true>() : gemv_fn<T, 8, false>();
+    }
+}
+
+constexpr size_t kXsBudget = 100 * 1024;  // staged-input bytes per GEMV block
+
+cudaError_t set_smem_attrs(bool bf) {
+    const int nbs[4] = {1, 2, 4, 8};
+    for (int i = 0; i < 4; ++i)
+        for (int two = 0; two < 2; ++two) {
+            void* f = bf ? pick_gemv<bf16>(nbs[i], two) : pick_gemv<float>(nbs[i], two);
+            cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kXsBudget);
+            if (e != cudaSuccess) return e;
+        }
+    return cudaSuccess;
+}
+
+pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
+    const bool bf = ctx->cfg.dtype == 1;
+    const bool two = p.epi == EPI_SWIGLU;
+    int nb = next_pow2_le8(std::max(1, p.B));
+    while (nb > 1 && (size_t)nb * p.K * 4 > kXsBudget) nb >>= 1;
+    if ((size_t)p.K * 4 > kXsBudget) return fail(ctx, PIPO_EINVAL, "GEMV input length %d too large", p.K);
+    const size_t smem = (size_t)nb * p.K * 4;
+    void* fn = bf ? pick_gemv<bf16>(nb, two) : pick_gemv<float>(nb, two);
+    const long long key = (reinterpret_cast<long long>(fn) << 1) ^ (long long)smem;
+    int per_sm;
+    auto it = ctx->occ.find(key);
+    if (it == ctx->occ.end()) {
+        CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, smem));
+        ctx->occ[key] = per_sm;
+    } else {
+        per_sm = it->second;
+    }
+    per_sm = std::max(1, per_sm);
+    if (p.splitk < 1) p.splitk = 1;
+    const long long tasks = (long long)p.N * p.splitk;
+    const int grid = (int)std::max(1LL, std::min<long long>((tasks + kWarps - 1) / kWarps, (long long)ctx->sms * per_sm));
+    void* args[] = {&p};
+    CK(cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, ctx->stream));
+    ctx->launches++;
+    return PIPO_OK;
+}
+
+Seg act_seg(const float* src, int ld, int K, const void* gamma = nullptr) {
+    Seg s{};
+    s.src = src; s.ld = ld; s.K = K; s.gamma = gamma;
+    return s;
+}
+
+GemvParams gemv_base(pipo_ctx* ctx, const void* W, int N, int epi, float* y, int ldy) {
+    GemvParams p{};
+    p.W = W; p.N = N; p.epi = epi; p.y = y; p.ldy = ldy;
+    p.B = ctx->B; p.splitk = 1; p.eps = ctx->cfg.rms_eps; p.nseg = 1;
+    return p;
+}
+
+int resadd_splits(pipo_ctx* ctx, int N, int K) {
+    const long long target = (long long)ctx->sms * kWarps * 2 * 4;
+    int s = (int)std::max(1LL, (target + N - 1) / N);
+    s = std::min(s, std::max(1, K / 256));
+    return s;
+}
+
+int attn_splits(const pipo_ctx* ctx, int B) {
+    const pipo_config& c = ctx->cfg;
+    int s = (2 * ctx->sms + B * c.n_kv_heads - 1) / (B * c.n_kv_heads);
+    s = std::max(1, std::min(s, (c.max_ctx + 15) / 16));
+    return s;
+}
+
+template <typename T, int DH, int G>
+void* attn_fn() { return reinterpret_cast<void*>(&attn_decode_kernel<T, DH, G>); }
+
+template <typename T, int DH>
+void* attn_pick_g(int G) {
+    switch (G) {
+        case 1: return attn_fn<T, DH, 1>();
+        case 2: return attn_fn<T, DH, 2>();
+        case 4: return attn_fn<T, DH, 4>();
+        case 8: return attn_fn<T, DH, 8>();
+        default: return nullptr;
+    }
+}
+
+void* attn_pick(bool bf, int DH, int G) {
+    if (DH == 64) return bf ? attn_pick_g<bf16, 64>(G) : attn_pick_g<float, 64>(G);
+    if (DH == 128) return bf ? attn_pick_g<bf16, 128>(G) : attn_pick_g<float, 128>(G);
+    return nullptr;
+}
+
+void* rope_pick(bool bf, int DH) {
+    if (DH == 64) return bf ? (void*)&rope_append_kernel<bf16, 64> : (void*)&rope_append_kernel<float, 64>;
+    if (DH == 128) return bf ? (void*)&rope_append_kernel<bf16, 128> : (void*)&rope_append_kernel<float, 128>;
+    return nullptr;
+}
+
+KVView kv_view(pipo_ctx* ctx, int layer) {
+    KVView v;
+    v.K = static_cast<char*>(ctx->Kc) + (size_t)layer * ctx->layer_elems * ctx->esz;
+    v.V = static_cast<char*>(ctx->Vc) + (size_t)layer * ctx->layer_elems * ctx->esz;
+    v.table = ctx->block_table;
+    v.blocks_per_seq = ctx->blocks_per_seq;
+    v.page = ctx->cfg.page_size;
+    v.n_kv = ctx->cfg.n_kv_heads;
+    return v;
+}
+
+// One decoder block on the residual stream xr (pre-norm attention + SwiGLU).
+pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, float* xr) {
+    const pipo_config& c = ctx->cfg;
+    const int H = c.hidden, DH = c.head_dim, qd = c.n_q_heads * DH, kd = c.n_kv_heads * DH, rows = qd + 2 * kd;
+    const bool bf = c.dtype == 1;
+    // RMSNorm -> fused QKV projection
+    GemvParams p = gemv_base(ctx, bw.Wqkv, rows, EPI_STORE, ctx->qkv, rows);
+    p.seg[0] = act_seg(xr, H, H, bw.attn_norm);
+    p.K = H;
+    TRY(launch_gemv(ctx, p));
+    // RoPE + KV append
+    KVView kv = kv_view(ctx, cache_layer);
+    {
+        const float* qkv = ctx->qkv;
+        int ld = rows;
+        float* qo = ctx->q;
+        const int32_t* np = ctx->n_pos;
+        int nq = c.n_q_heads;
+        double theta = c.rope_theta;
+        void* args[] = {(void*)&qkv, &ld, &qo, &kv, (void*)&np, &nq, &theta};
+        CK(cudaLaunchKernel(rope_pick(bf, DH), dim3(ctx->B, c.n_q_heads + 2 * c.n_kv_heads), dim3(DH / 2), args, 0,
+                            ctx->stream));
+        ctx->launches++;
+    }
+    // split-KV attention
+    {
+        const int S = attn_splits(ctx, ctx->B);
+        const float* qp = ctx->q;
+        const int32_t* np = ctx->n_pos;
+        float* out = ctx->attn;
+        float* po = ctx->part_o;
+        float* pml = ctx->part_ml;
+        unsigned* cnt = ctx->counters;
+        int Sv = S;
+        float scale = 1.0f / sqrtf((float)DH);
+        void* args[] = {(void*)&qp, &kv, (void*)&np, &out, &po, &pml, &cnt, &Sv, &scale};
+        CK(cudaLaunchKernel(attn_pick(bf, DH, c.n_q_heads / c.n_kv_heads), dim3(S, c.n_kv_heads, ctx->B), dim3(128),
+                            args, 0, ctx->stream));
+        ctx->launches++;
+    }
+    // O projection + residual
+    p = gemv_base(ctx, bw.Wo, H, EPI_RESADD, xr, H);
+    p.seg[0] = act_seg(ctx->attn, qd, qd);
+    p.K = qd;
+    p.splitk = resadd_splits(ctx, H, qd);
+    p.part = ctx->gemv_part; p.rowcnt = ctx->gemv_rowcnt;
+    TRY(launch_gemv(ctx, p));
+    // RMSNorm -> gate|up -> SwiGLU
+    p = gemv_base(ctx, bw.Wgu, c.ffn, EPI_SWIGLU, ctx->act, c.ffn);
+    p.seg[0] = act_seg(xr, H, H, bw.ffn_norm);
+    p.K = H;
+    p.rstride = c.ffn;
+    TRY(launch_gemv(ctx, p));
+    // down projection + residual
+    p = gemv_base(ctx, bw.Wdown, H, EPI_RESADD, xr, H);
+    p.seg[0] = act_seg(ctx->act, c.ffn, c.ffn);
+    p.K = c.ffn;
+    p.splitk = resadd_splits(ctx, H, c.ffn);
+    p.part = ctx->gemv_part; p.rowcnt = ctx->gemv_rowcnt;
+    TRY(launch_gemv(ctx, p));
+    return PIPO_OK;
+}
+
+pipo_status enqueue_lm_head(pipo_ctx* ctx, const float* h, const void* gamma, unsigned long long* am, float* dbg) {
+    const pipo_config& c = ctx->cfg;
+    GemvParams p = gemv_base(ctx, ctx->E, c.vocab, EPI_ARGMAX, nullptr, 0);
+    p.seg[0] = act_seg(h, c.hidden, c.hidden, gamma);
+    p.K = c.hidden;
+    p.am = am;
+    p.dbg = dbg;
+    p.ld_dbg = c.vocab;
+    return launch_gemv(ctx, p);
+}
+
+// One pair position of every sequence.  DECODE: the pending pair; PREFILL_*:
+// prompt pair j.  PREFILL_MID stops after the MTP block (teacher-forced token).
+pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
+    const pipo_config& c = ctx->cfg;
+    const int H = c.hidden, B = ctx->B;
+    const bool bf = c.dtype == 1;
+    unsigned long long* am_b = ctx->am;
+    unsigned long long* am_d = ctx->am + c.max_batch;
+
+    // pair embed + compressor (Eq. 1)
+    const int32_t* pairs = (mode == DECODE) ? ctx->pending : ctx->pf_pairs + (size_t)j * B * 2;
+    Seg s0{}, s1{};
+    s0.table = ctx->E; s0.pad = ctx->x_pad; s0.tok = pairs; s0.tok_ld = 2; s0.K = H;
+    s1 = s0; s1.tok = pairs + 1;
+    GemvParams p;
+    if (c.compressor == 0) {
+        p = gemv_base(ctx, ctx->comp_W, H, EPI_BIAS, ctx->x, H);
+        p.bias = ctx->comp_b;
+    } else {
+        p = gemv_base(ctx, ctx->comp_W1, H, EPI_SILU, ctx->t, H);
+    }
+    p.seg[0] = s0; p.seg[1] = s1; p.nseg = 2; p.K = 2 * H;
+    if (mode != PREFILL_MID) { p.zero_ptr = ctx->am; p.zero_n = 2 * c.max_batch; }
+    TRY(launch_gemv(ctx, p));
+    if (c.compressor == 1) {
+        p = gemv_base(ctx, ctx->comp_W2, H, EPI_STORE, ctx->x, H);
+        p.seg[0] = act_seg(ctx->t, H, H);
+        p.K = H;
+        TRY(launch_gemv(ctx, p));
+    }
+    // backbone (Eq. 2)
+    for (int l = 0; l < c.n_layers; ++l) TRY(enqueue_block(ctx, ctx->blocks[l], l, ctx->x));
+    // LM head + argmax (Eq. 3)
+    if (mode != PREFILL_MID) TRY(enqueue_lm_head(ctx, ctx->x, ctx->final_norm, am_b, c.debug ? ctx->dbg_lb : nullptr));
+    // MTP head input (App. A.2): W_fc [RMSNorm(h_b); RMSNorm(E[x_b])]
+    p = gemv_base(ctx, ctx->mtp_W_fc, H, EPI_STORE, ctx->x2, H);
+    p.seg[0] = act_seg(ctx->x, H, H, ctx->mtp_norm_h);
+    Seg se{};
+    se.table = ctx->E; se.pad = ctx->x_pad; se.gamma = ctx->mtp_norm_e; se.K = H;
+    if (mode == PREFILL_MID) { se.tok = ctx->pf_mtp + (size_t)j * B; se.tok_ld = 1; }
+    else se.tok_am = am_b;
+    p.seg[1] = se; p.nseg = 2; p.K = 2 * H;
+    TRY(launch_gemv(ctx, p));
+    if (c.mtp_block) TRY(enqueue_block(ctx, ctx->mtp, c.n_layers, ctx->x2));
+    if (mode == PREFILL_MID) {
+        advance_kernel<<<(B + 127) / 128, 128, 0, ctx->stream>>>(ctx->n_pos, B);
+        CK(cudaGetLastError());
+        ctx->launches++;
+        return PIPO_OK;
+    }
+    // draft token (Eq. 5)
+    TRY(enqueue_lm_head(ctx, ctx->x2, ctx->mtp_norm_post, am_d, c.debug ? ctx->dbg_ld : nullptr));
+    // confidence (Eq. 6, App. A.3): t = SiLU(W1 RMSNorm([h_b; h_d]))
+    p = gemv_base(ctx, ctx->conf_W1, H, EPI_SILU, ctx->t, H);
+    p.seg[0] = act_seg(ctx->x, H, H, ctx->conf_norm);
+    p.seg[1] = act_seg(ctx->x2, H, H, nullptr);
+    p.nseg = 2; p.K = 2 * H; p.joint_norm = 1;
+    TRY(launch_gemv(ctx, p));
+    StepState st{};
+    st.pending = ctx->pending; st.n_pos = ctx->n_pos; st.emitted = ctx->emitted;
+    st.out_tokens = ctx->out_tokens; st.out_nacc = ctx->out_nacc;
+    st.am_b = am_b; st.am_d = am_d;
+    if (c.debug) {
+        st.dbg_conf = ctx->dbg_conf; st.dbg_hb = ctx->dbg_hb; st.dbg_hd = ctx->dbg_hd;
+        st.dbg_xb = ctx->dbg_xb; st.dbg_xd = ctx->dbg_xd;
+    }
+    if (bf)
+        accept_kernel<bf16><<<B, 256, 0, ctx->stream>>>(ctx->t, ctx->conf_W2, H, c.tau, c.force_mode, st, ctx->x, ctx->x2);
+    else
+        accept_kernel<float><<<B, 256, 0, ctx->stream>>>(ctx->t, ctx->conf_W2, H, c.tau, c.force_mode, st, ctx->x, ctx->x2);
+    CK(cudaGetLastError());
+    ctx->launches++;
+    return PIPO_OK;
+}
+
+void drop_graph(pipo_ctx* ctx) {
+    if (ctx->graph) cudaGraphExecDestroy(ctx->graph);
+    ctx->graph = nullptr;
+    ctx->graph_B = -1;
+}
+
+pipo_status ensure_graph(pipo_ctx* ctx) {
+    if (ctx->graph && ctx->graph_B == ctx->B) return PIPO_OK;
+    drop_graph(ctx);
+    cudaGraph_t g = nullptr;
+    CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
+    ctx->launches = 0;
+    pipo_status s = enqueue_position(ctx, DECODE, 0);
+    cudaError_t e = cudaStreamEndCapture(ctx->stream, &g);
+    if (s != PIPO_OK) {
+        if (g) cudaGraphDestroy(g);
+        return s;
+    }
+    if (e != cudaSuccess) return fail(ctx, PIPO_ECUDA, "graph capture: %s", cudaGetErrorString(e));
+    e = cudaGraphInstantiate(&ctx->graph, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) return fail(ctx, PIPO_ECUDA, "graph instantiate: %s", cudaGetErrorString(e));
+    ctx->graph_B = ctx->B;
+    return PIPO_OK;
+}
+
+__global__ void cache_copy_kernel(KVView kv, int b, int n, int dh, float* buf, int to_cache, int bf) {
+    const int j = blockIdx.x;
+    const int kd = kv.n_kv * dh;
+    for (int i = threadIdx.x; i < kd; i += blockDim.x) {
+        const int g = i / dh, d = i % dh;
+        const int blk = kv.table[(size_t)b * kv.blocks_per_seq + j / kv.page];
+        const size_t off = (((size_t)blk * kv.n_kv + g) * kv.page + (j % kv.page)) * dh + d;
+        float* bk = buf + (size_t)j * kd + i;
+        float* bv = buf + (size_t)n * kd + (size_t)j * kd + i;
+        if (bf) {
+            bf16* K = static_cast<bf16*>(kv.K);
+            bf16* V = static_cast<bf16*>(kv.V);
+            if (to_cache) { K[off] = __float2bfloat16_rn(*bk); V[off] = __float2bfloat16_rn(*bv); }
+            else { *bk = __bfloat162float(K[off]); *bv = __bfloat162float(V[off]); }
+        } else {
+            float* K = static_cast<float*>(kv.K);
+            float* V = static_cast<float*>(kv.V);
+            if (to_cache) { K[off] = *bk; V[off] = *bv; }
+            else { *bk = K[off]; *bv = V[off]; }
+        }
+    }
+}
+
+pipo_status ensure_cache_tmp(pipo_ctx* ctx, size_t elems) {
+    if (ctx->cache_tmp_elems >= elems) return PIPO_OK;
+    if (ctx->cache_tmp) {
+        cudaFree(ctx->cache_tmp);
+        ctx->allocs.erase(std::find(ctx->allocs.begin(), ctx->allocs.end(), (void*)ctx->cache_tmp));
+        ctx->cache_tmp = nullptr;
+    }
+    TRY(dalloc(ctx, &ctx->cache_tmp, elems * sizeof(float)));
+    ctx->cache_tmp_elems = elems;
+    return PIPO_OK;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ C ABI
+extern "C" {
+
+const char* pipo_last_error(const pipo_ctx* ctx) { return ctx ? ctx->err.c_str() : g_init_error.c_str(); }
+
+int32_t pipo_step_launches(const pipo_ctx* ctx) { return ctx ? ctx->launches : 0; }
+
+void pipo_free(pipo_ctx* ctx) {
+    if (!ctx) return;
+    cudaSetDevice(ctx->dev);
+    if (ctx->stream) cudaStreamSynchronize(ctx->stream);
+    drop_graph(ctx);
+    for (void* p : ctx->allocs) cudaFree(p);
+    if (ctx->own_stream) cudaStreamDestroy(ctx->own_stream);
+    delete ctx;
+}
+
+pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** out) {
+    pipo_ctx* ctx = nullptr;
+    if (!cfg || !w || !out) return fail(nullptr, PIPO_EINVAL, "null argument");
+    *out = nullptr;
+    const pipo_config& c = *cfg;
+    if (c.hidden <= 0 || c.hidden % 8 || c.n_layers < 0 || c.n_q_heads <= 0 || c.n_kv_heads <= 0 ||
+        c.n_q_heads % c.n_kv_heads || c.ffn <= 0 || c.ffn % 8 || c.vocab <= 0 || c.max_batch <= 0 ||
+        c.max_ctx <= 0 || c.page_size <= 0 || (c.dtype != 0 && c.dtype != 1) ||
+        (c.compressor != 0 && c.compressor != 1) || (c.mtp_block != 0 && c.mtp_block != 1))
+        return fail(nullptr, PIPO_EINVAL, "invalid config");
+    if (c.head_dim != 64 && c.head_dim != 128) return fail(nullptr, PIPO_EINVAL, "head_dim must be 64 or 128");
+    const int G = c.n_q_heads / c.n_kv_heads;
+    if (G != 1 && G != 2 && G != 4 && G != 8) return fail(nullptr, PIPO_EINVAL, "n_q/n_kv must be 1, 2, 4 or 8");
+    if ((size_t)c.ffn * 4 > kXsBudget || (size_t)2 * c.hidden * 4 > kXsBudget)
+        return fail(nullptr, PIPO_EINVAL, "hidden/ffn too large for the staged GEMV input");
+
+    ctx = new pipo_ctx();
+    ctx->cfg = c;
+    ctx->esz = c.dtype == 1 ? 2 : 4;
+    pipo_status s = [&]() -> pipo_status {
+        CK(cudaGetDevice(&ctx->dev));
+        CK(cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, ctx->dev));
+        CK(cudaStreamCreateWithFlags(&ctx->own_stream, cudaStreamNonBlocking));
+        ctx->stream = ctx->own_stream;
+        CK(set_smem_attrs(c.dtype == 1));
+        const size_t H = c.hidden, V = c.vocab;
+        TRY(upload(ctx, &ctx->E, w->E, V * H));
+        TRY(upload(ctx, &ctx->x_pad, w->x_pad, H));
+        if (c.compressor == 0) {
+            TRY(upload(ctx, &ctx->comp_W, w->comp_W, H * 2 * H));
+            TRY(upload(ctx, &ctx->comp_b, w->comp_b, H));
+        } else {
+            TRY(upload(ctx, &ctx->comp_W1, w->comp_W1, H * 2 * H));
+            TRY(upload(ctx, &ctx->comp_W2, w->comp_W2, H * H));
+        }
+        ctx->blocks.resize(c.n_layers);
+        for (int l = 0; l < c.n_layers; ++l)
+            TRY(upload_block(ctx, ctx->blocks[l], l, w->attn_norm, w->Wq, w->Wk, w->Wv, w->Wo, w->ffn_norm, w->Wgate,
+                             w->Wup, w->Wdown));
+        if (c.mtp_block)
+            TRY(upload_block(ctx, ctx->mtp, 0, w->m_attn_norm, w->m_Wq, w->m_Wk, w->m_Wv, w->m_Wo, w->m_ffn_norm,
+                             w->m_Wgate, w->m_Wup, w->m_Wdown));
+        TRY(upload(ctx, &ctx->final_norm, w->final_norm, H));
+        TRY(upload(ctx, &ctx->mtp_norm_h, w->mtp_norm_h, H));
+        TRY(upload(ctx, &ctx->mtp_norm_e, w->mtp_norm_e, H));
+        TRY(upload(ctx, &ctx->mtp_W_fc, w->mtp_W_fc, H * 2 * H));
+        TRY(upload(ctx, &ctx->mtp_norm_post, w->mtp_norm_post, H));
+        TRY(upload(ctx, &ctx->conf_norm, w->conf_norm, 2 * H));
+        TRY(upload(ctx, &ctx->conf_W1, w->conf_W1, H * 2 * H));
+        TRY(upload(ctx, &ctx->conf_W2, w->conf_W2, H));
+
+        // paged KV cache
+        const int MB = c.max_batch, DH = c.head_dim;
+        ctx->n_cache_layers = c.n_layers + (c.mtp_block ? 1 : 0);
+        ctx->blocks_per_seq = (c.max_ctx + c.page_size - 1) / c.page_size;
+        ctx->num_blocks = MB * ctx->blocks_per_seq;
+        ctx->layer_elems = (size_t)ctx->num_blocks * c.n_kv_heads * c.page_size * DH;
+        TRY(dalloc(ctx, reinterpret_cast<char**>(&ctx->Kc), std::max<size_t>(1, ctx->n_cache_layers) * ctx->layer_elems * ctx->esz));
+        TRY(dalloc(ctx, reinterpret_cast<char**>(&ctx->Vc), std::max<size_t>(1, ctx->n_cache_layers) * ctx->layer_elems * ctx->esz));
+        std::vector<int32_t> table(ctx->num_blocks);
+        std::iota(table.begin(), table.end(), 0);
+        if (c.page_shuffle_seed) {
+            std::mt19937 rng(c.page_shuffle_seed);
+            std::shuffle(table.begin(), table.end(), rng);
+        }
+        TRY(dalloc(ctx, &ctx->block_table, table.size() * sizeof(int32_t)));
+        CK(cudaMemcpy(ctx->block_table, table.data(), table.size() * sizeof(int32_t), cudaMemcpyHostToDevice));
+
+        // activations and state
+        const int qd = c.n_q_heads * DH, kd = c.n_kv_heads * DH;
+        TRY(dalloc(ctx, &ctx->x, (size_t)MB * H * 4));
+        TRY(dalloc(ctx, &ctx->x2, (size_t)MB * H * 4));
+        TRY(dalloc(ctx, &ctx->qkv, (size_t)MB * (qd + 2 * kd) * 4));
+        TRY(dalloc(ctx, &ctx->q, (size_t)MB * qd * 4));
+        TRY(dalloc(ctx, &ctx->attn, (size_t)MB * qd * 4));
+        TRY(dalloc(ctx, &ctx->act, (size_t)MB * c.ffn * 4));
+        TRY(dalloc(ctx, &ctx->t, (size_t)MB * H * 4));
+        size_t parts = 0;
+        for (int b = 1; b <= MB; ++b) parts = std::max(parts, (size_t)b * c.n_q_heads * attn_splits(ctx, b));
+        TRY(dalloc(ctx, &ctx->part_o, parts * DH * 4));
+        TRY(dalloc(ctx, &ctx->part_ml, parts * 2 * 4));
+        TRY(dalloc(ctx, &ctx->counters, (size_t)MB * c.n_kv_heads * 4));
+        CK(cudaMemset(ctx->counters, 0, (size_t)MB * c.n_kv_heads * 4));
+        TRY(dalloc(ctx, &ctx->am, (size_t)2 * MB * 8));
+        const int smax = std::max(resadd_splits(ctx, H, qd), resadd_splits(ctx, H, c.ffn));
+        TRY(dalloc(ctx, &ctx->gemv_part, (size_t)smax * MB * H * 4));
+        TRY(dalloc(ctx, &ctx->gemv_rowcnt, (size_t)H * 4));
+        CK(cudaMemset(ctx->gemv_rowcnt, 0, (size_t)H * 4));
+        TRY(dalloc(ctx, &ctx->pending, (size_t)MB * 2 * 4));
+        TRY(dalloc(ctx, &ctx->n_pos, (size_t)MB * 4));
+        TRY(dalloc(ctx, &ctx->out_tokens, (size_t)MB * 2 * 4));
+        TRY(dalloc(ctx, &ctx->out_nacc, (size_t)MB * 4));
+        TRY(dalloc(ctx, &ctx->emitted, (size_t)MB * 8));
+        CK(cudaMemset(ctx->n_pos, 0, (size_t)MB * 4));
+        CK(cudaMemset(ctx->emitted, 0, (size_t)MB * 8));
+        if (c.debug) {
+            TRY(dalloc(ctx, &ctx->dbg_lb, (size_t)MB * V * 4));
+            TRY(dalloc(ctx, &ctx->dbg_ld, (size_t)MB * V * 4));
+            TRY(dalloc(ctx, &ctx->dbg_conf, (size_t)MB * 4));
+            TRY(dalloc(ctx, &ctx->dbg_hb, (size_t)MB * H * 4));
+            TRY(dalloc(ctx, &ctx->dbg_hd, (size_t)MB * H * 4));
+            TRY(dalloc(ctx, &ctx->dbg_xb, (size_t)MB * 4));
+            TRY(dalloc(ctx, &ctx->dbg_xd, (size_t)MB * 4));
+        }
+        CK(cudaDeviceSynchronize());
+        return PIPO_OK;
+    }();
+    if (s != PIPO_OK) {
+        g_init_error = ctx->err;
+        pipo_free(ctx);
+        return s;
+    }
+    *out = ctx;
+    return PIPO_OK;
+}
+
+pipo_status pipo_set_stream(pipo_ctx* ctx, void* stream) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    CK(cudaSetDevice(ctx->dev));
+    CK(cudaStreamSynchronize(ctx->stream));
+    ctx->stream = stream ? static_cast<cudaStream_t>(stream) : ctx->own_stream;
+    drop_graph(ctx);
+    return PIPO_OK;
+}
+
+pipo_status pipo_set_threshold(pipo_ctx* ctx, float tau, int32_t force_mode) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    if (force_mode < 0 || force_mode > 2 || !(tau == tau)) return fail(ctx, PIPO_EINVAL, "bad threshold or force mode");
+    if (ctx->cfg.tau != tau || ctx->cfg.force_mode != force_mode) drop_graph(ctx);
+    ctx->cfg.tau = tau;
+    ctx->cfg.force_mode = force_mode;
+    return PIPO_OK;
+}
+
+pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride, const int32_t* h_lens,
+                         int32_t* h_tokens, int32_t* h_n_accepted) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    const pipo_config& c = ctx->cfg;
+    if (batch < 1 || batch > c.max_batch || !h_ids || !h_lens || stride < 1)
+        return fail(ctx, PIPO_EINVAL, "bad prefill arguments (batch %d, stride %d)", batch, stride);
+    int N = -1;
+    for (int b = 0; b < batch; ++b) {
+        const int len = h_lens[b];
+        if (len < 1 || len > stride) return fail(ctx, PIPO_EINVAL, "sequence %d: length %d not in [1, %d]", b, len, stride);
+        const int nb = (len + 1) / 2;
+        if (N >= 0 && nb != N) return fail(ctx, PIPO_EINVAL, "sequences must give the same number of pairs");
+        N = nb;
+        for (int i = 0; i < len; ++i) {
+            const int32_t t = h_ids[(size_t)b * stride + i];
+            if (t < 0 || t >= c.vocab) return fail(ctx, PIPO_EINVAL, "token id %d out of range at (%d, %d)", t, b, i);
+        }
+    }
+    if (N > c.max_ctx) return fail(ctx, PIPO_ECAPACITY, "prompt needs %d entries > max_ctx %d", N, c.max_ctx);
+    CK(cudaSetDevice(ctx->dev));
+    // pairs [N][B][2] (PAD = -1 in an odd prompt's last slot), MTP inputs [N][B]
+    std::vector<int32_t> pairs((size_t)N * batch * 2), mtp((size_t)N * batch, 0);
+    for (int j = 0; j < N; ++j)
+        for (int b = 0; b < batch; ++b) {
+            const int32_t* t = h_ids + (size_t)b * stride;
+            const int len = h_lens[b];
+            pairs[((size_t)j * batch + b) * 2] = t[2 * j];
+            pairs[((size_t)j * batch + b) * 2 + 1] = (2 * j + 1 < len) ? t[2 * j + 1] : -1;
+            if (j + 1 < N) mtp[(size_t)j * batch + b] = t[2 * j + 2];
+        }
+    if (pairs.size() > ctx->pf_cap) {
+        for (void* p : {(void*)ctx->pf_pairs, (void*)ctx->pf_mtp})
+            if (p) {
+                cudaFree(p);
+                ctx->allocs.erase(std::find(ctx->allocs.begin(), ctx->allocs.end(), p));
+            }
+        ctx->pf_pairs = ctx->pf_mtp = nullptr;
+        ctx->pf_cap = 0;
+        TRY(dalloc(ctx, &ctx->pf_pairs, pairs.size() * 4));
+        TRY(dalloc(ctx, &ctx->pf_mtp, pairs.size() * 4));
+        ctx->pf_cap = pairs.size();
+    }
+    CK(cudaMemcpyAsync(ctx->pf_pairs, pairs.data(), pairs.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
+    CK(cudaMemcpyAsync(ctx->pf_mtp, mtp.data(), mtp.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
+    CK(cudaMemsetAsync(ctx->n_pos, 0, (size_t)batch * 4, ctx->stream));
+    CK(cudaMemsetAsync(ctx->emitted, 0, (size_t)batch * 8, ctx->stream));
+    ctx->B = batch;
+    const int saved = ctx->launches;
+    for (int j = 0; j < N; ++j) TRY(enqueue_position(ctx, j + 1 < N ? PREFILL_MID : PREFILL_LAST, j));
+    ctx->launches = saved;
+    if (h_tokens) CK(cudaMemcpyAsync(h_tokens, ctx->out_tokens, (size_t)batch * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    if (h_n_accepted) CK(cudaMemcpyAsync(h_n_accepted, ctx->out_nacc, (size_t)batch * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    ctx->h_len.assign(batch, N);
+    ctx->prefilled = true;
+    return PIPO_OK;
+}
+
+pipo_status pipo_decode_step_async(pipo_ctx* ctx, int32_t* d_tokens, int32_t* d_n_accepted) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    if (!ctx->prefilled) return fail(ctx, PIPO_ESTATE, "decode step before prefill");
+    for (int b = 0; b < ctx->B; ++b)
+        if (ctx->h_len[b] + 1 > ctx->cfg.max_ctx)
+            return fail(ctx, PIPO_ECAPACITY, "sequence %d: KV cache full (%d entries)", b, ctx->h_len[b]);
+    CK(cudaSetDevice(ctx->dev));
+    TRY(ensure_graph(ctx));
+    CK(cudaGraphLaunch(ctx->graph, ctx->stream));
+    if (d_tokens) CK(cudaMemcpyAsync(d_tokens, ctx->out_tokens, (size_t)ctx->B * 8, cudaMemcpyDeviceToDevice, ctx->stream));
+    if (d_n_accepted) CK(cudaMemcpyAsync(d_n_accepted, ctx->out_nacc, (size_t)ctx->B * 4, cudaMemcpyDeviceToDevice, ctx->stream));
+    for (int b = 0; b < ctx->B; ++b) ctx->h_len[b] += 1;
+    return PIPO_OK;
+}
+
+pipo_status pipo_decode_step(pipo_ctx* ctx, int32_t* h_tokens, int32_t* h_n_accepted) {
+    TRY(pipo_decode_step_async(ctx, nullptr, nullptr));
+    if (h_tokens) CK(cudaMemcpyAsync(h_tokens, ctx->out_tokens, (size_t)ctx->B * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    if (h_n_accepted) CK(cudaMemcpyAsync(h_n_accepted, ctx->out_nacc, (size_t)ctx->B * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    return PIPO_OK;
+}
+
+pipo_status pipo_rollback(pipo_ctx* ctx, const int32_t* h_n_pairs) {
+    if (!ctx || !h_n_pairs) return fail(ctx, PIPO_EINVAL, "null argument");
+    if (!ctx->prefilled) return fail(ctx, PIPO_ESTATE, "rollback before prefill");
+    for (int b = 0; b < ctx->B; ++b)
+        if (h_n_pairs[b] < 0 || h_n_pairs[b] > ctx->h_len[b])
+            return fail(ctx, PIPO_EINVAL, "sequence %d: rollback to %d of %d entries", b, h_n_pairs[b], ctx->h_len[b]);
+    CK(cudaSetDevice(ctx->dev));
+    CK(cudaMemcpyAsync(ctx->n_pos, h_n_pairs, (size_t)ctx->B * 4, cudaMemcpyHostToDevice, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    for (int b = 0; b < ctx->B; ++b) ctx->h_len[b] = h_n_pairs[b];
+    return PIPO_OK;
+}
+
+pipo_status pipo_set_pending(pipo_ctx* ctx, const int32_t* h_pairs) {
+    if (!ctx || !h_pairs) return fail(ctx, PIPO_EINVAL, "null argument");
+    if (!ctx->prefilled) return fail(ctx, PIPO_ESTATE, "set_pending before prefill");
+    for (int b = 0; b < ctx->B; ++b) {
+        if (h_pairs[2 * b] < 0 || h_pairs[2 * b] >= ctx->cfg.vocab || h_pairs[2 * b + 1] < -1 ||
+            h_pairs[2 * b + 1] >= ctx->cfg.vocab)
+            return fail(ctx, PIPO_EINVAL, "sequence %d: pending pair out of range", b);
+    }
+    CK(cudaSetDevice(ctx->dev));
+    CK(cudaMemcpyAsync(ctx->pending, h_pairs, (size_t)ctx->B * 8, cudaMemcpyHostToDevice, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    return PIPO_OK;
+}
+
+pipo_status pipo_get_counters(pipo_ctx* ctx, int32_t* h_kv_len, int64_t* h_emitted) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    CK(cudaSetDevice(ctx->dev));
+    if (h_kv_len) CK(cudaMemcpyAsync(h_kv_len, ctx->n_pos, (size_t)ctx->B * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    if (h_emitted) CK(cudaMemcpyAsync(h_emitted, ctx->emitted, (size_t)ctx->B * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    return PIPO_OK;
+}
+
+pipo_status pipo_debug_dump(pipo_ctx* ctx, const pipo_debug* o) {
+    if (!ctx || !o) return fail(ctx, PIPO_EINVAL, "null argument");
+    if (!ctx->cfg.debug) return fail(ctx, PIPO_ESTATE, "context was created without debug buffers");
+    CK(cudaSetDevice(ctx->dev));
+    const size_t B = ctx->B, V = ctx->cfg.vocab, H = ctx->cfg.hidden;
+    cudaStream_t s = ctx->stream;
+    if (o->logits_b) CK(cudaMemcpyAsync(o->logits_b, ctx->dbg_lb, B * V * 4, cudaMemcpyDeviceToHost, s));
+    if (o->logits_d) CK(cudaMemcpyAsync(o->logits_d, ctx->dbg_ld, B * V * 4, cudaMemcpyDeviceToHost, s));
+    if (o->conf) CK(cudaMemcpyAsync(o->conf, ctx->dbg_conf, B * 4, cudaMemcpyDeviceToHost, s));
+    if (o->h_b) CK(cudaMemcpyAsync(o->h_b, ctx->dbg_hb, B * H * 4, cudaMemcpyDeviceToHost, s));
+    if (o->h_d) CK(cudaMemcpyAsync(o->h_d, ctx->dbg_hd, B * H * 4, cudaMemcpyDeviceToHost, s));
+    if (o->x_b) CK(cudaMemcpyAsync(o->x_b, ctx->dbg_xb, B * 4, cudaMemcpyDeviceToHost, s));
+    if (o->x_d) CK(cudaMemcpyAsync(o->x_d, ctx->dbg_xd, B * 4, cudaMemcpyDeviceToHost, s));
+    CK(cudaStreamSynchronize(s));
+    return PIPO_OK;
+}
+
+pipo_status pipo_read_cache(pipo_ctx* ctx, int32_t b, int32_t layer, int32_t n, float* h_K, float* h_V) {
+    if (!ctx || !h_K || !h_V) return fail(ctx, PIPO_EINVAL, "null argument");
+    if (b < 0 || b >= ctx->cfg.max_batch || layer < 0 || layer >= ctx->n_cache_layers || n < 0 || n > ctx->cfg.max_ctx)
+        return fail(ctx, PIPO_EINVAL, "read_cache: bad index");
+    if (n == 0) return PIPO_OK;
+    CK(cudaSetDevice(ctx->dev));
+    const size_t kd = (size_t)ctx->cfg.n_kv_heads * ctx->cfg.head_dim;
+    TRY(ensure_cache_tmp(ctx, 2 * kd * n));
+    cache_copy_kernel<<<n, 256, 0, ctx->stream>>>(kv_view(ctx, layer), b, n, ctx->cfg.head_dim, ctx->cache_tmp, 0,
+                                                   ctx->cfg.dtype == 1);
+    CK(cudaGetLastError());
+    CK(cudaMemcpyAsync(h_K, ctx->cache_tmp, kd * n * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaMemcpyAsync(h_V, ctx->cache_tmp + kd * n, kd * n * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    return PIPO_OK;
+}
+
+pipo_status pipo_load_cache(pipo_ctx* ctx, int32_t b, int32_t n, const float* h_K, const float* h_V) {
+    if (!ctx || !h_K || !h_V) return fail(ctx, PIPO_EINVAL, "null argument");
+    if (!ctx->prefilled || b < 0 || b >= ctx->B) return fail(ctx, PIPO_ESTATE, "load_cache needs a prefilled sequence b");
+    if (n < 1 || n > ctx->cfg.max_ctx) return fail(ctx, PIPO_ECAPACITY, "load_cache: %d entries", n);
+    CK(cudaSetDevice(ctx->dev));
+    const size_t kd = (size_t)ctx->cfg.n_kv_heads * ctx->cfg.head_dim;
+    TRY(ensure_cache_tmp(ctx, 2 * kd * n));
+    for (int l = 0; l < ctx->n_cache_layers; ++l) {
+        CK(cudaMemcpyAsync(ctx->cache_tmp, h_K + (size_t)l * n * kd, kd * n * 4, cudaMemcpyHostToDevice, ctx->stream));
+        CK(cudaMemcpyAsync(ctx->cache_tmp + kd * n, h_V + (size_t)l * n * kd, kd * n * 4, cudaMemcpyHostToDevice, ctx->stream));
+        cache_copy_kernel<<<n, 256, 0, ctx->stream>>>(kv_view(ctx, l), b, n, ctx->cfg.head_dim, ctx->cache_tmp, 1,
+                                                       ctx->cfg.dtype == 1);
+        CK(cudaGetLastError());
+    }
+    std::vector<int32_t> nn(1, n);
+    CK(cudaMemcpyAsync(ctx->n_pos + b, nn.data(), 4, cudaMemcpyHostToDevice, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    ctx->h_len[b] = n;
+    return PIPO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,56 @@
+"""Algorithmic bytes and flops of one PIPO pair-decode step.
+
+What the method must move per step, whatever the implementation:
+  * every weight of the compressor, the L backbone blocks, the MTP input
+    projection and block, and the confidence head, once;
+  * the tied embedding E twice: the draft head needs the backbone token x_b
+    from the first LM-head pass before its own pass can start (Eq. 3-5);
+  * the KV cache of every block: entries 0..n of each sequence, read once
+    (keys and values, backbone blocks + the MTP block), plus the new entry
+    written.
+Activations are a few KB per sequence and are left out.
+"""
+from __future__ import annotations
+
+from .synth import ModelShape
+
+
+def esize(s: ModelShape) -> int:
+    return 2 if s.dtype == "bf16" else 4
+
+
+def block_params(s: ModelShape) -> int:
+    qd, kd = s.n_q * s.d_h, s.n_kv * s.d_h
+    return 2 * s.H + (qd + 2 * kd) * s.H + s.H * qd + 3 * s.F * s.H
+
+
+def weight_params(s: ModelShape) -> int:
+    """Parameters streamed once per step (E excluded)."""
+    H = s.H
+    comp = H * 2 * H + (H * H if s.compressor == "mlp" else H)
+    mtp = 2 * H + H * 2 * H + (block_params(s) if s.mtp_block else 0) + H
+    conf = 2 * H + H * 2 * H + H
+    return comp + s.L * block_params(s) + H + mtp + conf
+
+
+def kv_entry_bytes(s: ModelShape) -> int:
+    """Bytes of one KV entry across every cached block (K and V)."""
+    layers = s.L + (1 if s.mtp_block else 0)
+    return layers * 2 * s.n_kv * s.d_h * esize(s)
+
+
+def step_bytes(s: ModelShape, batch: int, ctx_avg: float) -> float:
+    """Algorithmic HBM bytes of one step; ctx_avg = mean entries per sequence
+    before the step (the step reads ctx_avg + 1 entries and writes one)."""
+    e = esize(s)
+    w = (weight_params(s) + 2 * s.V * s.H) * e
+    kv = batch * (ctx_avg + 1) * kv_entry_bytes(s) + batch * kv_entry_bytes(s)
+    return float(w + kv)
+
+
+def step_flops(s: ModelShape, batch: int, ctx_avg: float) -> float:
+    """Multiply-add flops of one step (2 per MAC): weights x batch + attention."""
+    macs = (weight_params(s) + 2 * s.V * s.H) * batch
+    layers = s.L + (1 if s.mtp_block else 0)
+    macs += batch * layers * (ctx_avg + 1) * s.n_q * s.d_h * 2
+    return 2.0 * macs

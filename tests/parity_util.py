@@ -1,0 +1,81 @@
+"""Shared driver of the GPU-vs-oracle parity tests.
+
+Forced replay: after every step both sides continue from the oracle's pending
+pair, so each step is compared from identical history.  Per step:
+  * logits of both heads and the confidence: max-abs <= tol
+    (2e-2 for bf16 models, 1e-4 for fp32 models);
+  * x_b / x_d bit-exact wherever the oracle's top-1/top-2 logit margin > 1e-2;
+  * the accept decision bit-exact wherever |c - tau| > 1e-2.
+"""
+import numpy as np
+
+from oracle import oracle as O
+from paper_2605_27255_gb300 import capi
+
+MARGIN = 1e-2
+
+
+def tol_for(shape):
+    return 2e-2 if shape.dtype == "bf16" else 1e-4
+
+
+class Stats:
+    def __init__(self):
+        self.tok_checked = 0
+        self.tok_total = 0
+        self.acc_checked = 0
+        self.max_logit_err = 0.0
+        self.max_conf_err = 0.0
+
+
+def compare(shape, tau, o, d, tok, nacc, force, stats, tol, where=""):
+    B = tok.shape[0]
+    for b in range(B):
+        eb = float(np.abs(d["logits_b"][b] - o["logits_b"][b]).max())
+        ed = float(np.abs(d["logits_d"][b] - o["logits_d"][b]).max())
+        ec = abs(float(d["conf"][b]) - float(o["conf"][b]))
+        stats.max_logit_err = max(stats.max_logit_err, eb, ed)
+        stats.max_conf_err = max(stats.max_conf_err, ec)
+        assert eb <= tol and ed <= tol, f"{where} b={b}: logit error {eb:.3g}/{ed:.3g} > {tol}"
+        assert ec <= tol, f"{where} b={b}: confidence error {ec:.3g} > {tol}"
+        stats.tok_total += 2
+        if o["margin_b"][b] > MARGIN:
+            assert d["x_b"][b] == o["x_b"][b], f"{where} b={b}: x_b {d['x_b'][b]} != {o['x_b'][b]}"
+            assert tok[b, 0] == o["tokens"][b, 0]
+            stats.tok_checked += 1
+        if o["margin_d"][b] > MARGIN:
+            assert d["x_d"][b] == o["x_d"][b], f"{where} b={b}: x_d {d['x_d'][b]} != {o['x_d'][b]}"
+            stats.tok_checked += 1
+        if force or abs(float(o["conf"][b]) - tau) > MARGIN:
+            assert nacc[b] == o["n_acc"][b], f"{where} b={b}: accept {nacc[b]} != {o['n_acc'][b]}"
+            stats.acc_checked += 1
+            if o["margin_d"][b] > MARGIN and o["margin_b"][b] > MARGIN:
+                assert tok[b, 1] == o["tokens"][b, 1]
+
+
+def run_forced_replay(shape, weights, prompts, steps, *, tau=None, force=0, max_ctx=None,
+                      page_shuffle_seed=0, lens=None, oracle_weights=None):
+    """Prefill + `steps` decode steps on both sides; returns Stats."""
+    tau = shape.tau if tau is None else tau
+    B, T = prompts.shape
+    n_pairs = (T + 1) // 2
+    max_ctx = max_ctx or n_pairs + steps + 1
+    tol = tol_for(shape)
+    gpu = capi.Pipo(shape, weights, max_batch=B, max_ctx=max_ctx, tau=tau, force_mode=force, debug=True,
+                    page_shuffle_seed=page_shuffle_seed)
+    try:
+        orc = O.State(O.Model(shape, oracle_weights or weights, max_ctx=max_ctx), B)
+        st = Stats()
+        tok, nacc = gpu.prefill(prompts, lens)
+        o = orc.prefill(prompts, lens, tau=tau, force=force)
+        compare(shape, tau, o, gpu.debug(), tok, nacc, force, st, tol, "prefill")
+        for i in range(steps):
+            gpu.set_pending([[orc.seq(b)["p0"], orc.seq(b)["p1"]] for b in range(B)])
+            tok, nacc = gpu.step()
+            o = orc.step(tau=tau, force=force)
+            compare(shape, tau, o, gpu.debug(), tok, nacc, force, st, tol, f"step {i}")
+        n, e = gpu.counters()
+        assert list(n) == [orc.seq(b)["n"] for b in range(B)]
+        return st
+    finally:
+        gpu.close()

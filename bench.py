@@ -136,7 +136,8 @@ def oracle_sample(shape, weights_host, batch, n_ctx, tau, force, budget_s, max_s
 
     from oracle import oracle as O
     from paper_2605_27255_gb300 import synth
-    model = O.Model(shape, weights_host, max_ctx=n_ctx + 64)
+    cap = max_steps or 256
+    model = O.Model(shape, weights_host, max_ctx=n_ctx + cap + 1)
     st = O.State(model, batch)
     dev = "cuda" if torch.cuda.is_available() else "cpu"
     K, V = synth.gen_kv_fill(shape, n_ctx, seed=7, device=dev)
@@ -152,7 +153,7 @@ def oracle_sample(shape, weights_host, batch, n_ctx, tau, force, budget_s, max_s
         steps += 1
         toks += int(batch + o["n_acc"].sum())
         el = time.perf_counter() - t0
-        if el >= budget_s or (max_steps and steps >= max_steps):
+        if el >= budget_s or steps >= cap:
             break
     return dict(seconds=el, steps=steps, tokens=toks)
 

@@ -181,6 +181,20 @@ PIPO_API pipo_status pipo_load_cache(pipo_ctx *ctx, int32_t b, int32_t n, const 
  * restores the context's own stream.  Drops the captured step graph. */
 PIPO_API pipo_status pipo_set_stream(pipo_ctx *ctx, void *stream);
 
+/* ---- kernel-level entry points (device buffers, no context) ------------
+ * They run one kernel of the decode path on caller-owned device memory, on
+ * `stream` (a cudaStream_t; NULL = the legacy default stream), without a
+ * host sync.  Used to time and test kernels in isolation. */
+
+/* Weight-streaming GEMV of the backbone projections (Eq. 2 blocks):
+ *   mode 0: y[b*N + r] = sum_k W[r*K + k] * x[b*K + k]             (W: [N, K])
+ *   mode 1: y[b*N + r] = SiLU(W[2r,:] . x[b,:]) * (W[2r+1,:] . x[b,:])
+ *           (SwiGLU with gate and up rows interleaved; W: [2N, K])
+ * dtype 0: W fp32, 1: W bf16; x [B, K] and y [B, N] fp32.  K must be a
+ * multiple of 8 and B*K*4 <= 200 KB per 4 sequences.  EINVAL otherwise. */
+PIPO_API pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void *d_W, int32_t N, int32_t K,
+                                  const float *d_x, int32_t B, float *d_y, void *stream);
+
 /* Number of kernel launches one decode step enqueues (for launch accounting). */
 PIPO_API int32_t pipo_step_launches(const pipo_ctx *ctx);
 

@@ -81,6 +81,8 @@ SIGNATURES = {
     "pipo_read_cache": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_int32, _FP, _FP]),
     "pipo_load_cache": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, _FP, _FP]),
     "pipo_set_stream": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "pipo_op_gemv": (C.c_int, [C.c_int32, C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_int32,
+                               C.c_void_p, C.c_void_p]),
     "pipo_step_launches": (C.c_int32, [C.c_void_p]),
     "pipo_last_error": (C.c_char_p, [C.c_void_p]),
     "pipo_free": (None, [C.c_void_p]),
@@ -196,6 +198,12 @@ def pipo_load_cache(ctx, b: int, K: np.ndarray, V: np.ndarray) -> None:
 
 def pipo_set_stream(ctx, stream: int) -> None:
     _check(load().pipo_set_stream(ctx, C.c_void_p(stream or None)), ctx)
+
+
+def pipo_op_gemv(dtype: int, mode: int, W: int, N: int, K: int, x: int, B: int, y: int, stream: int = 0) -> None:
+    """Device pointers (ints); see include/pipo.h."""
+    _check(load().pipo_op_gemv(dtype, mode, C.c_void_p(W), N, K, C.c_void_p(x), B, C.c_void_p(y),
+                               C.c_void_p(stream or None)), None)
 
 
 def pipo_step_launches(ctx) -> int:

@@ -1,0 +1,310 @@
+// Split-KV GQA flash-decode over the paged pair-KV cache, one thread-block
+// cluster per (sequence, kv head) (sm_103a).
+//
+// Grid (CS, n_kv, B), cluster (CS, 1, 1), 128 threads.  CTA s of the cluster
+// attends the G = n_q/n_kv query heads of its kv head over a contiguous slice
+// of entries 0..n (n = entries before this step; entry n is this step's new
+// key/value).  Fused in:
+//   * RoPE of q and of the new k (rotate-half, angle table cos/sin
+//     [max_ctx][d_h/2] precomputed in fp64 and stored as fp32);
+//   * the KV append: the CTA owning entry n rounds k, v to the cache type,
+//     writes them to block table[b][n/64], slot n%64, and attends to them.
+// Each lane covers 8 dims of one entry (d_h/8 lanes per entry), keys and
+// values are read with 16-byte loads, kU entries in flight per lane group.
+// The CS partials (m, l, o) are merged through distributed shared memory:
+// each CTA merges a 1/CS slice of the output dims.  No global scratch.
+//
+// Programmatic dependent launch: the first keys/values of the slice are loaded
+// before griddepcontrol.wait (the cache entries < n and n itself come from
+// earlier steps); q and the new k, v are read after it.
+#pragma once
+
+#include <cooperative_groups.h>
+
+#include "kernels.cuh"
+
+namespace pipo {
+
+namespace cg = cooperative_groups;
+
+template <typename T> struct KV8;  // 8 consecutive cache elements
+template <> struct KV8<__nv_bfloat16> {
+    uint4 v;
+    __device__ __forceinline__ void load(const __nv_bfloat16* p) { v = ldg_cg(p); }
+    __device__ __forceinline__ void zero() { v = make_uint4(0, 0, 0, 0); }
+    __device__ __forceinline__ void to_float(float (&f)[8]) const {
+        f[0] = bf_lo(v.x); f[1] = bf_hi(v.x); f[2] = bf_lo(v.y); f[3] = bf_hi(v.y);
+        f[4] = bf_lo(v.z); f[5] = bf_hi(v.z); f[6] = bf_lo(v.w); f[7] = bf_hi(v.w);
+    }
+};
+template <> struct KV8<float> {
+    uint4 a, b;
+    __device__ __forceinline__ void load(const float* p) {
+        a = ldg_cg(p);
+        b = ldg_cg(p + 4);
+    }
+    __device__ __forceinline__ void zero() { a = b = make_uint4(0, 0, 0, 0); }
+    __device__ __forceinline__ void to_float(float (&f)[8]) const {
+        f[0] = __uint_as_float(a.x); f[1] = __uint_as_float(a.y); f[2] = __uint_as_float(a.z); f[3] = __uint_as_float(a.w);
+        f[4] = __uint_as_float(b.x); f[5] = __uint_as_float(b.y); f[6] = __uint_as_float(b.z); f[7] = __uint_as_float(b.w);
+    }
+};
+
+struct AttnParams {
+    const float* qkv;       // [B][(n_q + 2 n_kv) * d_h] projections of this step (not rotated)
+    int ld_qkv;
+    KVView kv;
+    const int32_t* n_pos;   // [B] entries before this step
+    const float* rope;      // [max_ctx][d_h/2][2] (cos, sin)
+    float* out;             // [B][n_q * d_h]
+    float scale;            // 1/sqrt(d_h)
+};
+
+// rotate-half RoPE of the 8 dims [8*li, 8*li+8) of a d_h vector held as one
+// 8-dim slice per lane; partner lane holds the other half (li ^ (LPE/2)).
+template <int DH>
+__device__ __forceinline__ void rope8(float (&x)[8], int li, int pos, const float* rope) {
+    constexpr int LPE = DH / 8;
+    float other[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) other[e] = __shfl_xor_sync(0xffffffffu, x[e], LPE / 2, LPE);
+    const bool first = li < LPE / 2;
+    const int i0 = (li % (LPE / 2)) * 8;  // pair index of dim e is i0 + e
+    const float4* cs = reinterpret_cast<const float4*>(rope + ((size_t)pos * (DH / 2) + i0) * 2);
+#pragma unroll
+    for (int e = 0; e < 8; e += 2) {
+        const float4 t = cs[e / 2];  // cos(i0+e), sin(i0+e), cos(i0+e+1), sin(i0+e+1)
+        if (first) {
+            x[e] = x[e] * t.x - other[e] * t.y;
+            x[e + 1] = x[e + 1] * t.z - other[e + 1] * t.w;
+        } else {
+            x[e] = x[e] * t.x + other[e] * t.y;
+            x[e + 1] = x[e + 1] * t.z + other[e + 1] * t.w;
+        }
+    }
+}
+
+template <typename T, int DH, int G, int CS>
+__global__ void __launch_bounds__(128) attn_cluster_kernel(AttnParams p) {
+    constexpr int LPE = DH / 8;        // lanes per entry
+    constexpr int EPW = 32 / LPE;      // entries per warp step
+    constexpr int kU = 4;              // warp steps in flight
+    constexpr int NW = 4;
+    constexpr int STEP = NW * EPW;     // entries per CTA step
+    __shared__ float sm_o[G][DH];
+    __shared__ float sm_m[G], sm_l[G];
+    __shared__ float wm[NW][G], wl[NW][G];
+    __shared__ float wo[NW][G][DH];
+
+    pdl_launch();
+    cg::cluster_group cluster = cg::this_cluster();
+    const int s = (int)cluster.block_rank();
+    const int g = blockIdx.y, b = blockIdx.z;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int li = lane % LPE, slot = lane / LPE;
+    const int n_kv = p.kv.n_kv, n_q = n_kv * G;
+    const int n = p.n_pos[b];          // cached entries; entry n is new
+    const int len = n + 1;
+    const int chunk = (len + CS - 1) / CS;
+    const int j0 = s * chunk, j1 = min(len, j0 + chunk);
+    const int jc = min(j1, n);         // cached part of the slice: [j0, jc)
+    const T* Kb = static_cast<const T*>(p.kv.K);
+    const T* Vb = static_cast<const T*>(p.kv.V);
+
+    // prefetch the first kU warp steps of keys/values (independent of this step)
+    KV8<T> kr[kU], vr[kU];
+    const int jwb = j0 + warp * EPW;  // warp-uniform base; lane group entry = base + slot
+    // loads are unconditional: an entry outside the slice reads entry 0 of the
+    // sequence instead and is masked out of the softmax (a select on a load
+    // result would make the thread wait for it)
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+        const int j = jwb + slot + u * STEP;
+        const size_t off = kv_off<T, DH>(p.kv, b, j < jc ? j : 0, g) + li * 8;
+        kr[u].load(Kb + off);
+        vr[u].load(Vb + off);
+    }
+    pdl_wait();
+
+    // q of the G heads, 8 dims per lane, rotated, pre-scaled
+    float q[G][8];
+    const float* qrow = p.qkv + (size_t)b * p.ld_qkv;
+#pragma unroll
+    for (int hh = 0; hh < G; ++hh) {
+        const float4* qp = reinterpret_cast<const float4*>(qrow + (size_t)(g * G + hh) * DH + li * 8);
+        const float4 a = qp[0], c = qp[1];
+        q[hh][0] = a.x; q[hh][1] = a.y; q[hh][2] = a.z; q[hh][3] = a.w;
+        q[hh][4] = c.x; q[hh][5] = c.y; q[hh][6] = c.z; q[hh][7] = c.w;
+        rope8<DH>(q[hh], li, n, p.rope);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) q[hh][e] *= p.scale;
+    }
+
+    float m[G], l[G], o[G][8];
+#pragma unroll
+    for (int hh = 0; hh < G; ++hh) {
+        m[hh] = -INFINITY;
+        l[hh] = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) o[hh][e] = 0.f;
+    }
+
+    // one block of kU entries per lane group: scores, one max update, sums
+    auto consume = [&](KV8<T> (&kk)[kU], KV8<T> (&vv)[kU], int jbase) {
+        float sc[kU][G];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            float kf[8];
+            kk[u].to_float(kf);
+#pragma unroll
+            for (int hh = 0; hh < G; ++hh) {
+                float d = 0.f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) d += q[hh][e] * kf[e];
+#pragma unroll
+                for (int off = LPE / 2; off > 0; off >>= 1) d += __shfl_xor_sync(0xffffffffu, d, off, LPE);
+                sc[u][hh] = (jbase + u * STEP < jc) ? d : -INFINITY;
+            }
+        }
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) {
+            float mx = m[hh];
+#pragma unroll
+            for (int u = 0; u < kU; ++u) mx = fmaxf(mx, sc[u][hh]);
+            if (mx == -INFINITY) continue;
+            const float corr = expf(m[hh] - mx);
+            l[hh] *= corr;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) o[hh][e] *= corr;
+            m[hh] = mx;
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            float vf[8];
+            vv[u].to_float(vf);
+#pragma unroll
+            for (int hh = 0; hh < G; ++hh) {
+                const float pj = (sc[u][hh] == -INFINITY) ? 0.f : expf(sc[u][hh] - m[hh]);
+                l[hh] += pj;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) o[hh][e] += pj * vf[e];
+            }
+        }
+    };
+
+    for (int jb = jwb; jb < jc; jb += kU * STEP) {  // warp-uniform trip count
+        KV8<T> kn[kU], vn[kU];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            const int j = jb + slot + (kU + u) * STEP;
+            const size_t off = kv_off<T, DH>(p.kv, b, j < jc ? j : 0, g) + li * 8;
+            kn[u].load(Kb + off);
+            vn[u].load(Vb + off);
+        }
+        consume(kr, vr, jb + slot);
+#pragma unroll
+        for (int u = 0; u < kU; ++u) { kr[u] = kn[u]; vr[u] = vn[u]; }
+    }
+
+    // the new entry n: rotate k, round k and v to the cache type, append, attend
+    // (the whole warp 0 runs it so that the shuffles see full warps; lane
+    // group 0 writes the cache and keeps the entry in its softmax state)
+    if (n >= j0 && n < j1 && warp == 0) {
+        const float* kp = qrow + (size_t)(n_q + g) * DH + li * 8;
+        const float* vp = qrow + (size_t)(n_q + n_kv + g) * DH + li * 8;
+        float kf[8], vf[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) { kf[e] = kp[e]; vf[e] = vp[e]; }
+        rope8<DH>(kf, li, n, p.rope);
+        const size_t off = kv_off<T, DH>(p.kv, b, n, g) + li * 8;
+        T* Kw = static_cast<T*>(p.kv.K) + off;
+        T* Vw = static_cast<T*>(p.kv.V) + off;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const T kt = from_f<T>(kf[e]), vt = from_f<T>(vf[e]);
+            if (slot == 0) {
+                Kw[e] = kt;
+                Vw[e] = vt;
+            }
+            kf[e] = to_f(kt);
+            vf[e] = to_f(vt);
+        }
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) {
+            float d = 0.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) d += q[hh][e] * kf[e];
+#pragma unroll
+            for (int off2 = LPE / 2; off2 > 0; off2 >>= 1) d += __shfl_xor_sync(0xffffffffu, d, off2, LPE);
+            if (slot != 0) continue;
+            const float mx = fmaxf(m[hh], d);
+            const float corr = expf(m[hh] - mx);
+            const float pj = expf(d - mx);
+            l[hh] = l[hh] * corr + pj;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) o[hh][e] = o[hh][e] * corr + pj * vf[e];
+            m[hh] = mx;
+        }
+    }
+
+    // merge the EPW lane groups of the warp (same dims, different entries)
+#pragma unroll
+    for (int hh = 0; hh < G; ++hh) {
+#pragma unroll
+        for (int off = LPE; off < 32; off <<= 1) {
+            const float m2 = __shfl_xor_sync(0xffffffffu, m[hh], off);
+            const float l2 = __shfl_xor_sync(0xffffffffu, l[hh], off);
+            const float mx = fmaxf(m[hh], m2);
+            const float f1 = (m[hh] == -INFINITY) ? 0.f : expf(m[hh] - mx);
+            const float f2 = (m2 == -INFINITY) ? 0.f : expf(m2 - mx);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const float o2 = __shfl_xor_sync(0xffffffffu, o[hh][e], off);
+                o[hh][e] = o[hh][e] * f1 + o2 * f2;
+            }
+            l[hh] = l[hh] * f1 + l2 * f2;
+            m[hh] = mx;
+        }
+        if (slot == 0) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) wo[warp][hh][li * 8 + e] = o[hh][e];
+            if (li == 0) { wm[warp][hh] = m[hh]; wl[warp][hh] = l[hh]; }
+        }
+    }
+    __syncthreads();
+    // merge the warps: CTA partial (m, l, o) in shared memory
+    for (int i = threadIdx.x; i < G * DH; i += blockDim.x) {
+        const int hh = i / DH, t = i % DH;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) M = fmaxf(M, wm[w][hh]);
+        float L = 0.f, Ov = 0.f;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) {
+            const float f = (wm[w][hh] == -INFINITY) ? 0.f : expf(wm[w][hh] - M);
+            L += wl[w][hh] * f;
+            Ov += wo[w][hh][t] * f;
+        }
+        sm_o[hh][t] = Ov;
+        if (t == 0) { sm_m[hh] = M; sm_l[hh] = L; }
+    }
+    cluster.sync();
+    // cluster merge: CTA s finishes dims [s*G*DH/CS, (s+1)*G*DH/CS) of the G heads
+    constexpr int PER = (G * DH + CS - 1) / CS;
+    for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
+        const int hh = i / DH, t = i % DH;
+        float M = -INFINITY;
+        for (int r = 0; r < CS; ++r) M = fmaxf(M, *cluster.map_shared_rank(&sm_m[hh], r));
+        float L = 0.f, Ov = 0.f;
+        for (int r = 0; r < CS; ++r) {
+            const float mr = *cluster.map_shared_rank(&sm_m[hh], r);
+            const float f = (mr == -INFINITY) ? 0.f : expf(mr - M);
+            L += *cluster.map_shared_rank(&sm_l[hh], r) * f;
+            Ov += *cluster.map_shared_rank(&sm_o[hh][t], r) * f;
+        }
+        p.out[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + t] = Ov / L;
+    }
+    cluster.sync();  // keep every CTA's shared memory alive until all merges read it
+}
+
+}  // namespace pipo

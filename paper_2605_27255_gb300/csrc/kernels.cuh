@@ -19,7 +19,7 @@ enum Epi : int {
     EPI_BIAS = 1,    // y = W x + bias
     EPI_SILU = 2,    // y = SiLU(W x)
     EPI_RESADD = 3,  // y += W x            (residual stream; split-K: fixed-order sum)
-    EPI_SWIGLU = 4,  // y = SiLU(W_r x) * (W_{r+F} x)   (gate rows, then up rows)
+    EPI_SWIGLU = 4,  // y = SiLU(W_2r x) * (W_2r+1 x)   (gate and up rows interleaved)
     EPI_ARGMAX = 5,  // packed (logit, -row) max per sequence; optional logits
 };
 
@@ -44,7 +44,6 @@ struct GemvParams {
     const void* W;       // [rows, K]
     int N;               // output rows
     int K;               // input length (sum of the segments)
-    int rstride;         // EPI_SWIGLU: offset of the up rows
     int epi;
     float* y;
     int ldy;
@@ -63,11 +62,23 @@ struct GemvParams {
 
 // ---------------------------------------------------------------- loads
 
+// 128-bit streaming load of read-only weights.  volatile keeps the issue
+// point where the code puts it (ahead of the compute that consumes an older
+// load), so the register ring really holds several loads in flight.
 __device__ __forceinline__ uint4 ldg_stream(const void* p) {
     uint4 r;
-    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
         : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
         : "l"(p));
+    return r;
+}
+
+// 128-bit load of cache data written by earlier kernels (L1 bypassed).
+__device__ __forceinline__ uint4 ldg_cg(const void* p) {
+    uint4 r;
+    asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
     return r;
 }
 
@@ -115,6 +126,12 @@ __device__ __forceinline__ int argmax_row(unsigned long long k) {
     return (int)(0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFull));
 }
 
+// Programmatic dependent launch: let the next kernel of the stream start its
+// independent prologue, and wait for the previous kernel's results.  Both are
+// no-ops for a kernel launched without the programmatic-serialization attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -138,6 +155,8 @@ __global__ void __launch_bounds__(kThreads) gemv_kernel(GemvParams p) {
     const int K = p.K;
     const T* W = static_cast<const T*>(p.W);
 
+    pdl_launch();
+    pdl_wait();
     if (p.zero_ptr && blockIdx.x == 0)
         for (int i = threadIdx.x; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
 
@@ -209,8 +228,9 @@ __global__ void __launch_bounds__(kThreads) gemv_kernel(GemvParams p) {
             float acc0[NB], acc1[NB];
 #pragma unroll
             for (int bb = 0; bb < NB; ++bb) { acc0[bb] = 0.f; acc1[bb] = 0.f; }
-            const T* w0 = W + (size_t)r * K;
-            const T* w1 = W + (size_t)(r + p.rstride) * K;
+            // SwiGLU: gate row 2r and up row 2r+1 (interleaved at upload)
+            const T* w0 = W + (size_t)(TWO ? 2 * r : r) * K;
+            const T* w1 = W + (size_t)(2 * r + 1) * K;
             for (int kb = k0 + lane * 8; kb < k1; kb += 256 * kU) {
                 W8<T> wa[kU], wb[kU];
 #pragma unroll
@@ -326,6 +346,8 @@ __device__ __forceinline__ size_t kv_off(const KVView& kv, int b, int pos, int g
 template <typename T, int DH>
 __global__ void rope_append_kernel(const float* __restrict__ qkv, int ld_qkv, float* __restrict__ q_out,
                                    KVView kv, const int32_t* __restrict__ n_pos, int n_q, double theta) {
+    pdl_launch();
+    pdl_wait();
     const int b = blockIdx.x, h = blockIdx.y, i = threadIdx.x;
     const int pos = n_pos[b];
     const float* src = qkv + (size_t)b * ld_qkv + (size_t)h * DH;
@@ -363,6 +385,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
                                                           float* __restrict__ part_o, float* __restrict__ part_ml,
                                                           unsigned int* __restrict__ counters, int S, float scale) {
     constexpr int EPL = DH / 32;  // elements per lane
+    pdl_launch();
+    pdl_wait();
     const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n_kv = kv.n_kv, n_q = n_kv * G;
@@ -482,6 +506,8 @@ struct StepState {
 template <typename T>
 __global__ void accept_kernel(const float* __restrict__ t, const void* W2, int H, float tau, int force,
                               StepState st, const float* hb, const float* hd) {
+    pdl_launch();
+    pdl_wait();
     const int b = blockIdx.x;
     float acc = 0.f;
     for (int k = threadIdx.x; k < H; k += blockDim.x) acc += ldw<T>(W2, k) * t[(size_t)b * H + k];
@@ -514,6 +540,8 @@ __global__ void accept_kernel(const float* __restrict__ t, const void* W2, int H
 
 // Prefill positions before the last: n[b] += 1.
 __global__ void advance_kernel(int32_t* n_pos, int B) {
+    pdl_launch();
+    pdl_wait();
     const int b = blockIdx.x * blockDim.x + threadIdx.x;
     if (b < B) n_pos[b] += 1;
 }

@@ -10,6 +10,8 @@
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
+#include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <numeric>
@@ -17,6 +19,8 @@
 #include <string>
 #include <vector>
 
+#include "attn_cluster.cuh"
+#include "gemv_stream.cuh"
 #include "kernels.cuh"
 #include "pipo.h"
 
@@ -70,6 +74,11 @@ struct pipo_ctx {
 
     int32_t *pf_pairs = nullptr, *pf_mtp = nullptr;
     size_t pf_cap = 0;
+
+    float* rope = nullptr;            // [max_ctx][d_h/2][2] cos, sin
+    bool pdl = false;                 // programmatic dependent launch (decode graph only)
+    int attn_cs = 8;                  // cluster size of the attention kernel
+    bool attn_v0 = false;             // (development) the unclustered attention path
 
     int B = 0;
     bool prefilled = false;
@@ -148,9 +157,12 @@ pipo_status upload_block(pipo_ctx* ctx, BlockW& bw, int l, const void* an, const
     TRY(put(ctx, bw.Wqkv, (qd + kd) * H, at(wv, l * kd * H, e), kd * H));
     TRY(upload(ctx, &bw.Wo, at(wo, l * H * qd, e), H * qd));
     TRY(upload(ctx, &bw.ffn_norm, at(fn, l * H, e), H));
+    // gate|up interleaved by row: row 2f = gate_f, row 2f+1 = up_f
     TRY(dalloc(ctx, reinterpret_cast<char**>(&bw.Wgu), 2 * F * H * e));
-    TRY(put(ctx, bw.Wgu, 0, at(wg, l * F * H, e), F * H));
-    TRY(put(ctx, bw.Wgu, F * H, at(wu, l * F * H, e), F * H));
+    if (!wg || !wu) return fail(ctx, PIPO_EINVAL, "missing gate/up weights");
+    CK(cudaMemcpy2D(bw.Wgu, 2 * H * e, at(wg, l * F * H, e), H * e, H * e, F, cudaMemcpyDefault));
+    CK(cudaMemcpy2D(static_cast<char*>(bw.Wgu) + H * e, 2 * H * e, at(wu, l * F * H, e), H * e, H * e, F,
+                    cudaMemcpyDefault));
     TRY(upload(ctx, &bw.Wdown, at(wd, l * H * F, e), H * F));
     return PIPO_OK;
 }
@@ -174,9 +186,64 @@ void* pick_gemv(int nb, bool two) {
     }
 }
 
-constexpr size_t kXsBudget = 100 * 1024;  // staged-input bytes per GEMV block
+constexpr size_t kXsBudget = 100 * 1024;      // staged-input bytes per v0 GEMV block
+constexpr size_t kStreamBudget = 200 * 1024;  // staged-input bytes per streaming GEMV block
+constexpr int kStreamDepth = 4;  // chunks per register batch (two batches)
+
+// Launch with programmatic dependent launch (decode graph) and an optional
+// cluster dimension.
+pipo_status launch_ex(pipo_ctx* ctx, const void* fn, dim3 grid, dim3 block, size_t smem, void** args,
+                      int cluster_x = 1) {
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = grid;
+    lc.blockDim = block;
+    lc.dynamicSmemBytes = smem;
+    lc.stream = ctx->stream;
+    cudaLaunchAttribute at[2];
+    int na = 0;
+    if (ctx->pdl) {
+        at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        at[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
+    }
+    if (cluster_x > 1) {
+        at[na].id = cudaLaunchAttributeClusterDimension;
+        at[na].val.clusterDim.x = cluster_x;
+        at[na].val.clusterDim.y = 1;
+        at[na].val.clusterDim.z = 1;
+        ++na;
+    }
+    lc.attrs = at;
+    lc.numAttrs = na;
+    CK(cudaLaunchKernelExC(&lc, fn, args));
+    ctx->launches++;
+    return PIPO_OK;
+}
+
+template <typename T, int NB, int RU>
+void* stream_fn(bool rows) {
+    return rows ? reinterpret_cast<void*>(&gemv_rows_kernel<T, NB, RU, kStreamDepth>)
+                : reinterpret_cast<void*>(&gemv_stream_kernel<T, NB, RU, kStreamDepth>);
+}
+
+// rows: every weight row is a whole number of 512-byte chunks (fast kernel)
+template <typename T>
+void* pick_stream(int nb, int ru, bool rows) {
+    switch (nb) {
+        case 1: return ru == 2 ? stream_fn<T, 1, 2>(rows) : stream_fn<T, 1, 1>(rows);
+        case 2: return ru == 2 ? stream_fn<T, 2, 2>(rows) : stream_fn<T, 2, 1>(rows);
+        default: return ru == 2 ? stream_fn<T, 4, 2>(rows) : stream_fn<T, 4, 1>(rows);
+    }
+}
 
 cudaError_t set_smem_attrs(bool bf) {
+    for (int nb : {1, 2, 4})
+        for (int ru : {1, 2})
+            for (bool rows : {false, true}) {
+                void* f = bf ? pick_stream<bf16>(nb, ru, rows) : pick_stream<float>(nb, ru, rows);
+                cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kStreamBudget);
+                if (e != cudaSuccess) return e;
+            }
     const int nbs[4] = {1, 2, 4, 8};
     for (int i = 0; i < 4; ++i)
         for (int two = 0; two < 2; ++two) {
@@ -190,6 +257,16 @@ cudaError_t set_smem_attrs(bool bf) {
 pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
     const bool bf = ctx->cfg.dtype == 1;
     const bool two = p.epi == EPI_SWIGLU;
+    if (p.B <= 4) {
+        // streaming kernel: one CTA per SM, chunk-balanced, deterministic
+        int nb = std::min(4, next_pow2_le8(std::max(1, p.B)));
+        while (nb > 1 && (size_t)nb * p.K * 4 > kStreamBudget) nb >>= 1;
+        if ((size_t)p.K * 4 > kStreamBudget) return fail(ctx, PIPO_EINVAL, "GEMV input length %d too large", p.K);
+        const bool rows = ((size_t)p.K * ctx->esz) % 512 == 0;
+        void* fn = bf ? pick_stream<bf16>(nb, two ? 2 : 1, rows) : pick_stream<float>(nb, two ? 2 : 1, rows);
+        void* args[] = {&p};
+        return launch_ex(ctx, fn, dim3(ctx->sms), dim3(kStreamThreads), (size_t)nb * p.K * 4, args);
+    }
     int nb = next_pow2_le8(std::max(1, p.B));
     while (nb > 1 && (size_t)nb * p.K * 4 > kXsBudget) nb >>= 1;
     if ((size_t)p.K * 4 > kXsBudget) return fail(ctx, PIPO_EINVAL, "GEMV input length %d too large", p.K);
@@ -209,9 +286,7 @@ pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
     const long long tasks = (long long)p.N * p.splitk;
     const int grid = (int)std::max(1LL, std::min<long long>((tasks + kWarps - 1) / kWarps, (long long)ctx->sms * per_sm));
     void* args[] = {&p};
-    CK(cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, ctx->stream));
-    ctx->launches++;
-    return PIPO_OK;
+    return launch_ex(ctx, fn, dim3(grid), dim3(kThreads), smem, args);
 }
 
 Seg act_seg(const float* src, int ld, int K, const void* gamma = nullptr) {
@@ -261,6 +336,26 @@ void* attn_pick(bool bf, int DH, int G) {
     return nullptr;
 }
 
+template <typename T, int DH, int G, int CS>
+void* attnc_fn() { return reinterpret_cast<void*>(&attn_cluster_kernel<T, DH, G, CS>); }
+
+template <typename T, int DH>
+void* attnc_pick_g(int G) {
+    switch (G) {
+        case 1: return attnc_fn<T, DH, 1, 8>();
+        case 2: return attnc_fn<T, DH, 2, 8>();
+        case 4: return attnc_fn<T, DH, 4, 8>();
+        case 8: return attnc_fn<T, DH, 8, 8>();
+        default: return nullptr;
+    }
+}
+
+void* attnc_pick(bool bf, int DH, int G) {
+    if (DH == 64) return bf ? attnc_pick_g<bf16, 64>(G) : attnc_pick_g<float, 64>(G);
+    if (DH == 128) return bf ? attnc_pick_g<bf16, 128>(G) : attnc_pick_g<float, 128>(G);
+    return nullptr;
+}
+
 void* rope_pick(bool bf, int DH) {
     if (DH == 64) return bf ? (void*)&rope_append_kernel<bf16, 64> : (void*)&rope_append_kernel<float, 64>;
     if (DH == 128) return bf ? (void*)&rope_append_kernel<bf16, 128> : (void*)&rope_append_kernel<float, 128>;
@@ -288,8 +383,22 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
     p.seg[0] = act_seg(xr, H, H, bw.attn_norm);
     p.K = H;
     TRY(launch_gemv(ctx, p));
-    // RoPE + KV append
     KVView kv = kv_view(ctx, cache_layer);
+    if (!ctx->attn_v0) {
+        // RoPE + KV append + split-KV attention, one cluster per (sequence, kv head)
+        AttnParams ap;
+        ap.qkv = ctx->qkv;
+        ap.ld_qkv = rows;
+        ap.kv = kv;
+        ap.n_pos = ctx->n_pos;
+        ap.rope = ctx->rope;
+        ap.out = ctx->attn;
+        ap.scale = 1.0f / sqrtf((float)DH);
+        void* args[] = {&ap};
+        TRY(launch_ex(ctx, attnc_pick(bf, DH, c.n_q_heads / c.n_kv_heads), dim3(ctx->attn_cs, c.n_kv_heads, ctx->B),
+                      dim3(128), 0, args, ctx->attn_cs));
+    } else {
+    // RoPE + KV append
     {
         const float* qkv = ctx->qkv;
         int ld = rows;
@@ -298,9 +407,7 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         int nq = c.n_q_heads;
         double theta = c.rope_theta;
         void* args[] = {(void*)&qkv, &ld, &qo, &kv, (void*)&np, &nq, &theta};
-        CK(cudaLaunchKernel(rope_pick(bf, DH), dim3(ctx->B, c.n_q_heads + 2 * c.n_kv_heads), dim3(DH / 2), args, 0,
-                            ctx->stream));
-        ctx->launches++;
+        TRY(launch_ex(ctx, rope_pick(bf, DH), dim3(ctx->B, c.n_q_heads + 2 * c.n_kv_heads), dim3(DH / 2), 0, args));
     }
     // split-KV attention
     {
@@ -314,9 +421,9 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         int Sv = S;
         float scale = 1.0f / sqrtf((float)DH);
         void* args[] = {(void*)&qp, &kv, (void*)&np, &out, &po, &pml, &cnt, &Sv, &scale};
-        CK(cudaLaunchKernel(attn_pick(bf, DH, c.n_q_heads / c.n_kv_heads), dim3(S, c.n_kv_heads, ctx->B), dim3(128),
-                            args, 0, ctx->stream));
-        ctx->launches++;
+        TRY(launch_ex(ctx, attn_pick(bf, DH, c.n_q_heads / c.n_kv_heads), dim3(S, c.n_kv_heads, ctx->B), dim3(128),
+                      0, args));
+    }
     }
     // O projection + residual
     p = gemv_base(ctx, bw.Wo, H, EPI_RESADD, xr, H);
@@ -329,7 +436,6 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
     p = gemv_base(ctx, bw.Wgu, c.ffn, EPI_SWIGLU, ctx->act, c.ffn);
     p.seg[0] = act_seg(xr, H, H, bw.ffn_norm);
     p.K = H;
-    p.rstride = c.ffn;
     TRY(launch_gemv(ctx, p));
     // down projection + residual
     p = gemv_base(ctx, bw.Wdown, H, EPI_RESADD, xr, H);
@@ -397,10 +503,10 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
     TRY(launch_gemv(ctx, p));
     if (c.mtp_block) TRY(enqueue_block(ctx, ctx->mtp, c.n_layers, ctx->x2));
     if (mode == PREFILL_MID) {
-        advance_kernel<<<(B + 127) / 128, 128, 0, ctx->stream>>>(ctx->n_pos, B);
-        CK(cudaGetLastError());
-        ctx->launches++;
-        return PIPO_OK;
+        int32_t* np = ctx->n_pos;
+        int Bv = B;
+        void* args[] = {&np, &Bv};
+        return launch_ex(ctx, (const void*)&advance_kernel, dim3((B + 127) / 128), dim3(128), 0, args);
     }
     // draft token (Eq. 5)
     TRY(enqueue_lm_head(ctx, ctx->x2, ctx->mtp_norm_post, am_d, c.debug ? ctx->dbg_ld : nullptr));
@@ -418,13 +524,17 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
         st.dbg_conf = ctx->dbg_conf; st.dbg_hb = ctx->dbg_hb; st.dbg_hd = ctx->dbg_hd;
         st.dbg_xb = ctx->dbg_xb; st.dbg_xd = ctx->dbg_xd;
     }
-    if (bf)
-        accept_kernel<bf16><<<B, 256, 0, ctx->stream>>>(ctx->t, ctx->conf_W2, H, c.tau, c.force_mode, st, ctx->x, ctx->x2);
-    else
-        accept_kernel<float><<<B, 256, 0, ctx->stream>>>(ctx->t, ctx->conf_W2, H, c.tau, c.force_mode, st, ctx->x, ctx->x2);
-    CK(cudaGetLastError());
-    ctx->launches++;
-    return PIPO_OK;
+    {
+        const float* tp = ctx->t;
+        const void* w2 = ctx->conf_W2;
+        int Hv = H, force = c.force_mode;
+        float tau = c.tau;
+        const float* hb = ctx->x;
+        const float* hd = ctx->x2;
+        void* args[] = {(void*)&tp, (void*)&w2, &Hv, &tau, &force, &st, (void*)&hb, (void*)&hd};
+        return launch_ex(ctx, bf ? (const void*)&accept_kernel<bf16> : (const void*)&accept_kernel<float>, dim3(B),
+                         dim3(256), 0, args);
+    }
 }
 
 void drop_graph(pipo_ctx* ctx) {
@@ -439,7 +549,9 @@ pipo_status ensure_graph(pipo_ctx* ctx) {
     cudaGraph_t g = nullptr;
     CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
     ctx->launches = 0;
+    ctx->pdl = true;
     pipo_status s = enqueue_position(ctx, DECODE, 0);
+    ctx->pdl = false;
     cudaError_t e = cudaStreamEndCapture(ctx->stream, &g);
     if (s != PIPO_OK) {
         if (g) cudaGraphDestroy(g);
@@ -566,6 +678,9 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         ctx->layer_elems = (size_t)ctx->num_blocks * c.n_kv_heads * c.page_size * DH;
         TRY(dalloc(ctx, reinterpret_cast<char**>(&ctx->Kc), std::max<size_t>(1, ctx->n_cache_layers) * ctx->layer_elems * ctx->esz));
         TRY(dalloc(ctx, reinterpret_cast<char**>(&ctx->Vc), std::max<size_t>(1, ctx->n_cache_layers) * ctx->layer_elems * ctx->esz));
+        // zeroed: masked lanes of the attention kernel read (and multiply by 0) entry 0
+        CK(cudaMemset(ctx->Kc, 0, std::max<size_t>(1, ctx->n_cache_layers) * ctx->layer_elems * ctx->esz));
+        CK(cudaMemset(ctx->Vc, 0, std::max<size_t>(1, ctx->n_cache_layers) * ctx->layer_elems * ctx->esz));
         std::vector<int32_t> table(ctx->num_blocks);
         std::iota(table.begin(), table.end(), 0);
         if (c.page_shuffle_seed) {
@@ -574,6 +689,20 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         }
         TRY(dalloc(ctx, &ctx->block_table, table.size() * sizeof(int32_t)));
         CK(cudaMemcpy(ctx->block_table, table.data(), table.size() * sizeof(int32_t), cudaMemcpyHostToDevice));
+
+        // RoPE angle table: angle = pos * theta^(-2i/d_h), cos/sin in double, stored fp32
+        {
+            std::vector<float> tab((size_t)c.max_ctx * DH);
+            for (int pos = 0; pos < c.max_ctx; ++pos)
+                for (int i = 0; i < DH / 2; ++i) {
+                    const double ang = (double)pos * std::pow((double)c.rope_theta, -2.0 * i / DH);
+                    tab[((size_t)pos * (DH / 2) + i) * 2] = (float)std::cos(ang);
+                    tab[((size_t)pos * (DH / 2) + i) * 2 + 1] = (float)std::sin(ang);
+                }
+            TRY(dalloc(ctx, &ctx->rope, tab.size() * 4));
+            CK(cudaMemcpy(ctx->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice));
+        }
+        if (const char* ev = getenv("PIPO_ATTN_V0")) ctx->attn_v0 = ev[0] == '1';
 
         // activations and state
         const int qd = c.n_q_heads * DH, kd = c.n_kv_heads * DH;
@@ -811,6 +940,40 @@ pipo_status pipo_load_cache(pipo_ctx* ctx, int32_t b, int32_t n, const float* h_
     CK(cudaStreamSynchronize(ctx->stream));
     ctx->h_len[b] = n;
     return PIPO_OK;
+}
+
+pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N, int32_t K, const float* d_x,
+                         int32_t B, float* d_y, void* stream) {
+    static thread_local pipo_ctx op;  // device facts and launch settings only; owns no memory
+    pipo_ctx* ctx = &op;
+    if (!d_W || !d_x || !d_y || N < 1 || K < 8 || K % 8 || B < 1 || (dtype != 0 && dtype != 1) ||
+        (mode != 0 && mode != 1))
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_gemv: bad arguments");
+    int dev = 0;
+    CK(cudaGetDevice(&dev));
+    if (op.sms == 0 || op.dev != dev || (int)op.esz != (dtype == 1 ? 2 : 4)) {
+        op.dev = dev;
+        CK(cudaDeviceGetAttribute(&op.sms, cudaDevAttrMultiProcessorCount, dev));
+        op.cfg.dtype = dtype;
+        op.esz = dtype == 1 ? 2 : 4;
+        CK(set_smem_attrs(dtype == 1));
+    }
+    op.stream = static_cast<cudaStream_t>(stream);
+    op.pdl = false;
+    GemvParams p{};
+    p.W = d_W;
+    p.N = N;
+    p.K = K;
+    p.epi = mode == 1 ? EPI_SWIGLU : EPI_STORE;
+    p.y = d_y;
+    p.ldy = N;
+    p.B = B;
+    p.splitk = 1;
+    p.nseg = 1;
+    p.seg[0] = act_seg(d_x, K, K);
+    pipo_status st = launch_gemv(ctx, p);
+    if (st != PIPO_OK) g_init_error = op.err;
+    return st;
 }
 
 }  // extern "C"

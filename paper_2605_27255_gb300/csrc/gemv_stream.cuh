@@ -19,10 +19,20 @@
 #pragma once
 
 #include "kernels.cuh"
+#include "tma.cuh"
 
 namespace pipo {
 
-constexpr int kStreamThreads = 512;
+#ifndef PIPO_STREAM_THREADS
+#define PIPO_STREAM_THREADS 768
+#endif
+#ifndef PIPO_TMA_WARPS
+#define PIPO_TMA_WARPS 8
+#endif
+#ifndef PIPO_TMA_STAGE_CHUNKS
+#define PIPO_TMA_STAGE_CHUNKS 8
+#endif
+constexpr int kStreamThreads = PIPO_STREAM_THREADS;
 constexpr int kStreamWarps = kStreamThreads / 32;
 
 template <typename T> struct Chunk16;  // 16 bytes of weights
@@ -384,6 +394,218 @@ __device__ __forceinline__ void stage_input_split(const GemvParams& p, float* xs
     __syncthreads();
 }
 
+// 4 consecutive elements of a weight-typed vector as floats (16- or 8-byte load)
+template <typename T>
+__device__ __forceinline__ float4 ld4(const void* base, size_t i) {
+    if (sizeof(T) == 4) return *reinterpret_cast<const float4*>(static_cast<const float*>(base) + i);
+    const uint2 u = *reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(base) + i);
+    return make_float4(bf_lo(u.x), bf_hi(u.x), bf_lo(u.y), bf_hi(u.y));
+}
+
+// Fast staging of the GEMV input in the split layout of gemv_rows: every
+// thread owns up to kMaxQ float4 groups of the K inputs, issues all their loads
+// (activation or gathered embedding, and the RMSNorm gain) at once, reduces the
+// sums of squares over the block, and stores the scaled values: one global
+// round trip per sequence instead of one per loop iteration.
+template <typename T, int NB, int kThreadsPerBlock>
+__device__ __forceinline__ void stage_input_fast(const GemvParams& p, float* xs, int b0, int nb) {
+    constexpr int kMaxQ = 4096 / kThreadsPerBlock;  // K <= 16384 inputs
+    __shared__ float red_ss[32][2];
+    __shared__ float rstd_s[2];
+    __shared__ int tok_s[NB][2];
+    const int K = p.K, K4 = K / 4, K0q = p.seg[0].K / 4;
+    const int tid = threadIdx.x, nt = blockDim.x, warp = tid >> 5, lane = tid & 31;
+    const bool norm0 = p.seg[0].gamma != nullptr, norm1 = p.nseg > 1 && p.seg[1].gamma != nullptr;
+    // gathered rows: token ids first (one round trip for all sequences)
+    if (tid < NB * 2) {
+        const int bb = tid >> 1, s = tid & 1;
+        int t = 0;
+        if (bb < nb && s < p.nseg && !p.seg[s].src) {
+            const Seg& sg = p.seg[s];
+            t = sg.tok_am ? argmax_row(sg.tok_am[b0 + bb]) : sg.tok[(size_t)(b0 + bb) * sg.tok_ld];
+        }
+        tok_s[bb][s] = t;
+    }
+    // gains (shared by every sequence)
+    float4 gm[kMaxQ];
+#pragma unroll
+    for (int i = 0; i < kMaxQ; ++i) {
+        const int q = tid + i * nt;
+        gm[i] = make_float4(1.f, 1.f, 1.f, 1.f);
+        if (q < K4) {
+            if (p.joint_norm) {
+                if (norm0) gm[i] = ld4<T>(p.seg[0].gamma, (size_t)q * 4);
+            } else if (q < K0q) {
+                if (norm0) gm[i] = ld4<T>(p.seg[0].gamma, (size_t)q * 4);
+            } else if (norm1) {
+                gm[i] = ld4<T>(p.seg[1].gamma, (size_t)(q - K0q) * 4);
+            }
+        }
+    }
+    __syncthreads();
+    for (int bb = 0; bb < NB; ++bb) {
+        const int b = b0 + bb;
+        float4 v[kMaxQ];
+        float ss0 = 0.f, ss1 = 0.f;
+#pragma unroll
+        for (int i = 0; i < kMaxQ; ++i) {
+            const int q = tid + i * nt;
+            v[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (q < K4 && bb < nb) {
+                const int s = q < K0q ? 0 : 1;
+                const Seg& sg = p.seg[s];
+                const int qq = s == 0 ? q : q - K0q;
+                if (sg.src) {
+                    v[i] = *reinterpret_cast<const float4*>(sg.src + (size_t)b * sg.ld + (size_t)qq * 4);
+                } else {
+                    const int t = tok_s[bb][s];
+                    v[i] = t < 0 ? ld4<T>(sg.pad, (size_t)qq * 4) : ld4<T>(sg.table, (size_t)t * sg.K + (size_t)qq * 4);
+                }
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < kMaxQ; ++i) {
+            const int q = tid + i * nt;
+            const float sq = v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+            if (p.joint_norm || q < K0q) ss0 += sq; else ss1 += sq;
+        }
+        if (norm0 || norm1) {
+            ss0 = warp_sum(ss0);
+            ss1 = warp_sum(ss1);
+            if (lane == 0) { red_ss[warp][0] = ss0; red_ss[warp][1] = ss1; }
+            __syncthreads();
+            if (tid < 2) {
+                float t = 0.f;
+                for (int w = 0; w < nt / 32; ++w) t += red_ss[w][tid];
+                const int len = p.joint_norm ? (tid == 0 ? K : 1) : (tid == 0 ? p.seg[0].K : (p.nseg > 1 ? p.seg[1].K : 1));
+                rstd_s[tid] = 1.0f / sqrtf(t / (float)len + p.eps);
+            }
+            __syncthreads();
+        }
+        const float r0 = norm0 ? rstd_s[0] : 1.f;
+        const float r1 = norm1 ? rstd_s[1] : 1.f;
+#pragma unroll
+        for (int i = 0; i < kMaxQ; ++i) {
+            const int q = tid + i * nt;
+            if (q < K4) {
+                const float r = (p.joint_norm || q < K0q) ? r0 : r1;
+                float4 o = v[i];
+                if (norm0 || norm1) {
+                    o.x *= r * gm[i].x; o.y *= r * gm[i].y; o.z *= r * gm[i].z; o.w *= r * gm[i].w;
+                }
+                const int idx = sizeof(T) == 2 ? (q & 1) * (K / 2) + (q >> 1) * 4 : q * 4;
+                *reinterpret_cast<float4*>(xs + bb * K + idx) = o;
+            }
+        }
+    }
+    __syncthreads();
+}
+
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(smem_dst)), "l"(gsrc), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\n cp.async.wait_group 0;" ::: "memory");
+}
+
+// Register-light staging for the register-ring GEMV: activations and RMSNorm
+// gains travel global -> shared with cp.async (no registers held), gathered
+// embedding rows (compressor and MTP inputs only) through registers; then one
+// block reduction for the norms and one scaling pass in shared memory.
+// gsm: K elements of type T for the gains.  Same split layout as stage_input_fast.
+template <typename T, int NB>
+__device__ __forceinline__ void stage_input_async(const GemvParams& p, float* xs, T* gsm, int b0, int nb) {
+    __shared__ float red_ss[32][NB][2];
+    __shared__ float rstd_s[NB][2];
+    const int K = p.K, K0q = p.seg[0].K / 4;
+    const int tid = threadIdx.x, nt = blockDim.x, warp = tid >> 5, lane = tid & 31;
+    const bool norm0 = p.seg[0].gamma != nullptr, norm1 = p.nseg > 1 && p.seg[1].gamma != nullptr;
+    auto xidx = [&](int q) { return sizeof(T) == 2 ? (q & 1) * (K / 2) + (q >> 1) * 4 : q * 4; };
+    // gains: raw bytes of each normalised segment into gsm (element k at gsm[k])
+    {
+        int koff = 0;
+        for (int s = 0; s < p.nseg; ++s) {
+            const Seg& sg = p.seg[s];
+            const int len = p.joint_norm ? K : sg.K;
+            const void* gp = sg.gamma;
+            if (gp && !(p.joint_norm && s > 0)) {
+                const int n16 = len * (int)sizeof(T) / 16;
+                for (int i = tid; i < n16; i += nt)
+                    cp_async16(reinterpret_cast<char*>(gsm + koff) + 16 * i, static_cast<const char*>(gp) + 16 * i, 16);
+            }
+            koff += sg.K;
+        }
+    }
+    // activations: 16-byte pieces straight into the split layout (zero-filled past nb)
+    for (int bb = 0; bb < NB; ++bb) {
+        int qoff = 0;
+        for (int s = 0; s < p.nseg; ++s) {
+            const Seg& sg = p.seg[s];
+            const int nq = sg.K / 4;
+            if (sg.src) {
+                const float* row = sg.src + (size_t)(b0 + min(bb, nb - 1)) * sg.ld;
+                for (int q = tid; q < nq; q += nt)
+                    cp_async16(xs + bb * K + xidx(qoff + q), row + 4 * q, bb < nb ? 16 : 0);
+            } else {
+                const int t = bb < nb ? (sg.tok_am ? argmax_row(sg.tok_am[b0 + bb]) : sg.tok[(size_t)(b0 + bb) * sg.tok_ld])
+                                      : 0;
+                for (int q = tid; q < nq; q += nt) {
+                    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (bb < nb) v = t < 0 ? ld4<T>(sg.pad, (size_t)q * 4) : ld4<T>(sg.table, (size_t)t * sg.K + (size_t)q * 4);
+                    *reinterpret_cast<float4*>(xs + bb * K + xidx(qoff + q)) = v;
+                }
+            }
+            qoff += nq;
+        }
+    }
+    cp_async_wait_all();
+    __syncthreads();
+    if (!norm0 && !norm1) return;
+    // sums of squares per sequence and norm group
+    const int K4 = K / 4;
+    float ss[NB][2];
+#pragma unroll
+    for (int bb = 0; bb < NB; ++bb) { ss[bb][0] = 0.f; ss[bb][1] = 0.f; }
+    for (int q = tid; q < K4; q += nt) {
+        const int gsel = (p.joint_norm || q < K0q) ? 0 : 1;
+#pragma unroll
+        for (int bb = 0; bb < NB; ++bb) {
+            const float4 v = *reinterpret_cast<const float4*>(xs + bb * K + xidx(q));
+            const float sq = v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+            if (gsel == 0) ss[bb][0] += sq; else ss[bb][1] += sq;
+        }
+    }
+#pragma unroll
+    for (int bb = 0; bb < NB; ++bb) {
+        const float a = warp_sum(ss[bb][0]), c = warp_sum(ss[bb][1]);
+        if (lane == 0) { red_ss[warp][bb][0] = a; red_ss[warp][bb][1] = c; }
+    }
+    __syncthreads();
+    if (tid < NB * 2) {
+        const int bb = tid >> 1, g = tid & 1;
+        float t = 0.f;
+        for (int w = 0; w < nt / 32; ++w) t += red_ss[w][bb][g];
+        const int len = p.joint_norm ? K : (g == 0 ? p.seg[0].K : (p.nseg > 1 ? p.seg[1].K : 1));
+        rstd_s[bb][g] = 1.0f / sqrtf(t / (float)len + p.eps);
+    }
+    __syncthreads();
+    for (int q = tid; q < K4; q += nt) {
+        const int gsel = (p.joint_norm || q < K0q) ? 0 : 1;
+        if (!(gsel == 0 ? norm0 : norm1)) continue;
+        const float4 gm = ld4<T>(gsm, (size_t)q * 4);
+#pragma unroll
+        for (int bb = 0; bb < NB; ++bb) {
+            float4* xp = reinterpret_cast<float4*>(xs + bb * K + xidx(q));
+            const float r = rstd_s[bb][gsel];
+            float4 v = *xp;
+            v.x *= r * gm.x; v.y *= r * gm.y; v.z *= r * gm.z; v.w *= r * gm.w;
+            *xp = v;
+        }
+    }
+    __syncthreads();
+}
+
 template <typename T, int NB, int RU, int kU>
 __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p) {
     extern __shared__ float4 smem4[];
@@ -427,7 +649,7 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
                 for (int i = threadIdx.x; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
         }
         __syncthreads();
-        stage_input_split<T, NB>(p, xs, b0, nb);
+        stage_input_async<T, NB>(p, xs, reinterpret_cast<T*>(xs + NB * K), b0, nb);
 
         float best_v[NB];
         int best_r[NB];
@@ -573,6 +795,269 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
         }
         __syncthreads();
     }
+}
+
+// ---------------------------------------------------------------------------
+// Per-warp accumulation over a contiguous range [c0, c1) of 512-byte chunks of
+// whole-chunk rows (shared by the register-ring and the bulk-copy kernels).
+template <typename T, int NB, int RU>
+struct WarpRows {
+    static constexpr int EPC = Chunk16<T>::kElems;
+    const GemvParams* p;
+    int K, cpr, cpu, u0, c0, c1, b0, nb, lane, warp;
+    int cc, crow, cj, xi, plane;
+    const float4* xs4;
+    float acc[NB], part[RU][NB];
+    float best_v[NB];
+    int best_r[NB];
+
+    __device__ __forceinline__ void init(const GemvParams* pp, const float* xs, int cpr_, int u0_, int c0_, int c1_,
+                                         int b0_, int nb_) {
+        p = pp;
+        K = pp->K;
+        cpr = cpr_;
+        cpu = cpr_ * RU;
+        u0 = u0_;
+        c0 = c0_;
+        c1 = c1_;
+        b0 = b0_;
+        nb = nb_;
+        lane = threadIdx.x & 31;
+        warp = threadIdx.x >> 5;
+        cc = c0;
+        crow = c0 / cpr;
+        cj = c0 - crow * cpr;
+        xi = cj * 32 + lane;
+        plane = K / 8;
+        xs4 = reinterpret_cast<const float4*>(xs);
+#pragma unroll
+        for (int bb = 0; bb < NB; ++bb) {
+            acc[bb] = 0.f;
+            best_v[bb] = -INFINITY;
+            best_r[bb] = 0x7fffffff;
+#pragma unroll
+            for (int r = 0; r < RU; ++r) part[r][bb] = 0.f;
+        }
+    }
+
+    // consume the next chunk cc of the range (its 16 bytes for this lane)
+    template <int NW>
+    __device__ __forceinline__ void chunk(const uint4& wv, int (&head_unit)[NW], int (&head_fin)[NW],
+                                          float (&head_val)[NW][RU][NB]) {
+        float w[EPC];
+        Chunk16<T>::to_float(wv, w);
+#pragma unroll
+        for (int bb = 0; bb < NB; ++bb) {
+            const float4 xa = xs4[bb * (K / 4) + xi];
+            float sum = w[0] * xa.x + w[1] * xa.y + w[2] * xa.z + w[3] * xa.w;
+            if (EPC == 8) {
+                const float4 xb = xs4[bb * (K / 4) + plane + xi];
+                sum += w[4 % EPC] * xb.x + w[5 % EPC] * xb.y + w[6 % EPC] * xb.z + w[7 % EPC] * xb.w;
+            }
+            acc[bb] += sum;
+        }
+        ++cc;
+        xi += 32;
+        if (++cj == cpr) {
+            const int r = crow % RU;
+#pragma unroll
+            for (int bb = 0; bb < NB; ++bb) {
+                const float t = warp_sum(acc[bb]);
+                acc[bb] = 0.f;
+#pragma unroll
+                for (int rr = 0; rr < RU; ++rr)
+                    if (rr == r) part[rr][bb] = t;
+            }
+            if (r == RU - 1) {
+                const int unit = crow / RU;
+                if (unit * cpu >= c0) {
+                    unit_epilogue<T, RU, NB>(*p, u0 + unit, part, b0, nb, best_v, best_r);
+                } else if (lane == 0) {
+                    head_unit[warp] = unit;
+                    head_fin[warp] = 1;
+#pragma unroll
+                    for (int rr = 0; rr < RU; ++rr)
+#pragma unroll
+                        for (int bb = 0; bb < NB; ++bb) head_val[warp][rr][bb] = part[rr][bb];
+                }
+#pragma unroll
+                for (int rr = 0; rr < RU; ++rr)
+#pragma unroll
+                    for (int bb = 0; bb < NB; ++bb) part[rr][bb] = 0.f;
+            }
+            cj = 0;
+            xi = lane;
+            ++crow;
+        }
+    }
+
+    // the range ended inside a unit: record this warp's partial of it
+    template <int NW>
+    __device__ __forceinline__ void finish(int (&head_unit)[NW], int (&head_fin)[NW], int (&tail_unit)[NW],
+                                           float (&head_val)[NW][RU][NB], float (&tail_val)[NW][RU][NB]) {
+        if (!(c0 < c1 && (c1 % cpu) != 0)) return;
+        const int unit = (c1 - 1) / cpu;
+        const int r = crow % RU;
+        float a[RU][NB];
+#pragma unroll
+        for (int bb = 0; bb < NB; ++bb) {
+            const float t = warp_sum(acc[bb]);
+#pragma unroll
+            for (int rr = 0; rr < RU; ++rr) a[rr][bb] = part[rr][bb] + ((rr == r && cj > 0) ? t : 0.f);
+        }
+        if (lane != 0) return;
+        if (unit * cpu >= c0) {
+            tail_unit[warp] = unit;
+#pragma unroll
+            for (int rr = 0; rr < RU; ++rr)
+#pragma unroll
+                for (int bb = 0; bb < NB; ++bb) tail_val[warp][rr][bb] = a[rr][bb];
+        } else {
+            head_unit[warp] = unit;
+            head_fin[warp] = 0;
+#pragma unroll
+            for (int rr = 0; rr < RU; ++rr)
+#pragma unroll
+                for (int bb = 0; bb < NB; ++bb) head_val[warp][rr][bb] = a[rr][bb];
+        }
+    }
+};
+
+// After a block barrier: units split between warps are finished by the warp
+// holding their last chunk (partials added in warp order); then the argmax
+// reduction of the block.
+template <typename T, int NB, int RU, int NW>
+__device__ __forceinline__ void finish_block(const GemvParams& p, WarpRows<T, NB, RU>& wr, int (&head_unit)[NW],
+                                             int (&head_fin)[NW], int (&tail_unit)[NW], float (&head_val)[NW][RU][NB],
+                                             float (&tail_val)[NW][RU][NB], float (&red_v)[NW][NB],
+                                             int (&red_r)[NW][NB]) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (head_fin[warp] && head_unit[warp] >= 0) {
+        const int unit = head_unit[warp];
+        int ws = warp - 1;
+        while (ws >= 0 && tail_unit[ws] != unit) --ws;
+        float a[RU][NB];
+#pragma unroll
+        for (int r = 0; r < RU; ++r)
+#pragma unroll
+            for (int bb = 0; bb < NB; ++bb) {
+                float sum = (ws >= 0) ? tail_val[ws][r][bb] : 0.f;
+                for (int v = (ws >= 0 ? ws + 1 : 0); v <= warp; ++v)
+                    if (head_unit[v] == unit) sum += head_val[v][r][bb];
+                a[r][bb] = sum;
+            }
+        unit_epilogue<T, RU, NB>(p, wr.u0 + unit, a, wr.b0, wr.nb, wr.best_v, wr.best_r);
+    }
+    if (p.epi == EPI_ARGMAX) {
+        if (lane == 0)
+#pragma unroll
+            for (int bb = 0; bb < NB; ++bb) { red_v[warp][bb] = wr.best_v[bb]; red_r[warp][bb] = wr.best_r[bb]; }
+        __syncthreads();
+        if (threadIdx.x < wr.nb) {
+            const int bb = threadIdx.x;
+            float bv = -INFINITY;
+            int br = 0x7fffffff;
+            for (int w = 0; w < NW; ++w)
+                if (red_r[w][bb] != 0x7fffffff && (red_v[w][bb] > bv || (red_v[w][bb] == bv && red_r[w][bb] < br))) {
+                    bv = red_v[w][bb];
+                    br = red_r[w][bb];
+                }
+            if (br != 0x7fffffff) atomicMax(p.am + wr.b0 + bb, argmax_key(bv, br));
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Bulk-copy (TMA) GEMV.  Each warp owns a contiguous chunk range of the CTA's
+// rows and a private ring of `ns` shared-memory stages of kStageChunks chunks;
+// lane 0 refills a stage with one cp.async.bulk as soon as the warp has read it
+// (mbarrier completion).  Bytes in flight per SM: up to 8 warps x ns x 4 KB,
+// with one copy instruction per 4 KB.  Single pass: B <= NB.
+constexpr int kTmaWarps = PIPO_TMA_WARPS;
+constexpr int kTmaThreads = kTmaWarps * 32;
+constexpr int kStageChunks = PIPO_TMA_STAGE_CHUNKS;
+constexpr int kStageBytes = kStageChunks * 512;
+
+template <typename T, int NB, int RU>
+__global__ void __launch_bounds__(kTmaThreads) gemv_tma_kernel(GemvParams p, int ns) {
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    __shared__ int head_unit[kTmaWarps], tail_unit[kTmaWarps], head_fin[kTmaWarps];
+    __shared__ float head_val[kTmaWarps][RU][NB], tail_val[kTmaWarps][RU][NB];
+    __shared__ float red_v[kTmaWarps][NB];
+    __shared__ int red_r[kTmaWarps][NB];
+
+    pdl_launch();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int K = p.K;
+    const int cpr = K * (int)sizeof(T) / 512;
+    const int cpu = cpr * RU;
+    const int G = gridDim.x;
+    const int u0 = (int)((long long)blockIdx.x * p.N / G);
+    const int u1 = (int)((long long)(blockIdx.x + 1) * p.N / G);
+    const int C = (u1 - u0) * cpu;
+    const int c0 = (int)((long long)warp * C / kTmaWarps);
+    const int c1 = (int)((long long)(warp + 1) * C / kTmaWarps);
+    const char* gsrc = static_cast<const char*>(p.W) + ((size_t)u0 * cpu + c0) * 512;
+
+    unsigned char* ring = smem_raw + (size_t)warp * ns * kStageBytes;
+    float* xs = reinterpret_cast<float*>(smem_raw + (size_t)kTmaWarps * ns * kStageBytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(xs + NB * K) + warp * ns;
+    const int nst = (c1 - c0 + kStageChunks - 1) / kStageChunks;  // stages of this warp
+
+    auto issue = [&](int i) {  // lane 0: stage i of this warp into slot i % ns
+        const int first = i * kStageChunks;
+        const int n = min(kStageChunks, (c1 - c0) - first);
+        const uint32_t bytes = (uint32_t)n * 512u;
+        uint64_t* bar = bars + (i % ns);
+        mbar_arrive_expect_tx(bar, bytes);
+        bulk_g2s(ring + (size_t)(i % ns) * kStageBytes, gsrc + (size_t)first * 512, bytes, bar);
+    };
+    if (lane == 0) {
+        for (int s2 = 0; s2 < ns; ++s2) mbar_init(bars + s2, 1);
+        mbar_init_fence();
+        for (int i = 0; i < min(ns, nst); ++i) issue(i);
+    }
+    __syncwarp();
+    pdl_wait();
+    if (p.zero_ptr && blockIdx.x == 0)
+        for (int i = threadIdx.x; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
+    if (lane == 0) { head_fin[warp] = 0; head_unit[warp] = -1; tail_unit[warp] = -1; }
+    __syncthreads();
+    stage_input_fast<T, NB, kTmaThreads>(p, xs, 0, min(NB, p.B));
+
+    WarpRows<T, NB, RU> wr;
+    wr.init(&p, xs, cpr, u0, c0, c1, 0, min(NB, p.B));
+    int failed = -1;  // first stage whose wait gave up
+    for (int i = 0; i < nst; ++i) {
+        const int slot = i % ns;
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(bars + slot, (uint32_t)((i / ns) & 1)));
+        if (!ok) {
+            failed = i;
+            break;
+        }
+        const unsigned char* sp = ring + (size_t)slot * kStageBytes + lane * 16;
+        const int n = min(kStageChunks, (c1 - c0) - i * kStageChunks);
+        if (n == kStageChunks) {
+#pragma unroll
+            for (int ch = 0; ch < kStageChunks; ++ch)
+                wr.chunk(*reinterpret_cast<const uint4*>(sp + ch * 512), head_unit, head_fin, head_val);
+        } else {
+            for (int ch = 0; ch < n; ++ch)
+                wr.chunk(*reinterpret_cast<const uint4*>(sp + ch * 512), head_unit, head_fin, head_val);
+        }
+        __syncwarp();
+        if (lane == 0 && i + ns < nst) {
+            fence_proxy_async();  // our generic reads of the slot before the async overwrite
+            issue(i + ns);
+        }
+    }
+    if (failed >= 0 && lane == 0) {
+        // a wait gave up (error recorded): wait, bounded, for the copies still in flight
+        for (int i = failed + 1; i < min(nst, failed + ns); ++i) mbar_wait(bars + (i % ns), (uint32_t)((i / ns) & 1));
+    }
+    wr.finish(head_unit, head_fin, tail_unit, head_val, tail_val);
+    __syncthreads();
+    finish_block<T, NB, RU, kTmaWarps>(p, wr, head_unit, head_fin, tail_unit, head_val, tail_val, red_v, red_r);
 }
 
 }  // namespace pipo

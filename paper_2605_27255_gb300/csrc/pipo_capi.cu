@@ -22,6 +22,7 @@
 #include "attn_cluster.cuh"
 #include "gemv_stream.cuh"
 #include "kernels.cuh"
+#include "megakernel.cuh"
 #include "pipo.h"
 
 using namespace pipo;
@@ -79,6 +80,17 @@ struct pipo_ctx {
     bool pdl = false;                 // programmatic dependent launch (decode graph only)
     int attn_cs = 8;                  // cluster size of the attention kernel
     bool attn_v0 = false;             // (development) the unclustered attention path
+    bool gemv_tma = false;            // bulk-copy GEMV (else the register-ring GEMV)
+    // persistent step kernel: phases recorded from the enqueue code
+    std::vector<Phase>* rec = nullptr;  // recording target (nullptr: launch kernels)
+    bool rec_ok = true;                 // every recorded phase fits the step kernel
+    int rec_kmax = 0;
+    bool use_mk = false;                // use the persistent step kernel when it fits
+    bool mk_active = false;             // the current decode graph is the step kernel
+    Phase* d_phases = nullptr;
+    size_t d_phases_cap = 0;
+    unsigned* bar_ctr = nullptr;
+    std::string mk_note;
 
     int B = 0;
     bool prefilled = false;
@@ -188,7 +200,7 @@ void* pick_gemv(int nb, bool two) {
 
 constexpr size_t kXsBudget = 100 * 1024;      // staged-input bytes per v0 GEMV block
 constexpr size_t kStreamBudget = 200 * 1024;  // staged-input bytes per streaming GEMV block
-constexpr int kStreamDepth = 4;  // chunks per register batch (two batches)
+constexpr int kStreamDepth = 4;  // chunks per register batch (two batches in flight)
 
 // Launch with programmatic dependent launch (decode graph) and an optional
 // cluster dimension.
@@ -221,6 +233,30 @@ pipo_status launch_ex(pipo_ctx* ctx, const void* fn, dim3 grid, dim3 block, size
 }
 
 template <typename T, int NB, int RU>
+void* tma_fn() { return reinterpret_cast<void*>(&gemv_tma_kernel<T, NB, RU>); }
+
+template <typename T>
+void* pick_tma(int nb, int ru) {
+    switch (nb) {
+        case 1: return ru == 2 ? tma_fn<T, 1, 2>() : tma_fn<T, 1, 1>();
+        case 2: return ru == 2 ? tma_fn<T, 2, 2>() : tma_fn<T, 2, 1>();
+        default: return ru == 2 ? tma_fn<T, 4, 2>() : tma_fn<T, 4, 1>();
+    }
+}
+
+size_t g_smem_optin = 0;  // opt-in shared memory per block of the device
+
+// Allow `fn` the largest dynamic shared memory the device permits next to its
+// static shared memory; returns that size (0 on failure).
+size_t allow_max_smem(const void* fn) {
+    cudaFuncAttributes fa{};
+    if (cudaFuncGetAttributes(&fa, fn) != cudaSuccess) return 0;
+    const size_t dyn = g_smem_optin > fa.sharedSizeBytes ? g_smem_optin - fa.sharedSizeBytes : 0;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn) != cudaSuccess) return 0;
+    return dyn;
+}
+
+template <typename T, int NB, int RU>
 void* stream_fn(bool rows) {
     return rows ? reinterpret_cast<void*>(&gemv_rows_kernel<T, NB, RU, kStreamDepth>)
                 : reinterpret_cast<void*>(&gemv_stream_kernel<T, NB, RU, kStreamDepth>);
@@ -237,6 +273,16 @@ void* pick_stream(int nb, int ru, bool rows) {
 }
 
 cudaError_t set_smem_attrs(bool bf) {
+    int dev = 0, optin = 0;
+    cudaError_t e0 = cudaGetDevice(&dev);
+    if (e0 == cudaSuccess) e0 = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e0 != cudaSuccess) return e0;
+    g_smem_optin = (size_t)optin;
+    for (int nb : {1, 2, 4})
+        for (int ru : {1, 2}) {
+            void* f = bf ? pick_tma<bf16>(nb, ru) : pick_tma<float>(nb, ru);
+            if (allow_max_smem(f) < 160 * 1024) return cudaErrorInvalidValue;
+        }
     for (int nb : {1, 2, 4})
         for (int ru : {1, 2})
             for (bool rows : {false, true}) {
@@ -257,15 +303,42 @@ cudaError_t set_smem_attrs(bool bf) {
 pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
     const bool bf = ctx->cfg.dtype == 1;
     const bool two = p.epi == EPI_SWIGLU;
+    if (ctx->rec) {
+        Phase ph{};
+        ph.type = PH_GEMV;
+        ph.ru = two ? 2 : 1;
+        p.splitk = 1;  // the step kernel finishes every row inside one CTA
+        ph.g = p;
+        if (((size_t)p.K * ctx->esz) % 512 != 0 || p.B > 4) ctx->rec_ok = false;
+        ctx->rec_kmax = std::max(ctx->rec_kmax, p.K);
+        ctx->rec->push_back(ph);
+        return PIPO_OK;
+    }
     if (p.B <= 4) {
         // streaming kernel: one CTA per SM, chunk-balanced, deterministic
         int nb = std::min(4, next_pow2_le8(std::max(1, p.B)));
-        while (nb > 1 && (size_t)nb * p.K * 4 > kStreamBudget) nb >>= 1;
+        while (nb > 1 && (size_t)nb * p.K * 4 + (size_t)p.K * ctx->esz > kStreamBudget) nb >>= 1;
         if ((size_t)p.K * 4 > kStreamBudget) return fail(ctx, PIPO_EINVAL, "GEMV input length %d too large", p.K);
         const bool rows = ((size_t)p.K * ctx->esz) % 512 == 0;
+        const size_t xbytes = (size_t)nb * p.K * 4;
+        if (rows && ctx->gemv_tma && p.B <= nb) {
+            // bulk-copy kernel: stages per warp from what shared memory allows
+            const size_t per_stage = (size_t)kTmaWarps * (kStageBytes + 8);
+            const size_t room = g_smem_optin > 4096 + xbytes ? g_smem_optin - 4096 - xbytes : 0;
+            const int ns = (int)std::min<size_t>(4, room / per_stage);
+            if (ns >= 2) {
+                void* fn = bf ? pick_tma<bf16>(nb, two ? 2 : 1) : pick_tma<float>(nb, two ? 2 : 1);
+                int nsv = ns;
+                void* args[] = {&p, &nsv};
+                return launch_ex(ctx, fn, dim3(ctx->sms), dim3(kTmaThreads),
+                                 (size_t)kTmaWarps * ns * kStageBytes + xbytes + (size_t)kTmaWarps * ns * 8, args);
+            }
+        }
         void* fn = bf ? pick_stream<bf16>(nb, two ? 2 : 1, rows) : pick_stream<float>(nb, two ? 2 : 1, rows);
         void* args[] = {&p};
-        return launch_ex(ctx, fn, dim3(ctx->sms), dim3(kStreamThreads), (size_t)nb * p.K * 4, args);
+        // staged input, then (row kernel) the RMSNorm gains in their storage type
+        const size_t smem = xbytes + (rows ? (size_t)p.K * ctx->esz + 16 : 0);
+        return launch_ex(ctx, fn, dim3(ctx->sms), dim3(kStreamThreads), smem, args);
     }
     int nb = next_pow2_le8(std::max(1, p.B));
     while (nb > 1 && (size_t)nb * p.K * 4 > kXsBudget) nb >>= 1;
@@ -307,6 +380,13 @@ int resadd_splits(pipo_ctx* ctx, int N, int K) {
     int s = (int)std::max(1LL, (target + N - 1) / N);
     s = std::min(s, std::max(1, K / 256));
     return s;
+}
+
+// splits per (sequence, kv head) of the step kernel: one unit per CTA
+int mk_attn_splits(const pipo_ctx* ctx, int B) {
+    const pipo_config& c = ctx->cfg;
+    int s = (ctx->sms + B * c.n_kv_heads - 1) / (B * c.n_kv_heads);
+    return std::max(1, std::min(s, (c.max_ctx + 15) / 16));
 }
 
 int attn_splits(const pipo_ctx* ctx, int B) {
@@ -384,7 +464,24 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
     p.K = H;
     TRY(launch_gemv(ctx, p));
     KVView kv = kv_view(ctx, cache_layer);
-    if (!ctx->attn_v0) {
+    if (ctx->rec) {
+        Phase ph{};
+        ph.type = PH_ATTN;
+        AttnPhase& a = ph.a;
+        a.qkv = ctx->qkv;
+        a.ld_qkv = rows;
+        a.kv = kv;
+        a.n_pos = ctx->n_pos;
+        a.rope = ctx->rope;
+        a.out = ctx->attn;
+        a.scale = 1.0f / sqrtf((float)DH);
+        a.part_o = ctx->part_o;
+        a.part_ml = ctx->part_ml;
+        a.counters = ctx->counters;
+        a.S = mk_attn_splits(ctx, ctx->B);
+        a.B = ctx->B;
+        ctx->rec->push_back(ph);
+    } else if (!ctx->attn_v0) {
         // RoPE + KV append + split-KV attention, one cluster per (sequence, kv head)
         AttnParams ap;
         ap.qkv = ctx->qkv;
@@ -524,6 +621,22 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
         st.dbg_conf = ctx->dbg_conf; st.dbg_hb = ctx->dbg_hb; st.dbg_hd = ctx->dbg_hd;
         st.dbg_xb = ctx->dbg_xb; st.dbg_xd = ctx->dbg_xd;
     }
+    if (ctx->rec) {
+        Phase ph{};
+        ph.type = PH_ACCEPT;
+        AcceptPhase& a = ph.c;
+        a.t = ctx->t;
+        a.W2 = ctx->conf_W2;
+        a.H = H;
+        a.tau = c.tau;
+        a.force = c.force_mode;
+        a.st = st;
+        a.hb = ctx->x;
+        a.hd = ctx->x2;
+        a.B = B;
+        ctx->rec->push_back(ph);
+        return PIPO_OK;
+    }
     {
         const float* tp = ctx->t;
         const void* w2 = ctx->conf_W2;
@@ -543,9 +656,101 @@ void drop_graph(pipo_ctx* ctx) {
     ctx->graph_B = -1;
 }
 
+template <typename T, int NB, int DH, int G>
+void* mk_fn() { return reinterpret_cast<void*>(&step_kernel<T, NB, DH, G>); }
+
+void* mk_pick(bool bf, int nb, int DH, int G) {
+    if (bf && DH == 128 && G == 4) return nb == 1 ? mk_fn<bf16, 1, 128, 4>() : nb == 2 ? mk_fn<bf16, 2, 128, 4>() : mk_fn<bf16, 4, 128, 4>();
+    if (!bf && DH == 64 && G == 2) return nb == 1 ? mk_fn<float, 1, 64, 2>() : nb == 2 ? mk_fn<float, 2, 64, 2>() : mk_fn<float, 4, 64, 2>();
+    return nullptr;
+}
+
+// Record the decode step as phases; when they all fit, upload them and capture
+// (or prepare) the persistent step kernel.  Returns false when it does not fit.
+pipo_status try_step_kernel(pipo_ctx* ctx, bool& used) {
+    used = false;
+    if (!ctx->use_mk || ctx->B > 4) return PIPO_OK;
+    const pipo_config& c = ctx->cfg;
+    const int nb = ctx->B <= 1 ? 1 : ctx->B <= 2 ? 2 : 4;
+    void* fn = mk_pick(c.dtype == 1, nb, c.head_dim, c.n_q_heads / c.n_kv_heads);
+    if (!fn) { ctx->mk_note = "(no step-kernel instance for this head shape)"; return PIPO_OK; }
+    std::vector<Phase> phases;
+    ctx->rec = &phases;
+    ctx->rec_ok = true;
+    ctx->rec_kmax = 0;
+    pipo_status s = enqueue_position(ctx, DECODE, 0);
+    ctx->rec = nullptr;
+    if (s != PIPO_OK) return s;
+    if (!ctx->rec_ok) { ctx->mk_note = "(a projection row is not a whole number of 512-byte chunks)"; return PIPO_OK; }
+    // attention: warp partials [NW][G][DH] + (m, l), and the split merge [G][S][DH + 2]
+    const int G = c.n_q_heads / c.n_kv_heads;
+    const size_t attn_bytes = std::max((size_t)(2 * kMkWarps * G + kMkWarps * G * c.head_dim),
+                                       (size_t)G * mk_attn_splits(ctx, ctx->B) * (c.head_dim + 2)) * 4;
+    const size_t stage_bytes = std::max((size_t)nb * ctx->rec_kmax * 4, attn_bytes);
+    const size_t smem = mk_stage_offset() + stage_bytes;
+    if (allow_max_smem(fn) < smem) { ctx->mk_note = "(shared memory)"; return PIPO_OK; }
+    int per_sm = 0;
+    CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kMkThreads, smem));
+    if (per_sm < 1) { ctx->mk_note = "(occupancy)"; return PIPO_OK; }
+    if (phases.size() > ctx->d_phases_cap) {
+        if (ctx->d_phases) {
+            cudaFree(ctx->d_phases);
+            ctx->allocs.erase(std::find(ctx->allocs.begin(), ctx->allocs.end(), (void*)ctx->d_phases));
+        }
+        ctx->d_phases = nullptr;
+        TRY(dalloc(ctx, &ctx->d_phases, phases.size() * sizeof(Phase)));
+        ctx->d_phases_cap = phases.size();
+    }
+    CK(cudaMemcpy(ctx->d_phases, phases.data(), phases.size() * sizeof(Phase), cudaMemcpyHostToDevice));
+    // capture: zero the barrier counter, then one cooperative launch
+    cudaGraph_t g = nullptr;
+    CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
+    cudaError_t e = cudaMemsetAsync(ctx->bar_ctr, 0, sizeof(unsigned), ctx->stream);
+    if (e == cudaSuccess) {
+        const Phase* ph = ctx->d_phases;
+        int nph = (int)phases.size();
+        unsigned* bc = ctx->bar_ctr;
+        void* args[] = {(void*)&ph, &nph, &bc};
+        cudaLaunchConfig_t lc = {};
+        lc.gridDim = dim3(ctx->sms);
+        lc.blockDim = dim3(kMkThreads);
+        lc.dynamicSmemBytes = smem;
+        lc.stream = ctx->stream;
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeCooperative;
+        at[0].val.cooperative = 1;
+        lc.attrs = at;
+        lc.numAttrs = 1;
+        e = cudaLaunchKernelExC(&lc, fn, args);
+    }
+    cudaError_t e2 = cudaStreamEndCapture(ctx->stream, &g);
+    if (e == cudaSuccess && e2 == cudaSuccess) e = cudaGraphInstantiate(&ctx->graph, g, 0);
+    if (g) cudaGraphDestroy(g);
+    if (e != cudaSuccess || e2 != cudaSuccess) {
+        // not capturable here: keep the multi-kernel graph for this context
+        ctx->mk_note = std::string("step kernel unavailable: ") + cudaGetErrorString(e != cudaSuccess ? e : e2);
+        cudaGetLastError();
+        ctx->graph = nullptr;
+        ctx->use_mk = false;
+        return PIPO_OK;
+    }
+    ctx->graph_B = ctx->B;
+    ctx->launches = 1;
+    ctx->mk_active = true;
+    used = true;
+    return PIPO_OK;
+}
+
 pipo_status ensure_graph(pipo_ctx* ctx) {
     if (ctx->graph && ctx->graph_B == ctx->B) return PIPO_OK;
     drop_graph(ctx);
+    ctx->mk_active = false;
+    bool used = false;
+    TRY(try_step_kernel(ctx, used));
+    if (getenv("PIPO_VERBOSE"))
+        fprintf(stderr, "pipo: decode step = %s %s\n", used ? "persistent step kernel" : "kernel graph",
+                ctx->mk_note.c_str());
+    if (used) return PIPO_OK;
     cudaGraph_t g = nullptr;
     CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
     ctx->launches = 0;
@@ -598,6 +803,16 @@ pipo_status ensure_cache_tmp(pipo_ctx* ctx, size_t elems) {
     TRY(dalloc(ctx, &ctx->cache_tmp, elems * sizeof(float)));
     ctx->cache_tmp_elems = elems;
     return PIPO_OK;
+}
+
+// Read and clear the device error word (bounded waits that gave up).
+pipo_status check_device_error(pipo_ctx* ctx) {
+    unsigned e = 0;
+    CK(cudaMemcpyFromSymbol(&e, g_pipo_error, sizeof(e)));
+    if (!e) return PIPO_OK;
+    const unsigned zero = 0;
+    CK(cudaMemcpyToSymbol(g_pipo_error, &zero, sizeof(zero)));
+    return fail(ctx, PIPO_ECUDA, "device wait timed out (code %u): results of this step are invalid", e);
 }
 
 }  // namespace
@@ -703,6 +918,10 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
             CK(cudaMemcpy(ctx->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice));
         }
         if (const char* ev = getenv("PIPO_ATTN_V0")) ctx->attn_v0 = ev[0] == '1';
+        if (const char* ev = getenv("PIPO_GEMV_TMA")) ctx->gemv_tma = ev[0] == '1';
+        if (const char* ev = getenv("PIPO_STEP_KERNEL")) ctx->use_mk = ev[0] == '1';
+        TRY(dalloc(ctx, &ctx->bar_ctr, 64));
+        CK(cudaMemset(ctx->bar_ctr, 0, 64));
 
         // activations and state
         const int qd = c.n_q_heads * DH, kd = c.n_kv_heads * DH;
@@ -848,7 +1067,7 @@ pipo_status pipo_decode_step(pipo_ctx* ctx, int32_t* h_tokens, int32_t* h_n_acce
     if (h_tokens) CK(cudaMemcpyAsync(h_tokens, ctx->out_tokens, (size_t)ctx->B * 8, cudaMemcpyDeviceToHost, ctx->stream));
     if (h_n_accepted) CK(cudaMemcpyAsync(h_n_accepted, ctx->out_nacc, (size_t)ctx->B * 4, cudaMemcpyDeviceToHost, ctx->stream));
     CK(cudaStreamSynchronize(ctx->stream));
-    return PIPO_OK;
+    return check_device_error(ctx);
 }
 
 pipo_status pipo_rollback(pipo_ctx* ctx, const int32_t* h_n_pairs) {
@@ -884,7 +1103,7 @@ pipo_status pipo_get_counters(pipo_ctx* ctx, int32_t* h_kv_len, int64_t* h_emitt
     if (h_kv_len) CK(cudaMemcpyAsync(h_kv_len, ctx->n_pos, (size_t)ctx->B * 4, cudaMemcpyDeviceToHost, ctx->stream));
     if (h_emitted) CK(cudaMemcpyAsync(h_emitted, ctx->emitted, (size_t)ctx->B * 8, cudaMemcpyDeviceToHost, ctx->stream));
     CK(cudaStreamSynchronize(ctx->stream));
-    return PIPO_OK;
+    return check_device_error(ctx);
 }
 
 pipo_status pipo_debug_dump(pipo_ctx* ctx, const pipo_debug* o) {
@@ -942,9 +1161,9 @@ pipo_status pipo_load_cache(pipo_ctx* ctx, int32_t b, int32_t n, const float* h_
     return PIPO_OK;
 }
 
-pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N, int32_t K, const float* d_x,
-                         int32_t B, float* d_y, void* stream) {
-    static thread_local pipo_ctx op;  // device facts and launch settings only; owns no memory
+namespace {
+pipo_status op_gemv_impl(pipo_ctx& op, int32_t dtype, int32_t mode, const void* d_W, int32_t N, int32_t K,
+                         const float* d_x, int32_t B, float* d_y, void* stream) {
     pipo_ctx* ctx = &op;
     if (!d_W || !d_x || !d_y || N < 1 || K < 8 || K % 8 || B < 1 || (dtype != 0 && dtype != 1) ||
         (mode != 0 && mode != 1))
@@ -960,6 +1179,8 @@ pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N
     }
     op.stream = static_cast<cudaStream_t>(stream);
     op.pdl = false;
+    op.gemv_tma = false;
+    if (const char* ev = getenv("PIPO_GEMV_TMA")) op.gemv_tma = ev[0] == '1';
     GemvParams p{};
     p.W = d_W;
     p.N = N;
@@ -971,7 +1192,14 @@ pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N
     p.splitk = 1;
     p.nseg = 1;
     p.seg[0] = act_seg(d_x, K, K);
-    pipo_status st = launch_gemv(ctx, p);
+    return launch_gemv(ctx, p);
+}
+}  // namespace
+
+pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N, int32_t K, const float* d_x,
+                         int32_t B, float* d_y, void* stream) {
+    static thread_local pipo_ctx op;  // device facts and launch settings only; owns no memory
+    const pipo_status st = op_gemv_impl(op, dtype, mode, d_W, N, K, d_x, B, d_y, stream);
     if (st != PIPO_OK) g_init_error = op.err;
     return st;
 }

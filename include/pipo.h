@@ -195,6 +195,16 @@ PIPO_API pipo_status pipo_set_stream(pipo_ctx *ctx, void *stream);
 PIPO_API pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void *d_W, int32_t N, int32_t K,
                                   const float *d_x, int32_t B, float *d_y, void *stream);
 
+/* Kernel timing of one decode step run eagerly (no graph) on the context
+ * stream, with CUDA events recorded around every launch.  For launch i in step
+ * order: h_kind[i] (0 weight-streaming GEMV, 1 attention, 2 other), h_bytes[i]
+ * the algorithmic bytes it must move (weights it streams; for attention the
+ * KV entries it reads plus the one it writes), h_ms[i] its event-timed
+ * duration.  *h_n receives the launch count (at most cap are written).
+ * Advances the decode state exactly like pipo_decode_step. */
+PIPO_API pipo_status pipo_profile_step(pipo_ctx *ctx, int32_t cap, int32_t *h_kind, double *h_bytes, float *h_ms,
+                                       int32_t *h_n);
+
 /* Number of kernel launches one decode step enqueues (for launch accounting). */
 PIPO_API int32_t pipo_step_launches(const pipo_ctx *ctx);
 

@@ -83,6 +83,7 @@ SIGNATURES = {
     "pipo_set_stream": (C.c_int, [C.c_void_p, C.c_void_p]),
     "pipo_op_gemv": (C.c_int, [C.c_int32, C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_int32,
                                C.c_void_p, C.c_void_p]),
+    "pipo_profile_step": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.POINTER(C.c_double), _FP, _IP]),
     "pipo_step_launches": (C.c_int32, [C.c_void_p]),
     "pipo_last_error": (C.c_char_p, [C.c_void_p]),
     "pipo_free": (None, [C.c_void_p]),
@@ -206,6 +207,18 @@ def pipo_op_gemv(dtype: int, mode: int, W: int, N: int, K: int, x: int, B: int, 
                                C.c_void_p(stream or None)), None)
 
 
+def pipo_profile_step(ctx, cap: int = 4096):
+    """Per-launch (kind, algorithmic bytes, ms) of one eagerly run decode step."""
+    kind = np.zeros(cap, np.int32)
+    by = np.zeros(cap, np.float64)
+    ms = np.zeros(cap, np.float32)
+    n = np.zeros(1, np.int32)
+    _check(load().pipo_profile_step(ctx, cap, _ip(kind), by.ctypes.data_as(C.POINTER(C.c_double)), _fp(ms), _ip(n)),
+           ctx)
+    k = int(min(n[0], cap))
+    return kind[:k], by[:k], ms[:k]
+
+
 def pipo_step_launches(ctx) -> int:
     return int(load().pipo_step_launches(ctx))
 
@@ -308,3 +321,6 @@ class Pipo:
 
     def launches(self) -> int:
         return pipo_step_launches(self.ctx)
+
+    def profile_step(self):
+        return pipo_profile_step(self.ctx)

@@ -91,6 +91,14 @@ struct pipo_ctx {
     size_t d_phases_cap = 0;
     unsigned* bar_ctr = nullptr;
     std::string mk_note;
+    // per-launch timing (pipo_profile_step): events around every launch
+    bool prof = false;
+    int prof_kind = 2;
+    double prof_bytes = 0.0;
+    std::vector<cudaEvent_t> prof_ev;
+    std::vector<int> prof_k;
+    std::vector<double> prof_b;
+    size_t prof_n = 0;
 
     int B = 0;
     bool prefilled = false;
@@ -227,7 +235,23 @@ pipo_status launch_ex(pipo_ctx* ctx, const void* fn, dim3 grid, dim3 block, size
     }
     lc.attrs = at;
     lc.numAttrs = na;
+    if (ctx->prof) {
+        while (ctx->prof_ev.size() < 2 * (ctx->prof_n + 1)) {
+            cudaEvent_t e;
+            CK(cudaEventCreate(&e));
+            ctx->prof_ev.push_back(e);
+        }
+        CK(cudaEventRecord(ctx->prof_ev[2 * ctx->prof_n], ctx->stream));
+    }
     CK(cudaLaunchKernelExC(&lc, fn, args));
+    if (ctx->prof) {
+        CK(cudaEventRecord(ctx->prof_ev[2 * ctx->prof_n + 1], ctx->stream));
+        ctx->prof_k.push_back(ctx->prof_kind);
+        ctx->prof_b.push_back(ctx->prof_bytes);
+        ctx->prof_n++;
+        ctx->prof_kind = 2;
+        ctx->prof_bytes = 0.0;
+    }
     ctx->launches++;
     return PIPO_OK;
 }
@@ -314,6 +338,8 @@ pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
         ctx->rec->push_back(ph);
         return PIPO_OK;
     }
+    ctx->prof_kind = 0;
+    ctx->prof_bytes = (double)p.N * (two ? 2 : 1) * p.K * ctx->esz;
     if (p.B <= 4) {
         // streaming kernel: one CTA per SM, chunk-balanced, deterministic
         int nb = std::min(4, next_pow2_le8(std::max(1, p.B)));
@@ -483,6 +509,10 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         ctx->rec->push_back(ph);
     } else if (!ctx->attn_v0) {
         // RoPE + KV append + split-KV attention, one cluster per (sequence, kv head)
+        ctx->prof_kind = 1;
+        ctx->prof_bytes = 0.0;
+        for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b)
+            ctx->prof_bytes += (double)(ctx->h_len[b] + 2) * kd * 2 * ctx->esz;
         AttnParams ap;
         ap.qkv = ctx->qkv;
         ap.ld_qkv = rows;
@@ -829,6 +859,7 @@ void pipo_free(pipo_ctx* ctx) {
     cudaSetDevice(ctx->dev);
     if (ctx->stream) cudaStreamSynchronize(ctx->stream);
     drop_graph(ctx);
+    for (cudaEvent_t e : ctx->prof_ev) cudaEventDestroy(e);
     for (void* p : ctx->allocs) cudaFree(p);
     if (ctx->own_stream) cudaStreamDestroy(ctx->own_stream);
     delete ctx;
@@ -1202,6 +1233,40 @@ pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N
     const pipo_status st = op_gemv_impl(op, dtype, mode, d_W, N, K, d_x, B, d_y, stream);
     if (st != PIPO_OK) g_init_error = op.err;
     return st;
+}
+
+pipo_status pipo_profile_step(pipo_ctx* ctx, int32_t cap, int32_t* h_kind, double* h_bytes, float* h_ms,
+                              int32_t* h_n) {
+    if (!ctx || !h_n || cap < 0) return fail(ctx, PIPO_EINVAL, "null argument");
+    if (!ctx->prefilled) return fail(ctx, PIPO_ESTATE, "profile step before prefill");
+    for (int b = 0; b < ctx->B; ++b)
+        if (ctx->h_len[b] + 1 > ctx->cfg.max_ctx)
+            return fail(ctx, PIPO_ECAPACITY, "sequence %d: KV cache full (%d entries)", b, ctx->h_len[b]);
+    CK(cudaSetDevice(ctx->dev));
+    CK(cudaStreamSynchronize(ctx->stream));
+    ctx->prof = true;
+    ctx->prof_n = 0;
+    ctx->prof_k.clear();
+    ctx->prof_b.clear();
+    const int saved = ctx->launches;
+    const bool pdl = ctx->pdl;
+    ctx->pdl = false;
+    pipo_status s = enqueue_position(ctx, DECODE, 0);
+    ctx->pdl = pdl;
+    ctx->prof = false;
+    ctx->launches = saved;
+    if (s != PIPO_OK) return s;
+    CK(cudaStreamSynchronize(ctx->stream));
+    for (int b = 0; b < ctx->B; ++b) ctx->h_len[b] += 1;
+    *h_n = (int32_t)ctx->prof_n;
+    for (size_t i = 0; i < ctx->prof_n && (int)i < cap; ++i) {
+        float ms = 0.f;
+        CK(cudaEventElapsedTime(&ms, ctx->prof_ev[2 * i], ctx->prof_ev[2 * i + 1]));
+        if (h_kind) h_kind[i] = ctx->prof_k[i];
+        if (h_bytes) h_bytes[i] = ctx->prof_b[i];
+        if (h_ms) h_ms[i] = ms;
+    }
+    return check_device_error(ctx);
 }
 
 }  // extern "C"

@@ -1,7 +1,7 @@
 // Split-KV GQA flash-decode over the paged pair-KV cache, one thread-block
 // cluster per (sequence, kv head) (sm_103a).
 //
-// Grid (CS, n_kv, B), cluster (CS, 1, 1), 128 threads.  CTA s of the cluster
+// Grid (CS, n_kv, B), cluster (CS, 1, 1), 256 threads.  CTA s of the cluster
 // attends the G = n_q/n_kv query heads of its kv head over a contiguous slice
 // of entries 0..n (n = entries before this step; entry n is this step's new
 // key/value).  Fused in:
@@ -84,12 +84,15 @@ __device__ __forceinline__ void rope8(float (&x)[8], int li, int pos, const floa
     }
 }
 
+constexpr int kAttnWarps = 8;
+constexpr int kAttnThreads = kAttnWarps * 32;
+
 template <typename T, int DH, int G, int CS>
-__global__ void __launch_bounds__(128) attn_cluster_kernel(AttnParams p) {
+__global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p) {
     constexpr int LPE = DH / 8;        // lanes per entry
     constexpr int EPW = 32 / LPE;      // entries per warp step
     constexpr int kU = 4;              // warp steps in flight
-    constexpr int NW = 4;
+    constexpr int NW = kAttnWarps;
     constexpr int STEP = NW * EPW;     // entries per CTA step
     __shared__ float sm_o[G][DH];
     __shared__ float sm_m[G], sm_l[G];

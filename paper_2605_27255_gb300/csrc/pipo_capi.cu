@@ -78,7 +78,7 @@ struct pipo_ctx {
 
     float* rope = nullptr;            // [max_ctx][d_h/2][2] cos, sin
     bool pdl = false;                 // programmatic dependent launch (decode graph only)
-    int attn_cs = 8;                  // cluster size of the attention kernel
+    bool attn_cs16 = false;           // 16-CTA attention clusters available
     bool attn_v0 = false;             // (development) the unclustered attention path
     bool gemv_tma = false;            // bulk-copy GEMV (else the register-ring GEMV)
     // persistent step kernel: phases recorded from the enqueue code
@@ -445,21 +445,54 @@ void* attn_pick(bool bf, int DH, int G) {
 template <typename T, int DH, int G, int CS>
 void* attnc_fn() { return reinterpret_cast<void*>(&attn_cluster_kernel<T, DH, G, CS>); }
 
-template <typename T, int DH>
+template <typename T, int DH, int CS>
 void* attnc_pick_g(int G) {
     switch (G) {
-        case 1: return attnc_fn<T, DH, 1, 8>();
-        case 2: return attnc_fn<T, DH, 2, 8>();
-        case 4: return attnc_fn<T, DH, 4, 8>();
-        case 8: return attnc_fn<T, DH, 8, 8>();
+        case 1: return attnc_fn<T, DH, 1, CS>();
+        case 2: return attnc_fn<T, DH, 2, CS>();
+        case 4: return attnc_fn<T, DH, 4, CS>();
+        case 8: return attnc_fn<T, DH, 8, CS>();
         default: return nullptr;
     }
 }
 
-void* attnc_pick(bool bf, int DH, int G) {
-    if (DH == 64) return bf ? attnc_pick_g<bf16, 64>(G) : attnc_pick_g<float, 64>(G);
-    if (DH == 128) return bf ? attnc_pick_g<bf16, 128>(G) : attnc_pick_g<float, 128>(G);
+// cs: cluster size, 8 (portable) or 16 (non-portable, small batches)
+void* attnc_pick(bool bf, int DH, int G, int cs) {
+    if (cs == 16) {
+        if (DH == 64) return bf ? attnc_pick_g<bf16, 64, 16>(G) : attnc_pick_g<float, 64, 16>(G);
+        if (DH == 128) return bf ? attnc_pick_g<bf16, 128, 16>(G) : attnc_pick_g<float, 128, 16>(G);
+        return nullptr;
+    }
+    if (DH == 64) return bf ? attnc_pick_g<bf16, 64, 8>(G) : attnc_pick_g<float, 64, 8>(G);
+    if (DH == 128) return bf ? attnc_pick_g<bf16, 128, 8>(G) : attnc_pick_g<float, 128, 8>(G);
     return nullptr;
+}
+
+// Can a 16-CTA cluster of this kernel be scheduled here?  (sets the
+// non-portable cluster attribute; any failure selects 8)
+bool cluster16_ok(bool bf, int DH, int G) {
+    void* fn = attnc_pick(bf, DH, G, 16);
+    if (!fn) return false;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(16, 1, 1);
+    lc.blockDim = dim3(kAttnThreads);
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 16;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    lc.attrs = at;
+    lc.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, fn, &lc) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return n > 0;
 }
 
 void* rope_pick(bool bf, int DH) {
@@ -522,8 +555,10 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         ap.out = ctx->attn;
         ap.scale = 1.0f / sqrtf((float)DH);
         void* args[] = {&ap};
-        TRY(launch_ex(ctx, attnc_pick(bf, DH, c.n_q_heads / c.n_kv_heads), dim3(ctx->attn_cs, c.n_kv_heads, ctx->B),
-                      dim3(128), 0, args, ctx->attn_cs));
+        // 16-CTA clusters when the batch leaves most SMs idle with 8
+        const int cs = (ctx->attn_cs16 && ctx->B * c.n_kv_heads * 16 <= 2 * ctx->sms) ? 16 : 8;
+        TRY(launch_ex(ctx, attnc_pick(bf, DH, c.n_q_heads / c.n_kv_heads, cs), dim3(cs, c.n_kv_heads, ctx->B),
+                      dim3(kAttnThreads), 0, args, cs));
     } else {
     // RoPE + KV append
     {
@@ -949,6 +984,8 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
             CK(cudaMemcpy(ctx->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice));
         }
         if (const char* ev = getenv("PIPO_ATTN_V0")) ctx->attn_v0 = ev[0] == '1';
+        ctx->attn_cs16 = cluster16_ok(c.dtype == 1, c.head_dim, c.n_q_heads / c.n_kv_heads);
+        if (const char* ev = getenv("PIPO_ATTN_CS16")) ctx->attn_cs16 = ctx->attn_cs16 && ev[0] == '1';
         if (const char* ev = getenv("PIPO_GEMV_TMA")) ctx->gemv_tma = ev[0] == '1';
         if (const char* ev = getenv("PIPO_STEP_KERNEL")) ctx->use_mk = ev[0] == '1';
         TRY(dalloc(ctx, &ctx->bar_ctr, 64));

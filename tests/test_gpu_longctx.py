@@ -1,0 +1,46 @@
+"""Long-context parity: caches filled with 1500 seeded entries (many 64-entry
+pages per attention split) on both sides, then forced-replay decode steps;
+the split-KV attention with 8- and 16-CTA clusters against the oracle."""
+import os
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2605_27255_gb300 import capi, synth
+from parity_util import Stats, compare, tol_for
+
+pytestmark = pytest.mark.gpu
+
+MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003,
+                       compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1e6, tau=0.5)
+
+
+@pytest.mark.parametrize("cs16", ["1", "0"])
+def test_long_context_forced_replay(cs16, monkeypatch):
+    monkeypatch.setenv("PIPO_ATTN_CS16", cs16)
+    s = MID
+    n_ctx, B, steps = 1500, 2, 3
+    w = synth.gen_weights(s, seed=8)
+    K, V = synth.gen_kv_fill(s, n_ctx, seed=9)
+    K, V = K.numpy(), V.numpy()
+    prompts = synth.gen_prompts(B, 4, s.V, seed=4).numpy()
+    gpu = capi.Pipo(s, w, max_batch=B, max_ctx=n_ctx + steps + 2, debug=True, page_shuffle_seed=3)
+    orc = O.State(O.Model(s, w, max_ctx=n_ctx + steps + 2), B)
+    try:
+        tok, _ = gpu.prefill(prompts)
+        orc.prefill(prompts, tau=s.tau)
+        for b in range(B):
+            gpu.load_cache(b, K, V)
+            orc.set_cache(b, K, V)
+        st = Stats()
+        for i in range(steps):
+            pend = [[orc.seq(b)["p0"], orc.seq(b)["p1"]] for b in range(B)]
+            gpu.set_pending(pend)
+            tok, nacc = gpu.step()
+            o = orc.step(tau=s.tau)
+            compare(s, s.tau, o, gpu.debug(), tok, nacc, 0, st, tol_for(s), f"step {i}")
+        n, _ = gpu.counters()
+        assert list(n) == [n_ctx + steps] * B
+    finally:
+        gpu.close()

@@ -195,6 +195,18 @@ PIPO_API pipo_status pipo_set_stream(pipo_ctx *ctx, void *stream);
 PIPO_API pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void *d_W, int32_t N, int32_t K,
                                   const float *d_x, int32_t B, float *d_y, void *stream);
 
+/* Fused LM head + argmax over the tied embedding (Eq. 3 and Eq. 5, App. B.2):
+ *   d_tokens[b] = argmax_v  E[v,:] . RMSNorm(h[b,:]; gamma)
+ * with the lowest v winning ties; the logits are never stored unless
+ * d_logits [B, V] fp32 is given.  dtype 0: E and gamma fp32, 1: bf16;
+ * E [V, H]; d_h [B, H] fp32; d_gamma [H] or NULL (no norm); eps inside the
+ * root.  d_scratch: at least 8*B bytes of 8-byte-aligned device memory for the
+ * packed (logit, row) keys, overwritten (contents unspecified on return).
+ * Enqueued on `stream`.  EINVAL for bad shapes or a short scratch buffer. */
+PIPO_API pipo_status pipo_op_lm_head_argmax(int32_t dtype, const void *d_E, int32_t V, int32_t H, const float *d_h,
+                                            const void *d_gamma, float eps, int32_t B, int32_t *d_tokens,
+                                            float *d_logits, void *d_scratch, size_t scratch_bytes, void *stream);
+
 /* Kernel timing of one decode step run eagerly (no graph) on the context
  * stream, with CUDA events recorded around every launch.  For launch i in step
  * order: h_kind[i] (0 weight-streaming GEMV, 1 attention, 2 other), h_bytes[i]

@@ -83,6 +83,9 @@ SIGNATURES = {
     "pipo_set_stream": (C.c_int, [C.c_void_p, C.c_void_p]),
     "pipo_op_gemv": (C.c_int, [C.c_int32, C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_int32,
                                C.c_void_p, C.c_void_p]),
+    "pipo_op_lm_head_argmax": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
+                                         C.c_float, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
+                                         C.c_void_p]),
     "pipo_profile_step": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.POINTER(C.c_double), _FP, _IP]),
     "pipo_step_launches": (C.c_int32, [C.c_void_p]),
     "pipo_last_error": (C.c_char_p, [C.c_void_p]),
@@ -205,6 +208,15 @@ def pipo_op_gemv(dtype: int, mode: int, W: int, N: int, K: int, x: int, B: int, 
     """Device pointers (ints); see include/pipo.h."""
     _check(load().pipo_op_gemv(dtype, mode, C.c_void_p(W), N, K, C.c_void_p(x), B, C.c_void_p(y),
                                C.c_void_p(stream or None)), None)
+
+
+def pipo_op_lm_head_argmax(dtype: int, E: int, V: int, H: int, h: int, gamma: int, eps: float, B: int,
+                           tokens: int, logits: int, scratch: int, scratch_bytes: int, stream: int = 0) -> None:
+    """Device pointers (ints; 0 = NULL); see include/pipo.h."""
+    _check(load().pipo_op_lm_head_argmax(dtype, C.c_void_p(E), V, H, C.c_void_p(h), C.c_void_p(gamma or None),
+                                         float(eps), B, C.c_void_p(tokens), C.c_void_p(logits or None),
+                                         C.c_void_p(scratch or None), scratch_bytes, C.c_void_p(stream or None)),
+           None)
 
 
 def pipo_profile_step(ctx, cap: int = 4096):

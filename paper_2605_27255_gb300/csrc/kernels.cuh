@@ -538,6 +538,12 @@ __global__ void accept_kernel(const float* __restrict__ t, const void* W2, int H
     if (st.dbg_xb) { st.dbg_xb[b] = xb; st.dbg_xd[b] = xd; }
 }
 
+// Packed argmax keys -> token ids.
+__global__ void keys_to_tokens_kernel(const unsigned long long* keys, int32_t* tokens, int B) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b < B) tokens[b] = argmax_row(keys[b]);
+}
+
 // Prefill positions before the last: n[b] += 1.
 __global__ void advance_kernel(int32_t* n_pos, int B) {
     pdl_launch();

@@ -984,8 +984,9 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
             CK(cudaMemcpy(ctx->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice));
         }
         if (const char* ev = getenv("PIPO_ATTN_V0")) ctx->attn_v0 = ev[0] == '1';
-        ctx->attn_cs16 = cluster16_ok(c.dtype == 1, c.head_dim, c.n_q_heads / c.n_kv_heads);
-        if (const char* ev = getenv("PIPO_ATTN_CS16")) ctx->attn_cs16 = ctx->attn_cs16 && ev[0] == '1';
+        // 16-CTA clusters measured slower than 8 at 4B B=1 (2.77 vs 2.55 ms per step): opt-in only
+        if (const char* ev = getenv("PIPO_ATTN_CS16"))
+            ctx->attn_cs16 = ev[0] == '1' && cluster16_ok(c.dtype == 1, c.head_dim, c.n_q_heads / c.n_kv_heads);
         if (const char* ev = getenv("PIPO_GEMV_TMA")) ctx->gemv_tma = ev[0] == '1';
         if (const char* ev = getenv("PIPO_STEP_KERNEL")) ctx->use_mk = ev[0] == '1';
         TRY(dalloc(ctx, &ctx->bar_ctr, 64));
@@ -1230,12 +1231,9 @@ pipo_status pipo_load_cache(pipo_ctx* ctx, int32_t b, int32_t n, const float* h_
 }
 
 namespace {
-pipo_status op_gemv_impl(pipo_ctx& op, int32_t dtype, int32_t mode, const void* d_W, int32_t N, int32_t K,
-                         const float* d_x, int32_t B, float* d_y, void* stream) {
+// launch settings of the kernel-level entry points (owns no memory)
+pipo_status op_setup(pipo_ctx& op, int32_t dtype, void* stream) {
     pipo_ctx* ctx = &op;
-    if (!d_W || !d_x || !d_y || N < 1 || K < 8 || K % 8 || B < 1 || (dtype != 0 && dtype != 1) ||
-        (mode != 0 && mode != 1))
-        return fail(nullptr, PIPO_EINVAL, "pipo_op_gemv: bad arguments");
     int dev = 0;
     CK(cudaGetDevice(&dev));
     if (op.sms == 0 || op.dev != dev || (int)op.esz != (dtype == 1 ? 2 : 4)) {
@@ -1249,6 +1247,41 @@ pipo_status op_gemv_impl(pipo_ctx& op, int32_t dtype, int32_t mode, const void* 
     op.pdl = false;
     op.gemv_tma = false;
     if (const char* ev = getenv("PIPO_GEMV_TMA")) op.gemv_tma = ev[0] == '1';
+    return PIPO_OK;
+}
+
+pipo_status op_lm_head_impl(pipo_ctx& op, int32_t dtype, const void* d_E, int32_t V, int32_t H, const float* d_h,
+                            const void* d_gamma, float eps, int32_t B, int32_t* d_tokens, float* d_logits,
+                            unsigned long long* keys, void* stream) {
+    pipo_ctx* ctx = &op;
+    TRY(op_setup(op, dtype, stream));
+    CK(cudaMemsetAsync(keys, 0, (size_t)B * 8, op.stream));
+    GemvParams p{};
+    p.W = d_E;
+    p.N = V;
+    p.K = H;
+    p.epi = EPI_ARGMAX;
+    p.am = keys;
+    p.dbg = d_logits;
+    p.ld_dbg = V;
+    p.B = B;
+    p.splitk = 1;
+    p.nseg = 1;
+    p.eps = eps;
+    p.seg[0] = act_seg(d_h, H, H, d_gamma);
+    TRY(launch_gemv(ctx, p));
+    keys_to_tokens_kernel<<<(B + 127) / 128, 128, 0, op.stream>>>(keys, d_tokens, B);
+    CK(cudaGetLastError());
+    return PIPO_OK;
+}
+
+pipo_status op_gemv_impl(pipo_ctx& op, int32_t dtype, int32_t mode, const void* d_W, int32_t N, int32_t K,
+                         const float* d_x, int32_t B, float* d_y, void* stream) {
+    pipo_ctx* ctx = &op;
+    if (!d_W || !d_x || !d_y || N < 1 || K < 8 || K % 8 || B < 1 || (dtype != 0 && dtype != 1) ||
+        (mode != 0 && mode != 1))
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_gemv: bad arguments");
+    TRY(op_setup(op, dtype, stream));
     GemvParams p{};
     p.W = d_W;
     p.N = N;
@@ -1263,6 +1296,22 @@ pipo_status op_gemv_impl(pipo_ctx& op, int32_t dtype, int32_t mode, const void* 
     return launch_gemv(ctx, p);
 }
 }  // namespace
+
+pipo_status pipo_op_lm_head_argmax(int32_t dtype, const void* d_E, int32_t V, int32_t H, const float* d_h,
+                                   const void* d_gamma, float eps, int32_t B, int32_t* d_tokens, float* d_logits,
+                                   void* d_scratch, size_t scratch_bytes, void* stream) {
+    if (!d_E || !d_h || !d_tokens || !d_scratch || V < 1 || H < 8 || H % 8 || B < 1 || (dtype != 0 && dtype != 1) ||
+        !(eps >= 0.f) || reinterpret_cast<uintptr_t>(d_scratch) % 8 != 0)
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_lm_head_argmax: bad arguments");
+    if (scratch_bytes < (size_t)B * 8)
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_lm_head_argmax: scratch needs %zu bytes, got %zu", (size_t)B * 8,
+                    scratch_bytes);
+    static thread_local pipo_ctx op;
+    const pipo_status st = op_lm_head_impl(op, dtype, d_E, V, H, d_h, d_gamma, eps, B, d_tokens, d_logits,
+                                           static_cast<unsigned long long*>(d_scratch), stream);
+    if (st != PIPO_OK) g_init_error = op.err;
+    return st;
+}
 
 pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N, int32_t K, const float* d_x,
                          int32_t B, float* d_y, void* stream) {

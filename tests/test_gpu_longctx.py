@@ -1,6 +1,7 @@
 """Long-context parity: caches filled with 1500 seeded entries (many 64-entry
 pages per attention split) on both sides, then forced-replay decode steps;
-the split-KV attention with 8- and 16-CTA clusters against the oracle."""
+the split-KV attention with 8-CTA clusters (default) and 16-CTA clusters
+(opt-in) against the oracle."""
 import os
 
 import numpy as np

@@ -207,6 +207,24 @@ PIPO_API pipo_status pipo_op_lm_head_argmax(int32_t dtype, const void *d_E, int3
                                             const void *d_gamma, float eps, int32_t B, int32_t *d_tokens,
                                             float *d_logits, void *d_scratch, size_t scratch_bytes, void *stream);
 
+/* The same fused LM head + argmax as pipo_op_lm_head_argmax, for callers
+ * that cannot allocate device memory: for example a host program that hands
+ * every byte of the GPU to its own pool at start-up and allows no other
+ * allocation, or a latency-critical loop in which a cudaMalloc (which can
+ * synchronize the device) is not acceptable.  The paper has no counterpart:
+ * it is a deployment variant of this library.  It allocates nothing; its
+ * scratch is a fixed array of 64 packed keys (512 bytes) that the library
+ * keeps in device memory on every GPU that loads it, for the life of the
+ * process.  Hence B <= 64 (EINVAL otherwise).  The first call on each device
+ * looks up that array's device address (cudaGetSymbolAddress) with the device
+ * current; make that first call before any stream capture.  Every call on a
+ * device shares the one array and zeroes it first, so calls that overlap on
+ * the GPU (other streams, or other host threads) race and must be
+ * serialized by the caller.  Arguments otherwise as pipo_op_lm_head_argmax. */
+PIPO_API pipo_status pipo_op_lm_head_argmax_noalloc(int32_t dtype, const void *d_E, int32_t V, int32_t H,
+                                                    const float *d_h, const void *d_gamma, float eps, int32_t B,
+                                                    int32_t *d_tokens, float *d_logits, void *stream);
+
 /* Kernel timing of one decode step run eagerly (no graph) on the context
  * stream, with CUDA events recorded around every launch.  For launch i in step
  * order: h_kind[i] (0 weight-streaming GEMV, 1 attention, 2 other), h_bytes[i]

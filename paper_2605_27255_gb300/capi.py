@@ -86,6 +86,9 @@ SIGNATURES = {
     "pipo_op_lm_head_argmax": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
                                          C.c_float, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
                                          C.c_void_p]),
+    "pipo_op_lm_head_argmax_noalloc": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p,
+                                                 C.c_void_p, C.c_float, C.c_int32, C.c_void_p, C.c_void_p,
+                                                 C.c_void_p]),
     "pipo_profile_step": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.POINTER(C.c_double), _FP, _IP]),
     "pipo_step_launches": (C.c_int32, [C.c_void_p]),
     "pipo_last_error": (C.c_char_p, [C.c_void_p]),
@@ -217,6 +220,16 @@ def pipo_op_lm_head_argmax(dtype: int, E: int, V: int, H: int, h: int, gamma: in
                                          float(eps), B, C.c_void_p(tokens), C.c_void_p(logits or None),
                                          C.c_void_p(scratch or None), scratch_bytes, C.c_void_p(stream or None)),
            None)
+
+
+def pipo_op_lm_head_argmax_noalloc(dtype: int, E: int, V: int, H: int, h: int, gamma: int, eps: float, B: int,
+                                   tokens: int, logits: int, stream: int = 0) -> None:
+    """The LM-head argmax for callers that cannot allocate device memory: no
+    scratch argument, at most 64 sequences, calls on one device must not
+    overlap (see include/pipo.h).  Device pointers are ints (0 = NULL)."""
+    _check(load().pipo_op_lm_head_argmax_noalloc(dtype, C.c_void_p(E), V, H, C.c_void_p(h),
+                                                 C.c_void_p(gamma or None), float(eps), B, C.c_void_p(tokens),
+                                                 C.c_void_p(logits or None), C.c_void_p(stream or None)), None)
 
 
 def pipo_profile_step(ctx, cap: int = 4096):

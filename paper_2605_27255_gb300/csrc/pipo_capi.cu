@@ -14,6 +14,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <map>
+#include <mutex>
 #include <numeric>
 #include <random>
 #include <string>
@@ -1309,6 +1310,54 @@ pipo_status pipo_op_lm_head_argmax(int32_t dtype, const void* d_E, int32_t V, in
     static thread_local pipo_ctx op;
     const pipo_status st = op_lm_head_impl(op, dtype, d_E, V, H, d_h, d_gamma, eps, B, d_tokens, d_logits,
                                            static_cast<unsigned long long*>(d_scratch), stream);
+    if (st != PIPO_OK) g_init_error = op.err;
+    return st;
+}
+
+}  // extern "C"
+
+// ---- LM-head argmax without caller scratch --------------------------------
+// For callers that may not allocate device memory.  The packed-key scratch is
+// this fixed array: 64 keys, kept on every device that loads the library.  In
+// host code its name is only a stand-in for the symbol, never a device
+// address: the address is looked up per device with cudaGetSymbolAddress.
+namespace {
+constexpr int kNoAllocMaxBatch = 64;
+constexpr int kNoAllocMaxDevices = 64;
+unsigned long long* g_noalloc_keys_addr[kNoAllocMaxDevices] = {};  // per device, set on first use
+std::mutex g_noalloc_mu;
+}  // namespace
+static __device__ __align__(256) unsigned long long g_lm_head_noalloc_keys[kNoAllocMaxBatch];
+
+extern "C" {
+
+pipo_status pipo_op_lm_head_argmax_noalloc(int32_t dtype, const void* d_E, int32_t V, int32_t H, const float* d_h,
+                                           const void* d_gamma, float eps, int32_t B, int32_t* d_tokens,
+                                           float* d_logits, void* stream) {
+    if (!d_E || !d_h || !d_tokens || V < 1 || H < 8 || H % 8 || B < 1 || (dtype != 0 && dtype != 1) || !(eps >= 0.f))
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_lm_head_argmax_noalloc: bad arguments");
+    if (B > kNoAllocMaxBatch)
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_lm_head_argmax_noalloc: %d sequences, at most %d", B,
+                    kNoAllocMaxBatch);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(nullptr, PIPO_ECUDA, "cudaGetDevice: %s", cudaGetErrorString(e));
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(nullptr, PIPO_EINVAL, "device ordinal %d unsupported", dev);
+    unsigned long long* keys = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_noalloc_mu);
+        if (!g_noalloc_keys_addr[dev]) {
+            // set-up, once per device, with that device current
+            void* addr = nullptr;
+            e = cudaGetSymbolAddress(&addr, g_lm_head_noalloc_keys);
+            if (e != cudaSuccess)
+                return fail(nullptr, PIPO_ECUDA, "cudaGetSymbolAddress(scratch): %s", cudaGetErrorString(e));
+            g_noalloc_keys_addr[dev] = static_cast<unsigned long long*>(addr);
+        }
+        keys = g_noalloc_keys_addr[dev];
+    }
+    static thread_local pipo_ctx op;
+    const pipo_status st = op_lm_head_impl(op, dtype, d_E, V, H, d_h, d_gamma, eps, B, d_tokens, d_logits, keys, stream);
     if (st != PIPO_OK) g_init_error = op.err;
     return st;
 }

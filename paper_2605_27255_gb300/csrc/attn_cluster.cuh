@@ -60,17 +60,25 @@ struct AttnParams {
     float scale;            // 1/sqrt(d_h)
 };
 
+// cos/sin of the 8 rotation pairs of lane slice li at position pos
+template <int DH>
+__device__ __forceinline__ void rope_load(float4 (&cs)[4], int li, int pos, const float* rope) {
+    constexpr int LPE = DH / 8;
+    const int i0 = (li % (LPE / 2)) * 8;  // pair index of dim e is i0 + e
+    const float4* t = reinterpret_cast<const float4*>(rope + ((size_t)pos * (DH / 2) + i0) * 2);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) cs[e] = t[e];
+}
+
 // rotate-half RoPE of the 8 dims [8*li, 8*li+8) of a d_h vector held as one
 // 8-dim slice per lane; partner lane holds the other half (li ^ (LPE/2)).
 template <int DH>
-__device__ __forceinline__ void rope8(float (&x)[8], int li, int pos, const float* rope) {
+__device__ __forceinline__ void rope8(float (&x)[8], int li, const float4 (&cs)[4]) {
     constexpr int LPE = DH / 8;
     float other[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) other[e] = __shfl_xor_sync(0xffffffffu, x[e], LPE / 2, LPE);
     const bool first = li < LPE / 2;
-    const int i0 = (li % (LPE / 2)) * 8;  // pair index of dim e is i0 + e
-    const float4* cs = reinterpret_cast<const float4*>(rope + ((size_t)pos * (DH / 2) + i0) * 2);
 #pragma unroll
     for (int e = 0; e < 8; e += 2) {
         const float4 t = cs[e / 2];  // cos(i0+e), sin(i0+e), cos(i0+e+1), sin(i0+e+1)
@@ -87,11 +95,15 @@ __device__ __forceinline__ void rope8(float (&x)[8], int li, int pos, const floa
 constexpr int kAttnWarps = 8;
 constexpr int kAttnThreads = kAttnWarps * 32;
 
+#ifndef PIPO_ATTN_KU
+#define PIPO_ATTN_KU 4
+#endif
+
 template <typename T, int DH, int G, int CS>
 __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p) {
     constexpr int LPE = DH / 8;        // lanes per entry
     constexpr int EPW = 32 / LPE;      // entries per warp step
-    constexpr int kU = 4;              // warp steps in flight
+    constexpr int kU = PIPO_ATTN_KU;   // warp steps in flight
     constexpr int NW = kAttnWarps;
     constexpr int STEP = NW * EPW;     // entries per CTA step
     __shared__ float sm_o[G][DH];
@@ -127,6 +139,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
         kr[u].load(Kb + off);
         vr[u].load(Vb + off);
     }
+    float4 rope_cs[4];  // rotation of position n (static table)
+    rope_load<DH>(rope_cs, li, n, p.rope);
     pdl_wait();
 
     // q of the G heads, 8 dims per lane, rotated, pre-scaled
@@ -138,7 +152,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
         const float4 a = qp[0], c = qp[1];
         q[hh][0] = a.x; q[hh][1] = a.y; q[hh][2] = a.z; q[hh][3] = a.w;
         q[hh][4] = c.x; q[hh][5] = c.y; q[hh][6] = c.z; q[hh][7] = c.w;
-        rope8<DH>(q[hh], li, n, p.rope);
+        rope8<DH>(q[hh], li, rope_cs);
 #pragma unroll
         for (int e = 0; e < 8; ++e) q[hh][e] *= p.scale;
     }
@@ -218,7 +232,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
         float kf[8], vf[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) { kf[e] = kp[e]; vf[e] = vp[e]; }
-        rope8<DH>(kf, li, n, p.rope);
+        rope8<DH>(kf, li, rope_cs);
         const size_t off = kv_off<T, DH>(p.kv, b, n, g) + li * 8;
         T* Kw = static_cast<T*>(p.kv.K) + off;
         T* Vw = static_cast<T*>(p.kv.V) + off;

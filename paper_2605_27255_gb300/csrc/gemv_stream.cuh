@@ -32,7 +32,11 @@ namespace pipo {
 #ifndef PIPO_TMA_STAGE_CHUNKS
 #define PIPO_TMA_STAGE_CHUNKS 8
 #endif
+#ifndef PIPO_STREAM_CTAS_PER_SM
+#define PIPO_STREAM_CTAS_PER_SM 1
+#endif
 constexpr int kStreamThreads = PIPO_STREAM_THREADS;
+constexpr int kStreamCtasPerSm = PIPO_STREAM_CTAS_PER_SM;  // CTAs per SM of one GEMV launch
 constexpr int kStreamWarps = kStreamThreads / 32;
 
 template <typename T> struct Chunk16;  // 16 bytes of weights

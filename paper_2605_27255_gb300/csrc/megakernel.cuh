@@ -233,6 +233,8 @@ __device__ __forceinline__ void mk_attn_phase(const AttnPhase& a, float* smem) {
             kk[uu].load(Kb + off);
             vv[uu].load(Vb + off);
         }
+        float4 rope_cs[4];
+        rope_load<DH>(rope_cs, li, n, a.rope);
         float q[G][8];
 #pragma unroll
         for (int hh = 0; hh < G; ++hh) {
@@ -240,7 +242,7 @@ __device__ __forceinline__ void mk_attn_phase(const AttnPhase& a, float* smem) {
             const float4 x0 = qp[0], x1 = qp[1];
             q[hh][0] = x0.x; q[hh][1] = x0.y; q[hh][2] = x0.z; q[hh][3] = x0.w;
             q[hh][4] = x1.x; q[hh][5] = x1.y; q[hh][6] = x1.z; q[hh][7] = x1.w;
-            rope8<DH>(q[hh], li, n, a.rope);
+            rope8<DH>(q[hh], li, rope_cs);
 #pragma unroll
             for (int e = 0; e < 8; ++e) q[hh][e] *= a.scale;
         }
@@ -308,7 +310,7 @@ __device__ __forceinline__ void mk_attn_phase(const AttnPhase& a, float* smem) {
             float kf[8], vf[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e) { kf[e] = kp[e]; vf[e] = vp[e]; }
-            rope8<DH>(kf, li, n, a.rope);
+            rope8<DH>(kf, li, rope_cs);
             const size_t off = kv_off<T, DH>(a.kv, b, n, g) + li * 8;
             T* Kw = static_cast<T*>(a.kv.K) + off;
             T* Vw = static_cast<T*>(a.kv.V) + off;

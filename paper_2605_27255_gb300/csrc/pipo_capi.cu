@@ -351,7 +351,12 @@ pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
         if (rows && ctx->gemv_tma && p.B <= nb) {
             // bulk-copy kernel: stages per warp from what shared memory allows
             const size_t per_stage = (size_t)kTmaWarps * (kStageBytes + 8);
-            const size_t room = g_smem_optin > 4096 + xbytes ? g_smem_optin - 4096 - xbytes : 0;
+#ifdef PIPO_TMA_SMEM_CAP
+            const size_t cap = std::min<size_t>(g_smem_optin, PIPO_TMA_SMEM_CAP);  // leave room for a second CTA
+#else
+            const size_t cap = g_smem_optin;
+#endif
+            const size_t room = cap > 4096 + xbytes ? cap - 4096 - xbytes : 0;
             const int ns = (int)std::min<size_t>(4, room / per_stage);
             if (ns >= 2) {
                 void* fn = bf ? pick_tma<bf16>(nb, two ? 2 : 1) : pick_tma<float>(nb, two ? 2 : 1);
@@ -365,7 +370,7 @@ pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
         void* args[] = {&p};
         // staged input, then (row kernel) the RMSNorm gains in their storage type
         const size_t smem = xbytes + (rows ? (size_t)p.K * ctx->esz + 16 : 0);
-        return launch_ex(ctx, fn, dim3(ctx->sms), dim3(kStreamThreads), smem, args);
+        return launch_ex(ctx, fn, dim3(ctx->sms * kStreamCtasPerSm), dim3(kStreamThreads), smem, args);
     }
     int nb = next_pow2_le8(std::max(1, p.B));
     while (nb > 1 && (size_t)nb * p.K * 4 > kXsBudget) nb >>= 1;

@@ -195,6 +195,27 @@ PIPO_API pipo_status pipo_set_stream(pipo_ctx *ctx, void *stream);
 PIPO_API pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void *d_W, int32_t N, int32_t K,
                                   const float *d_x, int32_t B, float *d_y, void *stream);
 
+/* Tensor-core form of the same projections (Eq. 2 blocks) for batches that
+ * make them dense contractions: tcgen05 MMAs with fp32 accumulation in TMEM.
+ * Each fp32 activation enters as two bf16 parts, hi = bf16(x) and
+ * lo = bf16(x - hi), multiplied by the same bf16 weights (about 2^-17
+ * relative representation error; the weight traffic is that of one pass):
+ *   mode 0: y[b*N + r] = sum_k W[r*K + k] * x[b*K + k]              (W: [N, K])
+ *   mode 1: SwiGLU as in pipo_op_gemv (W: [2N, K], gate/up rows interleaved).
+ * W bf16, 16-byte aligned; x [B, K] and y [B, N] fp32.  K a multiple of 64,
+ * N (mode 1: 2N) >= 128, 1 <= B <= 128.  splits: K splits per 128-row tile
+ * (0 = automatic; partials are added in split order, deterministic).
+ * d_scratch: 1024-byte-aligned device memory of at least
+ * pipo_op_gemm_tc_scratch(mode, N, K, B, splits) bytes, overwritten.
+ * EINVAL for bad shapes, alignment or a short scratch buffer. */
+PIPO_API pipo_status pipo_op_gemm_tc(int32_t mode, const void *d_W, int32_t N, int32_t K, const float *d_x,
+                                     int32_t B, float *d_y, int32_t splits, void *d_scratch, size_t scratch_bytes,
+                                     void *stream);
+
+/* Scratch bytes pipo_op_gemm_tc needs on the current device (0 for
+ * arguments it rejects or when no device is usable). */
+PIPO_API size_t pipo_op_gemm_tc_scratch(int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits);
+
 /* Fused LM head + argmax over the tied embedding (Eq. 3 and Eq. 5, App. B.2):
  *   d_tokens[b] = argmax_v  E[v,:] . RMSNorm(h[b,:]; gamma)
  * with the lowest v winning ties; the logits are never stored unless

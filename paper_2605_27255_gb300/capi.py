@@ -89,6 +89,9 @@ SIGNATURES = {
     "pipo_op_lm_head_argmax_noalloc": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p,
                                                  C.c_void_p, C.c_float, C.c_int32, C.c_void_p, C.c_void_p,
                                                  C.c_void_p]),
+    "pipo_op_gemm_tc": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_int32, C.c_void_p,
+                                  C.c_int32, C.c_void_p, C.c_size_t, C.c_void_p]),
+    "pipo_op_gemm_tc_scratch": (C.c_size_t, [C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32]),
     "pipo_profile_step": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.POINTER(C.c_double), _FP, _IP]),
     "pipo_step_launches": (C.c_int32, [C.c_void_p]),
     "pipo_last_error": (C.c_char_p, [C.c_void_p]),
@@ -220,6 +223,18 @@ def pipo_op_lm_head_argmax(dtype: int, E: int, V: int, H: int, h: int, gamma: in
                                          float(eps), B, C.c_void_p(tokens), C.c_void_p(logits or None),
                                          C.c_void_p(scratch or None), scratch_bytes, C.c_void_p(stream or None)),
            None)
+
+
+def pipo_op_gemm_tc_scratch(mode: int, N: int, K: int, B: int, splits: int = 0) -> int:
+    """Scratch bytes pipo_op_gemm_tc needs (0: rejected arguments)."""
+    return int(load().pipo_op_gemm_tc_scratch(mode, N, K, B, splits))
+
+
+def pipo_op_gemm_tc(mode: int, W: int, N: int, K: int, x: int, B: int, y: int, splits: int, scratch: int,
+                    scratch_bytes: int, stream: int = 0) -> None:
+    """Tensor-core projection on device pointers (ints); see include/pipo.h."""
+    _check(load().pipo_op_gemm_tc(mode, C.c_void_p(W), N, K, C.c_void_p(x), B, C.c_void_p(y), splits,
+                                  C.c_void_p(scratch), scratch_bytes, C.c_void_p(stream or None)), None)
 
 
 def pipo_op_lm_head_argmax_noalloc(dtype: int, E: int, V: int, H: int, h: int, gamma: int, eps: float, B: int,

@@ -57,7 +57,7 @@ struct GemvParams {
     unsigned long long* zero_ptr;  // zeroed by block 0 before anything else (or nullptr)
     int zero_n;
     float* part;         // EPI_RESADD with splitk > 1: partials [splitk][B][N]
-    unsigned* rowcnt;    // per-row arrival counters (zero between launches)
+    unsigned* rowcnt;    // arrival counters per (batch group, row), [ceil(B/NB)][N] (zero between launches)
 };
 
 // ---------------------------------------------------------------- loads
@@ -300,10 +300,13 @@ __global__ void __launch_bounds__(kThreads) gemv_kernel(GemvParams p) {
             }
             // split-K residual add: every slice stores its partial; the last
             // slice of the row to arrive adds them in slice order (deterministic).
+            // CTAs reach the batch groups at different times: one counter per
+            // (group, row).
             if (p.epi == EPI_RESADD && S > 1 && lane == 0) {
                 for (int bb = 0; bb < nb; ++bb) p.part[((size_t)s * p.B + b0 + bb) * p.N + r] = acc0[bb];
                 __threadfence();
-                const unsigned prev = atomicAdd(p.rowcnt + r, 1u);
+                unsigned* cnt = p.rowcnt + (size_t)(b0 / NB) * p.N + r;
+                const unsigned prev = atomicAdd(cnt, 1u);
                 if (prev == (unsigned)S - 1) {
                     __threadfence();
                     for (int bb = 0; bb < nb; ++bb) {
@@ -311,7 +314,7 @@ __global__ void __launch_bounds__(kThreads) gemv_kernel(GemvParams p) {
                         for (int ss = 0; ss < S; ++ss) sum += __ldcg(p.part + ((size_t)ss * p.B + b0 + bb) * p.N + r);
                         p.y[(size_t)(b0 + bb) * p.ldy + r] += sum;
                     }
-                    p.rowcnt[r] = 0u;
+                    *cnt = 0u;
                 }
             }
         }

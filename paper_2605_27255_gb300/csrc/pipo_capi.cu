@@ -5,6 +5,8 @@
 // activation buffers and the per-sequence device state (pending pair, KV
 // length, emitted count).  A decode step is one captured CUDA graph: no host
 // round trip inside the step.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -25,6 +27,7 @@
 #include "kernels.cuh"
 #include "megakernel.cuh"
 #include "pipo.h"
+#include "tcgen05_gemm.cuh"
 
 using namespace pipo;
 using bf16 = __nv_bfloat16;
@@ -66,6 +69,14 @@ struct pipo_ctx {
     float* gemv_part = nullptr;     // split-K partials of the residual-add GEMVs
     unsigned* gemv_rowcnt = nullptr;
     unsigned long long* am = nullptr;  // [2][max_batch]
+    // tensor-core projections (bf16, batch >= tc_min_b)
+    bf16* tc_xb = nullptr;          // [2 * tc_bn_max][tc_kmax] bf16 activations (hi rows, lo rows)
+    float* tc_part = nullptr;       // split-K partials
+    size_t tc_part_cap = 0;         // floats
+    unsigned* tc_cnt = nullptr;     // per-tile arrival counters (zero between launches)
+    int tc_cnt_cap = 0, tc_kmax = 0, tc_bn_max = 0;
+    int tc_min_b = 16;
+    int tc_splits = 0;              // forced K splits (0: automatic)
 
     int32_t *pending = nullptr, *n_pos = nullptr, *out_tokens = nullptr, *out_nacc = nullptr;
     long long* emitted = nullptr;
@@ -297,6 +308,20 @@ void* pick_stream(int nb, int ru, bool rows) {
     }
 }
 
+// bh: batch columns of the tensor-core GEMM (its MMA N is 2 * bh: hi | lo)
+size_t tc_smem(int bh) {
+    return 1024 + (size_t)kTcStages * (kTcABytes + (size_t)2 * bh * kTcBK * 2) + (2 * kTcStages + 1) * 8;
+}
+
+void* pick_tc(int bh) {
+    switch (bh) {
+        case 16: return reinterpret_cast<void*>(&gemm_tc_kernel<16>);
+        case 32: return reinterpret_cast<void*>(&gemm_tc_kernel<32>);
+        case 64: return reinterpret_cast<void*>(&gemm_tc_kernel<64>);
+        default: return reinterpret_cast<void*>(&gemm_tc_kernel<128>);
+    }
+}
+
 cudaError_t set_smem_attrs(bool bf) {
     int dev = 0, optin = 0;
     cudaError_t e0 = cudaGetDevice(&dev);
@@ -322,12 +347,105 @@ cudaError_t set_smem_attrs(bool bf) {
             cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kXsBudget);
             if (e != cudaSuccess) return e;
         }
+    if (bf)
+        for (int bn : {16, 32, 64, 128}) {
+            cudaError_t e =
+                cudaFuncSetAttribute(pick_tc(bn), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem(bn));
+            if (e != cudaSuccess) return e;
+        }
     return cudaSuccess;
+}
+
+// ---------------------------------------------------- tensor-core projections
+PFN_cuTensorMapEncodeTiled_v12000 g_encode_tiled = nullptr;
+std::mutex g_encode_mu;
+
+// 2-D bf16 tensor map over a row-major [rows, K] matrix: boxes of 64 x box_rows
+// elements, 128-byte swizzle (the layout the tcgen05 descriptors expect).
+pipo_status make_tmap(pipo_ctx* ctx, CUtensorMap* tm, const void* base, int K, int rows, int box_rows) {
+    {
+        std::lock_guard<std::mutex> lk(g_encode_mu);
+        if (!g_encode_tiled) {
+            void* fn = nullptr;
+            cudaDriverEntryPointQueryResult q{};
+            CK(cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q));
+            if (q != cudaDriverEntryPointSuccess || !fn)
+                return fail(ctx, PIPO_ECUDA, "cuTensorMapEncodeTiled is not available");
+            g_encode_tiled = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+        }
+    }
+    if (reinterpret_cast<uintptr_t>(base) % 16 != 0 || K % kTcBK != 0 || rows < box_rows)
+        return fail(ctx, PIPO_EINVAL, "tensor map: base %% 16, K %% 64 and rows >= %d required", box_rows);
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kTcBK, (cuuint32_t)box_rows};
+    const cuuint32_t es[2] = {1, 1};
+    const CUresult r = g_encode_tiled(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                                      box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(ctx, PIPO_ECUDA, "cuTensorMapEncodeTiled: error %d", (int)r);
+    return PIPO_OK;
+}
+
+int tc_bn(int B) { return B <= 16 ? 16 : B <= 32 ? 32 : B <= 64 ? 64 : 128; }
+
+// resident CTAs per SM of the tensor-core GEMM at this BN (shared memory bound)
+int tc_ctas_per_sm(int bn) {
+    const size_t per = tc_smem(bn) + 40 * (size_t)bn + 1024;  // dynamic + static + reserve
+    return std::max(1, (int)(g_smem_optin ? 228 * 1024 / per : 1));
+}
+
+// K splits: enough CTAs for every SM's resident slots, each split at least
+// kTcMinKb 64-wide K blocks, partials within the workspace
+constexpr int kTcMinKb = 6;
+int tc_auto_splits(int sms, int bn, int tiles, int nkb) {
+    const int target = sms * tc_ctas_per_sm(bn);
+    if (tiles >= target) return 1;
+    const int s = (target + tiles - 1) / tiles;
+    return std::max(1, std::min(s, nkb / kTcMinKb));
+}
+
+// Projection on the tensor cores: bf16 activations (prep kernel), then the
+// tcgen05 GEMM.  Eligible: bf16 weights, K % 64 == 0, rows >= 128, B <= 128.
+pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, float* part, size_t part_cap,
+                           unsigned* cnt, int cnt_cap, int splits_req) {
+    const int ru = p.epi == EPI_SWIGLU ? 2 : 1;
+    const int rows = p.N * ru, bn = tc_bn(p.B), tiles = (rows + kTcM - 1) / kTcM, nkb = p.K / kTcBK;
+    int splits = splits_req > 0 ? std::min(splits_req, nkb) : tc_auto_splits(ctx->sms, bn, tiles, nkb);
+    while (splits > 1 && ((size_t)splits * rows * bn > part_cap || tiles > cnt_cap)) --splits;
+    CUtensorMap tmW, tmX;
+    TRY(make_tmap(ctx, &tmW, p.W, p.K, rows, kTcM));
+    TRY(make_tmap(ctx, &tmX, xb, p.K, 2 * bn, 2 * bn));
+    {
+        GemvParams pp = p;
+        int bh = bn;
+        void* args[] = {&pp, &xb, &bh};
+        ctx->prof_kind = 2;
+        ctx->prof_bytes = 0.0;
+        TRY(launch_ex(ctx, reinterpret_cast<const void*>(&prep_bf16_kernel<bf16>), dim3(bn), dim3(256), 0, args));
+    }
+    TcParams tp{};
+    tp.rows = rows; tp.K = p.K; tp.B = p.B; tp.ru = ru; tp.epi = p.epi;
+    tp.y = p.y; tp.ldy = p.ldy; tp.bias = p.bias; tp.am = p.am; tp.dbg = p.dbg; tp.ld_dbg = p.ld_dbg;
+    tp.splits = splits; tp.part = part; tp.cnt = cnt;
+    void* args[] = {&tmW, &tmX, &tp};
+    ctx->prof_kind = 0;
+    ctx->prof_bytes = (double)rows * p.K * 2;
+    return launch_ex(ctx, pick_tc(bn), dim3(tiles * splits), dim3(kTcThreads), tc_smem(bn), args);
+}
+
+bool tc_eligible(const pipo_ctx* ctx, const GemvParams& p) {
+    const int rows = p.N * (p.epi == EPI_SWIGLU ? 2 : 1);
+    return ctx->cfg.dtype == 1 && ctx->tc_xb && !ctx->rec && p.B >= ctx->tc_min_b && p.B <= ctx->tc_bn_max &&
+           p.K % kTcBK == 0 && p.K <= ctx->tc_kmax && rows >= kTcM;
 }
 
 pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
     const bool bf = ctx->cfg.dtype == 1;
     const bool two = p.epi == EPI_SWIGLU;
+    if (tc_eligible(ctx, p))
+        return launch_gemm_tc(ctx, p, ctx->tc_xb, ctx->tc_part, ctx->tc_part_cap, ctx->tc_cnt, ctx->tc_cnt_cap,
+                              ctx->tc_splits);
     if (ctx->rec) {
         Phase ph{};
         ph.type = PH_GEMV;
@@ -1016,8 +1134,22 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         TRY(dalloc(ctx, &ctx->am, (size_t)2 * MB * 8));
         const int smax = std::max(resadd_splits(ctx, H, qd), resadd_splits(ctx, H, c.ffn));
         TRY(dalloc(ctx, &ctx->gemv_part, (size_t)smax * MB * H * 4));
-        TRY(dalloc(ctx, &ctx->gemv_rowcnt, (size_t)H * 4));
-        CK(cudaMemset(ctx->gemv_rowcnt, 0, (size_t)H * 4));
+        // one counter per (batch group, row): at most MB groups
+        TRY(dalloc(ctx, &ctx->gemv_rowcnt, (size_t)MB * H * 4));
+        CK(cudaMemset(ctx->gemv_rowcnt, 0, (size_t)MB * H * 4));
+        // tensor-core projections: bf16 activation tile, split-K workspace, counters
+        if (const char* ev = getenv("PIPO_TC_MIN_BATCH")) ctx->tc_min_b = std::max(1, atoi(ev));
+        if (const char* ev = getenv("PIPO_TC_SPLITS")) ctx->tc_splits = std::max(0, atoi(ev));
+        if (c.dtype == 1 && MB >= ctx->tc_min_b) {
+            ctx->tc_bn_max = tc_bn(std::min(MB, 128));
+            ctx->tc_kmax = std::max({2 * (int)H, qd, c.ffn});
+            ctx->tc_part_cap = (size_t)4 * ctx->sms * kTcM * ctx->tc_bn_max;
+            ctx->tc_cnt_cap = 4 * ctx->sms;
+            TRY(dalloc(ctx, &ctx->tc_xb, (size_t)2 * ctx->tc_bn_max * ctx->tc_kmax * 2));
+            TRY(dalloc(ctx, &ctx->tc_part, ctx->tc_part_cap * 4));
+            TRY(dalloc(ctx, &ctx->tc_cnt, (size_t)ctx->tc_cnt_cap * 4));
+            CK(cudaMemset(ctx->tc_cnt, 0, (size_t)ctx->tc_cnt_cap * 4));
+        }
         TRY(dalloc(ctx, &ctx->pending, (size_t)MB * 2 * 4));
         TRY(dalloc(ctx, &ctx->n_pos, (size_t)MB * 4));
         TRY(dalloc(ctx, &ctx->out_tokens, (size_t)MB * 2 * 4));
@@ -1371,6 +1503,77 @@ pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N
                          int32_t B, float* d_y, void* stream) {
     static thread_local pipo_ctx op;  // device facts and launch settings only; owns no memory
     const pipo_status st = op_gemv_impl(op, dtype, mode, d_W, N, K, d_x, B, d_y, stream);
+    if (st != PIPO_OK) g_init_error = op.err;
+    return st;
+}
+
+}  // extern "C"
+
+namespace {
+struct TcScratch {
+    size_t xb, part, cnt, total;  // byte offsets of the parts, total bytes
+    int splits;
+};
+
+TcScratch tc_scratch_plan(int sms, int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits) {
+    const int rows = N * (mode == 1 ? 2 : 1), bn = tc_bn(B), tiles = (rows + kTcM - 1) / kTcM, nkb = K / kTcBK;
+    TcScratch t{};
+    t.splits = splits > 0 ? std::min<int>(splits, nkb) : tc_auto_splits(sms, bn, tiles, nkb);
+    t.xb = 0;
+    t.part = ((size_t)2 * bn * K * 2 + 1023) / 1024 * 1024;
+    t.cnt = t.part + (t.splits > 1 ? (size_t)t.splits * rows * bn * 4 : 0);
+    t.total = t.cnt + (size_t)tiles * 4;
+    return t;
+}
+
+bool tc_op_args_ok(int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits) {
+    return (mode == 0 || mode == 1) && N >= 1 && N * (mode == 1 ? 2 : 1) >= kTcM && K >= kTcBK && K % kTcBK == 0 &&
+           B >= 1 && B <= 128 && splits >= 0;
+}
+}  // namespace
+
+extern "C" {
+
+size_t pipo_op_gemm_tc_scratch(int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits) {
+    if (!tc_op_args_ok(mode, N, K, B, splits)) return 0;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    return tc_scratch_plan(sms, mode, N, K, B, splits).total;
+}
+
+pipo_status pipo_op_gemm_tc(int32_t mode, const void* d_W, int32_t N, int32_t K, const float* d_x, int32_t B,
+                            float* d_y, int32_t splits, void* d_scratch, size_t scratch_bytes, void* stream) {
+    if (!d_W || !d_x || !d_y || !d_scratch || !tc_op_args_ok(mode, N, K, B, splits) ||
+        reinterpret_cast<uintptr_t>(d_W) % 16 != 0 || reinterpret_cast<uintptr_t>(d_scratch) % 1024 != 0)
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_gemm_tc: bad arguments");
+    static thread_local pipo_ctx op;  // device facts and launch settings only; owns no memory
+    pipo_ctx* ctx = &op;
+    pipo_status st = op_setup(op, 1, stream);
+    if (st == PIPO_OK) {
+        const TcScratch t = tc_scratch_plan(op.sms, mode, N, K, B, splits);
+        if (scratch_bytes < t.total) {
+            st = fail(ctx, PIPO_EINVAL, "pipo_op_gemm_tc: scratch needs %zu bytes, got %zu", t.total, scratch_bytes);
+        } else {
+            char* base = static_cast<char*>(d_scratch);
+            const int tiles = (N * (mode == 1 ? 2 : 1) + kTcM - 1) / kTcM;
+            cudaError_t e = cudaMemsetAsync(base + t.cnt, 0, (size_t)tiles * 4, op.stream);
+            if (e != cudaSuccess) {
+                st = fail(ctx, PIPO_ECUDA, "cudaMemsetAsync: %s", cudaGetErrorString(e));
+            } else {
+                GemvParams p{};
+                p.W = d_W; p.N = N; p.K = K; p.epi = mode == 1 ? EPI_SWIGLU : EPI_STORE;
+                p.y = d_y; p.ldy = N; p.B = B; p.splitk = 1; p.nseg = 1;
+                p.seg[0] = act_seg(d_x, K, K);
+                st = launch_gemm_tc(ctx, p, reinterpret_cast<bf16*>(base + t.xb), reinterpret_cast<float*>(base + t.part),
+                                    t.splits > 1 ? (size_t)t.splits * N * (mode == 1 ? 2 : 1) * tc_bn(B) : 0,
+                                    reinterpret_cast<unsigned*>(base + t.cnt), tiles, t.splits);
+            }
+        }
+    }
     if (st != PIPO_OK) g_init_error = op.err;
     return st;
 }

@@ -1,0 +1,404 @@
+// Tensor-core (tcgen05 / TMEM) skinny GEMM for batched projections, sm_103a.
+//
+// When B * pairs makes a projection a real dense contraction (B >= 16), the
+// weight stream is fed to the 5th-generation tensor cores instead of CUDA
+// cores.  Swap-AB: D[rows, B] = W[rows, K] . X[B, K]^T, so the 128 weight rows
+// of a tile fill the MMA's M = 128 and the batch (padded to a multiple of 16)
+// is its N.  Both operands are K-major bf16 tiles loaded by TMA tensor copies
+// with 128-byte swizzle into a 4-stage shared-memory ring (mbarrier
+// completion).  One thread issues the copies, one thread issues
+// tcgen05.mma.cta_group::1.kind::f16 (fp32 accumulation in TMEM), and four
+// warps read the accumulator back with tcgen05.ld for the epilogue.  A CTA
+// owns one (128-row tile, K split); when there are fewer tiles than SMs, K is
+// split and the last CTA of a tile to finish adds the fp32 partials in split
+// order (deterministic) and applies the epilogue.
+//
+// The activations enter as two bf16 parts, x = hi + lo with hi = bf16(x) and
+// lo = bf16(x - hi) (prep_bf16_kernel, after the RMSNorm / gather of the GEMV
+// input segments in fp32).  Both parts are B columns of the MMA (N = 2 * BH),
+// so the bf16 weights meet an activation accurate to about 2^-17 relative:
+// the weight stream is unchanged, only the (idle) tensor-core work doubles.
+// The epilogue adds the two accumulator halves.  Every wait is bounded
+// (error word + drain, no hang).
+#pragma once
+
+#include <cuda.h>
+
+#include "kernels.cuh"
+#include "tma.cuh"
+
+namespace pipo {
+
+constexpr int kTcM = 128;                   // weight rows per tile (MMA M)
+constexpr int kTcBK = 64;                   // bf16 K per stage: 128-byte rows
+constexpr int kTcStages = 4;
+constexpr int kTcThreads = 128;
+constexpr int kTcABytes = kTcM * kTcBK * 2;  // 16 KB per stage
+
+struct TcParams {
+    int rows;            // W rows (output units * ru)
+    int K;
+    int B;               // sequences (batch columns < B are real)
+    int ru;              // 1, or 2 (SwiGLU: gate/up rows interleaved)
+    int epi;
+    float* y;
+    int ldy;
+    const void* bias;    // bf16 [rows]
+    unsigned long long* am;
+    float* dbg;
+    int ld_dbg;
+    int splits;          // K splits per tile
+    float* part;         // [splits][rows][BH] fp32 partials (splits > 1)
+    unsigned* cnt;       // [tiles] arrival counters, zero between launches
+};
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, int x, int y, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_u32(dst)),
+        "l"(tm), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle (8-row groups of
+// 128-byte rows, 1024 B apart), tile base 1024-byte aligned.
+__device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr >> 4) & 0x3FFFu);  // start address (16-byte units)
+    d |= (uint64_t)1 << 16;                    // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024 >> 4) << 32;          // stride byte offset between 8-row groups
+    d |= (uint64_t)1 << 46;                    // descriptor version
+    d |= (uint64_t)2 << 61;                    // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor of kind::f16: D fp32, A and B bf16, both K-major.
+__host__ __device__ constexpr uint32_t umma_idesc_bf16(int M, int N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(
+            d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+
+// arrive on `bar` once all tcgen05.mma issued before it by this thread complete
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)), "r"(ncols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// 16 consecutive fp32 columns of this thread's TMEM lane
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Epilogue of batch columns [c0, c0+16) of weight row `row` (thread = TMEM
+// lane).  All threads of the warp call it (the SwiGLU pairing shuffles).
+template <int BH>
+__device__ __forceinline__ void tc_epilogue16(const TcParams& p, int row, int c0, const float (&v)[16],
+                                              float (*red_v)[BH], int (*red_r)[BH]) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool in = row < p.rows;
+    if (p.epi == EPI_ARGMAX) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int b = c0 + j;
+            float bv = in ? v[j] : -INFINITY;
+            int br = in ? row : 0x7fffffff;
+            if (p.dbg && in && b < p.B) p.dbg[(size_t)b * p.ld_dbg + row] = v[j];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                const int orow = __shfl_xor_sync(0xffffffffu, br, o);
+                if (ov > bv || (ov == bv && orow < br)) { bv = ov; br = orow; }
+            }
+            if (lane == 0) { red_v[warp][b] = bv; red_r[warp][b] = br; }
+        }
+        return;
+    }
+    if (p.ru == 2) {  // gate on even rows, up on the odd row after it
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const float up = __shfl_xor_sync(0xffffffffu, v[j], 1);
+            const int b = c0 + j;
+            if (in && (row & 1) == 0 && b < p.B) p.y[(size_t)b * p.ldy + (row >> 1)] = silu(v[j]) * up;
+        }
+        return;
+    }
+    if (!in) return;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        const int b = c0 + j;
+        if (b >= p.B) continue;
+        float* yp = p.y + (size_t)b * p.ldy + row;
+        const float a = v[j];
+        switch (p.epi) {
+            case EPI_STORE: *yp = a; break;
+            case EPI_BIAS: *yp = a + __bfloat162float(static_cast<const __nv_bfloat16*>(p.bias)[row]); break;
+            case EPI_SILU: *yp = silu(a); break;
+            case EPI_RESADD: *yp += a; break;
+            default: break;
+        }
+    }
+}
+
+// BH: batch columns (a multiple of 16, >= B); the MMA N is 2 * BH (hi | lo).
+template <int BH>
+__global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW,
+                                                                const __grid_constant__ CUtensorMap tmX, TcParams p) {
+    extern __shared__ __align__(1024) unsigned char tc_smem_raw[];
+    constexpr int BN = 2 * BH;
+    constexpr int kBBytes = BN * kTcBK * 2;
+    constexpr uint32_t kCols = BN <= 32 ? 32u : BN <= 64 ? 64u : BN <= 128 ? 128u : 256u;
+    unsigned char* sm = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~(uintptr_t)1023);
+    unsigned char* sA = sm;
+    unsigned char* sB = sm + kTcStages * kTcABytes;
+    uint64_t* full = reinterpret_cast<uint64_t*>(sB + kTcStages * kBBytes);
+    uint64_t* empty = full + kTcStages;
+    uint64_t* accb = empty + kTcStages;
+    __shared__ uint32_t tmem_base;
+    __shared__ float red_v[4][BH];
+    __shared__ int red_r[4][BH];
+    __shared__ int last;
+
+    pdl_launch();
+    const int warp = threadIdx.x >> 5;
+    const int tile = blockIdx.x / p.splits, split = blockIdx.x % p.splits;
+    const int nkb = p.K / kTcBK;
+    const int kb0 = (int)((long long)split * nkb / p.splits), kb1 = (int)((long long)(split + 1) * nkb / p.splits);
+    const int nk = kb1 - kb0;  // >= 1 (splits <= nkb)
+
+    if (warp == 0) tmem_alloc(&tmem_base, kCols);
+    if (threadIdx.x == 32) {
+        for (int s = 0; s < kTcStages; ++s) {
+            mbar_init(full + s, 1);
+            mbar_init(empty + s, 1);
+        }
+        mbar_init(accb, 1);
+        mbar_init_fence();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+
+    const int lane = threadIdx.x & 31;
+    if (warp == 0) {
+        if (lane == 0) {
+            // TMA producer: weight tiles need nothing from the previous
+            // kernel; the activation tile waits for it (programmatic
+            // dependent launch)
+            int issued = 0;
+            for (int i = 0; i < nk; ++i) {
+                const int s = i % kTcStages;
+                if (i >= kTcStages && !mbar_wait(empty + s, (uint32_t)(((i / kTcStages) & 1) ^ 1))) break;
+                mbar_arrive_expect_tx(full + s, (uint32_t)(kTcABytes + kBBytes));
+                tma_load_2d(sA + s * kTcABytes, &tmW, (kb0 + i) * kTcBK, tile * kTcM, full + s);
+                if (i == 0) pdl_wait();
+                tma_load_2d(sB + s * kBBytes, &tmX, (kb0 + i) * kTcBK, 0, full + s);
+                issued = i + 1;
+            }
+            // no copy into this CTA's shared memory may still be in flight at exit
+            for (int i = max(0, issued - kTcStages); i < issued; ++i)
+                mbar_wait(full + (i % kTcStages), (uint32_t)((i / kTcStages) & 1));
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // MMA issuer: 4 MMAs of K = 16 per stage, the operand
+            // descriptors advanced by 32 bytes inside the swizzled rows
+            const uint32_t idesc = umma_idesc_bf16(kTcM, BN);
+            for (int i = 0; i < nk; ++i) {
+                const int s = i % kTcStages;
+                if (!mbar_wait(full + s, (uint32_t)((i / kTcStages) & 1))) break;
+                tc_fence_after();
+                const uint32_t a0 = smem_u32(sA + s * kTcABytes), b0 = smem_u32(sB + s * kBBytes);
+#pragma unroll
+                for (int k = 0; k < kTcBK / 16; ++k)
+                    umma_bf16(tmem, umma_desc_sw128(a0 + k * 32), umma_desc_sw128(b0 + k * 32), idesc,
+                              (i > 0 || k > 0) ? 1u : 0u);
+                umma_commit(empty + s);  // frees the stage once these MMAs have read it
+            }
+            umma_commit(accb);
+        }
+        __syncwarp();
+    }
+
+    // epilogue: thread t holds TMEM lane t = weight row tile*128 + t
+    mbar_wait(accb, 0);
+    __syncwarp();
+    tc_fence_after();
+    pdl_wait();
+    const int row = tile * kTcM + threadIdx.x;
+    const uint32_t lane_addr = tmem + ((uint32_t)(warp * 32) << 16);
+    // 16 batch columns: hi part at column c0, lo part at column BH + c0
+    auto ld_cols = [&](int c0, float (&v)[16]) {
+        float lo[16];
+        tmem_ld16(lane_addr + c0, v);
+        tmem_ld16(lane_addr + BH + c0, lo);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] += lo[j];
+    };
+    if (p.splits == 1) {
+#pragma unroll 1
+        for (int c0 = 0; c0 < BH; c0 += 16) {
+            float v[16];
+            ld_cols(c0, v);
+            tc_epilogue16<BH>(p, row, c0, v, red_v, red_r);
+        }
+    } else {
+        // tcgen05.ld is warp-collective: every lane loads, only rows in range store
+        float* dst = p.part + ((size_t)split * p.rows + min(row, p.rows - 1)) * BH;
+#pragma unroll 1
+        for (int c0 = 0; c0 < BH; c0 += 16) {
+            float v[16];
+            ld_cols(c0, v);
+            if (row < p.rows) {
+#pragma unroll
+                for (int j = 0; j < 16; j += 4)
+                    *reinterpret_cast<float4*>(dst + c0 + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+            }
+        }
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) last = (atomicAdd(p.cnt + tile, 1u) == (unsigned)p.splits - 1);
+        __syncthreads();
+        if (last) {
+            __threadfence();
+#pragma unroll 1
+            for (int c0 = 0; c0 < BH; c0 += 16) {
+                float v[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) v[j] = 0.f;
+                if (row < p.rows)
+                    for (int s = 0; s < p.splits; ++s) {
+                        const float* src = p.part + ((size_t)s * p.rows + row) * BH + c0;
+#pragma unroll
+                        for (int j = 0; j < 16; j += 4) {
+                            const float4 t = __ldcg(reinterpret_cast<const float4*>(src + j));
+                            v[j] += t.x; v[j + 1] += t.y; v[j + 2] += t.z; v[j + 3] += t.w;
+                        }
+                    }
+                tc_epilogue16<BH>(p, row, c0, v, red_v, red_r);
+            }
+            if (threadIdx.x == 0) p.cnt[tile] = 0u;
+        }
+    }
+    if (p.epi == EPI_ARGMAX && (p.splits == 1 || last)) {
+        __syncthreads();
+        if (threadIdx.x < p.B) {
+            const int b = threadIdx.x;
+            float bv = -INFINITY;
+            int br = 0x7fffffff;
+            for (int w = 0; w < 4; ++w)
+                if (red_r[w][b] != 0x7fffffff && (red_v[w][b] > bv || (red_v[w][b] == bv && red_r[w][b] < br))) {
+                    bv = red_v[w][b];
+                    br = red_r[w][b];
+                }
+            if (br != 0x7fffffff) atomicMax(p.am + b, argmax_key(bv, br));
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kCols);
+    }
+}
+
+// Activations of the tensor-core GEMM, [2 * BH][K] bf16: row b < B holds
+// hi = bf16(x_b) and row BH + b holds lo = bf16(x_b - hi), where x_b is the
+// (gathered, RMS-normalised) GEMV input of sequence b; rows of b >= B are
+// zero.  grid BH, 256 threads.
+template <typename T>
+__global__ void __launch_bounds__(256) prep_bf16_kernel(GemvParams p, __nv_bfloat16* xb, int BH) {
+    __shared__ float red[8][2];
+    __shared__ float rstd[2];
+    __shared__ int tok[2];
+    pdl_launch();
+    pdl_wait();
+    const int b = blockIdx.x, K = p.K, tid = threadIdx.x;
+    if (p.zero_ptr && b == 0)  // argmax keys of this step (read by later kernels only)
+        for (int i = tid; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
+    __nv_bfloat16* dst = xb + (size_t)b * K;
+    __nv_bfloat16* dst_lo = xb + (size_t)(BH + b) * K;
+    if (b >= p.B) {
+        for (int k = tid; k < K; k += blockDim.x) dst[k] = dst_lo[k] = __float2bfloat16_rn(0.f);
+        return;
+    }
+    if (tid < 2) {
+        int t = 0;
+        if (tid < p.nseg && !p.seg[tid].src) {
+            const Seg& sg = p.seg[tid];
+            t = sg.tok_am ? argmax_row(sg.tok_am[b]) : sg.tok[(size_t)b * sg.tok_ld];
+        }
+        tok[tid] = t;
+    }
+    __syncthreads();
+    const int K0 = p.seg[0].K;
+    auto val = [&](int k) -> float {
+        const int s = k < K0 ? 0 : 1;
+        const Seg& sg = p.seg[s];
+        const int kk = s == 0 ? k : k - K0;
+        if (sg.src) return sg.src[(size_t)b * sg.ld + kk];
+        return tok[s] < 0 ? ldw<T>(sg.pad, kk) : ldw<T>(sg.table, (size_t)tok[s] * sg.K + kk);
+    };
+    const bool norm0 = p.seg[0].gamma != nullptr, norm1 = p.nseg > 1 && p.seg[1].gamma != nullptr;
+    if (norm0 || norm1) {
+        float s0 = 0.f, s1 = 0.f;
+        for (int k = tid; k < K; k += blockDim.x) {
+            const float v = val(k);
+            if (p.joint_norm || k < K0) s0 += v * v; else s1 += v * v;
+        }
+        s0 = warp_sum(s0);
+        s1 = warp_sum(s1);
+        if ((tid & 31) == 0) { red[tid >> 5][0] = s0; red[tid >> 5][1] = s1; }
+        __syncthreads();
+        if (tid < 2) {
+            float t = 0.f;
+            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w][tid];
+            const int len = p.joint_norm ? (tid == 0 ? K : 1) : (tid == 0 ? K0 : (p.nseg > 1 ? p.seg[1].K : 1));
+            rstd[tid] = 1.0f / sqrtf(t / (float)len + p.eps);
+        }
+        __syncthreads();
+    }
+    for (int k = tid; k < K; k += blockDim.x) {
+        float v = val(k);
+        const int g = (p.joint_norm || k < K0) ? 0 : 1;
+        const Seg& sg = p.seg[p.joint_norm ? 0 : g];
+        if (sg.gamma) {
+            const int kk = (p.joint_norm || g == 0) ? k : k - K0;
+            v *= rstd[g] * ldw<T>(sg.gamma, kk);
+        }
+        const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+        dst[k] = hi;
+        dst_lo[k] = __float2bfloat16_rn(v - __bfloat162float(hi));
+    }
+}
+
+}  // namespace pipo

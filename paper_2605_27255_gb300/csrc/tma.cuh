@@ -14,7 +14,7 @@ namespace pipo {
 // Device error word: 0 = fine; kErrWaitTimeout when a bounded wait gave up.
 __device__ unsigned int g_pipo_error;
 constexpr unsigned kErrWaitTimeout = 1u;
-constexpr int kWaitSpins = 1 << 22;  // try_wait rounds before giving up (~seconds)
+constexpr unsigned long long kWaitNs = 2000000000ull;  // give up after 2 s of waiting
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -58,10 +58,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Bounded wait for phase `parity` of `bar`; false (and the error word set) on timeout.
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Bounded wait for phase `parity` of `bar`: false (and the error word set)
+// once kWaitNs of wall time have passed without the phase completing.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-    for (int i = 0; i < kWaitSpins; ++i)
-        if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    for (;;) {
+        for (int i = 0; i < 64; ++i)
+            if (mbar_try_wait(bar, parity)) return true;
+        if (global_ns() - t0 > kWaitNs) break;
+    }
     atomicOr(&g_pipo_error, kErrWaitTimeout);
     return false;
 }

@@ -1,0 +1,98 @@
+"""Tensor-core (tcgen05) projections: the kernel through its C-ABI entry point
+against a float64 evaluation of the fp32-activation projection, and the decode
+path with batches that route the projections to it, against the fp64 oracle
+(forced replay)."""
+import pytest
+import torch
+
+from paper_2605_27255_gb300 import capi, synth
+from parity_util import run_forced_replay
+
+pytestmark = pytest.mark.gpu
+
+
+def _run_tc(mode, N, K, B, splits, seed=0):
+    g = torch.Generator().manual_seed(seed + 7 * N + K + B)
+    rows = 2 * N if mode else N
+    W = (torch.randn(rows, K, generator=g) * 0.05).to(torch.bfloat16)
+    x = torch.randn(B, K, generator=g)
+    Wd, xd = W.cuda(), x.cuda()
+    y = torch.full((B, N), float("nan"), device="cuda")
+    nbytes = capi.pipo_op_gemm_tc_scratch(mode, N, K, B, splits)
+    assert nbytes > 0
+    scratch = torch.empty(nbytes + 1024, dtype=torch.uint8, device="cuda")
+    base = (scratch.data_ptr() + 1023) // 1024 * 1024
+    stream = torch.cuda.current_stream().cuda_stream
+    for _ in range(2):  # twice: the split-K arrival counters must come back to zero
+        y.fill_(float("nan"))
+        capi.pipo_op_gemm_tc(mode, Wd.data_ptr(), N, K, xd.data_ptr(), B, y.data_ptr(), splits, base, nbytes,
+                             stream)
+        torch.cuda.synchronize()
+    # fp32 activations: the kernel carries them as bf16 hi + lo parts
+    ref = x.double() @ W.double().t()
+    if mode:
+        gate, up = ref[:, 0::2], ref[:, 1::2]
+        ref = gate * torch.sigmoid(gate) * up
+    return y.cpu().double(), ref
+
+
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("N,K", [(2560, 2560), (333, 4096), (1000, 1408), (4096, 256), (128, 64)])
+@pytest.mark.parametrize("B", [1, 16, 37, 64, 128])
+@pytest.mark.parametrize("splits", [0, 1, 3])
+def test_gemm_tc_matches_float64(mode, N, K, B, splits):
+    y, ref = _run_tc(mode, N, K, B, splits)
+    assert not torch.isnan(y).any()
+    scale = ref.abs().max().item() + 1e-6
+    err = (y - ref).abs().max().item()
+    assert err <= 2e-5 * scale * max(1.0, K / 1024) + 1e-6, (err, scale)
+
+
+def test_gemm_tc_split_orders_agree():
+    """Different K splits change only the fp32 summation order."""
+    a, ref = _run_tc(0, 2560, 9728, 16, 1)
+    b, _ = _run_tc(0, 2560, 9728, 16, 19)
+    assert (a - b).abs().max().item() <= 2e-5 * ref.abs().max().item() * 9728 / 1024
+
+
+def test_gemm_tc_rejects_bad_arguments():
+    assert capi.pipo_op_gemm_tc_scratch(0, 256, 100, 4, 0) == 0  # K not a multiple of 64
+    assert capi.pipo_op_gemm_tc_scratch(0, 256, 128, 129, 0) == 0  # B > 128
+    assert capi.pipo_op_gemm_tc_scratch(0, 64, 128, 4, 0) == 0  # fewer than 128 rows
+    W = torch.zeros(256, 128, dtype=torch.bfloat16, device="cuda")
+    x = torch.zeros(4, 128, device="cuda")
+    y = torch.zeros(4, 256, device="cuda")
+    need = capi.pipo_op_gemm_tc_scratch(0, 256, 128, 4, 0)
+    s = torch.empty(need + 2048, dtype=torch.uint8, device="cuda")
+    base = (s.data_ptr() + 1023) // 1024 * 1024
+    with pytest.raises(capi.PipoError) as e:  # short scratch
+        capi.pipo_op_gemm_tc(0, W.data_ptr(), 256, 128, x.data_ptr(), 4, y.data_ptr(), 0, base, need - 4, 0)
+    assert e.value.status == capi.PIPO_EINVAL
+    with pytest.raises(capi.PipoError) as e:  # scratch not 1024-byte aligned
+        capi.pipo_op_gemm_tc(0, W.data_ptr(), 256, 128, x.data_ptr(), 4, y.data_ptr(), 0, base + 256, need, 0)
+    assert e.value.status == capi.PIPO_EINVAL
+
+
+# model-level: 512-wide blocks, ragged vocabulary; the FFN down projection
+# (K = 1376, not a multiple of 64) stays on the CUDA-core kernel
+MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003,
+                       compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1.0e4, tau=0.5)
+
+
+@pytest.mark.parametrize("B", [16, 37])
+def test_mid_bf16_tensor_core_batches(B):
+    w = synth.gen_weights(MID, seed=21)
+    prompts = synth.gen_prompts(B, 24, MID.V, seed=B).numpy()
+    st = run_forced_replay(MID, w, prompts, 4, force=0, page_shuffle_seed=5)
+    assert st.tok_checked >= 0.8 * st.tok_total
+    assert st.max_logit_err < 2e-2
+
+
+def test_mid_bf16_cuda_core_batches_over_8(monkeypatch):
+    """The CUDA-core GEMV at B = 37: five 8-sequence groups, split-K residual adds."""
+    monkeypatch.setenv("PIPO_TC_MIN_BATCH", "100000")
+    w = synth.gen_weights(MID, seed=22)
+    prompts = synth.gen_prompts(37, 24, MID.V, seed=9).numpy()
+    st = run_forced_replay(MID, w, prompts, 3, force=1)
+    assert st.tok_checked >= 0.8 * st.tok_total
+    assert st.max_logit_err < 2e-2

@@ -203,8 +203,10 @@ PIPO_API pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void *d_W, 
  *   mode 0: y[b*N + r] = sum_k W[r*K + k] * x[b*K + k]              (W: [N, K])
  *   mode 1: SwiGLU as in pipo_op_gemv (W: [2N, K], gate/up rows interleaved).
  * W bf16, 16-byte aligned; x [B, K] and y [B, N] fp32.  K a multiple of 64,
- * N (mode 1: 2N) >= 128, 1 <= B <= 128.  splits: K splits per 128-row tile
- * (0 = automatic; partials are added in split order, deterministic).
+ * N (mode 1: 2N) >= 128, 1 <= B <= 128.  splits: K splits per 128-row tile,
+ * at most 8 (0 = automatic; larger values are clamped); the splits of a tile
+ * are one thread-block cluster and add their partials in split order
+ * (deterministic).
  * d_scratch: 1024-byte-aligned device memory of at least
  * pipo_op_gemm_tc_scratch(mode, N, K, B, splits) bytes, overwritten.
  * EINVAL for bad shapes, alignment or a short scratch buffer. */

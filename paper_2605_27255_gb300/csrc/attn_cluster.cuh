@@ -1,7 +1,8 @@
 // Split-KV GQA flash-decode over the paged pair-KV cache, one thread-block
 // cluster per (sequence, kv head) (sm_103a).
 //
-// Grid (CS, n_kv, B), cluster (CS, 1, 1), 256 threads.  CTA s of the cluster
+// Grid (CS, n_kv, B), cluster (CS, 1, 1), 256 threads; CS (1 .. 16) is read
+// from the cluster at run time, so one kernel serves every split.  CTA s of the cluster
 // attends the G = n_q/n_kv query heads of its kv head over a contiguous slice
 // of entries 0..n (n = entries before this step; entry n is this step's new
 // key/value).  Fused in:
@@ -99,7 +100,7 @@ constexpr int kAttnThreads = kAttnWarps * 32;
 #define PIPO_ATTN_KU 4
 #endif
 
-template <typename T, int DH, int G, int CS>
+template <typename T, int DH, int G>
 __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p) {
     constexpr int LPE = DH / 8;        // lanes per entry
     constexpr int EPW = 32 / LPE;      // entries per warp step
@@ -114,6 +115,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     pdl_launch();
     cg::cluster_group cluster = cg::this_cluster();
     const int s = (int)cluster.block_rank();
+    const int CS = (int)cluster.num_blocks();
     const int g = blockIdx.y, b = blockIdx.z;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int li = lane % LPE, slot = lane / LPE;
@@ -307,7 +309,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     }
     cluster.sync();
     // cluster merge: CTA s finishes dims [s*G*DH/CS, (s+1)*G*DH/CS) of the G heads
-    constexpr int PER = (G * DH + CS - 1) / CS;
+    const int PER = (G * DH + CS - 1) / CS;
     for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
         const int hh = i / DH, t = i % DH;
         float M = -INFINITY;

@@ -71,10 +71,7 @@ struct pipo_ctx {
     unsigned long long* am = nullptr;  // [2][max_batch]
     // tensor-core projections (bf16, batch >= tc_min_b)
     bf16* tc_xb = nullptr;          // [2 * tc_bn_max][tc_kmax] bf16 activations (hi rows, lo rows)
-    float* tc_part = nullptr;       // split-K partials
-    size_t tc_part_cap = 0;         // floats
-    unsigned* tc_cnt = nullptr;     // per-tile arrival counters (zero between launches)
-    int tc_cnt_cap = 0, tc_kmax = 0, tc_bn_max = 0;
+    int tc_kmax = 0, tc_bn_max = 0;
     int tc_min_b = 16;
     int tc_splits = 0;              // forced K splits (0: automatic)
 
@@ -91,6 +88,8 @@ struct pipo_ctx {
     float* rope = nullptr;            // [max_ctx][d_h/2][2] cos, sin
     bool pdl = false;                 // programmatic dependent launch (decode graph only)
     bool attn_cs16 = false;           // 16-CTA attention clusters available
+    int attn_cs_force = 0;            // (development) fixed attention cluster size
+    int attn_cs_target = 1;           // attention CTAs per SM above which clusters shrink
     bool attn_v0 = false;             // (development) the unclustered attention path
     bool gemv_tma = false;            // bulk-copy GEMV (else the register-ring GEMV)
     // persistent step kernel: phases recorded from the enqueue code
@@ -310,15 +309,19 @@ void* pick_stream(int nb, int ru, bool rows) {
 
 // bh: batch columns of the tensor-core GEMM (its MMA N is 2 * bh: hi | lo)
 size_t tc_smem(int bh) {
-    return 1024 + (size_t)kTcStages * (kTcABytes + (size_t)2 * bh * kTcBK * 2) + (2 * kTcStages + 1) * 8;
+    const int st = tc_stages(bh);
+    return 1024 + (size_t)st * (kTcABytes + (size_t)2 * bh * kTcBK * 2) + (2 * st + 1) * 8;
 }
+
+template <int BH>
+void* tc_fn() { return reinterpret_cast<void*>(&gemm_tc_kernel<BH, tc_stages(BH)>); }
 
 void* pick_tc(int bh) {
     switch (bh) {
-        case 16: return reinterpret_cast<void*>(&gemm_tc_kernel<16>);
-        case 32: return reinterpret_cast<void*>(&gemm_tc_kernel<32>);
-        case 64: return reinterpret_cast<void*>(&gemm_tc_kernel<64>);
-        default: return reinterpret_cast<void*>(&gemm_tc_kernel<128>);
+        case 16: return tc_fn<16>();
+        case 32: return tc_fn<32>();
+        case 64: return tc_fn<64>();
+        default: return tc_fn<128>();
     }
 }
 
@@ -395,24 +398,23 @@ int tc_ctas_per_sm(int bn) {
     return std::max(1, (int)(g_smem_optin ? 228 * 1024 / per : 1));
 }
 
-// K splits: enough CTAs for every SM's resident slots, each split at least
-// kTcMinKb 64-wide K blocks, partials within the workspace
-constexpr int kTcMinKb = 6;
+// K splits (the cluster size): enough CTAs for every SM's resident slots,
+// each split at least kTcMinKb 64-wide K blocks, at most kTcMaxSplits
+constexpr int kTcMinKb = 4;
 int tc_auto_splits(int sms, int bn, int tiles, int nkb) {
     const int target = sms * tc_ctas_per_sm(bn);
     if (tiles >= target) return 1;
     const int s = (target + tiles - 1) / tiles;
-    return std::max(1, std::min(s, nkb / kTcMinKb));
+    return std::max(1, std::min({s, nkb / kTcMinKb, kTcMaxSplits}));
 }
 
 // Projection on the tensor cores: bf16 activations (prep kernel), then the
 // tcgen05 GEMM.  Eligible: bf16 weights, K % 64 == 0, rows >= 128, B <= 128.
-pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, float* part, size_t part_cap,
-                           unsigned* cnt, int cnt_cap, int splits_req) {
+pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int splits_req) {
     const int ru = p.epi == EPI_SWIGLU ? 2 : 1;
     const int rows = p.N * ru, bn = tc_bn(p.B), tiles = (rows + kTcM - 1) / kTcM, nkb = p.K / kTcBK;
-    int splits = splits_req > 0 ? std::min(splits_req, nkb) : tc_auto_splits(ctx->sms, bn, tiles, nkb);
-    while (splits > 1 && ((size_t)splits * rows * bn > part_cap || tiles > cnt_cap)) --splits;
+    const int splits = splits_req > 0 ? std::min({splits_req, nkb, kTcMaxSplits})
+                                      : tc_auto_splits(ctx->sms, bn, tiles, nkb);
     CUtensorMap tmW, tmX;
     TRY(make_tmap(ctx, &tmW, p.W, p.K, rows, kTcM));
     TRY(make_tmap(ctx, &tmX, xb, p.K, 2 * bn, 2 * bn));
@@ -427,11 +429,11 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, float* 
     TcParams tp{};
     tp.rows = rows; tp.K = p.K; tp.B = p.B; tp.ru = ru; tp.epi = p.epi;
     tp.y = p.y; tp.ldy = p.ldy; tp.bias = p.bias; tp.am = p.am; tp.dbg = p.dbg; tp.ld_dbg = p.ld_dbg;
-    tp.splits = splits; tp.part = part; tp.cnt = cnt;
+    tp.splits = splits;
     void* args[] = {&tmW, &tmX, &tp};
     ctx->prof_kind = 0;
     ctx->prof_bytes = (double)rows * p.K * 2;
-    return launch_ex(ctx, pick_tc(bn), dim3(tiles * splits), dim3(kTcThreads), tc_smem(bn), args);
+    return launch_ex(ctx, pick_tc(bn), dim3(tiles * splits), dim3(kTcThreads), tc_smem(bn), args, splits);
 }
 
 bool tc_eligible(const pipo_ctx* ctx, const GemvParams& p) {
@@ -444,8 +446,7 @@ pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
     const bool bf = ctx->cfg.dtype == 1;
     const bool two = p.epi == EPI_SWIGLU;
     if (tc_eligible(ctx, p))
-        return launch_gemm_tc(ctx, p, ctx->tc_xb, ctx->tc_part, ctx->tc_part_cap, ctx->tc_cnt, ctx->tc_cnt_cap,
-                              ctx->tc_splits);
+        return launch_gemm_tc(ctx, p, ctx->tc_xb, ctx->tc_splits);
     if (ctx->rec) {
         Phase ph{};
         ph.type = PH_GEMV;
@@ -566,36 +567,31 @@ void* attn_pick(bool bf, int DH, int G) {
     return nullptr;
 }
 
-template <typename T, int DH, int G, int CS>
-void* attnc_fn() { return reinterpret_cast<void*>(&attn_cluster_kernel<T, DH, G, CS>); }
+template <typename T, int DH, int G>
+void* attnc_fn() { return reinterpret_cast<void*>(&attn_cluster_kernel<T, DH, G>); }
 
-template <typename T, int DH, int CS>
+template <typename T, int DH>
 void* attnc_pick_g(int G) {
     switch (G) {
-        case 1: return attnc_fn<T, DH, 1, CS>();
-        case 2: return attnc_fn<T, DH, 2, CS>();
-        case 4: return attnc_fn<T, DH, 4, CS>();
-        case 8: return attnc_fn<T, DH, 8, CS>();
+        case 1: return attnc_fn<T, DH, 1>();
+        case 2: return attnc_fn<T, DH, 2>();
+        case 4: return attnc_fn<T, DH, 4>();
+        case 8: return attnc_fn<T, DH, 8>();
         default: return nullptr;
     }
 }
 
-// cs: cluster size, 8 (portable) or 16 (non-portable, small batches)
-void* attnc_pick(bool bf, int DH, int G, int cs) {
-    if (cs == 16) {
-        if (DH == 64) return bf ? attnc_pick_g<bf16, 64, 16>(G) : attnc_pick_g<float, 64, 16>(G);
-        if (DH == 128) return bf ? attnc_pick_g<bf16, 128, 16>(G) : attnc_pick_g<float, 128, 16>(G);
-        return nullptr;
-    }
-    if (DH == 64) return bf ? attnc_pick_g<bf16, 64, 8>(G) : attnc_pick_g<float, 64, 8>(G);
-    if (DH == 128) return bf ? attnc_pick_g<bf16, 128, 8>(G) : attnc_pick_g<float, 128, 8>(G);
+// one kernel for every cluster size (read from the cluster at run time)
+void* attnc_pick(bool bf, int DH, int G) {
+    if (DH == 64) return bf ? attnc_pick_g<bf16, 64>(G) : attnc_pick_g<float, 64>(G);
+    if (DH == 128) return bf ? attnc_pick_g<bf16, 128>(G) : attnc_pick_g<float, 128>(G);
     return nullptr;
 }
 
 // Can a 16-CTA cluster of this kernel be scheduled here?  (sets the
 // non-portable cluster attribute; any failure selects 8)
 bool cluster16_ok(bool bf, int DH, int G) {
-    void* fn = attnc_pick(bf, DH, G, 16);
+    void* fn = attnc_pick(bf, DH, G);
     if (!fn) return false;
     if (cudaFuncSetAttribute(fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
         cudaGetLastError();
@@ -634,6 +630,18 @@ KVView kv_view(pipo_ctx* ctx, int layer) {
     v.page = ctx->cfg.page_size;
     v.n_kv = ctx->cfg.n_kv_heads;
     return v;
+}
+
+// CTAs per (sequence, kv head) of the clustered attention: 8 while the batch
+// leaves SMs idle (16 where allowed and still under two per SM), fewer as the
+// (sequence, kv head) pairs alone fill the GPU.
+int attn_cluster_size(const pipo_ctx* ctx) {
+    if (ctx->attn_cs_force) return ctx->attn_cs_force;
+    const long long pairs = (long long)ctx->B * ctx->cfg.n_kv_heads;
+    if (ctx->attn_cs16 && pairs * 16 <= 2 * ctx->sms) return 16;
+    int cs = 8;
+    while (cs > 1 && pairs * cs > (long long)ctx->attn_cs_target * ctx->sms) cs >>= 1;
+    return cs;
 }
 
 // One decoder block on the residual stream xr (pre-norm attention + SwiGLU).
@@ -679,9 +687,8 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         ap.out = ctx->attn;
         ap.scale = 1.0f / sqrtf((float)DH);
         void* args[] = {&ap};
-        // 16-CTA clusters when the batch leaves most SMs idle with 8
-        const int cs = (ctx->attn_cs16 && ctx->B * c.n_kv_heads * 16 <= 2 * ctx->sms) ? 16 : 8;
-        TRY(launch_ex(ctx, attnc_pick(bf, DH, c.n_q_heads / c.n_kv_heads, cs), dim3(cs, c.n_kv_heads, ctx->B),
+        const int cs = attn_cluster_size(ctx);
+        TRY(launch_ex(ctx, attnc_pick(bf, DH, c.n_q_heads / c.n_kv_heads), dim3(cs, c.n_kv_heads, ctx->B),
                       dim3(kAttnThreads), 0, args, cs));
     } else {
     // RoPE + KV append
@@ -1111,6 +1118,13 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         // 16-CTA clusters measured slower than 8 at 4B B=1 (2.77 vs 2.55 ms per step): opt-in only
         if (const char* ev = getenv("PIPO_ATTN_CS16"))
             ctx->attn_cs16 = ev[0] == '1' && cluster16_ok(c.dtype == 1, c.head_dim, c.n_q_heads / c.n_kv_heads);
+        if (const char* ev = getenv("PIPO_ATTN_CS")) {
+            const int v = atoi(ev);
+            if (v == 1 || v == 2 || v == 4 || v == 8 || (v == 16 && cluster16_ok(c.dtype == 1, c.head_dim,
+                                                                               c.n_q_heads / c.n_kv_heads)))
+                ctx->attn_cs_force = v;
+        }
+        if (const char* ev = getenv("PIPO_ATTN_CS_TARGET")) ctx->attn_cs_target = std::max(1, atoi(ev));
         if (const char* ev = getenv("PIPO_GEMV_TMA")) ctx->gemv_tma = ev[0] == '1';
         if (const char* ev = getenv("PIPO_STEP_KERNEL")) ctx->use_mk = ev[0] == '1';
         TRY(dalloc(ctx, &ctx->bar_ctr, 64));
@@ -1137,18 +1151,13 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         // one counter per (batch group, row): at most MB groups
         TRY(dalloc(ctx, &ctx->gemv_rowcnt, (size_t)MB * H * 4));
         CK(cudaMemset(ctx->gemv_rowcnt, 0, (size_t)MB * H * 4));
-        // tensor-core projections: bf16 activation tile, split-K workspace, counters
+        // tensor-core projections: the bf16 activation tile
         if (const char* ev = getenv("PIPO_TC_MIN_BATCH")) ctx->tc_min_b = std::max(1, atoi(ev));
         if (const char* ev = getenv("PIPO_TC_SPLITS")) ctx->tc_splits = std::max(0, atoi(ev));
         if (c.dtype == 1 && MB >= ctx->tc_min_b) {
             ctx->tc_bn_max = tc_bn(std::min(MB, 128));
             ctx->tc_kmax = std::max({2 * (int)H, qd, c.ffn});
-            ctx->tc_part_cap = (size_t)4 * ctx->sms * kTcM * ctx->tc_bn_max;
-            ctx->tc_cnt_cap = 4 * ctx->sms;
             TRY(dalloc(ctx, &ctx->tc_xb, (size_t)2 * ctx->tc_bn_max * ctx->tc_kmax * 2));
-            TRY(dalloc(ctx, &ctx->tc_part, ctx->tc_part_cap * 4));
-            TRY(dalloc(ctx, &ctx->tc_cnt, (size_t)ctx->tc_cnt_cap * 4));
-            CK(cudaMemset(ctx->tc_cnt, 0, (size_t)ctx->tc_cnt_cap * 4));
         }
         TRY(dalloc(ctx, &ctx->pending, (size_t)MB * 2 * 4));
         TRY(dalloc(ctx, &ctx->n_pos, (size_t)MB * 4));
@@ -1510,21 +1519,8 @@ pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N
 }  // extern "C"
 
 namespace {
-struct TcScratch {
-    size_t xb, part, cnt, total;  // byte offsets of the parts, total bytes
-    int splits;
-};
-
-TcScratch tc_scratch_plan(int sms, int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits) {
-    const int rows = N * (mode == 1 ? 2 : 1), bn = tc_bn(B), tiles = (rows + kTcM - 1) / kTcM, nkb = K / kTcBK;
-    TcScratch t{};
-    t.splits = splits > 0 ? std::min<int>(splits, nkb) : tc_auto_splits(sms, bn, tiles, nkb);
-    t.xb = 0;
-    t.part = ((size_t)2 * bn * K * 2 + 1023) / 1024 * 1024;
-    t.cnt = t.part + (t.splits > 1 ? (size_t)t.splits * rows * bn * 4 : 0);
-    t.total = t.cnt + (size_t)tiles * 4;
-    return t;
-}
+// scratch of pipo_op_gemm_tc: the [2 * BH][K] bf16 activation tile
+size_t tc_scratch_bytes(int32_t K, int32_t B) { return (size_t)2 * tc_bn(B) * K * 2; }
 
 bool tc_op_args_ok(int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits) {
     return (mode == 0 || mode == 1) && N >= 1 && N * (mode == 1 ? 2 : 1) >= kTcM && K >= kTcBK && K % kTcBK == 0 &&
@@ -1536,13 +1532,7 @@ extern "C" {
 
 size_t pipo_op_gemm_tc_scratch(int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits) {
     if (!tc_op_args_ok(mode, N, K, B, splits)) return 0;
-    int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
-        cudaGetLastError();
-        return 0;
-    }
-    return tc_scratch_plan(sms, mode, N, K, B, splits).total;
+    return tc_scratch_bytes(K, B);
 }
 
 pipo_status pipo_op_gemm_tc(int32_t mode, const void* d_W, int32_t N, int32_t K, const float* d_x, int32_t B,
@@ -1554,24 +1544,15 @@ pipo_status pipo_op_gemm_tc(int32_t mode, const void* d_W, int32_t N, int32_t K,
     pipo_ctx* ctx = &op;
     pipo_status st = op_setup(op, 1, stream);
     if (st == PIPO_OK) {
-        const TcScratch t = tc_scratch_plan(op.sms, mode, N, K, B, splits);
-        if (scratch_bytes < t.total) {
-            st = fail(ctx, PIPO_EINVAL, "pipo_op_gemm_tc: scratch needs %zu bytes, got %zu", t.total, scratch_bytes);
+        const size_t need = tc_scratch_bytes(K, B);
+        if (scratch_bytes < need) {
+            st = fail(ctx, PIPO_EINVAL, "pipo_op_gemm_tc: scratch needs %zu bytes, got %zu", need, scratch_bytes);
         } else {
-            char* base = static_cast<char*>(d_scratch);
-            const int tiles = (N * (mode == 1 ? 2 : 1) + kTcM - 1) / kTcM;
-            cudaError_t e = cudaMemsetAsync(base + t.cnt, 0, (size_t)tiles * 4, op.stream);
-            if (e != cudaSuccess) {
-                st = fail(ctx, PIPO_ECUDA, "cudaMemsetAsync: %s", cudaGetErrorString(e));
-            } else {
-                GemvParams p{};
-                p.W = d_W; p.N = N; p.K = K; p.epi = mode == 1 ? EPI_SWIGLU : EPI_STORE;
-                p.y = d_y; p.ldy = N; p.B = B; p.splitk = 1; p.nseg = 1;
-                p.seg[0] = act_seg(d_x, K, K);
-                st = launch_gemm_tc(ctx, p, reinterpret_cast<bf16*>(base + t.xb), reinterpret_cast<float*>(base + t.part),
-                                    t.splits > 1 ? (size_t)t.splits * N * (mode == 1 ? 2 : 1) * tc_bn(B) : 0,
-                                    reinterpret_cast<unsigned*>(base + t.cnt), tiles, t.splits);
-            }
+            GemvParams p{};
+            p.W = d_W; p.N = N; p.K = K; p.epi = mode == 1 ? EPI_SWIGLU : EPI_STORE;
+            p.y = d_y; p.ldy = N; p.B = B; p.splitk = 1; p.nseg = 1;
+            p.seg[0] = act_seg(d_x, K, K);
+            st = launch_gemm_tc(ctx, p, static_cast<bf16*>(d_scratch), splits);
         }
     }
     if (st != PIPO_OK) g_init_error = op.err;

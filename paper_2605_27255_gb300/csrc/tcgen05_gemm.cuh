@@ -5,13 +5,15 @@
 // cores.  Swap-AB: D[rows, B] = W[rows, K] . X[B, K]^T, so the 128 weight rows
 // of a tile fill the MMA's M = 128 and the batch (padded to a multiple of 16)
 // is its N.  Both operands are K-major bf16 tiles loaded by TMA tensor copies
-// with 128-byte swizzle into a 4-stage shared-memory ring (mbarrier
-// completion).  One thread issues the copies, one thread issues
-// tcgen05.mma.cta_group::1.kind::f16 (fp32 accumulation in TMEM), and four
-// warps read the accumulator back with tcgen05.ld for the epilogue.  A CTA
-// owns one (128-row tile, K split); when there are fewer tiles than SMs, K is
-// split and the last CTA of a tile to finish adds the fp32 partials in split
-// order (deterministic) and applies the epilogue.
+// with 128-byte swizzle into a shared-memory ring of ST stages (mbarrier
+// completion; ST chosen so that two CTAs fit on an SM).  One thread issues the
+// copies, one thread issues tcgen05.mma.cta_group::1.kind::f16 (fp32
+// accumulation in TMEM), and four warps read the accumulator back with
+// tcgen05.ld for the epilogue.  A CTA owns one (128-row tile, K split).  When
+// there are fewer tiles than SM slots, K is split over the CTAs of a thread-
+// block cluster: each parks its partial tile in its own shared memory, and
+// CTA s adds the rows of slice s over the cluster through distributed shared
+// memory in split order (deterministic), then applies the epilogue to them.
 //
 // The activations enter as two bf16 parts, x = hi + lo with hi = bf16(x) and
 // lo = bf16(x - hi) (prep_bf16_kernel, after the RMSNorm / gather of the GEMV
@@ -22,6 +24,7 @@
 // (error word + drain, no hang).
 #pragma once
 
+#include <cooperative_groups.h>
 #include <cuda.h>
 
 #include "kernels.cuh"
@@ -31,9 +34,12 @@ namespace pipo {
 
 constexpr int kTcM = 128;                   // weight rows per tile (MMA M)
 constexpr int kTcBK = 64;                   // bf16 K per stage: 128-byte rows
-constexpr int kTcStages = 4;
 constexpr int kTcThreads = 128;
 constexpr int kTcABytes = kTcM * kTcBK * 2;  // 16 KB per stage
+constexpr int kTcMaxSplits = 8;             // portable cluster size
+
+// operand stages per batch width BH: about 100 KB of shared memory, two CTAs per SM
+__host__ __device__ constexpr int tc_stages(int bh) { return bh <= 16 ? 5 : bh <= 32 ? 4 : bh <= 64 ? 3 : 2; }
 
 struct TcParams {
     int rows;            // W rows (output units * ru)
@@ -47,9 +53,7 @@ struct TcParams {
     unsigned long long* am;
     float* dbg;
     int ld_dbg;
-    int splits;          // K splits per tile
-    float* part;         // [splits][rows][BH] fp32 partials (splits > 1)
-    unsigned* cnt;       // [tiles] arrival counters, zero between launches
+    int splits;          // K splits per tile = cluster size (1 .. kTcMaxSplits)
 };
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, int x, int y, uint64_t* bar) {
@@ -167,27 +171,77 @@ __device__ __forceinline__ void tc_epilogue16(const TcParams& p, int row, int c0
     }
 }
 
-// BH: batch columns (a multiple of 16, >= B); the MMA N is 2 * BH (hi | lo).
+// float index of float4 group c4 of row r in a [128][BH] fp32 tile parked in
+// shared memory: groups XOR-swizzled by row (conflict-free row-wise stores)
 template <int BH>
+__device__ __forceinline__ int tc_park_idx(int r, int c4) {
+    constexpr int NC4 = BH / 4;
+    return r * BH + ((c4 ^ (r & (NC4 - 1))) << 2);
+}
+
+// Split-K epilogue of 4 batch columns [4*c4, 4*c4+4) of tile row rr (and, for
+// SwiGLU, its up row rr+1), summed over the cluster in split order.
+template <int BH>
+__device__ __forceinline__ void tc_cluster_epilogue(const TcParams& p, cooperative_groups::cluster_group& cl,
+                                                    float* park, int tile, int rr, int c4) {
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f), u = a;
+    for (int s = 0; s < p.splits; ++s) {
+        const float* rem = cl.map_shared_rank(park, s);
+        const float4 t = *reinterpret_cast<const float4*>(rem + tc_park_idx<BH>(rr, c4));
+        a.x += t.x; a.y += t.y; a.z += t.z; a.w += t.w;
+        if (p.ru == 2) {
+            const float4 t2 = *reinterpret_cast<const float4*>(rem + tc_park_idx<BH>(rr + 1, c4));
+            u.x += t2.x; u.y += t2.y; u.z += t2.z; u.w += t2.w;
+        }
+    }
+    const float va[4] = {a.x, a.y, a.z, a.w}, vu[4] = {u.x, u.y, u.z, u.w};
+    const int row = tile * kTcM + rr;
+    if (row >= p.rows) return;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const int b = 4 * c4 + j;
+        if (b >= p.B) break;
+        if (p.ru == 2) {
+            p.y[(size_t)b * p.ldy + (row >> 1)] = silu(va[j]) * vu[j];
+            continue;
+        }
+        float* yp = p.y + (size_t)b * p.ldy + row;
+        switch (p.epi) {
+            case EPI_STORE: *yp = va[j]; break;
+            case EPI_BIAS: *yp = va[j] + __bfloat162float(static_cast<const __nv_bfloat16*>(p.bias)[row]); break;
+            case EPI_SILU: *yp = silu(va[j]); break;
+            case EPI_RESADD: *yp += va[j]; break;
+            case EPI_ARGMAX:
+                if (p.dbg) p.dbg[(size_t)b * p.ld_dbg + row] = va[j];
+                atomicMax(p.am + b, argmax_key(va[j], row));
+                break;
+            default: break;
+        }
+    }
+}
+
+// BH: batch columns (a multiple of 16, >= B); the MMA N is 2 * BH (hi | lo).
+// ST: operand stages.  Launched with cluster size p.splits when p.splits > 1.
+template <int BH, int ST>
 __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_constant__ CUtensorMap tmW,
                                                                 const __grid_constant__ CUtensorMap tmX, TcParams p) {
     extern __shared__ __align__(1024) unsigned char tc_smem_raw[];
     constexpr int BN = 2 * BH;
     constexpr int kBBytes = BN * kTcBK * 2;
     constexpr uint32_t kCols = BN <= 32 ? 32u : BN <= 64 ? 64u : BN <= 128 ? 128u : 256u;
+    static_assert(kTcM * BH * 4 <= ST * (kTcABytes + kBBytes), "parked tile must fit in the operand stages");
     unsigned char* sm = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~(uintptr_t)1023);
     unsigned char* sA = sm;
-    unsigned char* sB = sm + kTcStages * kTcABytes;
-    uint64_t* full = reinterpret_cast<uint64_t*>(sB + kTcStages * kBBytes);
-    uint64_t* empty = full + kTcStages;
-    uint64_t* accb = empty + kTcStages;
+    unsigned char* sB = sm + ST * kTcABytes;
+    uint64_t* full = reinterpret_cast<uint64_t*>(sB + ST * kBBytes);
+    uint64_t* empty = full + ST;
+    uint64_t* accb = empty + ST;
     __shared__ uint32_t tmem_base;
     __shared__ float red_v[4][BH];
     __shared__ int red_r[4][BH];
-    __shared__ int last;
 
     pdl_launch();
-    const int warp = threadIdx.x >> 5;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tile = blockIdx.x / p.splits, split = blockIdx.x % p.splits;
     const int nkb = p.K / kTcBK;
     const int kb0 = (int)((long long)split * nkb / p.splits), kb1 = (int)((long long)(split + 1) * nkb / p.splits);
@@ -195,7 +249,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
 
     if (warp == 0) tmem_alloc(&tmem_base, kCols);
     if (threadIdx.x == 32) {
-        for (int s = 0; s < kTcStages; ++s) {
+        for (int s = 0; s < ST; ++s) {
             mbar_init(full + s, 1);
             mbar_init(empty + s, 1);
         }
@@ -207,7 +261,6 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
     tc_fence_after();
     const uint32_t tmem = tmem_base;
 
-    const int lane = threadIdx.x & 31;
     if (warp == 0) {
         if (lane == 0) {
             // TMA producer: weight tiles need nothing from the previous
@@ -215,8 +268,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
             // dependent launch)
             int issued = 0;
             for (int i = 0; i < nk; ++i) {
-                const int s = i % kTcStages;
-                if (i >= kTcStages && !mbar_wait(empty + s, (uint32_t)(((i / kTcStages) & 1) ^ 1))) break;
+                const int s = i % ST;
+                if (i >= ST && !mbar_wait(empty + s, (uint32_t)(((i / ST) & 1) ^ 1))) break;
                 mbar_arrive_expect_tx(full + s, (uint32_t)(kTcABytes + kBBytes));
                 tma_load_2d(sA + s * kTcABytes, &tmW, (kb0 + i) * kTcBK, tile * kTcM, full + s);
                 if (i == 0) pdl_wait();
@@ -224,8 +277,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
                 issued = i + 1;
             }
             // no copy into this CTA's shared memory may still be in flight at exit
-            for (int i = max(0, issued - kTcStages); i < issued; ++i)
-                mbar_wait(full + (i % kTcStages), (uint32_t)((i / kTcStages) & 1));
+            for (int i = max(0, issued - ST); i < issued; ++i) mbar_wait(full + (i % ST), (uint32_t)((i / ST) & 1));
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -234,8 +286,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
             // descriptors advanced by 32 bytes inside the swizzled rows
             const uint32_t idesc = umma_idesc_bf16(kTcM, BN);
             for (int i = 0; i < nk; ++i) {
-                const int s = i % kTcStages;
-                if (!mbar_wait(full + s, (uint32_t)((i / kTcStages) & 1))) break;
+                const int s = i % ST;
+                if (!mbar_wait(full + s, (uint32_t)((i / ST) & 1))) break;
                 tc_fence_after();
                 const uint32_t a0 = smem_u32(sA + s * kTcABytes), b0 = smem_u32(sB + s * kBBytes);
 #pragma unroll
@@ -271,57 +323,45 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
             ld_cols(c0, v);
             tc_epilogue16<BH>(p, row, c0, v, red_v, red_r);
         }
+        if (p.epi == EPI_ARGMAX) {
+            __syncthreads();
+            if (threadIdx.x < p.B) {
+                const int b = threadIdx.x;
+                float bv = -INFINITY;
+                int br = 0x7fffffff;
+                for (int w = 0; w < 4; ++w)
+                    if (red_r[w][b] != 0x7fffffff && (red_v[w][b] > bv || (red_v[w][b] == bv && red_r[w][b] < br))) {
+                        bv = red_v[w][b];
+                        br = red_r[w][b];
+                    }
+                if (br != 0x7fffffff) atomicMax(p.am + b, argmax_key(bv, br));
+            }
+        }
     } else {
-        // tcgen05.ld is warp-collective: every lane loads, only rows in range store
-        float* dst = p.part + ((size_t)split * p.rows + min(row, p.rows - 1)) * BH;
+        // park this split's partial tile in the (now idle) operand stages
+        namespace cg = cooperative_groups;
+        cg::cluster_group cl = cg::this_cluster();
+        float* park = reinterpret_cast<float*>(sm);
 #pragma unroll 1
         for (int c0 = 0; c0 < BH; c0 += 16) {
             float v[16];
             ld_cols(c0, v);
-            if (row < p.rows) {
 #pragma unroll
-                for (int j = 0; j < 16; j += 4)
-                    *reinterpret_cast<float4*>(dst + c0 + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
-            }
+            for (int q = 0; q < 4; ++q)
+                *reinterpret_cast<float4*>(park + tc_park_idx<BH>(threadIdx.x, c0 / 4 + q)) =
+                    make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
-        __threadfence();
-        __syncthreads();
-        if (threadIdx.x == 0) last = (atomicAdd(p.cnt + tile, 1u) == (unsigned)p.splits - 1);
-        __syncthreads();
-        if (last) {
-            __threadfence();
-#pragma unroll 1
-            for (int c0 = 0; c0 < BH; c0 += 16) {
-                float v[16];
-#pragma unroll
-                for (int j = 0; j < 16; ++j) v[j] = 0.f;
-                if (row < p.rows)
-                    for (int s = 0; s < p.splits; ++s) {
-                        const float* src = p.part + ((size_t)s * p.rows + row) * BH + c0;
-#pragma unroll
-                        for (int j = 0; j < 16; j += 4) {
-                            const float4 t = __ldcg(reinterpret_cast<const float4*>(src + j));
-                            v[j] += t.x; v[j + 1] += t.y; v[j + 2] += t.z; v[j + 3] += t.w;
-                        }
-                    }
-                tc_epilogue16<BH>(p, row, c0, v, red_v, red_r);
-            }
-            if (threadIdx.x == 0) p.cnt[tile] = 0u;
+        cl.sync();  // every split's partial is parked
+        // rows [r0, r1) of the tile are this CTA's: an even count (SwiGLU pairs)
+        const int R = (((kTcM + p.splits - 1) / p.splits) + 1) & ~1;
+        const int r0 = min(kTcM, split * R), r1 = min(kTcM, r0 + R);
+        const int step = p.ru == 2 ? 2 : 1;
+        const int items = (r1 - r0) / step * (BH / 4);
+        for (int it = threadIdx.x; it < items; it += kTcThreads) {
+            const int rr = r0 + (it / (BH / 4)) * step, c4 = it % (BH / 4);
+            tc_cluster_epilogue<BH>(p, cl, park, tile, rr, c4);
         }
-    }
-    if (p.epi == EPI_ARGMAX && (p.splits == 1 || last)) {
-        __syncthreads();
-        if (threadIdx.x < p.B) {
-            const int b = threadIdx.x;
-            float bv = -INFINITY;
-            int br = 0x7fffffff;
-            for (int w = 0; w < 4; ++w)
-                if (red_r[w][b] != 0x7fffffff && (red_v[w][b] > bv || (red_v[w][b] == bv && red_r[w][b] < br))) {
-                    bv = red_v[w][b];
-                    br = red_r[w][b];
-                }
-            if (br != 0x7fffffff) atomicMax(p.am + b, argmax_key(bv, br));
-        }
+        cl.sync();  // no CTA leaves while others still read its shared memory
     }
     tc_fence_before();
     __syncthreads();

@@ -202,8 +202,8 @@ PIPO_API pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void *d_W, 
  * relative representation error; the weight traffic is that of one pass):
  *   mode 0: y[b*N + r] = sum_k W[r*K + k] * x[b*K + k]              (W: [N, K])
  *   mode 1: SwiGLU as in pipo_op_gemv (W: [2N, K], gate/up rows interleaved).
- * W bf16, 16-byte aligned; x [B, K] and y [B, N] fp32.  K a multiple of 64,
- * N (mode 1: 2N) >= 128, 1 <= B <= 128.  splits: K splits per 128-row tile,
+ * W bf16, 16-byte aligned; x [B, K] and y [B, N] fp32.  K a multiple of 64
+ * and at most 16384, N (mode 1: 2N) >= 128, 1 <= B <= 128.  splits: K splits per 128-row tile,
  * at most 8 (0 = automatic; larger values are clamped); the splits of a tile
  * are one thread-block cluster and add their partials in split order
  * (deterministic).

@@ -32,6 +32,7 @@ template <typename T> struct KV8;  // 8 consecutive cache elements
 template <> struct KV8<__nv_bfloat16> {
     uint4 v;
     __device__ __forceinline__ void load(const __nv_bfloat16* p) { v = ldg_cg(p); }
+    __device__ __forceinline__ void load_s(const unsigned char* p) { v = *reinterpret_cast<const uint4*>(p); }
     __device__ __forceinline__ void zero() { v = make_uint4(0, 0, 0, 0); }
     __device__ __forceinline__ void to_float(float (&f)[8]) const {
         f[0] = bf_lo(v.x); f[1] = bf_hi(v.x); f[2] = bf_lo(v.y); f[3] = bf_hi(v.y);
@@ -43,6 +44,10 @@ template <> struct KV8<float> {
     __device__ __forceinline__ void load(const float* p) {
         a = ldg_cg(p);
         b = ldg_cg(p + 4);
+    }
+    __device__ __forceinline__ void load_s(const unsigned char* p) {
+        a = *reinterpret_cast<const uint4*>(p);
+        b = *reinterpret_cast<const uint4*>(p + 16);
     }
     __device__ __forceinline__ void zero() { a = b = make_uint4(0, 0, 0, 0); }
     __device__ __forceinline__ void to_float(float (&f)[8]) const {

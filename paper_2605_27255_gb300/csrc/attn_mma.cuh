@@ -1,0 +1,356 @@
+// Split-KV GQA flash-decode on the tensor cores (mma.sync m16n8k16, bf16 in,
+// fp32 accumulate) with the keys and values streamed into shared memory by
+// bulk asynchronous copies (sm_103a; bf16 cache, d_h = 128).
+//
+// One thread-block cluster of CS CTAs per (sequence, kv head), as in
+// attn_cluster_kernel: CTA s owns a contiguous slice of the entries 0..n
+// (entry n is this step's new key/value, which the CTA owning it rotates,
+// rounds to bf16, appends and attends to); the CS partial softmax states are
+// merged through distributed shared memory.
+//
+// Per CTA: a producer thread copies aligned 16-entry groups of the slice into
+// a ring of kMmaStages stages with TMA tensor copies: the cache layer is a 2-D
+// tensor of rows (block, kv head, slot) x d_h bf16, and a group is four boxes
+// of 16 rows x 64 dims (K and V, two halves each) stored with the 128-byte
+// swizzle, which keeps the ldmatrix reads free of bank conflicts.  Four
+// compute warps take the groups in turn.  For a group:
+//   S = Q K^T    A = Q: rows 0..G-1 the bf16 part of the G query heads of
+//                this kv head (rotated, pre-scaled by 1/sqrt(d_h)), rows
+//                G..2G-1 the bf16 remainder q - bf16(q); B = K from ldmatrix.
+//                Score of head h = row h + row h+G (fp32-accurate).
+//   online softmax per head on the accumulator fragments;
+//   O += P V     A = P in the same hi / lo row split (the accumulator layout
+//                of S is the A-fragment layout of P), B = V (ldmatrix.trans).
+// About six warp instructions per cached entry, against ~160 for the
+// CUDA-core kernels, so the kernel streams the cache at memory rate.
+// Entries of a group outside the slice are masked (p = 0; the cache holds
+// only finite values).  Every wait is bounded (error word, shared abort flag).
+#pragma once
+
+#include "attn_cluster.cuh"
+#include "tma.cuh"
+
+namespace pipo {
+
+constexpr int kMmaDH = 128;
+constexpr int kMmaRun = 16;                         // entries per group
+constexpr int kMmaHalf = kMmaRun * 128;             // one box: 16 rows x 64 dims bf16 (2 KB)
+constexpr int kMmaStageBytes = 4 * kMmaHalf;        // K (2 halves) + V (2 halves)
+constexpr int kMmaStages = 10;
+constexpr int kMmaWarps = 4;                        // compute warps
+constexpr int kMmaThreads = (kMmaWarps + 1) * 32;   // + the producer warp
+
+constexpr size_t mma_attn_smem() { return 1024 + (size_t)kMmaStages * kMmaStageBytes + 2 * kMmaStages * 8; }
+
+// byte offset of 8-dim chunk c (0..15) of row `row` (0..15) of a K or V tile:
+// two 64-dim halves of 16 x 128 bytes, 16-byte chunks XOR-swizzled by row % 8
+__device__ __forceinline__ uint32_t mma_tile_off(int row, int c) {
+    return (uint32_t)((c >> 3) * kMmaHalf + row * 128 + (((c & 7) ^ (row & 7)) << 4));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo_col, float hi_col) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(lo_col, hi_col);
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+__device__ __forceinline__ float bf16_rest(float x) { return x - __bfloat162float(__float2bfloat16_rn(x)); }
+
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+// D += A B with A rows 8..15 zero (a1 = a3 = 0)
+__device__ __forceinline__ void mma_rows8(float (&d)[4], uint32_t a0, uint32_t a2, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+}
+
+// tmK, tmV: this layer's K and V cache as [blocks * n_kv * page][d_h] bf16,
+// boxes of 64 dims x 16 rows, 128-byte swizzle
+template <int G>
+__global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, const __grid_constant__ CUtensorMap tmK,
+                                                               const __grid_constant__ CUtensorMap tmV) {
+    static_assert(G == 1 || G == 2 || G == 4, "2G query rows must fit the 8 live MMA rows");
+    constexpr int DH = kMmaDH;
+    constexpr int NW = kMmaWarps;
+    constexpr int NP = NW + 1;  // softmax partials: one per compute warp + the new entry
+    extern __shared__ __align__(1024) unsigned char am_smem_raw[];
+    __shared__ float qs[G][DH];       // rotated, pre-scaled queries (fp32)
+    __shared__ float kn_s[DH], vn_s[DH];  // the new entry, rounded to bf16
+    __shared__ float sm_o[G][DH];
+    __shared__ float sm_m[G], sm_l[G];
+    __shared__ float wm[NP][G], wl[NP][G];
+    __shared__ float wo[NP][G][DH];
+    __shared__ int abort_flag;
+
+    unsigned char* ring = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(am_smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)kMmaStages * kMmaStageBytes);
+    uint64_t* empty = full + kMmaStages;
+
+    pdl_launch();
+    cg::cluster_group cluster = cg::this_cluster();
+    const int s = (int)cluster.block_rank();
+    const int CS = (int)cluster.num_blocks();
+    const int g = blockIdx.y, b = blockIdx.z;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_kv = p.kv.n_kv, n_q = n_kv * G;
+    const int n = p.n_pos[b];          // cached entries; entry n is new
+    const int len = n + 1;
+    const int chunk = (len + CS - 1) / CS;
+    const int j0 = s * chunk, j1 = min(len, j0 + chunk);
+    const int jc = min(j1, n);         // cached part of the slice: [j0, jc)
+    const int grp0 = j0 / kMmaRun;
+    const int ngrp = jc > j0 ? (jc - 1) / kMmaRun - grp0 + 1 : 0;
+    const bool owns_new = n >= j0 && n < j1;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kMmaStages; ++i) {
+            mbar_init(full + i, 1);
+            mbar_init(empty + i, 1);
+        }
+        abort_flag = 0;
+        mbar_init_fence();
+    }
+    __syncthreads();
+
+    if (warp == NW) {
+        // ---- producer: whole 16-entry groups (earlier steps wrote them, so
+        // the copies start before the dependency wait)
+        if (lane == 0) {
+            int t = 0;
+            for (; t < ngrp; ++t) {
+                const int st = t % kMmaStages;
+                if (t >= kMmaStages && (*(volatile int*)&abort_flag ||
+                                        !mbar_wait(empty + st, (uint32_t)(((t / kMmaStages) & 1) ^ 1)))) {
+                    *(volatile int*)&abort_flag = 1;
+                    break;
+                }
+                const int e = (grp0 + t) * kMmaRun;  // a group never crosses a page
+                const int blk = p.kv.table[(size_t)b * p.kv.blocks_per_seq + e / p.kv.page];
+                const int row = (blk * n_kv + g) * p.kv.page + e % p.kv.page;
+                unsigned char* stg = ring + (size_t)st * kMmaStageBytes;
+                mbar_arrive_expect_tx(full + st, (uint32_t)kMmaStageBytes);
+                tma_load_2d(stg, &tmK, 0, row, full + st);
+                tma_load_2d(stg + kMmaHalf, &tmK, 64, row, full + st);
+                tma_load_2d(stg + 2 * kMmaHalf, &tmV, 0, row, full + st);
+                tma_load_2d(stg + 3 * kMmaHalf, &tmV, 64, row, full + st);
+            }
+            // no copy into this CTA's shared memory may still be in flight at exit
+            for (int i = max(0, t - kMmaStages); i < t; ++i)
+                mbar_wait(full + (i % kMmaStages), (uint32_t)((i / kMmaStages) & 1));
+        }
+        __syncwarp();
+    } else {
+        const int ct = threadIdx.x;  // 0 .. 32*NW-1
+        // ---- prologue: rotated, pre-scaled q of the G heads; the new k, v
+        pdl_wait();
+        const float* qrow = p.qkv + (size_t)b * p.ld_qkv;
+        const float* rope = p.rope + (size_t)n * DH;  // [DH/2][2] cos, sin at position n
+        for (int i = ct; i < (G + 1) * (DH / 2); i += 32 * NW) {
+            const int h = i / (DH / 2), pr = i % (DH / 2);
+            const float c = rope[2 * pr], sn = rope[2 * pr + 1];
+            if (h < G) {
+                const float* q = qrow + (size_t)(g * G + h) * DH;
+                const float x1 = q[pr], x2 = q[pr + DH / 2];
+                qs[h][pr] = (x1 * c - x2 * sn) * p.scale;
+                qs[h][pr + DH / 2] = (x2 * c + x1 * sn) * p.scale;
+            } else if (owns_new) {
+                const float* k = qrow + (size_t)(n_q + g) * DH;
+                const float x1 = k[pr], x2 = k[pr + DH / 2];
+                kn_s[pr] = __bfloat162float(__float2bfloat16_rn(x1 * c - x2 * sn));
+                kn_s[pr + DH / 2] = __bfloat162float(__float2bfloat16_rn(x2 * c + x1 * sn));
+            }
+        }
+        if (owns_new)
+            for (int d = ct; d < DH; d += 32 * NW)
+                vn_s[d] = __bfloat162float(__float2bfloat16_rn(qrow[(size_t)(n_q + n_kv + g) * DH + d]));
+        asm volatile("bar.sync 1, %0;" ::"n"(32 * NW) : "memory");  // compute warps only
+
+        // the new entry: append it to the cache and make it partial NW
+        if (owns_new) {
+            const size_t off = kv_off<__nv_bfloat16, DH>(p.kv, b, n, g);
+            __nv_bfloat16* Kw = static_cast<__nv_bfloat16*>(p.kv.K) + off;
+            __nv_bfloat16* Vw = static_cast<__nv_bfloat16*>(p.kv.V) + off;
+            for (int d = ct; d < DH; d += 32 * NW) {
+                Kw[d] = __float2bfloat16_rn(kn_s[d]);
+                Vw[d] = __float2bfloat16_rn(vn_s[d]);
+            }
+        }
+        if (warp < G) {
+            const int h = warp;
+            float dsum = 0.f;
+            for (int d = lane; d < DH; d += 32) dsum += qs[h][d] * kn_s[d];
+            dsum = warp_sum(dsum);
+            for (int d = lane; d < DH; d += 32) wo[NW][h][d] = owns_new ? vn_s[d] : 0.f;
+            if (lane == 0) {
+                wm[NW][h] = owns_new ? dsum : -INFINITY;
+                wl[NW][h] = owns_new ? 1.f : 0.f;
+            }
+        }
+
+        // ---- A fragments of Q: row r = lane / 4 (hi part for r < G, remainder for r < 2G)
+        const int r = lane >> 2, tq = lane & 3;
+        uint32_t qa[DH / 16][2];
+#pragma unroll
+        for (int kc = 0; kc < DH / 16; ++kc) {
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                const int d0 = kc * 16 + half * 8 + 2 * tq;
+                float x0 = 0.f, x1 = 0.f;
+                if (r < G) {
+                    x0 = qs[r][d0];
+                    x1 = qs[r][d0 + 1];
+                } else if (r < 2 * G) {
+                    x0 = bf16_rest(qs[r - G][d0]);
+                    x1 = bf16_rest(qs[r - G][d0 + 1]);
+                }
+                qa[kc][half] = pack_bf16x2(x0, x1);
+            }
+        }
+
+        float o[DH / 8][4];
+#pragma unroll
+        for (int nd = 0; nd < DH / 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+        float m_run = -INFINITY, l_run = 0.f;
+        const int lm = lane >> 3, lr = lane & 7;  // ldmatrix: matrix index, row within it
+
+        for (int t = warp; t < ngrp; t += NW) {
+            const int st = t % kMmaStages;
+            if (*(volatile int*)&abort_flag || !mbar_wait(full + st, (uint32_t)((t / kMmaStages) & 1))) {
+                *(volatile int*)&abort_flag = 1;
+                break;
+            }
+            const uint32_t kS = smem_u32(ring + (size_t)st * kMmaStageBytes);
+            const uint32_t vS = kS + 2 * kMmaHalf;
+            const int e0 = (grp0 + t) * kMmaRun;
+            const int lo = max(j0, e0) - e0, hi = min(jc, e0 + kMmaRun) - e0;  // valid entries [lo, hi)
+
+            // S = Q K^T: two n-tiles of 8 entries, 8 k-chunks of 16 dims
+            float sacc[2][4];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                sacc[nt][0] = sacc[nt][1] = sacc[nt][2] = sacc[nt][3] = 0.f;
+#pragma unroll
+                for (int kc2 = 0; kc2 < DH / 32; ++kc2) {
+                    uint32_t bk[4];
+                    ldsm_x4(bk, kS + mma_tile_off(nt * 8 + lr, 4 * kc2 + 2 * (lm >> 1) + (lm & 1)));
+                    mma_rows8(sacc[nt], qa[kc2 * 2][0], qa[kc2 * 2][1], bk[0], bk[1]);
+                    mma_rows8(sacc[nt], qa[kc2 * 2 + 1][0], qa[kc2 * 2 + 1][1], bk[2], bk[3]);
+                }
+            }
+            // score of (head r mod G, entry nt*8 + 2tq + j): bf16 row + remainder row
+            float sv[2][2];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int j = 0; j < 2; ++j) {
+                    const float v = sacc[nt][j] + __shfl_xor_sync(0xffffffffu, sacc[nt][j], 4 * G);
+                    const int e = nt * 8 + 2 * tq + j;
+                    sv[nt][j] = (e >= lo && e < hi) ? v : -INFINITY;
+                }
+            float rmax = fmaxf(fmaxf(sv[0][0], sv[0][1]), fmaxf(sv[1][0], sv[1][1]));
+            rmax = fmaxf(rmax, __shfl_xor_sync(0xffffffffu, rmax, 1));
+            rmax = fmaxf(rmax, __shfl_xor_sync(0xffffffffu, rmax, 2));
+            const float m_new = fmaxf(m_run, rmax);
+            const float corr = (m_run == -INFINITY) ? 0.f : expf(m_run - m_new);
+            float pv[2][2], rsum = 0.f;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int j = 0; j < 2; ++j) {
+                    pv[nt][j] = (sv[nt][j] == -INFINITY) ? 0.f : expf(sv[nt][j] - m_new);
+                    rsum += pv[nt][j];
+                }
+            rsum += __shfl_xor_sync(0xffffffffu, rsum, 1);
+            rsum += __shfl_xor_sync(0xffffffffu, rsum, 2);
+            l_run = l_run * corr + rsum;
+            m_run = m_new;
+#pragma unroll
+            for (int nd = 0; nd < DH / 8; ++nd) {
+                o[nd][0] *= corr;
+                o[nd][1] *= corr;
+            }
+            // A fragments of P: k = entry; bf16 part in rows < G, remainder in rows G..2G-1
+            uint32_t pa0, pa2;
+            if (r < G) {
+                pa0 = pack_bf16x2(pv[0][0], pv[0][1]);
+                pa2 = pack_bf16x2(pv[1][0], pv[1][1]);
+            } else if (r < 2 * G) {
+                pa0 = pack_bf16x2(bf16_rest(pv[0][0]), bf16_rest(pv[0][1]));
+                pa2 = pack_bf16x2(bf16_rest(pv[1][0]), bf16_rest(pv[1][1]));
+            } else {
+                pa0 = pa2 = 0u;
+            }
+            // O += P V: 16 n-tiles of 8 dims
+#pragma unroll
+            for (int nd2 = 0; nd2 < DH / 16; ++nd2) {
+                uint32_t bv[4];
+                ldsm_x4_t(bv, vS + mma_tile_off(lr + (lm & 1) * 8, nd2 * 2 + (lm >> 1)));
+                mma_rows8(o[nd2 * 2], pa0, pa2, bv[0], bv[1]);
+                mma_rows8(o[nd2 * 2 + 1], pa0, pa2, bv[2], bv[3]);
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty + st);  // this group's stage is free
+        }
+
+        // warp partial: O of head r = bf16-part row r + remainder row r + G
+#pragma unroll
+        for (int nd = 0; nd < DH / 8; ++nd)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                const float v = o[nd][j] + __shfl_xor_sync(0xffffffffu, o[nd][j], 4 * G);
+                if (r < G) wo[warp][r][nd * 8 + 2 * tq + j] = v;
+            }
+        if (r < G && tq == 0) {
+            wm[warp][r] = m_run;
+            wl[warp][r] = l_run;
+        }
+    }
+    __syncthreads();
+    // merge the partials: CTA (m, l, o) in shared memory
+    for (int i = threadIdx.x; i < G * DH; i += blockDim.x) {
+        const int hh = i / DH, t = i % DH;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NP; ++w) M = fmaxf(M, wm[w][hh]);
+        float L = 0.f, Ov = 0.f;
+#pragma unroll
+        for (int w = 0; w < NP; ++w) {
+            const float f = (wm[w][hh] == -INFINITY) ? 0.f : expf(wm[w][hh] - M);
+            L += wl[w][hh] * f;
+            Ov += wo[w][hh][t] * f;
+        }
+        sm_o[hh][t] = Ov;
+        if (t == 0) { sm_m[hh] = M; sm_l[hh] = L; }
+    }
+    cluster.sync();
+    // cluster merge: CTA s finishes dims [s*G*DH/CS, (s+1)*G*DH/CS) of the G heads
+    const int PER = (G * DH + CS - 1) / CS;
+    for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
+        const int hh = i / DH, t = i % DH;
+        float M = -INFINITY;
+        for (int rr = 0; rr < CS; ++rr) M = fmaxf(M, *cluster.map_shared_rank(&sm_m[hh], rr));
+        float L = 0.f, Ov = 0.f;
+        for (int rr = 0; rr < CS; ++rr) {
+            const float mr = *cluster.map_shared_rank(&sm_m[hh], rr);
+            const float f = (mr == -INFINITY) ? 0.f : expf(mr - M);
+            L += *cluster.map_shared_rank(&sm_l[hh], rr) * f;
+            Ov += *cluster.map_shared_rank(&sm_o[hh][t], rr) * f;
+        }
+        p.out[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + t] = Ov / L;
+    }
+    cluster.sync();  // keep every CTA's shared memory alive until all merges read it
+}
+
+}  // namespace pipo

@@ -23,6 +23,7 @@
 #include <vector>
 
 #include "attn_cluster.cuh"
+#include "attn_mma.cuh"
 #include "gemv_stream.cuh"
 #include "kernels.cuh"
 #include "megakernel.cuh"
@@ -72,7 +73,7 @@ struct pipo_ctx {
     // tensor-core projections (bf16, batch >= tc_min_b)
     bf16* tc_xb = nullptr;          // [2 * tc_bn_max][tc_kmax] bf16 activations (hi rows, lo rows)
     int tc_kmax = 0, tc_bn_max = 0;
-    int tc_min_b = 16;
+    int tc_min_b = 4;               // measured: tensor cores ahead of the CUDA-core GEMV from B = 4
     int tc_splits = 0;              // forced K splits (0: automatic)
 
     int32_t *pending = nullptr, *n_pos = nullptr, *out_tokens = nullptr, *out_nacc = nullptr;
@@ -89,8 +90,10 @@ struct pipo_ctx {
     bool pdl = false;                 // programmatic dependent launch (decode graph only)
     bool attn_cs16 = false;           // 16-CTA attention clusters available
     int attn_cs_force = 0;            // (development) fixed attention cluster size
-    int attn_cs_target = 1;           // attention CTAs per SM above which clusters shrink
+    int attn_cs_target = 0;           // attention CTAs per SM above which clusters shrink (0: per kernel)
     bool attn_v0 = false;             // (development) the unclustered attention path
+    bool attn_regs = false;           // register-ring attention instead of the tensor-core one
+    std::vector<CUtensorMap> kv_tm;   // tensor-core attention: K and V tensor map of every cache layer
     bool gemv_tma = false;            // bulk-copy GEMV (else the register-ring GEMV)
     // persistent step kernel: phases recorded from the enqueue code
     std::vector<Phase>* rec = nullptr;  // recording target (nullptr: launch kernels)
@@ -325,6 +328,9 @@ void* pick_tc(int bh) {
     }
 }
 
+bool tc_cluster_spread();
+void* attnm_pick(int G);
+
 cudaError_t set_smem_attrs(bool bf) {
     int dev = 0, optin = 0;
     cudaError_t e0 = cudaGetDevice(&dev);
@@ -351,9 +357,19 @@ cudaError_t set_smem_attrs(bool bf) {
             if (e != cudaSuccess) return e;
         }
     if (bf)
+        for (int g : {1, 2, 4}) {
+            cudaError_t e = cudaFuncSetAttribute(attnm_pick(g), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)mma_attn_smem());
+            if (e != cudaSuccess) return e;
+        }
+    if (bf)
         for (int bn : {16, 32, 64, 128}) {
             cudaError_t e =
                 cudaFuncSetAttribute(pick_tc(bn), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem(bn));
+            if (e != cudaSuccess) return e;
+            e = cudaFuncSetAttribute(pick_tc(bn), cudaFuncAttributeClusterSchedulingPolicyPreference,
+                                     tc_cluster_spread() ? cudaClusterSchedulingPolicySpread
+                                                         : cudaClusterSchedulingPolicyLoadBalancing);
             if (e != cudaSuccess) return e;
         }
     return cudaSuccess;
@@ -398,14 +414,61 @@ int tc_ctas_per_sm(int bn) {
     return std::max(1, (int)(g_smem_optin ? 228 * 1024 / per : 1));
 }
 
+// Cluster placement of the tensor-core GEMM: load-balancing (several CTAs of
+// a cluster may share an SM) unless PIPO_TC_CLUSTER_SPREAD=1.
+bool tc_cluster_spread() {
+    static const bool v = [] {
+        const char* ev = getenv("PIPO_TC_CLUSTER_SPREAD");
+        return ev && ev[0] == '1';
+    }();
+    return v;
+}
+
+// Clusters of `cs` CTAs of the GEMM at batch width bh that can be resident at
+// once on the current device (cudaOccupancyMaxActiveClusters; cached).
+int tc_max_clusters(int bh, int cs) {
+    static std::mutex mu;
+    static std::map<long long, int> cache;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return 0; }
+    const long long key = ((long long)dev << 20) | ((long long)bh << 8) | cs;
+    std::lock_guard<std::mutex> lk(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(cs);
+    lc.blockDim = dim3(kTcThreads);
+    lc.dynamicSmemBytes = tc_smem(bh);
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = cs;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    lc.attrs = at;
+    lc.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, pick_tc(bh), &lc) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+    }
+    cache[key] = n;
+    return n;
+}
+
 // K splits (the cluster size): enough CTAs for every SM's resident slots,
-// each split at least kTcMinKb 64-wide K blocks, at most kTcMaxSplits
+// each split at least kTcMinKb 64-wide K blocks, at most kTcMaxSplits, and
+// no more than fit on the GPU at once as clusters (one wave).
 constexpr int kTcMinKb = 4;
 int tc_auto_splits(int sms, int bn, int tiles, int nkb) {
     const int target = sms * tc_ctas_per_sm(bn);
     if (tiles >= target) return 1;
-    const int s = (target + tiles - 1) / tiles;
-    return std::max(1, std::min({s, nkb / kTcMinKb, kTcMaxSplits}));
+    static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
+    for (int s = std::min({target / tiles, nkb / kTcMinKb, kTcMaxSplits}); s >= 2; --s) {
+        const int mc = tc_max_clusters(bn, s);
+        if (verbose) fprintf(stderr, "[pipo] tc splits: bh=%d tiles=%d nkb=%d s=%d max_clusters=%d\n", bn, tiles, nkb, s, mc);
+        if (mc >= tiles) return s;
+    }
+    return 1;
 }
 
 // Projection on the tensor cores: bf16 activations (prep kernel), then the
@@ -424,7 +487,8 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
         void* args[] = {&pp, &xb, &bh};
         ctx->prof_kind = 2;
         ctx->prof_bytes = 0.0;
-        TRY(launch_ex(ctx, reinterpret_cast<const void*>(&prep_bf16_kernel<bf16>), dim3(bn), dim3(256), 0, args));
+        TRY(launch_ex(ctx, reinterpret_cast<const void*>(&prep_bf16_kernel<bf16>), dim3(bn), dim3(kPrepThreads), 0,
+                      args));
     }
     TcParams tp{};
     tp.rows = rows; tp.K = p.K; tp.B = p.B; tp.ru = ru; tp.epi = p.epi;
@@ -439,7 +503,7 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
 bool tc_eligible(const pipo_ctx* ctx, const GemvParams& p) {
     const int rows = p.N * (p.epi == EPI_SWIGLU ? 2 : 1);
     return ctx->cfg.dtype == 1 && ctx->tc_xb && !ctx->rec && p.B >= ctx->tc_min_b && p.B <= ctx->tc_bn_max &&
-           p.K % kTcBK == 0 && p.K <= ctx->tc_kmax && rows >= kTcM;
+           p.K % kTcBK == 0 && p.K <= ctx->tc_kmax && p.K <= 4 * kPrepQ * kPrepThreads && rows >= kTcM;
 }
 
 pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
@@ -588,6 +652,16 @@ void* attnc_pick(bool bf, int DH, int G) {
     return nullptr;
 }
 
+// tensor-core attention (bf16 cache, d_h = 128, 1, 2 or 4 query heads per kv head)
+void* attnm_pick(int G) {
+    switch (G) {
+        case 1: return reinterpret_cast<void*>(&attn_mma_kernel<1>);
+        case 2: return reinterpret_cast<void*>(&attn_mma_kernel<2>);
+        case 4: return reinterpret_cast<void*>(&attn_mma_kernel<4>);
+        default: return nullptr;
+    }
+}
+
 // Can a 16-CTA cluster of this kernel be scheduled here?  (sets the
 // non-portable cluster attribute; any failure selects 8)
 bool cluster16_ok(bool bf, int DH, int G) {
@@ -632,6 +706,15 @@ KVView kv_view(pipo_ctx* ctx, int layer) {
     return v;
 }
 
+// the tensor-core attention applies: bf16 cache, d_h = 128, G in {1, 2, 4},
+// pages of whole 16-entry groups
+bool attn_mma_ok(const pipo_ctx* ctx) {
+    const pipo_config& c = ctx->cfg;
+    const int G = c.n_q_heads / c.n_kv_heads;
+    return !ctx->attn_regs && c.dtype == 1 && c.head_dim == kMmaDH && (G == 1 || G == 2 || G == 4) &&
+           c.page_size % kMmaRun == 0;
+}
+
 // CTAs per (sequence, kv head) of the clustered attention: 8 while the batch
 // leaves SMs idle (16 where allowed and still under two per SM), fewer as the
 // (sequence, kv head) pairs alone fill the GPU.
@@ -639,8 +722,11 @@ int attn_cluster_size(const pipo_ctx* ctx) {
     if (ctx->attn_cs_force) return ctx->attn_cs_force;
     const long long pairs = (long long)ctx->B * ctx->cfg.n_kv_heads;
     if (ctx->attn_cs16 && pairs * 16 <= 2 * ctx->sms) return 16;
+    // measured best: about two tensor-core attention CTAs per SM (they are
+    // resident two at a time), one register-ring CTA per SM
+    const long long target = ctx->attn_cs_target > 0 ? ctx->attn_cs_target : (attn_mma_ok(ctx) ? 2 : 1);
     int cs = 8;
-    while (cs > 1 && pairs * cs > (long long)ctx->attn_cs_target * ctx->sms) cs >>= 1;
+    while (cs > 1 && pairs * cs > target * ctx->sms) cs >>= 1;
     return cs;
 }
 
@@ -688,8 +774,15 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         ap.scale = 1.0f / sqrtf((float)DH);
         void* args[] = {&ap};
         const int cs = attn_cluster_size(ctx);
-        TRY(launch_ex(ctx, attnc_pick(bf, DH, c.n_q_heads / c.n_kv_heads), dim3(cs, c.n_kv_heads, ctx->B),
-                      dim3(kAttnThreads), 0, args, cs));
+        const int G = c.n_q_heads / c.n_kv_heads;
+        if (attn_mma_ok(ctx) && cs <= 8 && (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers) {
+            void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
+            TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, ctx->B), dim3(kMmaThreads), mma_attn_smem(),
+                          margs, cs));
+        }
+        else
+            TRY(launch_ex(ctx, attnc_pick(bf, DH, G), dim3(cs, c.n_kv_heads, ctx->B), dim3(kAttnThreads), 0, args,
+                          cs));
     } else {
     // RoPE + KV append
     {
@@ -1115,6 +1208,17 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
             CK(cudaMemcpy(ctx->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice));
         }
         if (const char* ev = getenv("PIPO_ATTN_V0")) ctx->attn_v0 = ev[0] == '1';
+        if (const char* ev = getenv("PIPO_ATTN_IMPL")) ctx->attn_regs = strcmp(ev, "regs") == 0;
+        if (attn_mma_ok(ctx)) {
+            // the cache layers as 2-D tensors [blocks * n_kv * page][d_h] for the tensor-core attention
+            const int rows = ctx->num_blocks * c.n_kv_heads * c.page_size;
+            ctx->kv_tm.resize(2 * ctx->n_cache_layers);
+            for (int l = 0; l < ctx->n_cache_layers; ++l) {
+                const KVView v = kv_view(ctx, l);
+                TRY(make_tmap(ctx, &ctx->kv_tm[2 * l], v.K, DH, rows, kMmaRun));
+                TRY(make_tmap(ctx, &ctx->kv_tm[2 * l + 1], v.V, DH, rows, kMmaRun));
+            }
+        }
         // 16-CTA clusters measured slower than 8 at 4B B=1 (2.77 vs 2.55 ms per step): opt-in only
         if (const char* ev = getenv("PIPO_ATTN_CS16"))
             ctx->attn_cs16 = ev[0] == '1' && cluster16_ok(c.dtype == 1, c.head_dim, c.n_q_heads / c.n_kv_heads);
@@ -1524,6 +1628,7 @@ size_t tc_scratch_bytes(int32_t K, int32_t B) { return (size_t)2 * tc_bn(B) * K 
 
 bool tc_op_args_ok(int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits) {
     return (mode == 0 || mode == 1) && N >= 1 && N * (mode == 1 ? 2 : 1) >= kTcM && K >= kTcBK && K % kTcBK == 0 &&
+           K <= 4 * kPrepQ * kPrepThreads &&
            B >= 1 && B <= 128 && splits >= 0;
 }
 }  // namespace

@@ -56,13 +56,6 @@ struct TcParams {
     int splits;          // K splits per tile = cluster size (1 .. kTcMaxSplits)
 };
 
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, int x, int y, uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-            smem_u32(dst)),
-        "l"(tm), "r"(x), "r"(y), "r"(smem_u32(bar))
-        : "memory");
-}
 
 // Shared-memory matrix descriptor: K-major, 128-byte swizzle (8-row groups of
 // 128-byte rows, 1024 B apart), tile base 1024-byte aligned.
@@ -374,70 +367,98 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
 // Activations of the tensor-core GEMM, [2 * BH][K] bf16: row b < B holds
 // hi = bf16(x_b) and row BH + b holds lo = bf16(x_b - hi), where x_b is the
 // (gathered, RMS-normalised) GEMV input of sequence b; rows of b >= B are
-// zero.  grid BH, 256 threads.
+// zero.  grid BH, kPrepThreads threads; one pass: every thread keeps its
+// (at most kPrepQ) groups of 4 inputs in registers between the sum of squares
+// and the write, and all its loads are in flight together.
+constexpr int kPrepThreads = 512;
+constexpr int kPrepQ = 8;  // K <= 4 * kPrepQ * kPrepThreads = 16384
+
 template <typename T>
-__global__ void __launch_bounds__(256) prep_bf16_kernel(GemvParams p, __nv_bfloat16* xb, int BH) {
-    __shared__ float red[8][2];
+__device__ __forceinline__ float4 ld4_any(const void* p, size_t i) {
+    if constexpr (sizeof(T) == 2) {
+        const uint2 u = *reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(p) + i);
+        return make_float4(bf_lo(u.x), bf_hi(u.x), bf_lo(u.y), bf_hi(u.y));
+    } else {
+        return *reinterpret_cast<const float4*>(static_cast<const float*>(p) + i);
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kPrepThreads) prep_bf16_kernel(GemvParams p, __nv_bfloat16* xb, int BH) {
+    __shared__ float red[kPrepThreads / 32][2];
     __shared__ float rstd[2];
-    __shared__ int tok[2];
     pdl_launch();
     pdl_wait();
-    const int b = blockIdx.x, K = p.K, tid = threadIdx.x;
+    const int b = blockIdx.x, K = p.K, K4 = K / 4, tid = threadIdx.x;
     if (p.zero_ptr && b == 0)  // argmax keys of this step (read by later kernels only)
         for (int i = tid; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
-    __nv_bfloat16* dst = xb + (size_t)b * K;
-    __nv_bfloat16* dst_lo = xb + (size_t)(BH + b) * K;
+    uint2* dst = reinterpret_cast<uint2*>(xb + (size_t)b * K);
+    uint2* dst_lo = reinterpret_cast<uint2*>(xb + (size_t)(BH + b) * K);
     if (b >= p.B) {
-        for (int k = tid; k < K; k += blockDim.x) dst[k] = dst_lo[k] = __float2bfloat16_rn(0.f);
+        for (int q = tid; q < K4; q += kPrepThreads) dst[q] = dst_lo[q] = make_uint2(0u, 0u);
         return;
     }
-    if (tid < 2) {
-        int t = 0;
-        if (tid < p.nseg && !p.seg[tid].src) {
-            const Seg& sg = p.seg[tid];
-            t = sg.tok_am ? argmax_row(sg.tok_am[b]) : sg.tok[(size_t)b * sg.tok_ld];
+    const int K0q = p.seg[0].K / 4;
+    int tok[2] = {0, 0};
+#pragma unroll
+    for (int s = 0; s < 2; ++s)
+        if (s < p.nseg && !p.seg[s].src) {
+            const Seg& sg = p.seg[s];
+            tok[s] = sg.tok_am ? argmax_row(sg.tok_am[b]) : sg.tok[(size_t)b * sg.tok_ld];
         }
-        tok[tid] = t;
+    float4 v[kPrepQ];
+    float ss0 = 0.f, ss1 = 0.f;
+#pragma unroll
+    for (int i = 0; i < kPrepQ; ++i) {
+        const int q = tid + i * kPrepThreads;
+        v[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (q < K4) {
+            const int s = q < K0q ? 0 : 1;
+            const Seg& sg = p.seg[s];
+            const size_t kk = (size_t)(s == 0 ? q : q - K0q) * 4;
+            if (sg.src) v[i] = *reinterpret_cast<const float4*>(sg.src + (size_t)b * sg.ld + kk);
+            else v[i] = tok[s] < 0 ? ld4_any<T>(sg.pad, kk) : ld4_any<T>(sg.table, (size_t)tok[s] * sg.K + kk);
+        }
     }
-    __syncthreads();
-    const int K0 = p.seg[0].K;
-    auto val = [&](int k) -> float {
-        const int s = k < K0 ? 0 : 1;
-        const Seg& sg = p.seg[s];
-        const int kk = s == 0 ? k : k - K0;
-        if (sg.src) return sg.src[(size_t)b * sg.ld + kk];
-        return tok[s] < 0 ? ldw<T>(sg.pad, kk) : ldw<T>(sg.table, (size_t)tok[s] * sg.K + kk);
-    };
     const bool norm0 = p.seg[0].gamma != nullptr, norm1 = p.nseg > 1 && p.seg[1].gamma != nullptr;
     if (norm0 || norm1) {
-        float s0 = 0.f, s1 = 0.f;
-        for (int k = tid; k < K; k += blockDim.x) {
-            const float v = val(k);
-            if (p.joint_norm || k < K0) s0 += v * v; else s1 += v * v;
+#pragma unroll
+        for (int i = 0; i < kPrepQ; ++i) {
+            const int q = tid + i * kPrepThreads;
+            const float sq = v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+            if (p.joint_norm || q < K0q) ss0 += sq; else ss1 += sq;
         }
-        s0 = warp_sum(s0);
-        s1 = warp_sum(s1);
-        if ((tid & 31) == 0) { red[tid >> 5][0] = s0; red[tid >> 5][1] = s1; }
+        ss0 = warp_sum(ss0);
+        ss1 = warp_sum(ss1);
+        if ((tid & 31) == 0) { red[tid >> 5][0] = ss0; red[tid >> 5][1] = ss1; }
         __syncthreads();
         if (tid < 2) {
             float t = 0.f;
-            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w][tid];
-            const int len = p.joint_norm ? (tid == 0 ? K : 1) : (tid == 0 ? K0 : (p.nseg > 1 ? p.seg[1].K : 1));
+            for (int w = 0; w < kPrepThreads / 32; ++w) t += red[w][tid];
+            const int len = p.joint_norm ? (tid == 0 ? K : 1) : (tid == 0 ? p.seg[0].K : (p.nseg > 1 ? p.seg[1].K : 1));
             rstd[tid] = 1.0f / sqrtf(t / (float)len + p.eps);
         }
         __syncthreads();
     }
-    for (int k = tid; k < K; k += blockDim.x) {
-        float v = val(k);
-        const int g = (p.joint_norm || k < K0) ? 0 : 1;
+#pragma unroll
+    for (int i = 0; i < kPrepQ; ++i) {
+        const int q = tid + i * kPrepThreads;
+        if (q >= K4) break;
+        float4 x = v[i];
+        const int g = (p.joint_norm || q < K0q) ? 0 : 1;
         const Seg& sg = p.seg[p.joint_norm ? 0 : g];
         if (sg.gamma) {
-            const int kk = (p.joint_norm || g == 0) ? k : k - K0;
-            v *= rstd[g] * ldw<T>(sg.gamma, kk);
+            const size_t kk = (size_t)((p.joint_norm || g == 0) ? q : q - K0q) * 4;
+            const float4 gm = ld4_any<T>(sg.gamma, kk);
+            const float r = rstd[g];
+            x.x *= r * gm.x; x.y *= r * gm.y; x.z *= r * gm.z; x.w *= r * gm.w;
         }
-        const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-        dst[k] = hi;
-        dst_lo[k] = __float2bfloat16_rn(v - __bfloat162float(hi));
+        const __nv_bfloat162 h01 = __floats2bfloat162_rn(x.x, x.y), h23 = __floats2bfloat162_rn(x.z, x.w);
+        const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+        const __nv_bfloat162 l01 = __floats2bfloat162_rn(x.x - f01.x, x.y - f01.y);
+        const __nv_bfloat162 l23 = __floats2bfloat162_rn(x.z - f23.x, x.w - f23.y);
+        dst[q] = make_uint2(*reinterpret_cast<const uint32_t*>(&h01), *reinterpret_cast<const uint32_t*>(&h23));
+        dst_lo[q] = make_uint2(*reinterpret_cast<const uint32_t*>(&l01), *reinterpret_cast<const uint32_t*>(&l23));
     }
 }
 

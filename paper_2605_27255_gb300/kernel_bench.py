@@ -1,6 +1,8 @@
-"""Time one decode-path kernel in isolation through the C ABI (pipo_op_gemv).
+"""Time one decode-path kernel in isolation through the C ABI (pipo_op_gemv,
+or with --tc the tensor-core projection pipo_op_gemm_tc: its activation-split
+kernel and its GEMM, both in the timed region).
 
-  python -m paper_2605_27255_gb300.kernel_bench --shape lm_head [--batch 1] [--iters 50]
+  python -m paper_2605_27255_gb300.kernel_bench --shape lm_head [--batch 1] [--iters 50] [--tc] [--splits S]
 
 Shapes are the weight-streaming projections of the 4B-class model.  Weights
 are random bf16; several copies are cycled so that every launch streams from
@@ -27,7 +29,7 @@ SHAPES = {
 }
 
 
-def run(name: str, batch: int, iters: int, min_bytes: float = 300e6) -> dict:
+def run(name: str, batch: int, iters: int, min_bytes: float = 300e6, tc: bool = False, splits: int = 0) -> dict:
     N, K, mode = SHAPES[name]
     rows = 2 * N if mode else N
     nbytes = rows * K * 2
@@ -36,18 +38,30 @@ def run(name: str, batch: int, iters: int, min_bytes: float = 300e6) -> dict:
     x = torch.randn(batch, K, device="cuda")
     y = torch.empty(batch, N, device="cuda")
     st = torch.cuda.current_stream()
+    if tc:
+        sb = capi.pipo_op_gemm_tc_scratch(mode, N, K, batch, splits)
+        scratch = torch.empty(sb + 1024, dtype=torch.uint8, device="cuda")
+        base = (scratch.data_ptr() + 1023) // 1024 * 1024
+
+        def launch(i):
+            capi.pipo_op_gemm_tc(mode, Ws[i % copies].data_ptr(), N, K, x.data_ptr(), batch, y.data_ptr(), splits,
+                                 base, sb, st.cuda_stream)
+    else:
+        def launch(i):
+            capi.pipo_op_gemv(1, mode, Ws[i % copies].data_ptr(), N, K, x.data_ptr(), batch, y.data_ptr(),
+                              st.cuda_stream)
     for i in range(3):
-        capi.pipo_op_gemv(1, mode, Ws[i % copies].data_ptr(), N, K, x.data_ptr(), batch, y.data_ptr(), st.cuda_stream)
+        launch(i)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     e0.record(st)
     for i in range(iters):
-        capi.pipo_op_gemv(1, mode, Ws[i % copies].data_ptr(), N, K, x.data_ptr(), batch, y.data_ptr(), st.cuda_stream)
+        launch(i)
     e1.record(st)
     torch.cuda.synchronize()
     us = e0.elapsed_time(e1) * 1e3 / iters
-    return dict(kernel="gemv", shape=name, batch=batch, N=N, K=K, us_per_launch=us, gbs=nbytes / us / 1e3,
-                bytes_per_launch=nbytes, copies=copies)
+    return dict(kernel="gemm_tc" if tc else "gemv", shape=name, batch=batch, N=N, K=K, us_per_launch=us,
+                gbs=nbytes / us / 1e3, bytes_per_launch=nbytes, copies=copies)
 
 
 def main() -> None:
@@ -55,10 +69,12 @@ def main() -> None:
     ap.add_argument("--shape", default="all", choices=["all"] + sorted(SHAPES))
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--iters", type=int, default=50)
+    ap.add_argument("--tc", action="store_true", help="tensor-core projection (bf16 hi/lo activations)")
+    ap.add_argument("--splits", type=int, default=0, help="K splits of the tensor-core GEMM (0: automatic)")
     a = ap.parse_args()
     capi.load()
     for name in (sorted(SHAPES) if a.shape == "all" else [a.shape]):
-        print(json.dumps(run(name, a.batch, a.iters)), flush=True)
+        print(json.dumps(run(name, a.batch, a.iters, tc=a.tc, splits=a.splits)), flush=True)
 
 
 if __name__ == "__main__":

@@ -274,11 +274,14 @@ def run_pipo(args):
     _, e2b = g.counters()
     e2e_tokens = int((e2b - e2a).sum())
     launches = g.launches()
+    desc = g.describe()
     # dominant kernel: per-launch CUDA-event timings of eagerly run steps
     prof_steps = max(1, min(K, args.profile_steps))
     kb = {0: [0.0, 0.0, 0], 1: [0.0, 0.0, 0], 2: [0.0, 0.0, 0]}
     for _ in range(prof_steps):
+        torch.cuda.nvtx.range_push("profile_step")  # ncu --nvtx-include "profile_step/" selects these launches
         kind, by, pms = g.profile_step()
+        torch.cuda.nvtx.range_pop()
         for kk, bb, mm in zip(kind, by, pms):
             kb[int(kk)][0] += float(bb)
             kb[int(kk)][1] += float(mm)
@@ -322,8 +325,8 @@ def run_pipo(args):
                    "acceptance": tokens / (K * B) - 1.0, "pair_step_us": 1e3 * ms / K,
                    "prefill_s": t_pf, "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
                    "parallelism": f"replicas x{ws}"},
-        "roofline": {"bound": "hbm", "kernel": "gemv_rows_kernel (weight-streaming GEMV: every projection and "
-                                                  "both LM-head launches of a step)",
+        "roofline": {"bound": "hbm", "kernel": f"weight-streaming projections (every projection and both LM-head "
+                                                  f"launches of a step): {desc}",
                      "achieved": gemv_gbs, "peak": hbm, "unit": "GB/s",
                      "frac": (gemv_gbs / hbm) if gemv_gbs else None, "traffic": None,
                      "algorithmic_bytes_per_launch": gb / max(1, gn), "avg_launch_us": 1e3 * gms / max(1, gn),

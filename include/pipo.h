@@ -258,6 +258,15 @@ PIPO_API pipo_status pipo_op_lm_head_argmax_noalloc(int32_t dtype, const void *d
 PIPO_API pipo_status pipo_profile_step(pipo_ctx *ctx, int32_t cap, int32_t *h_kind, double *h_bytes, float *h_ms,
                                        int32_t *h_n);
 
+/* Which kernels the next decode step launches for the projections and the
+ * attention, and the attention cluster size, as one NUL-terminated line of
+ * at most cap bytes in h_buf, e.g. "B=16 projections=gemm_tc_kernel<16>+
+ * prep_bf16_kernel (tcgen05) attention=attn_mma_kernel cluster=2".  Batch B
+ * is the prefilled batch (before a prefill: cfg.max_batch).  A report of
+ * this library's kernel choices; the paper has no counterpart.  EINVAL for
+ * a NULL context or buffer or cap == 0. */
+PIPO_API pipo_status pipo_describe_step(const pipo_ctx *ctx, char *h_buf, size_t cap);
+
 /* Number of kernel launches one decode step enqueues (for launch accounting). */
 PIPO_API int32_t pipo_step_launches(const pipo_ctx *ctx);
 

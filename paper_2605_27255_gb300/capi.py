@@ -92,6 +92,7 @@ SIGNATURES = {
     "pipo_op_gemm_tc": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_int32, C.c_void_p,
                                   C.c_int32, C.c_void_p, C.c_size_t, C.c_void_p]),
     "pipo_op_gemm_tc_scratch": (C.c_size_t, [C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32]),
+    "pipo_describe_step": (C.c_int, [C.c_void_p, C.c_char_p, C.c_size_t]),
     "pipo_profile_step": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.POINTER(C.c_double), _FP, _IP]),
     "pipo_step_launches": (C.c_int32, [C.c_void_p]),
     "pipo_last_error": (C.c_char_p, [C.c_void_p]),
@@ -361,6 +362,12 @@ class Pipo:
 
     def launches(self) -> int:
         return pipo_step_launches(self.ctx)
+
+    def describe(self) -> str:
+        """The kernels the next decode step launches (pipo_describe_step)."""
+        buf = C.create_string_buffer(512)
+        _check(load().pipo_describe_step(self.ctx, buf, 512), self.ctx)
+        return buf.value.decode()
 
     def profile_step(self):
         return pipo_profile_step(self.ctx)

@@ -132,7 +132,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             for (; t < ngrp; ++t) {
                 const int st = t % kMmaStages;
                 if (t >= kMmaStages && (*(volatile int*)&abort_flag ||
-                                        !mbar_wait(empty + st, (uint32_t)(((t / kMmaStages) & 1) ^ 1)))) {
+                                        !mbar_wait(empty + st, (uint32_t)(((t / kMmaStages) & 1) ^ 1), 21, t))) {
                     *(volatile int*)&abort_flag = 1;
                     break;
                 }
@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             }
             // no copy into this CTA's shared memory may still be in flight at exit
             for (int i = max(0, t - kMmaStages); i < t; ++i)
-                mbar_wait(full + (i % kMmaStages), (uint32_t)((i / kMmaStages) & 1));
+                mbar_wait(full + (i % kMmaStages), (uint32_t)((i / kMmaStages) & 1), 22, i);
         }
         __syncwarp();
     } else {
@@ -227,7 +227,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
 
         for (int t = warp; t < ngrp; t += NW) {
             const int st = t % kMmaStages;
-            if (*(volatile int*)&abort_flag || !mbar_wait(full + st, (uint32_t)((t / kMmaStages) & 1))) {
+            if (*(volatile int*)&abort_flag || !mbar_wait(full + st, (uint32_t)((t / kMmaStages) & 1), 23, t)) {
                 *(volatile int*)&abort_flag = 1;
                 break;
             }

@@ -1034,7 +1034,7 @@ __global__ void __launch_bounds__(kTmaThreads) gemv_tma_kernel(GemvParams p, int
     int failed = -1;  // first stage whose wait gave up
     for (int i = 0; i < nst; ++i) {
         const int slot = i % ns;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(bars + slot, (uint32_t)((i / ns) & 1)));
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(bars + slot, (uint32_t)((i / ns) & 1), 31, i));
         if (!ok) {
             failed = i;
             break;
@@ -1057,7 +1057,7 @@ __global__ void __launch_bounds__(kTmaThreads) gemv_tma_kernel(GemvParams p, int
     }
     if (failed >= 0 && lane == 0) {
         // a wait gave up (error recorded): wait, bounded, for the copies still in flight
-        for (int i = failed + 1; i < min(nst, failed + ns); ++i) mbar_wait(bars + (i % ns), (uint32_t)((i / ns) & 1));
+        for (int i = failed + 1; i < min(nst, failed + ns); ++i) mbar_wait(bars + (i % ns), (uint32_t)((i / ns) & 1), 32, i);
     }
     wr.finish(head_unit, head_fin, tail_unit, head_val, tail_val);
     __syncthreads();

@@ -175,7 +175,7 @@ __device__ __forceinline__ bool mk_gemv_phase(const Phase& ph, WarpRing& r, cons
     bool ok = true;
     for (int i = 0; i < nst; ++i) {
         const int slot = r.consumed % kMkStages;
-        ok = __all_sync(0xffffffffu, mbar_wait(r.bars + slot, (uint32_t)((r.consumed / kMkStages) & 1)));
+        ok = __all_sync(0xffffffffu, mbar_wait(r.bars + slot, (uint32_t)((r.consumed / kMkStages) & 1), 41, r.consumed));
         if (!ok) break;
         const unsigned char* sp = r.base + (size_t)slot * kMkStageBytes + lane * 16;
         const int n = min(kMkStageChunks, (c1 - c0) - i * kMkStageChunks);
@@ -513,7 +513,7 @@ __global__ void __launch_bounds__(kMkThreads, 1) step_kernel(const Phase* __rest
     // drain (bounded) any stage still in flight (only after a failed wait)
     if (lane == 0)
         while (r.consumed < r.issued) {
-            mbar_wait(r.bars + (r.consumed % kMkStages), (uint32_t)((r.consumed / kMkStages) & 1));
+            mbar_wait(r.bars + (r.consumed % kMkStages), (uint32_t)((r.consumed / kMkStages) & 1), 42, r.consumed);
             ++r.consumed;
         }
     (void)ok;

@@ -311,22 +311,25 @@ void* pick_stream(int nb, int ru, bool rows) {
 }
 
 // bh: batch columns of the tensor-core GEMM (its MMA N is 2 * bh: hi | lo)
-size_t tc_smem(int bh) {
-    const int st = tc_stages(bh);
+size_t tc_smem(int bh, bool deep = false) {
+    const int st = tc_stages(bh, deep);
     return 1024 + (size_t)st * (kTcABytes + (size_t)2 * bh * kTcBK * 2) + (2 * st + 1) * 8;
 }
 
-template <int BH>
-void* tc_fn() { return reinterpret_cast<void*>(&gemm_tc_kernel<BH, tc_stages(BH)>); }
+template <int BH, bool DEEP>
+void* tc_fn() { return reinterpret_cast<void*>(&gemm_tc_kernel<BH, tc_stages(BH, DEEP)>); }
 
-void* pick_tc(int bh) {
+template <bool DEEP>
+void* pick_tc_v(int bh) {
     switch (bh) {
-        case 16: return tc_fn<16>();
-        case 32: return tc_fn<32>();
-        case 64: return tc_fn<64>();
-        default: return tc_fn<128>();
+        case 16: return tc_fn<16, DEEP>();
+        case 32: return tc_fn<32, DEEP>();
+        case 64: return tc_fn<64, DEEP>();
+        default: return tc_fn<128, DEEP>();
     }
 }
+
+void* pick_tc(int bh, bool deep = false) { return deep ? pick_tc_v<true>(bh) : pick_tc_v<false>(bh); }
 
 bool tc_cluster_spread();
 void* attnm_pick(int G);
@@ -363,15 +366,16 @@ cudaError_t set_smem_attrs(bool bf) {
             if (e != cudaSuccess) return e;
         }
     if (bf)
-        for (int bn : {16, 32, 64, 128}) {
-            cudaError_t e =
-                cudaFuncSetAttribute(pick_tc(bn), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem(bn));
-            if (e != cudaSuccess) return e;
-            e = cudaFuncSetAttribute(pick_tc(bn), cudaFuncAttributeClusterSchedulingPolicyPreference,
-                                     tc_cluster_spread() ? cudaClusterSchedulingPolicySpread
-                                                         : cudaClusterSchedulingPolicyLoadBalancing);
-            if (e != cudaSuccess) return e;
-        }
+        for (int bn : {16, 32, 64, 128})
+            for (bool deep : {false, true}) {
+                cudaError_t e = cudaFuncSetAttribute(pick_tc(bn, deep), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                     (int)tc_smem(bn, deep));
+                if (e != cudaSuccess) return e;
+                e = cudaFuncSetAttribute(pick_tc(bn, deep), cudaFuncAttributeClusterSchedulingPolicyPreference,
+                                         tc_cluster_spread() ? cudaClusterSchedulingPolicySpread
+                                                             : cudaClusterSchedulingPolicyLoadBalancing);
+                if (e != cudaSuccess) return e;
+            }
     return cudaSuccess;
 }
 
@@ -409,8 +413,8 @@ pipo_status make_tmap(pipo_ctx* ctx, CUtensorMap* tm, const void* base, int K, i
 int tc_bn(int B) { return B <= 16 ? 16 : B <= 32 ? 32 : B <= 64 ? 64 : 128; }
 
 // resident CTAs per SM of the tensor-core GEMM at this BN (shared memory bound)
-int tc_ctas_per_sm(int bn) {
-    const size_t per = tc_smem(bn) + 40 * (size_t)bn + 1024;  // dynamic + static + reserve
+int tc_ctas_per_sm(int bn, bool deep = false) {
+    const size_t per = tc_smem(bn, deep) + 40 * (size_t)bn + 1024;  // dynamic + static + reserve
     return std::max(1, (int)(g_smem_optin ? 228 * 1024 / per : 1));
 }
 
@@ -426,19 +430,19 @@ bool tc_cluster_spread() {
 
 // Clusters of `cs` CTAs of the GEMM at batch width bh that can be resident at
 // once on the current device (cudaOccupancyMaxActiveClusters; cached).
-int tc_max_clusters(int bh, int cs) {
+int tc_max_clusters(int bh, int cs, bool deep) {
     static std::mutex mu;
     static std::map<long long, int> cache;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return 0; }
-    const long long key = ((long long)dev << 20) | ((long long)bh << 8) | cs;
+    const long long key = ((long long)dev << 20) | ((long long)deep << 16) | ((long long)bh << 8) | cs;
     std::lock_guard<std::mutex> lk(mu);
     auto it = cache.find(key);
     if (it != cache.end()) return it->second;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(cs);
     lc.blockDim = dim3(kTcThreads);
-    lc.dynamicSmemBytes = tc_smem(bh);
+    lc.dynamicSmemBytes = tc_smem(bh, deep);
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = cs;
@@ -447,7 +451,7 @@ int tc_max_clusters(int bh, int cs) {
     lc.attrs = at;
     lc.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, pick_tc(bh), &lc) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, pick_tc(bh, deep), &lc) != cudaSuccess) {
         cudaGetLastError();
         n = 0;
     }
@@ -455,20 +459,33 @@ int tc_max_clusters(int bh, int cs) {
     return n;
 }
 
-// K splits (the cluster size): enough CTAs for every SM's resident slots,
-// each split at least kTcMinKb 64-wide K blocks, at most kTcMaxSplits, and
-// no more than fit on the GPU at once as clusters (one wave).
+// Launch plan of a tensor-core projection: the K splits (the cluster size)
+// and the pipeline variant.  Tiles that fit one per SM take the deep ring,
+// split so that the CTAs still fit one per SM; more tiles take the two-per-SM
+// ring, split up to the SM slots.  Each split has at least kTcMinKb 64-wide K
+// blocks, at most kTcMaxSplits, and all clusters must fit at once (one wave).
 constexpr int kTcMinKb = 4;
-int tc_auto_splits(int sms, int bn, int tiles, int nkb) {
-    const int target = sms * tc_ctas_per_sm(bn);
-    if (tiles >= target) return 1;
+struct TcPlan {
+    int splits;
+    bool deep;
+};
+TcPlan tc_plan(int sms, int bn, int tiles, int nkb) {
+    static const int force_deep = [] {
+        const char* ev = getenv("PIPO_TC_DEEP");
+        return ev ? atoi(ev) : -1;
+    }();
+    const bool deep = force_deep >= 0 ? force_deep == 1 : tiles <= sms;
+    const int target = sms * tc_ctas_per_sm(bn, deep);
+    if (tiles >= target) return {1, deep};
     static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
     for (int s = std::min({target / tiles, nkb / kTcMinKb, kTcMaxSplits}); s >= 2; --s) {
-        const int mc = tc_max_clusters(bn, s);
-        if (verbose) fprintf(stderr, "[pipo] tc splits: bh=%d tiles=%d nkb=%d s=%d max_clusters=%d\n", bn, tiles, nkb, s, mc);
-        if (mc >= tiles) return s;
+        const int mc = tc_max_clusters(bn, s, deep);
+        if (verbose)
+            fprintf(stderr, "[pipo] tc plan: bh=%d deep=%d tiles=%d nkb=%d s=%d max_clusters=%d\n", bn, (int)deep, tiles,
+                    nkb, s, mc);
+        if (mc >= tiles) return {s, deep};
     }
-    return 1;
+    return {1, deep};
 }
 
 // Projection on the tensor cores: bf16 activations (prep kernel), then the
@@ -476,8 +493,9 @@ int tc_auto_splits(int sms, int bn, int tiles, int nkb) {
 pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int splits_req) {
     const int ru = p.epi == EPI_SWIGLU ? 2 : 1;
     const int rows = p.N * ru, bn = tc_bn(p.B), tiles = (rows + kTcM - 1) / kTcM, nkb = p.K / kTcBK;
-    const int splits = splits_req > 0 ? std::min({splits_req, nkb, kTcMaxSplits})
-                                      : tc_auto_splits(ctx->sms, bn, tiles, nkb);
+    TcPlan plan = tc_plan(ctx->sms, bn, tiles, nkb);
+    if (splits_req > 0) plan.splits = std::min({splits_req, nkb, kTcMaxSplits});
+    const int splits = plan.splits;
     CUtensorMap tmW, tmX;
     TRY(make_tmap(ctx, &tmW, p.W, p.K, rows, kTcM));
     TRY(make_tmap(ctx, &tmX, xb, p.K, 2 * bn, 2 * bn));
@@ -497,7 +515,8 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
     void* args[] = {&tmW, &tmX, &tp};
     ctx->prof_kind = 0;
     ctx->prof_bytes = (double)rows * p.K * 2;
-    return launch_ex(ctx, pick_tc(bn), dim3(tiles * splits), dim3(kTcThreads), tc_smem(bn), args, splits);
+    return launch_ex(ctx, pick_tc(bn, plan.deep), dim3(tiles * splits), dim3(kTcThreads), tc_smem(bn, plan.deep), args,
+                     splits);
 }
 
 bool tc_eligible(const pipo_ctx* ctx, const GemvParams& p) {
@@ -706,6 +725,49 @@ KVView kv_view(pipo_ctx* ctx, int layer) {
     return v;
 }
 
+// One shared-memory carveout preference for every kernel of a step
+// (PIPO_CARVEOUT=<percent>; default: the driver's choice).  Measured on the
+// 4B shapes: a 100 % carveout for all kernels helps the tensor-core attention
+// next to the small-batch GEMVs and slows the register-ring attention, while
+// the driver's choice with the kernel selection of attn_use_mma is as fast.
+cudaError_t set_carveouts(bool bf) {
+    int pct = -1;
+    if (const char* ev = getenv("PIPO_CARVEOUT")) pct = atoi(ev);
+    if (pct < 0) return cudaSuccess;
+    std::vector<const void*> fns;
+    for (int nb : {1, 2, 4, 8})
+        for (int two = 0; two < 2; ++two) fns.push_back(bf ? pick_gemv<bf16>(nb, two) : pick_gemv<float>(nb, two));
+    for (int nb : {1, 2, 4})
+        for (int ru : {1, 2}) {
+            fns.push_back(bf ? pick_tma<bf16>(nb, ru) : pick_tma<float>(nb, ru));
+            for (bool rows : {false, true})
+                fns.push_back(bf ? pick_stream<bf16>(nb, ru, rows) : pick_stream<float>(nb, ru, rows));
+        }
+    if (bf) {
+        for (int bn : {16, 32, 64, 128}) {
+            fns.push_back(pick_tc(bn, false));
+            fns.push_back(pick_tc(bn, true));
+        }
+        fns.push_back(reinterpret_cast<const void*>(&prep_bf16_kernel<bf16>));
+        for (int g : {1, 2, 4}) fns.push_back(attnm_pick(g));
+    }
+    for (int dh : {64, 128}) {
+        for (int g : {1, 2, 4, 8}) {
+            fns.push_back(attnc_pick(bf, dh, g));
+            fns.push_back(attn_pick(bf, dh, g));
+        }
+        fns.push_back(rope_pick(bf, dh));
+    }
+    fns.push_back(bf ? (const void*)&accept_kernel<bf16> : (const void*)&accept_kernel<float>);
+    fns.push_back((const void*)&advance_kernel);
+    for (const void* f : fns) {
+        if (!f) continue;
+        const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout, pct);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
 // the tensor-core attention applies: bf16 cache, d_h = 128, G in {1, 2, 4},
 // pages of whole 16-entry groups
 bool attn_mma_ok(const pipo_ctx* ctx) {
@@ -713,6 +775,14 @@ bool attn_mma_ok(const pipo_ctx* ctx) {
     const int G = c.n_q_heads / c.n_kv_heads;
     return !ctx->attn_regs && c.dtype == 1 && c.head_dim == kMmaDH && (G == 1 || G == 2 || G == 4) &&
            c.page_size % kMmaRun == 0;
+}
+
+// ... and is used: from the batch at which the projections move to the tensor
+// cores (measured: below it the register-ring attention is slightly faster
+// next to the CUDA-core GEMVs, from B = 4 the tensor-core one by far), with
+// the cache tensor maps in place
+bool attn_use_mma(const pipo_ctx* ctx) {
+    return attn_mma_ok(ctx) && ctx->B >= ctx->tc_min_b && (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers;
 }
 
 // CTAs per (sequence, kv head) of the clustered attention: 8 while the batch
@@ -724,7 +794,7 @@ int attn_cluster_size(const pipo_ctx* ctx) {
     if (ctx->attn_cs16 && pairs * 16 <= 2 * ctx->sms) return 16;
     // measured best: about two tensor-core attention CTAs per SM (they are
     // resident two at a time), one register-ring CTA per SM
-    const long long target = ctx->attn_cs_target > 0 ? ctx->attn_cs_target : (attn_mma_ok(ctx) ? 2 : 1);
+    const long long target = ctx->attn_cs_target > 0 ? ctx->attn_cs_target : (attn_use_mma(ctx) ? 2 : 1);
     int cs = 8;
     while (cs > 1 && pairs * cs > target * ctx->sms) cs >>= 1;
     return cs;
@@ -775,7 +845,7 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         void* args[] = {&ap};
         const int cs = attn_cluster_size(ctx);
         const int G = c.n_q_heads / c.n_kv_heads;
-        if (attn_mma_ok(ctx) && cs <= 8 && (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers) {
+        if (attn_use_mma(ctx) && cs <= 8) {
             void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
             TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, ctx->B), dim3(kMmaThreads), mma_attn_smem(),
                           margs, cs));
@@ -1099,9 +1169,15 @@ pipo_status check_device_error(pipo_ctx* ctx) {
     unsigned e = 0;
     CK(cudaMemcpyFromSymbol(&e, g_pipo_error, sizeof(e)));
     if (!e) return PIPO_OK;
-    const unsigned zero = 0;
-    CK(cudaMemcpyToSymbol(g_pipo_error, &zero, sizeof(zero)));
-    return fail(ctx, PIPO_ECUDA, "device wait timed out (code %u): results of this step are invalid", e);
+    unsigned info[4] = {0, 0, 0, 0};
+    CK(cudaMemcpyFromSymbol(info, g_pipo_error_info, sizeof(info)));
+    const unsigned zero[4] = {0, 0, 0, 0};
+    CK(cudaMemcpyToSymbol(g_pipo_error, zero, sizeof(unsigned)));
+    CK(cudaMemcpyToSymbol(g_pipo_error_info, zero, sizeof(zero)));
+    return fail(ctx, PIPO_ECUDA,
+                "device wait timed out (code %u; first at wait site %u, block %u, iteration %u, parity %u): "
+                "results of this step are invalid",
+                e, info[0], info[1], info[2], info[3]);
 }
 
 }  // namespace
@@ -1207,6 +1283,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
             TRY(dalloc(ctx, &ctx->rope, tab.size() * 4));
             CK(cudaMemcpy(ctx->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice));
         }
+        CK(set_carveouts(c.dtype == 1));
         if (const char* ev = getenv("PIPO_ATTN_V0")) ctx->attn_v0 = ev[0] == '1';
         if (const char* ev = getenv("PIPO_ATTN_IMPL")) ctx->attn_regs = strcmp(ev, "regs") == 0;
         if (attn_mma_ok(ctx)) {
@@ -1662,6 +1739,37 @@ pipo_status pipo_op_gemm_tc(int32_t mode, const void* d_W, int32_t N, int32_t K,
     }
     if (st != PIPO_OK) g_init_error = op.err;
     return st;
+}
+
+pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {
+    if (!ctx || !h_buf || cap == 0) return fail(nullptr, PIPO_EINVAL, "pipo_describe_step: bad arguments");
+    const pipo_config& c = ctx->cfg;
+    const int B = ctx->prefilled ? ctx->B : c.max_batch;
+    const int H = c.hidden, qd = c.n_q_heads * c.head_dim, kd = c.n_kv_heads * c.head_dim;
+    // the projections of a decoder block: (rows, K)
+    const int shp[4][2] = {{qd + 2 * kd, H}, {H, qd}, {2 * c.ffn, H}, {H, c.ffn}};
+    int n_tc = 0;
+    for (auto& sh : shp) {
+        GemvParams p{};
+        p.N = sh[0];
+        p.K = sh[1];
+        p.B = B;
+        p.epi = EPI_STORE;
+        n_tc += tc_eligible(ctx, p) ? 1 : 0;
+    }
+    std::string proj;
+    const std::string cuda_core = B <= 4 ? "gemv_rows_kernel" : "gemv_kernel";
+    if (n_tc == 4) proj = "gemm_tc_kernel<" + std::to_string(tc_bn(B)) + ">+prep_bf16_kernel (tcgen05)";
+    else if (n_tc > 0) proj = "gemm_tc_kernel<" + std::to_string(tc_bn(B)) + ">+prep_bf16_kernel (tcgen05; " +
+                              std::to_string(4 - n_tc) + " of 4 block projections on " + cuda_core + ")";
+    else proj = cuda_core;
+    const int cs = attn_cluster_size(ctx);
+    const bool mma = attn_use_mma(ctx) && cs <= 8;
+    const std::string d = "B=" + std::to_string(B) + " projections=" + proj + " attention=" +
+                          (ctx->attn_v0 ? std::string("attn_decode_kernel") : mma ? "attn_mma_kernel" : "attn_cluster_kernel") +
+                          " cluster=" + std::to_string(cs);
+    snprintf(h_buf, cap, "%s", d.c_str());
+    return PIPO_OK;
 }
 
 pipo_status pipo_profile_step(pipo_ctx* ctx, int32_t cap, int32_t* h_kind, double* h_bytes, float* h_ms,

@@ -38,8 +38,12 @@ constexpr int kTcThreads = 128;
 constexpr int kTcABytes = kTcM * kTcBK * 2;  // 16 KB per stage
 constexpr int kTcMaxSplits = 8;             // portable cluster size
 
-// operand stages per batch width BH: about 100 KB of shared memory, two CTAs per SM
-__host__ __device__ constexpr int tc_stages(int bh) { return bh <= 16 ? 5 : bh <= 32 ? 4 : bh <= 64 ? 3 : 2; }
+// operand stages per batch width BH: about 100 KB of shared memory (two CTAs
+// per SM), or, for grids of at most one CTA per SM, about 200 KB (deep): a
+// lone CTA needs the deeper ring to keep enough weight bytes in flight
+__host__ __device__ constexpr int tc_stages(int bh, bool deep = false) {
+    return deep ? (bh <= 16 ? 10 : bh <= 32 ? 8 : bh <= 64 ? 6 : 4) : (bh <= 16 ? 5 : bh <= 32 ? 4 : bh <= 64 ? 3 : 2);
+}
 
 struct TcParams {
     int rows;            // W rows (output units * ru)
@@ -256,21 +260,28 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
 
     if (warp == 0) {
         if (lane == 0) {
-            // TMA producer: weight tiles need nothing from the previous
-            // kernel; the activation tile waits for it (programmatic
-            // dependent launch)
-            int issued = 0;
-            for (int i = 0; i < nk; ++i) {
+            // TMA producer: the weight tiles of the first ST stages need
+            // nothing from the previous kernel and go out before the
+            // dependency wait (programmatic dependent launch); the
+            // activation tiles follow it
+            const int pre = min(nk, ST);
+            for (int i = 0; i < pre; ++i) {
+                mbar_arrive_expect_tx(full + i, (uint32_t)(kTcABytes + kBBytes));
+                tma_load_2d(sA + i * kTcABytes, &tmW, (kb0 + i) * kTcBK, tile * kTcM, full + i);
+            }
+            pdl_wait();
+            for (int i = 0; i < pre; ++i) tma_load_2d(sB + i * kBBytes, &tmX, (kb0 + i) * kTcBK, 0, full + i);
+            int issued = pre;
+            for (int i = pre; i < nk; ++i) {
                 const int s = i % ST;
-                if (i >= ST && !mbar_wait(empty + s, (uint32_t)(((i / ST) & 1) ^ 1))) break;
+                if (!mbar_wait(empty + s, (uint32_t)(((i / ST) & 1) ^ 1), 11, i)) break;
                 mbar_arrive_expect_tx(full + s, (uint32_t)(kTcABytes + kBBytes));
                 tma_load_2d(sA + s * kTcABytes, &tmW, (kb0 + i) * kTcBK, tile * kTcM, full + s);
-                if (i == 0) pdl_wait();
                 tma_load_2d(sB + s * kBBytes, &tmX, (kb0 + i) * kTcBK, 0, full + s);
                 issued = i + 1;
             }
             // no copy into this CTA's shared memory may still be in flight at exit
-            for (int i = max(0, issued - ST); i < issued; ++i) mbar_wait(full + (i % ST), (uint32_t)((i / ST) & 1));
+            for (int i = max(0, issued - ST); i < issued; ++i) mbar_wait(full + (i % ST), (uint32_t)((i / ST) & 1), 12, i);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -280,7 +291,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
             const uint32_t idesc = umma_idesc_bf16(kTcM, BN);
             for (int i = 0; i < nk; ++i) {
                 const int s = i % ST;
-                if (!mbar_wait(full + s, (uint32_t)((i / ST) & 1))) break;
+                if (!mbar_wait(full + s, (uint32_t)((i / ST) & 1), 13, i)) break;
                 tc_fence_after();
                 const uint32_t a0 = smem_u32(sA + s * kTcABytes), b0 = smem_u32(sB + s * kBBytes);
 #pragma unroll
@@ -295,7 +306,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
     }
 
     // epilogue: thread t holds TMEM lane t = weight row tile*128 + t
-    mbar_wait(accb, 0);
+    mbar_wait(accb, 0, 14, (unsigned)nk);
     __syncwarp();
     tc_fence_after();
     pdl_wait();

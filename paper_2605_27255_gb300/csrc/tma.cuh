@@ -14,6 +14,12 @@ namespace pipo {
 
 // Device error word: 0 = fine; kErrWaitTimeout when a bounded wait gave up.
 __device__ unsigned int g_pipo_error;
+// First wait that gave up: {site code, linear block index, iteration, parity}
+// (the site codes name the wait: 11-14 projection GEMM producer-empty,
+// producer-drain, MMA-full, epilogue-accumulator; 21-23 attention
+// producer-empty, producer-drain, consumer-full; 31-32 bulk-copy GEMV;
+// 41-42 step kernel).
+__device__ unsigned int g_pipo_error_info[4];
 constexpr unsigned kErrWaitTimeout = 1u;
 constexpr unsigned long long kWaitNs = 2000000000ull;  // give up after 2 s of waiting
 
@@ -80,8 +86,9 @@ __device__ __forceinline__ unsigned long long global_ns() {
 }
 
 // Bounded wait for phase `parity` of `bar`: false (and the error word set)
-// once kWaitNs of wall time have passed without the phase completing.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// once kWaitNs of wall time have passed without the phase completing; the
+// first wait to give up records `site`, its block and `iter` for the host.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned site = 0, unsigned iter = 0) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
     for (;;) {
@@ -90,6 +97,11 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
         if (global_ns() - t0 > kWaitNs) break;
     }
     atomicOr(&g_pipo_error, kErrWaitTimeout);
+    if (atomicCAS(&g_pipo_error_info[0], 0u, site ? site : 99u) == 0u) {
+        g_pipo_error_info[1] = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);
+        g_pipo_error_info[2] = iter;
+        g_pipo_error_info[3] = parity;
+    }
     return false;
 }
 

@@ -60,6 +60,15 @@ def test_4b_b4_forced_replay(w4b):
     assert st.tok_checked >= 0.8 * st.tok_total
 
 
+def test_4b_b16_forced_replay(w4b):
+    """4b-b16: sixteen sequences, tcgen05 projections and tensor-core attention."""
+    w, host = w4b
+    prompts = synth.gen_prompts(16, 8, synth.B4.V, seed=5).numpy()
+    st = run_forced_replay(synth.B4, w, prompts, 2, oracle_weights=host, force=1)
+    assert st.tok_checked >= 0.8 * st.tok_total
+    assert st.max_logit_err < 2e-2
+
+
 def test_9b_b1_forced_replay():
     """9B-class shapes (H=4096, F=12288)."""
     w, host = _weights(synth.B9)

@@ -96,3 +96,24 @@ def test_mid_bf16_cuda_core_batches_over_8(monkeypatch):
     st = run_forced_replay(MID, w, prompts, 3, force=1)
     assert st.tok_checked >= 0.8 * st.tok_total
     assert st.max_logit_err < 2e-2
+
+
+def test_decode_path_uses_tensor_core_kernels():
+    """At B = 16 the block projections and the attention take the tcgen05 and
+    mma.sync kernels (the down projection, K = 1376, stays on CUDA cores)."""
+    w = synth.gen_weights(MID, seed=23)
+    g = capi.Pipo(MID, w, max_batch=16, max_ctx=40)
+    try:
+        g.prefill(synth.gen_prompts(16, 8, MID.V, seed=1).numpy())
+        d = g.describe()
+        assert "gemm_tc_kernel<16>" in d and "1 of 4 block projections on gemv_kernel" in d, d
+        assert "attn_mma_kernel" in d, d
+    finally:
+        g.close()
+    g = capi.Pipo(MID, w, max_batch=2, max_ctx=40)
+    try:
+        g.prefill(synth.gen_prompts(2, 8, MID.V, seed=1).numpy())
+        d = g.describe()
+        assert "projections=gemv_rows_kernel" in d and "attention=attn_cluster_kernel cluster=8" in d, d
+    finally:
+        g.close()

@@ -73,6 +73,7 @@ struct pipo_ctx {
     // tensor-core projections (bf16, batch >= tc_min_b)
     bf16* tc_xb = nullptr;          // [2 * tc_bn_max][tc_kmax] bf16 activations (hi rows, lo rows)
     int tc_kmax = 0, tc_bn_max = 0;
+    int act_rows = 0;               // rows of the fp32 activation buffers (>= the batch width BH)
     int tc_min_b = 4;               // measured: tensor cores ahead of the CUDA-core GEMV from B = 4
     int tc_splits = 0;              // forced K splits (0: automatic)
 
@@ -331,6 +332,32 @@ void* pick_tc_v(int bh) {
 
 void* pick_tc(int bh, bool deep = false) { return deep ? pick_tc_v<true>(bh) : pick_tc_v<false>(bh); }
 
+template <int BH, bool DEEP>
+void* tcf_fn() { return reinterpret_cast<void*>(&gemm_tcf_kernel<BH, tcf_stages(BH, DEEP)>); }
+
+template <bool DEEP>
+void* pick_tcf_v(int bh) {
+    switch (bh) {
+        case 16: return tcf_fn<16, DEEP>();
+        case 32: return tcf_fn<32, DEEP>();
+        case 64: return tcf_fn<64, DEEP>();
+        default: return tcf_fn<128, DEEP>();
+    }
+}
+
+// kernel variants of the tensor-core projection: fused (activation split
+// inside the GEMM) or fed by prep_bf16_kernel; deep (one CTA per SM) or not
+void* pick_tcv(int bh, bool deep, bool fused) {
+    if (fused) return deep ? pick_tcf_v<true>(bh) : pick_tcf_v<false>(bh);
+    return pick_tc(bh, deep);
+}
+size_t tcv_smem(int bh, bool deep, bool fused) {
+    if (!fused) return tc_smem(bh, deep);
+    const int st = tcf_stages(bh, deep);
+    return 1024 + (size_t)st * tcf_stage_bytes(bh) + (3 * st + 1) * 8;
+}
+int tcv_threads(bool fused) { return fused ? kTcfThreads : kTcThreads; }
+
 bool tc_cluster_spread();
 void* attnm_pick(int G);
 
@@ -367,15 +394,17 @@ cudaError_t set_smem_attrs(bool bf) {
         }
     if (bf)
         for (int bn : {16, 32, 64, 128})
-            for (bool deep : {false, true}) {
-                cudaError_t e = cudaFuncSetAttribute(pick_tc(bn, deep), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                     (int)tc_smem(bn, deep));
-                if (e != cudaSuccess) return e;
-                e = cudaFuncSetAttribute(pick_tc(bn, deep), cudaFuncAttributeClusterSchedulingPolicyPreference,
-                                         tc_cluster_spread() ? cudaClusterSchedulingPolicySpread
-                                                             : cudaClusterSchedulingPolicyLoadBalancing);
-                if (e != cudaSuccess) return e;
-            }
+            for (bool deep : {false, true})
+                for (bool fused : {false, true}) {
+                    void* fn = pick_tcv(bn, deep, fused);
+                    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                         (int)tcv_smem(bn, deep, fused));
+                    if (e != cudaSuccess) return e;
+                    e = cudaFuncSetAttribute(fn, cudaFuncAttributeClusterSchedulingPolicyPreference,
+                                             tc_cluster_spread() ? cudaClusterSchedulingPolicySpread
+                                                                 : cudaClusterSchedulingPolicyLoadBalancing);
+                    if (e != cudaSuccess) return e;
+                }
     return cudaSuccess;
 }
 
@@ -383,20 +412,24 @@ cudaError_t set_smem_attrs(bool bf) {
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_tiled = nullptr;
 std::mutex g_encode_mu;
 
+// the driver's tensor-map encoder, looked up once
+pipo_status load_encoder(pipo_ctx* ctx) {
+    std::lock_guard<std::mutex> lk(g_encode_mu);
+    if (!g_encode_tiled) {
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        CK(cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q));
+        if (q != cudaDriverEntryPointSuccess || !fn)
+            return fail(ctx, PIPO_ECUDA, "cuTensorMapEncodeTiled is not available");
+        g_encode_tiled = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    return PIPO_OK;
+}
+
 // 2-D bf16 tensor map over a row-major [rows, K] matrix: boxes of 64 x box_rows
 // elements, 128-byte swizzle (the layout the tcgen05 descriptors expect).
 pipo_status make_tmap(pipo_ctx* ctx, CUtensorMap* tm, const void* base, int K, int rows, int box_rows) {
-    {
-        std::lock_guard<std::mutex> lk(g_encode_mu);
-        if (!g_encode_tiled) {
-            void* fn = nullptr;
-            cudaDriverEntryPointQueryResult q{};
-            CK(cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q));
-            if (q != cudaDriverEntryPointSuccess || !fn)
-                return fail(ctx, PIPO_ECUDA, "cuTensorMapEncodeTiled is not available");
-            g_encode_tiled = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-        }
-    }
+    TRY(load_encoder(ctx));
     if (reinterpret_cast<uintptr_t>(base) % 16 != 0 || K % kTcBK != 0 || rows < box_rows)
         return fail(ctx, PIPO_EINVAL, "tensor map: base %% 16, K %% 64 and rows >= %d required", box_rows);
     const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
@@ -410,11 +443,28 @@ pipo_status make_tmap(pipo_ctx* ctx, CUtensorMap* tm, const void* base, int K, i
     return PIPO_OK;
 }
 
+// 2-D fp32 tensor map over activations [rows][ld] (first K columns): boxes of
+// 64 x box_rows elements, no swizzle; rows past `rows` read as zeros.
+pipo_status make_tmap_x(pipo_ctx* ctx, CUtensorMap* tm, const float* base, int K, int ld, int rows, int box_rows) {
+    TRY(load_encoder(ctx));
+    if (!base || reinterpret_cast<uintptr_t>(base) % 16 != 0 || K % kTcBK != 0 || ld % 4 != 0 || rows < 1)
+        return fail(ctx, PIPO_EINVAL, "activation tensor map: base %% 16, K %% 64, ld %% 4 required");
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)ld * 4};
+    const cuuint32_t box[2] = {(cuuint32_t)kTcBK, (cuuint32_t)box_rows};
+    const cuuint32_t es[2] = {1, 1};
+    const CUresult r = g_encode_tiled(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides,
+                                      box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                                      CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(ctx, PIPO_ECUDA, "cuTensorMapEncodeTiled (activations): error %d", (int)r);
+    return PIPO_OK;
+}
+
 int tc_bn(int B) { return B <= 16 ? 16 : B <= 32 ? 32 : B <= 64 ? 64 : 128; }
 
 // resident CTAs per SM of the tensor-core GEMM at this BN (shared memory bound)
-int tc_ctas_per_sm(int bn, bool deep = false) {
-    const size_t per = tc_smem(bn, deep) + 40 * (size_t)bn + 1024;  // dynamic + static + reserve
+int tc_ctas_per_sm(int bn, bool deep = false, bool fused = false) {
+    const size_t per = tcv_smem(bn, deep, fused) + 48 * (size_t)bn + 1024;  // dynamic + static + reserve
     return std::max(1, (int)(g_smem_optin ? 228 * 1024 / per : 1));
 }
 
@@ -430,19 +480,20 @@ bool tc_cluster_spread() {
 
 // Clusters of `cs` CTAs of the GEMM at batch width bh that can be resident at
 // once on the current device (cudaOccupancyMaxActiveClusters; cached).
-int tc_max_clusters(int bh, int cs, bool deep) {
+int tc_max_clusters(int bh, int cs, bool deep, bool fused) {
     static std::mutex mu;
     static std::map<long long, int> cache;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return 0; }
-    const long long key = ((long long)dev << 20) | ((long long)deep << 16) | ((long long)bh << 8) | cs;
+    const long long key =
+        ((long long)dev << 20) | ((long long)fused << 17) | ((long long)deep << 16) | ((long long)bh << 8) | cs;
     std::lock_guard<std::mutex> lk(mu);
     auto it = cache.find(key);
     if (it != cache.end()) return it->second;
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(cs);
-    lc.blockDim = dim3(kTcThreads);
-    lc.dynamicSmemBytes = tc_smem(bh, deep);
+    lc.blockDim = dim3(tcv_threads(fused));
+    lc.dynamicSmemBytes = tcv_smem(bh, deep, fused);
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = cs;
@@ -451,7 +502,7 @@ int tc_max_clusters(int bh, int cs, bool deep) {
     lc.attrs = at;
     lc.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, pick_tc(bh, deep), &lc) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, pick_tcv(bh, deep, fused), &lc) != cudaSuccess) {
         cudaGetLastError();
         n = 0;
     }
@@ -469,17 +520,17 @@ struct TcPlan {
     int splits;
     bool deep;
 };
-TcPlan tc_plan(int sms, int bn, int tiles, int nkb) {
+TcPlan tc_plan(int sms, int bn, int tiles, int nkb, bool fused) {
     static const int force_deep = [] {
         const char* ev = getenv("PIPO_TC_DEEP");
         return ev ? atoi(ev) : -1;
     }();
     const bool deep = force_deep >= 0 ? force_deep == 1 : tiles <= sms;
-    const int target = sms * tc_ctas_per_sm(bn, deep);
+    const int target = sms * tc_ctas_per_sm(bn, deep, fused);
     if (tiles >= target) return {1, deep};
     static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
     for (int s = std::min({target / tiles, nkb / kTcMinKb, kTcMaxSplits}); s >= 2; --s) {
-        const int mc = tc_max_clusters(bn, s, deep);
+        const int mc = tc_max_clusters(bn, s, deep, fused);
         if (verbose)
             fprintf(stderr, "[pipo] tc plan: bh=%d deep=%d tiles=%d nkb=%d s=%d max_clusters=%d\n", bn, (int)deep, tiles,
                     nkb, s, mc);
@@ -488,13 +539,72 @@ TcPlan tc_plan(int sms, int bn, int tiles, int nkb) {
     return {1, deep};
 }
 
-// Projection on the tensor cores: bf16 activations (prep kernel), then the
-// tcgen05 GEMM.  Eligible: bf16 weights, K % 64 == 0, rows >= 128, B <= 128.
-pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int splits_req) {
+// The activation split can run inside the GEMM: activation segments only (no
+// embedding gathers), at most one RMSNorm (a single segment, or one joint norm
+// over both), TMA-addressable rows.
+bool tcf_eligible(const GemvParams& p) {
+    for (int s = 0; s < p.nseg; ++s) {
+        const Seg& sg = p.seg[s];
+        if (!sg.src || reinterpret_cast<uintptr_t>(sg.src) % 16 != 0 || sg.ld % 4 != 0 || sg.K % kTcBK != 0) return false;
+    }
+    if (p.nseg == 2 && !p.joint_norm && (p.seg[0].gamma || p.seg[1].gamma)) return false;
+    if (p.zero_ptr && p.epi == EPI_ARGMAX) return false;  // block 0 zeroes keys the other blocks update
+    return true;
+}
+
+bool tc_prep_forced() {
+    const char* ev = getenv("PIPO_TC_PREP");
+    return ev && ev[0] == '1';
+}
+
+// Widest batch width that runs the fused form.  Measured on the 4B shapes:
+// fused ahead at BH 16 (B = 4: 3.08 -> 2.84 ms, B = 16: 3.29 -> 2.86 ms per
+// step), behind at BH 64 (5.02 -> 5.33 ms), where the fp32 activation tile
+// halves the pipeline depth.  PIPO_TC_FUSED_MAX_BH overrides.
+int tc_fused_max_bh() {
+    static const int v = [] {
+        const char* ev = getenv("PIPO_TC_FUSED_MAX_BH");
+        return ev ? atoi(ev) : 32;
+    }();
+    return v;
+}
+
+// Projection on the tensor cores: the fused GEMM, or bf16 activations from
+// prep_bf16_kernel and then the tcgen05 GEMM.  Eligible: bf16 weights,
+// K % 64 == 0, rows >= 128, B <= 128.  x_rows: rows behind each activation
+// pointer (the tensor maps read no further; at least BH for box-sized maps).
+pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int splits_req, int x_rows) {
     const int ru = p.epi == EPI_SWIGLU ? 2 : 1;
     const int rows = p.N * ru, bn = tc_bn(p.B), tiles = (rows + kTcM - 1) / kTcM, nkb = p.K / kTcBK;
-    TcPlan plan = tc_plan(ctx->sms, bn, tiles, nkb);
+    const bool fused = tcf_eligible(p) && !tc_prep_forced() && x_rows >= bn && bn <= tc_fused_max_bh();
+    TcPlan plan = tc_plan(ctx->sms, bn, tiles, nkb, fused);
     if (splits_req > 0) plan.splits = std::min({splits_req, nkb, kTcMaxSplits});
+    TcParams tp{};
+    tp.rows = rows; tp.K = p.K; tp.B = p.B; tp.ru = ru; tp.epi = p.epi;
+    tp.y = p.y; tp.ldy = p.ldy; tp.bias = p.bias; tp.am = p.am; tp.dbg = p.dbg; tp.ld_dbg = p.ld_dbg;
+    tp.splits = plan.splits;
+    if (fused) {
+        CUtensorMap tmW, tmX0, tmX1;
+        TRY(make_tmap(ctx, &tmW, p.W, p.K, rows, kTcM));
+        TRY(make_tmap_x(ctx, &tmX0, p.seg[0].src, p.seg[0].K, p.seg[0].ld, x_rows, bn));
+        if (p.nseg == 2) TRY(make_tmap_x(ctx, &tmX1, p.seg[1].src, p.seg[1].K, p.seg[1].ld, x_rows, bn));
+        else tmX1 = tmX0;
+        TcfIn in{};
+        in.nseg = p.nseg;
+        in.K0 = p.seg[0].K;
+        in.norm = p.seg[0].gamma != nullptr;
+        in.klen = p.joint_norm ? p.K : p.seg[0].K;
+        in.gamma = p.seg[0].gamma;
+        in.eps = p.eps;
+        in.B = p.B;
+        in.zero_ptr = p.zero_ptr;
+        in.zero_n = p.zero_n;
+        void* args[] = {&tmW, &tmX0, &tmX1, &in, &tp};
+        ctx->prof_kind = 0;
+        ctx->prof_bytes = (double)rows * p.K * 2;
+        return launch_ex(ctx, pick_tcv(bn, plan.deep, true), dim3(tiles * plan.splits), dim3(kTcfThreads),
+                         tcv_smem(bn, plan.deep, true), args, plan.splits);
+    }
     const int splits = plan.splits;
     CUtensorMap tmW, tmX;
     TRY(make_tmap(ctx, &tmW, p.W, p.K, rows, kTcM));
@@ -508,10 +618,6 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
         TRY(launch_ex(ctx, reinterpret_cast<const void*>(&prep_bf16_kernel<bf16>), dim3(bn), dim3(kPrepThreads), 0,
                       args));
     }
-    TcParams tp{};
-    tp.rows = rows; tp.K = p.K; tp.B = p.B; tp.ru = ru; tp.epi = p.epi;
-    tp.y = p.y; tp.ldy = p.ldy; tp.bias = p.bias; tp.am = p.am; tp.dbg = p.dbg; tp.ld_dbg = p.ld_dbg;
-    tp.splits = splits;
     void* args[] = {&tmW, &tmX, &tp};
     ctx->prof_kind = 0;
     ctx->prof_bytes = (double)rows * p.K * 2;
@@ -529,7 +635,7 @@ pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
     const bool bf = ctx->cfg.dtype == 1;
     const bool two = p.epi == EPI_SWIGLU;
     if (tc_eligible(ctx, p))
-        return launch_gemm_tc(ctx, p, ctx->tc_xb, ctx->tc_splits);
+        return launch_gemm_tc(ctx, p, ctx->tc_xb, ctx->tc_splits, ctx->act_rows);
     if (ctx->rec) {
         Phase ph{};
         ph.type = PH_GEMV;
@@ -744,10 +850,9 @@ cudaError_t set_carveouts(bool bf) {
                 fns.push_back(bf ? pick_stream<bf16>(nb, ru, rows) : pick_stream<float>(nb, ru, rows));
         }
     if (bf) {
-        for (int bn : {16, 32, 64, 128}) {
-            fns.push_back(pick_tc(bn, false));
-            fns.push_back(pick_tc(bn, true));
-        }
+        for (int bn : {16, 32, 64, 128})
+            for (bool deep : {false, true})
+                for (bool fused : {false, true}) fns.push_back(pick_tcv(bn, deep, fused));
         fns.push_back(reinterpret_cast<const void*>(&prep_bf16_kernel<bf16>));
         for (int g : {1, 2, 4}) fns.push_back(attnm_pick(g));
     }
@@ -1313,13 +1418,17 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
 
         // activations and state
         const int qd = c.n_q_heads * DH, kd = c.n_kv_heads * DH;
-        TRY(dalloc(ctx, &ctx->x, (size_t)MB * H * 4));
-        TRY(dalloc(ctx, &ctx->x2, (size_t)MB * H * 4));
+        // GEMM inputs get at least as many rows as the tensor-core batch width
+        // (their activation tensor maps read box-sized tiles of BH rows)
+        ctx->act_rows = c.dtype == 1 ? std::max(MB, tc_bn(std::min(MB, 128))) : MB;
+        const size_t AR = (size_t)ctx->act_rows;
+        TRY(dalloc(ctx, &ctx->x, AR * H * 4));
+        TRY(dalloc(ctx, &ctx->x2, AR * H * 4));
         TRY(dalloc(ctx, &ctx->qkv, (size_t)MB * (qd + 2 * kd) * 4));
         TRY(dalloc(ctx, &ctx->q, (size_t)MB * qd * 4));
-        TRY(dalloc(ctx, &ctx->attn, (size_t)MB * qd * 4));
-        TRY(dalloc(ctx, &ctx->act, (size_t)MB * c.ffn * 4));
-        TRY(dalloc(ctx, &ctx->t, (size_t)MB * H * 4));
+        TRY(dalloc(ctx, &ctx->attn, AR * qd * 4));
+        TRY(dalloc(ctx, &ctx->act, AR * c.ffn * 4));
+        TRY(dalloc(ctx, &ctx->t, AR * H * 4));
         size_t parts = 0;
         for (int b = 1; b <= MB; ++b) parts = std::max(parts, (size_t)b * c.n_q_heads * attn_splits(ctx, b));
         TRY(dalloc(ctx, &ctx->part_o, parts * DH * 4));
@@ -1734,7 +1843,7 @@ pipo_status pipo_op_gemm_tc(int32_t mode, const void* d_W, int32_t N, int32_t K,
             p.W = d_W; p.N = N; p.K = K; p.epi = mode == 1 ? EPI_SWIGLU : EPI_STORE;
             p.y = d_y; p.ldy = N; p.B = B; p.splitk = 1; p.nseg = 1;
             p.seg[0] = act_seg(d_x, K, K);
-            st = launch_gemm_tc(ctx, p, static_cast<bf16*>(d_scratch), splits);
+            st = launch_gemm_tc(ctx, p, static_cast<bf16*>(d_scratch), splits, B);
         }
     }
     if (st != PIPO_OK) g_init_error = op.err;
@@ -1759,9 +1868,12 @@ pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {
     }
     std::string proj;
     const std::string cuda_core = B <= 4 ? "gemv_rows_kernel" : "gemv_kernel";
-    if (n_tc == 4) proj = "gemm_tc_kernel<" + std::to_string(tc_bn(B)) + ">+prep_bf16_kernel (tcgen05)";
-    else if (n_tc > 0) proj = "gemm_tc_kernel<" + std::to_string(tc_bn(B)) + ">+prep_bf16_kernel (tcgen05; " +
-                              std::to_string(4 - n_tc) + " of 4 block projections on " + cuda_core + ")";
+    const bool fused = !tc_prep_forced() && tc_bn(B) <= tc_fused_max_bh();
+    const std::string tck = fused ? "gemm_tcf_kernel<" + std::to_string(tc_bn(B)) + ">"
+                                  : "gemm_tc_kernel<" + std::to_string(tc_bn(B)) + ">+prep_bf16_kernel";
+    if (n_tc == 4) proj = tck + " (tcgen05)";
+    else if (n_tc > 0) proj = tck + " (tcgen05; " + std::to_string(4 - n_tc) + " of 4 block projections on " +
+                              cuda_core + ")";
     else proj = cuda_core;
     const int cs = attn_cluster_size(ctx);
     const bool mma = attn_use_mma(ctx) && cs <= 8;

@@ -119,11 +119,12 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 }
 
 // Epilogue of batch columns [c0, c0+16) of weight row `row` (thread = TMEM
-// lane).  All threads of the warp call it (the SwiGLU pairing shuffles).
+// lane; quad = the warp's TMEM lane quadrant).  All threads of the warp call
+// it (the SwiGLU pairing shuffles).
 template <int BH>
 __device__ __forceinline__ void tc_epilogue16(const TcParams& p, int row, int c0, const float (&v)[16],
-                                              float (*red_v)[BH], int (*red_r)[BH]) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+                                              float (*red_v)[BH], int (*red_r)[BH], int quad) {
+    const int warp = quad, lane = threadIdx.x & 31;
     const bool in = row < p.rows;
     if (p.epi == EPI_ARGMAX) {
 #pragma unroll
@@ -177,10 +178,12 @@ __device__ __forceinline__ int tc_park_idx(int r, int c4) {
 }
 
 // Split-K epilogue of 4 batch columns [4*c4, 4*c4+4) of tile row rr (and, for
-// SwiGLU, its up row rr+1), summed over the cluster in split order.
+// SwiGLU, its up row rr+1), summed over the cluster in split order, scaled by
+// rstd[b] (a per-sequence RMSNorm factor) when rstd is given.
 template <int BH>
 __device__ __forceinline__ void tc_cluster_epilogue(const TcParams& p, cooperative_groups::cluster_group& cl,
-                                                    float* park, int tile, int rr, int c4) {
+                                                    float* park, int tile, int rr, int c4,
+                                                    const float* rstd = nullptr) {
     float4 a = make_float4(0.f, 0.f, 0.f, 0.f), u = a;
     for (int s = 0; s < p.splits; ++s) {
         const float* rem = cl.map_shared_rank(park, s);
@@ -191,7 +194,14 @@ __device__ __forceinline__ void tc_cluster_epilogue(const TcParams& p, cooperati
             u.x += t2.x; u.y += t2.y; u.z += t2.z; u.w += t2.w;
         }
     }
-    const float va[4] = {a.x, a.y, a.z, a.w}, vu[4] = {u.x, u.y, u.z, u.w};
+    float va[4] = {a.x, a.y, a.z, a.w}, vu[4] = {u.x, u.y, u.z, u.w};
+    if (rstd) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            va[j] *= rstd[4 * c4 + j];
+            vu[j] *= rstd[4 * c4 + j];
+        }
+    }
     const int row = tile * kTcM + rr;
     if (row >= p.rows) return;
 #pragma unroll
@@ -325,7 +335,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
         for (int c0 = 0; c0 < BH; c0 += 16) {
             float v[16];
             ld_cols(c0, v);
-            tc_epilogue16<BH>(p, row, c0, v, red_v, red_r);
+            tc_epilogue16<BH>(p, row, c0, v, red_v, red_r, warp);
         }
         if (p.epi == EPI_ARGMAX) {
             __syncthreads();
@@ -364,6 +374,293 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
         for (int it = threadIdx.x; it < items; it += kTcThreads) {
             const int rr = r0 + (it / (BH / 4)) * step, c4 = it % (BH / 4);
             tc_cluster_epilogue<BH>(p, cl, park, tile, rr, c4);
+        }
+        cl.sync();  // no CTA leaves while others still read its shared memory
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kCols);
+    }
+}
+
+// ---------------------------------------------------------------- fused form
+//
+// The same projection with the activation split done inside the GEMM: per
+// stage the producer thread also copies the raw fp32 activation tile
+// [BH rows][64] (TMA, rows past the batch read as zeros) and, for a
+// normalised input, the 64 RMSNorm gains; four converter warps turn it into
+// the swizzled bf16 hi | lo operand tile (rows b and BH + b) in the stage and
+// accumulate sum(x^2) per sequence.  The norm factor rstd[b] =
+// 1/sqrt(mean(x^2) + eps) multiplies the accumulator in the epilogue
+// (W (g . x) rstd is the projection of the normalised input); with K split
+// over a cluster the sums are added over the cluster in split order.  The
+// converter warps are also the epilogue warps (TMEM lane quadrants 2, 3, 0, 1).
+// Inputs: one activation segment, or two under one joint norm (no gathers,
+// no separate norms of two segments: those keep prep_bf16_kernel).
+constexpr int kTcfThreads = 192;  // W producer, MMA issuer, 4 converter / epilogue warps
+
+__host__ __device__ constexpr int tcf_stages(int bh, bool deep) {
+    return deep ? (bh <= 16 ? 8 : bh <= 32 ? 6 : bh <= 64 ? 4 : 2) : (bh <= 16 ? 4 : bh <= 32 ? 3 : 2);
+}
+// stage: W tile, bf16 operand tile [2BH][64], raw fp32 tile [BH][64], gains (128 B), 1024-byte aligned
+__host__ __device__ constexpr int tcf_stage_bytes(int bh) { return kTcABytes + 512 * bh + 1024; }
+
+struct TcfIn {
+    int nseg, K0, norm, klen;  // segments, length of segment 0, norm applied, norm length
+    const void* gamma;         // [K] bf16 gains (joint or single segment) when norm
+    float eps;
+    int B;
+    unsigned long long* zero_ptr;  // zeroed by block 0 before anything else (or nullptr)
+    int zero_n;
+};
+
+template <int BH, int ST>
+__global__ void __launch_bounds__(kTcfThreads, 1)
+    gemm_tcf_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX0,
+                    const __grid_constant__ CUtensorMap tmX1, TcfIn in, TcParams p) {
+    extern __shared__ __align__(1024) unsigned char tcf_smem_raw[];
+    constexpr int BN = 2 * BH;
+    constexpr int SB = tcf_stage_bytes(BH);
+    constexpr int kBOff = kTcABytes, kRawOff = kTcABytes + 256 * BH, kGmOff = kTcABytes + 512 * BH;
+    constexpr uint32_t kCols = BN <= 32 ? 32u : BN <= 64 ? 64u : BN <= 128 ? 128u : 256u;
+    constexpr int NQ = BH / 16;  // conversion tasks per converter thread per stage
+    static_assert(kTcM * BH * 4 <= ST * SB, "parked tile must fit in the stages");
+    unsigned char* sm = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(tcf_smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint64_t* full_raw = reinterpret_cast<uint64_t*>(sm + (size_t)ST * SB);
+    uint64_t* full_mma = full_raw + ST;
+    uint64_t* empty = full_mma + ST;
+    uint64_t* accb = empty + ST;
+    __shared__ uint32_t tmem_base;
+    __shared__ float red_v[4][BH];
+    __shared__ int red_r[4][BH];
+    __shared__ float ss_s[BH], rstd_s[BH];
+
+    pdl_launch();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tile = blockIdx.x / p.splits, split = blockIdx.x % p.splits;
+    const int nkb = p.K / kTcBK;
+    const int kb0 = (int)((long long)split * nkb / p.splits), kb1 = (int)((long long)(split + 1) * nkb / p.splits);
+    const int nk = kb1 - kb0;  // >= 1 (splits <= nkb)
+    const uint32_t raw_bytes = (uint32_t)(BH * kTcBK * 4) + (in.norm ? 128u : 0u);
+
+    if (warp == 0) tmem_alloc(&tmem_base, kCols);
+    if (threadIdx.x == 32) {
+        for (int s = 0; s < ST; ++s) {
+            mbar_init(full_raw + s, 1);
+            mbar_init(full_mma + s, 4);
+            mbar_init(empty + s, 1);
+        }
+        mbar_init(accb, 1);
+        mbar_init_fence();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // producer: weights and gains of the first ST stages before the
+            // dependency wait, the activation tiles after it
+            auto x_tile = [&](int i, unsigned char* stg, uint64_t* bar) {
+                const int k = (kb0 + i) * kTcBK;
+                if (in.nseg == 2 && k >= in.K0) tma_load_2d(stg + kRawOff, &tmX1, k - in.K0, 0, bar);
+                else tma_load_2d(stg + kRawOff, &tmX0, k, 0, bar);
+            };
+            const int pre = min(nk, ST);
+            for (int i = 0; i < pre; ++i) {
+                unsigned char* stg = sm + (size_t)i * SB;
+                mbar_arrive_expect_tx(full_raw + i, (uint32_t)kTcABytes + raw_bytes);
+                tma_load_2d(stg, &tmW, (kb0 + i) * kTcBK, tile * kTcM, full_raw + i);
+                if (in.norm)
+                    bulk_g2s(stg + kGmOff, static_cast<const __nv_bfloat16*>(in.gamma) + (size_t)(kb0 + i) * kTcBK,
+                             128, full_raw + i);
+            }
+            pdl_wait();
+            for (int i = 0; i < pre; ++i) x_tile(i, sm + (size_t)i * SB, full_raw + i);
+            int issued = pre;
+            for (int i = pre; i < nk; ++i) {
+                const int s = i % ST;
+                if (!mbar_wait(empty + s, (uint32_t)(((i / ST) & 1) ^ 1), 11, i)) break;
+                unsigned char* stg = sm + (size_t)s * SB;
+                mbar_arrive_expect_tx(full_raw + s, (uint32_t)kTcABytes + raw_bytes);
+                tma_load_2d(stg, &tmW, (kb0 + i) * kTcBK, tile * kTcM, full_raw + s);
+                if (in.norm)
+                    bulk_g2s(stg + kGmOff, static_cast<const __nv_bfloat16*>(in.gamma) + (size_t)(kb0 + i) * kTcBK,
+                             128, full_raw + s);
+                x_tile(i, stg, full_raw + s);
+                issued = i + 1;
+            }
+            for (int i = max(0, issued - ST); i < issued; ++i)
+                mbar_wait(full_raw + (i % ST), (uint32_t)((i / ST) & 1), 12, i);
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // MMA issuer: a stage is ready once the converter warps filled its operand tile
+            const uint32_t idesc = umma_idesc_bf16(kTcM, BN);
+            for (int i = 0; i < nk; ++i) {
+                const int s = i % ST;
+                if (!mbar_wait(full_mma + s, (uint32_t)((i / ST) & 1), 13, i)) break;
+                tc_fence_after();
+                const uint32_t a0 = smem_u32(sm + (size_t)s * SB), b0 = a0 + kBOff;
+#pragma unroll
+                for (int k = 0; k < kTcBK / 16; ++k)
+                    umma_bf16(tmem, umma_desc_sw128(a0 + k * 32), umma_desc_sw128(b0 + k * 32), idesc,
+                              (i > 0 || k > 0) ? 1u : 0u);
+                umma_commit(empty + s);
+            }
+            umma_commit(accb);
+        }
+        __syncwarp();
+    } else {
+        // converter warps: raw fp32 tile -> bf16 hi | lo operand tile, sum(x^2)
+        const int xt = threadIdx.x - 64;  // 0..127
+        pdl_wait();
+        if (in.zero_ptr && blockIdx.x == 0)
+            for (int i = xt; i < in.zero_n; i += 128) in.zero_ptr[i] = 0ull;
+        float ss[NQ];
+#pragma unroll
+        for (int q = 0; q < NQ; ++q) ss[q] = 0.f;
+        for (int i = 0; i < nk; ++i) {
+            const int s = i % ST;
+            if (!mbar_wait(full_raw + s, (uint32_t)((i / ST) & 1), 15, i)) break;
+            unsigned char* stg = sm + (size_t)s * SB;
+            const float* raw = reinterpret_cast<const float*>(stg + kRawOff);
+            float gm[8];
+            const int c = xt & 7;  // 8-element chunk of the 64-wide stage (same for every task)
+            if (in.norm) {
+                const uint4 g4 = *reinterpret_cast<const uint4*>(stg + kGmOff + c * 16);
+                gm[0] = bf_lo(g4.x); gm[1] = bf_hi(g4.x); gm[2] = bf_lo(g4.y); gm[3] = bf_hi(g4.y);
+                gm[4] = bf_lo(g4.z); gm[5] = bf_hi(g4.z); gm[6] = bf_lo(g4.w); gm[7] = bf_hi(g4.w);
+            }
+#pragma unroll
+            for (int q = 0; q < NQ; ++q) {
+                const int b = (xt >> 3) + 16 * q;
+                const float4 r0 = *reinterpret_cast<const float4*>(raw + b * kTcBK + c * 8);
+                const float4 r1 = *reinterpret_cast<const float4*>(raw + b * kTcBK + c * 8 + 4);
+                float x[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+                if (b >= in.B) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) x[e] = 0.f;
+                }
+                if (in.norm) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        ss[q] += x[e] * x[e];
+                        x[e] *= gm[e];
+                    }
+                }
+                uint32_t hi[4], lo[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const __nv_bfloat162 h = __floats2bfloat162_rn(x[2 * e], x[2 * e + 1]);
+                    const float2 hf = __bfloat1622float2(h);
+                    const __nv_bfloat162 l = __floats2bfloat162_rn(x[2 * e] - hf.x, x[2 * e + 1] - hf.y);
+                    hi[e] = *reinterpret_cast<const uint32_t*>(&h);
+                    lo[e] = *reinterpret_cast<const uint32_t*>(&l);
+                }
+                const int sw = (c ^ (b & 7)) << 4;
+                *reinterpret_cast<uint4*>(stg + kBOff + b * 128 + sw) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                *reinterpret_cast<uint4*>(stg + kBOff + (BH + b) * 128 + sw) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            }
+            fence_proxy_async();  // the generic-proxy stores above, before the MMAs read them
+            __syncwarp();
+            if (lane == 0) mbar_arrive(full_mma + s);
+        }
+        // sum(x^2) of sequence b over this CTA's K range
+#pragma unroll
+        for (int q = 0; q < NQ; ++q) {
+            float v = ss[q];
+            v += __shfl_xor_sync(0xffffffffu, v, 1);
+            v += __shfl_xor_sync(0xffffffffu, v, 2);
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            if ((xt & 7) == 0) ss_s[(xt >> 3) + 16 * q] = v;
+        }
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+        if (p.splits == 1 && xt < BH)
+            rstd_s[xt] = in.norm ? 1.0f / sqrtf(ss_s[xt] / (float)in.klen + in.eps) : 1.0f;
+        asm volatile("bar.sync 1, 128;" ::: "memory");
+    }
+
+    // ---- epilogue: the converter warps hold TMEM lane quadrants 2, 3, 0, 1
+    const int quad = warp & 3;
+    const int row = tile * kTcM + quad * 32 + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(quad * 32) << 16);
+    const bool epi_warp = warp >= 2;
+    if (epi_warp) {
+        mbar_wait(accb, 0, 14, (unsigned)nk);
+        __syncwarp();
+        tc_fence_after();
+    }
+    auto ld_cols = [&](int c0, float (&v)[16]) {
+        float lo[16];
+        tmem_ld16(lane_addr + c0, v);
+        tmem_ld16(lane_addr + BH + c0, lo);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] += lo[j];
+    };
+    if (p.splits == 1) {
+        if (epi_warp) {
+#pragma unroll 1
+            for (int c0 = 0; c0 < BH; c0 += 16) {
+                float v[16];
+                ld_cols(c0, v);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) v[j] *= rstd_s[c0 + j];
+                tc_epilogue16<BH>(p, row, c0, v, red_v, red_r, quad);
+            }
+            if (p.epi == EPI_ARGMAX) {
+                asm volatile("bar.sync 1, 128;" ::: "memory");
+                const int b = threadIdx.x - 64;
+                if (b < p.B) {
+                    float bv = -INFINITY;
+                    int br = 0x7fffffff;
+                    for (int w = 0; w < 4; ++w)
+                        if (red_r[w][b] != 0x7fffffff &&
+                            (red_v[w][b] > bv || (red_v[w][b] == bv && red_r[w][b] < br))) {
+                            bv = red_v[w][b];
+                            br = red_r[w][b];
+                        }
+                    if (br != 0x7fffffff) atomicMax(p.am + b, argmax_key(bv, br));
+                }
+            }
+        }
+    } else {
+        namespace cg = cooperative_groups;
+        cg::cluster_group cl = cg::this_cluster();
+        float* park = reinterpret_cast<float*>(sm);
+        if (epi_warp) {
+            const int r = quad * 32 + lane;
+#pragma unroll 1
+            for (int c0 = 0; c0 < BH; c0 += 16) {
+                float v[16];
+                ld_cols(c0, v);
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    *reinterpret_cast<float4*>(park + tc_park_idx<BH>(r, c0 / 4 + q)) =
+                        make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            }
+        }
+        cl.sync();  // every split's partial tile and sum(x^2) are in place
+        if (epi_warp) {
+            const int xt = threadIdx.x - 64;
+            if (xt < BH) {
+                float t = 0.f;
+                for (int rk = 0; rk < p.splits; ++rk) t += *cl.map_shared_rank(&ss_s[xt], rk);
+                rstd_s[xt] = in.norm ? 1.0f / sqrtf(t / (float)in.klen + in.eps) : 1.0f;
+            }
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            const int R = (((kTcM + p.splits - 1) / p.splits) + 1) & ~1;
+            const int r0 = min(kTcM, split * R), r1 = min(kTcM, r0 + R);
+            const int step = p.ru == 2 ? 2 : 1;
+            const int items = (r1 - r0) / step * (BH / 4);
+            for (int it = xt; it < items; it += 128) {
+                const int rr = r0 + (it / (BH / 4)) * step, c4 = it % (BH / 4);
+                tc_cluster_epilogue<BH>(p, cl, park, tile, rr, c4, rstd_s);
+            }
         }
         cl.sync();  // no CTA leaves while others still read its shared memory
     }

@@ -106,7 +106,7 @@ def test_decode_path_uses_tensor_core_kernels():
     try:
         g.prefill(synth.gen_prompts(16, 8, MID.V, seed=1).numpy())
         d = g.describe()
-        assert "gemm_tc_kernel<16>" in d and "1 of 4 block projections on gemv_kernel" in d, d
+        assert "gemm_tcf_kernel<16>" in d and "1 of 4 block projections on gemv_kernel" in d, d
         assert "attn_mma_kernel" in d, d
     finally:
         g.close()

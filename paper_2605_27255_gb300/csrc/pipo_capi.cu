@@ -74,7 +74,7 @@ struct pipo_ctx {
     bf16* tc_xb = nullptr;          // [2 * tc_bn_max][tc_kmax] bf16 activations (hi rows, lo rows)
     int tc_kmax = 0, tc_bn_max = 0;
     int act_rows = 0;               // rows of the fp32 activation buffers (>= the batch width BH)
-    int tc_min_b = 4;               // measured: tensor cores ahead of the CUDA-core GEMV from B = 4
+    int tc_min_b = 2;               // measured: a tie with the CUDA-core GEMV at B = 1, far ahead from B = 4
     int tc_splits = 0;              // forced K splits (0: automatic)
 
     int32_t *pending = nullptr, *n_pos = nullptr, *out_tokens = nullptr, *out_nacc = nullptr;

@@ -4,6 +4,14 @@ kernel and its GEMM, both in the timed region).
 
   python -m paper_2605_27255_gb300.kernel_bench --shape lm_head [--batch 1] [--iters 50] [--tc] [--splits S]
 
+With --step, one eagerly launched decode step (pipo_profile_step, inside an
+NVTX range "profile_step") of a small bf16 model -- 512 wide, 3 layers, 8/2
+heads of 128, the attention shape of the 4B model -- with every cache filled
+to --ctx seeded entries: a small case for profiler captures of the attention
+and projection kernels.
+
+  python -m paper_2605_27255_gb300.kernel_bench --step --batch 64 --ctx 512
+
 Shapes are the weight-streaming projections of the 4B-class model.  Weights
 are random bf16; several copies are cycled so that every launch streams from
 HBM (more than twice the 129 MB L2 in total).  Prints one JSON line per shape
@@ -64,6 +72,40 @@ def run(name: str, batch: int, iters: int, min_bytes: float = 300e6, tc: bool = 
                 gbs=nbytes / us / 1e3, bytes_per_launch=nbytes, copies=copies)
 
 
+STEP_SHAPE = dict(name="step", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1408, V=5056, compressor="mlp",
+                  mtp_block=1, dtype="bf16", rope_theta=1.0e6, tau=0.5)
+
+
+def run_step(batch: int, ctx: int) -> dict:
+    from . import synth
+    shape = synth.ModelShape(**STEP_SHAPE)
+    w = synth.gen_weights(shape, seed=0, device="cuda")
+    g = capi.Pipo(shape, w, max_batch=batch, max_ctx=ctx + 16)
+    try:
+        g.prefill(synth.gen_prompts(batch, 2, shape.V, seed=1).numpy())
+        K, V = synth.gen_kv_fill(shape, ctx, seed=7, device="cuda")
+        K, V = K.cpu().numpy(), V.cpu().numpy()
+        for b in range(batch):
+            g.load_cache(b, K, V)
+        for _ in range(3):
+            g.step_async()
+        torch.cuda.synchronize()
+        torch.cuda.nvtx.range_push("profile_step")
+        kind, by, ms = g.profile_step()
+        torch.cuda.nvtx.range_pop()
+        torch.cuda.synchronize()
+        out = dict(kernel="decode_step", shape=STEP_SHAPE["name"], batch=batch, ctx=ctx, path=g.describe(),
+                   launches=len(kind))
+        for k, name in ((0, "projections"), (1, "attention"), (2, "other")):
+            sel = [i for i, kk in enumerate(kind) if int(kk) == k]
+            t = float(sum(ms[i] for i in sel))
+            b = float(sum(by[i] for i in sel))
+            out[name] = dict(launches=len(sel), ms=t, gbs=(b / (t / 1e3) / 1e9) if t > 0 and b > 0 else None)
+        return out
+    finally:
+        g.close()
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--shape", default="all", choices=["all"] + sorted(SHAPES))
@@ -71,8 +113,13 @@ def main() -> None:
     ap.add_argument("--iters", type=int, default=50)
     ap.add_argument("--tc", action="store_true", help="tensor-core projection (bf16 hi/lo activations)")
     ap.add_argument("--splits", type=int, default=0, help="K splits of the tensor-core GEMM (0: automatic)")
+    ap.add_argument("--step", action="store_true", help="one eager decode step of a small bf16 model")
+    ap.add_argument("--ctx", type=int, default=512, help="--step: cached entries per sequence")
     a = ap.parse_args()
     capi.load()
+    if a.step:
+        print(json.dumps(run_step(a.batch, a.ctx)), flush=True)
+        return
     for name in (sorted(SHAPES) if a.shape == "all" else [a.shape]):
         print(json.dumps(run(name, a.batch, a.iters, tc=a.tc, splits=a.splits)), flush=True)
 

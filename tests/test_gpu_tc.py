@@ -100,7 +100,8 @@ def test_mid_bf16_cuda_core_batches_over_8(monkeypatch):
 
 def test_decode_path_uses_tensor_core_kernels():
     """At B = 16 the block projections and the attention take the tcgen05 and
-    mma.sync kernels (the down projection, K = 1376, stays on CUDA cores)."""
+    mma.sync kernels (the down projection, K = 1376, stays on CUDA cores); a
+    single sequence stays on the CUDA-core GEMV and attention."""
     w = synth.gen_weights(MID, seed=23)
     g = capi.Pipo(MID, w, max_batch=16, max_ctx=40)
     try:
@@ -110,9 +111,9 @@ def test_decode_path_uses_tensor_core_kernels():
         assert "attn_mma_kernel" in d, d
     finally:
         g.close()
-    g = capi.Pipo(MID, w, max_batch=2, max_ctx=40)
+    g = capi.Pipo(MID, w, max_batch=1, max_ctx=40)
     try:
-        g.prefill(synth.gen_prompts(2, 8, MID.V, seed=1).numpy())
+        g.prefill(synth.gen_prompts(1, 8, MID.V, seed=1).numpy())
         d = g.describe()
         assert "projections=gemv_rows_kernel" in d and "attention=attn_cluster_kernel cluster=8" in d, d
     finally:

@@ -74,6 +74,7 @@ struct pipo_ctx {
     bf16* tc_xb = nullptr;          // [2 * tc_bn_max][tc_kmax] bf16 activations (hi rows, lo rows)
     int tc_kmax = 0, tc_bn_max = 0;
     int act_rows = 0;               // rows of the fp32 activation buffers (>= the batch width BH)
+    bool tc_shallow = false;        // this step's projections: two-per-SM ring (room for a co-resident neighbour)
     int tc_min_b = 2;               // measured: a tie with the CUDA-core GEMV at B = 1, far ahead from B = 4
     int tc_splits = 0;              // forced K splits (0: automatic)
 
@@ -520,12 +521,12 @@ struct TcPlan {
     int splits;
     bool deep;
 };
-TcPlan tc_plan(int sms, int bn, int tiles, int nkb, bool fused) {
+TcPlan tc_plan(int sms, int bn, int tiles, int nkb, bool fused, bool allow_deep = true) {
     static const int force_deep = [] {
         const char* ev = getenv("PIPO_TC_DEEP");
         return ev ? atoi(ev) : -1;
     }();
-    const bool deep = force_deep >= 0 ? force_deep == 1 : tiles <= sms;
+    const bool deep = force_deep >= 0 ? force_deep == 1 : (allow_deep && tiles <= sms);
     const int target = sms * tc_ctas_per_sm(bn, deep, fused);
     if (tiles >= target) return {1, deep};
     static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
@@ -577,7 +578,7 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
     const int ru = p.epi == EPI_SWIGLU ? 2 : 1;
     const int rows = p.N * ru, bn = tc_bn(p.B), tiles = (rows + kTcM - 1) / kTcM, nkb = p.K / kTcBK;
     const bool fused = tcf_eligible(p) && !tc_prep_forced() && x_rows >= bn && bn <= tc_fused_max_bh();
-    TcPlan plan = tc_plan(ctx->sms, bn, tiles, nkb, fused);
+    TcPlan plan = tc_plan(ctx->sms, bn, tiles, nkb, fused, !ctx->tc_shallow);
     if (splits_req > 0) plan.splits = std::min({splits_req, nkb, kTcMaxSplits});
     TcParams tp{};
     tp.rows = rows; tp.K = p.K; tp.B = p.B; tp.ru = ru; tp.epi = p.epi;
@@ -905,6 +906,30 @@ int attn_cluster_size(const pipo_ctx* ctx) {
     return cs;
 }
 
+// Long attention: the cached K/V bytes of a layer are at least six times the
+// QKV weight bytes (cached lengths at graph capture).  Then every projection
+// takes the two-per-SM ring, whose shared memory leaves room for a
+// neighbouring kernel's CTAs: under programmatic dependent launch the
+// attention starts streaming the cache during the QKV projection and each
+// projection prefetches its weights during the kernel before it.  Measured on
+// 4B (ratio of cache to QKV bytes in brackets): B=4 at ~15.9 K cached pairs
+// [8.3] 5.82 -> 4.73 ms per step; B=64 at ~530 pairs [4.4] 5.07 (deep) vs
+// 5.38 ms with the QKV and O projections shallow; B=16 [1.1] 2.87 (deep) vs
+// 3.08 ms all shallow.  PIPO_TC_SHALLOW_ATTN=0/1 overrides.
+bool attn_is_long(const pipo_ctx* ctx) {
+    static const int force = [] {
+        const char* ev = getenv("PIPO_TC_SHALLOW_ATTN");
+        return ev ? atoi(ev) : -1;
+    }();
+    if (force >= 0) return force == 1;
+    const pipo_config& c = ctx->cfg;
+    double ctx_sum = 0.0;
+    for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b) ctx_sum += ctx->h_len[b];
+    const double kv_bytes = ctx_sum * c.n_kv_heads * c.head_dim * 2.0 * ctx->esz;
+    const double qkv_bytes = (double)(c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim * c.hidden * ctx->esz;
+    return kv_bytes >= 6.0 * qkv_bytes;
+}
+
 // One decoder block on the residual stream xr (pre-norm attention + SwiGLU).
 pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, float* xr) {
     const pipo_config& c = ctx->cfg;
@@ -1023,6 +1048,7 @@ pipo_status enqueue_lm_head(pipo_ctx* ctx, const float* h, const void* gamma, un
 // prompt pair j.  PREFILL_MID stops after the MTP block (teacher-forced token).
 pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
     const pipo_config& c = ctx->cfg;
+    ctx->tc_shallow = attn_is_long(ctx);
     const int H = c.hidden, B = ctx->B;
     const bool bf = c.dtype == 1;
     unsigned long long* am_b = ctx->am;

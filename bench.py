@@ -123,6 +123,22 @@ def dist_env():
     return int(os.environ.get("RANK", "0")), ws, int(os.environ.get("LOCAL_RANK", "0"))
 
 
+def aggregate_ranks(ms, tokens, e2e_s, e2e_tokens, device):
+    """Whole-job figures over the ranks of a torch.distributed job: the
+    slowest rank's times (max) and the tokens of all ranks (sum).  A single
+    process returns its own figures."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return ms, tokens, e2e_s, e2e_tokens
+    t = torch.tensor([ms, tokens, e2e_s, e2e_tokens], dtype=torch.float64, device=device)
+    mx = t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    sm = t.clone()
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    return float(mx[0]), float(sm[1]), float(mx[2]), float(sm[3])
+
+
 def build_weights(shape, device):
     from paper_2605_27255_gb300 import synth
     return synth.gen_weights(shape, seed=0, device=device)
@@ -288,15 +304,7 @@ def run_pipo(args):
             kb[int(kk)][2] += 1
     tot_ms = sum(v[1] for v in kb.values())
 
-    if ws > 1:
-        t = torch.tensor([ms, tokens, e2e_s, e2e_tokens], dtype=torch.float64, device="cuda")
-        mx = t.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        sm = t.clone()
-        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-        ms_all, tokens_all, e2e_all, e2e_tok_all = float(mx[0]), float(sm[1]), float(mx[2]), float(sm[3])
-    else:
-        ms_all, tokens_all, e2e_all, e2e_tok_all = ms, tokens, e2e_s, e2e_tokens
+    ms_all, tokens_all, e2e_all, e2e_tok_all = aggregate_ranks(ms, tokens, e2e_s, e2e_tokens, "cuda")
     value = tokens_all / (ms_all / 1e3)
     hbm, tf, src = peaks()
     step_s = ms / 1e3 / K

@@ -887,20 +887,20 @@ bool attn_mma_ok(const pipo_ctx* ctx) {
 // cores (measured: below it the register-ring attention is slightly faster
 // next to the CUDA-core GEMVs, from B = 4 the tensor-core one by far), with
 // the cache tensor maps in place
-bool attn_use_mma(const pipo_ctx* ctx) {
-    return attn_mma_ok(ctx) && ctx->B >= ctx->tc_min_b && (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers;
+bool attn_use_mma(const pipo_ctx* ctx, int B) {
+    return attn_mma_ok(ctx) && B >= ctx->tc_min_b && (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers;
 }
 
 // CTAs per (sequence, kv head) of the clustered attention: 8 while the batch
 // leaves SMs idle (16 where allowed and still under two per SM), fewer as the
 // (sequence, kv head) pairs alone fill the GPU.
-int attn_cluster_size(const pipo_ctx* ctx) {
+int attn_cluster_size(const pipo_ctx* ctx, int B) {
     if (ctx->attn_cs_force) return ctx->attn_cs_force;
-    const long long pairs = (long long)ctx->B * ctx->cfg.n_kv_heads;
+    const long long pairs = (long long)B * ctx->cfg.n_kv_heads;
     if (ctx->attn_cs16 && pairs * 16 <= 2 * ctx->sms) return 16;
     // measured best: about two tensor-core attention CTAs per SM (they are
     // resident two at a time), one register-ring CTA per SM
-    const long long target = ctx->attn_cs_target > 0 ? ctx->attn_cs_target : (attn_use_mma(ctx) ? 2 : 1);
+    const long long target = ctx->attn_cs_target > 0 ? ctx->attn_cs_target : (attn_use_mma(ctx, B) ? 2 : 1);
     int cs = 8;
     while (cs > 1 && pairs * cs > target * ctx->sms) cs >>= 1;
     return cs;
@@ -973,9 +973,9 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         ap.out = ctx->attn;
         ap.scale = 1.0f / sqrtf((float)DH);
         void* args[] = {&ap};
-        const int cs = attn_cluster_size(ctx);
+        const int cs = attn_cluster_size(ctx, ctx->B);
         const int G = c.n_q_heads / c.n_kv_heads;
-        if (attn_use_mma(ctx) && cs <= 8) {
+        if (attn_use_mma(ctx, ctx->B) && cs <= 8) {
             void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
             TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, ctx->B), dim3(kMmaThreads), mma_attn_smem(),
                           margs, cs));
@@ -1901,8 +1901,8 @@ pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {
     else if (n_tc > 0) proj = tck + " (tcgen05; " + std::to_string(4 - n_tc) + " of 4 block projections on " +
                               cuda_core + ")";
     else proj = cuda_core;
-    const int cs = attn_cluster_size(ctx);
-    const bool mma = attn_use_mma(ctx) && cs <= 8;
+    const int cs = attn_cluster_size(ctx, B);
+    const bool mma = attn_use_mma(ctx, B) && cs <= 8;
     const std::string d = "B=" + std::to_string(B) + " projections=" + proj + " attention=" +
                           (ctx->attn_v0 ? std::string("attn_decode_kernel") : mma ? "attn_mma_kernel" : "attn_cluster_kernel") +
                           " cluster=" + std::to_string(cs);

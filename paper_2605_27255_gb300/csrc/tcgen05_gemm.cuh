@@ -1,12 +1,13 @@
 // Tensor-core (tcgen05 / TMEM) skinny GEMM for batched projections, sm_103a.
 //
-// When B * pairs makes a projection a real dense contraction (B >= 16), the
-// weight stream is fed to the 5th-generation tensor cores instead of CUDA
-// cores.  Swap-AB: D[rows, B] = W[rows, K] . X[B, K]^T, so the 128 weight rows
-// of a tile fill the MMA's M = 128 and the batch (padded to a multiple of 16)
-// is its N.  Both operands are K-major bf16 tiles loaded by TMA tensor copies
-// with 128-byte swizzle into a shared-memory ring of ST stages (mbarrier
-// completion; ST chosen so that two CTAs fit on an SM).  One thread issues the
+// For batches of two sequences and more the weight stream is fed to the
+// 5th-generation tensor cores instead of CUDA cores (every weight byte then
+// serves the whole batch at once).  Swap-AB: D[rows, B] = W[rows, K] .
+// X[B, K]^T, so the 128 weight rows of a tile fill the MMA's M = 128 and the
+// batch (padded to a multiple of 16) is its N.  Both operands are K-major bf16
+// tiles loaded by TMA tensor copies with 128-byte swizzle into a
+// shared-memory ring of ST stages (mbarrier completion; ST sized for two CTAs
+// per SM, or for one in the deep variant).  One thread issues the
 // copies, one thread issues tcgen05.mma.cta_group::1.kind::f16 (fp32
 // accumulation in TMEM), and four warps read the accumulator back with
 // tcgen05.ld for the epilogue.  A CTA owns one (128-row tile, K split).  When
@@ -17,7 +18,8 @@
 //
 // The activations enter as two bf16 parts, x = hi + lo with hi = bf16(x) and
 // lo = bf16(x - hi) (prep_bf16_kernel, after the RMSNorm / gather of the GEMV
-// input segments in fp32).  Both parts are B columns of the MMA (N = 2 * BH),
+// input segments in fp32; or, in gemm_tcf_kernel below, converter warps inside
+// the GEMM).  Both parts are B columns of the MMA (N = 2 * BH),
 // so the bf16 weights meet an activation accurate to about 2^-17 relative:
 // the weight stream is unchanged, only the (idle) tensor-core work doubles.
 // The epilogue adds the two accumulator halves.  Every wait is bounded

@@ -98,6 +98,34 @@ __device__ __forceinline__ void rope8(float (&x)[8], int li, const float4 (&cs)[
     }
 }
 
+// Cluster merge of one output element from the CS (<= 16) partial softmax
+// states (m, l, o) of cluster ranks 0..CS-1: every distributed-shared-memory
+// load is issued before any is used, then the ranks are combined in order.
+__device__ __forceinline__ float cluster_merge_elem(cg::cluster_group& cluster, const float* m_loc,
+                                                    const float* l_loc, const float* o_loc, int CS) {
+    float mr[16], lr[16], orr[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r)
+        if (r < CS) {
+            mr[r] = *cluster.map_shared_rank(m_loc, r);
+            lr[r] = *cluster.map_shared_rank(l_loc, r);
+            orr[r] = *cluster.map_shared_rank(o_loc, r);
+        }
+    float M = -INFINITY;
+#pragma unroll
+    for (int r = 0; r < 16; ++r)
+        if (r < CS) M = fmaxf(M, mr[r]);
+    float L = 0.f, Ov = 0.f;
+#pragma unroll
+    for (int r = 0; r < 16; ++r)
+        if (r < CS) {
+            const float f = (mr[r] == -INFINITY) ? 0.f : expf(mr[r] - M);
+            L += lr[r] * f;
+            Ov += orr[r] * f;
+        }
+    return Ov / L;
+}
+
 constexpr int kAttnWarps = 8;
 constexpr int kAttnThreads = kAttnWarps * 32;
 
@@ -317,16 +345,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     const int PER = (G * DH + CS - 1) / CS;
     for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
         const int hh = i / DH, t = i % DH;
-        float M = -INFINITY;
-        for (int r = 0; r < CS; ++r) M = fmaxf(M, *cluster.map_shared_rank(&sm_m[hh], r));
-        float L = 0.f, Ov = 0.f;
-        for (int r = 0; r < CS; ++r) {
-            const float mr = *cluster.map_shared_rank(&sm_m[hh], r);
-            const float f = (mr == -INFINITY) ? 0.f : expf(mr - M);
-            L += *cluster.map_shared_rank(&sm_l[hh], r) * f;
-            Ov += *cluster.map_shared_rank(&sm_o[hh][t], r) * f;
-        }
-        p.out[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + t] = Ov / L;
+        p.out[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + t] =
+            cluster_merge_elem(cluster, &sm_m[hh], &sm_l[hh], &sm_o[hh][t], CS);
     }
     cluster.sync();  // keep every CTA's shared memory alive until all merges read it
 }

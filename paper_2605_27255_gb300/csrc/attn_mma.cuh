@@ -115,6 +115,8 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     const bool owns_new = n >= j0 && n < j1;
 
     if (threadIdx.x == 0) {
+        prefetch_tmap(&tmK);
+        prefetch_tmap(&tmV);
         for (int i = 0; i < kMmaStages; ++i) {
             mbar_init(full + i, 1);
             mbar_init(empty + i, 1);
@@ -339,16 +341,8 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     const int PER = (G * DH + CS - 1) / CS;
     for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
         const int hh = i / DH, t = i % DH;
-        float M = -INFINITY;
-        for (int rr = 0; rr < CS; ++rr) M = fmaxf(M, *cluster.map_shared_rank(&sm_m[hh], rr));
-        float L = 0.f, Ov = 0.f;
-        for (int rr = 0; rr < CS; ++rr) {
-            const float mr = *cluster.map_shared_rank(&sm_m[hh], rr);
-            const float f = (mr == -INFINITY) ? 0.f : expf(mr - M);
-            L += *cluster.map_shared_rank(&sm_l[hh], rr) * f;
-            Ov += *cluster.map_shared_rank(&sm_o[hh][t], rr) * f;
-        }
-        p.out[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + t] = Ov / L;
+        p.out[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + t] =
+            cluster_merge_elem(cluster, &sm_m[hh], &sm_l[hh], &sm_o[hh][t], CS);
     }
     cluster.sync();  // keep every CTA's shared memory alive until all merges read it
 }

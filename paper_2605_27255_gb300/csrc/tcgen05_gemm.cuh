@@ -256,6 +256,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
     const int kb0 = (int)((long long)split * nkb / p.splits), kb1 = (int)((long long)(split + 1) * nkb / p.splits);
     const int nk = kb1 - kb0;  // >= 1 (splits <= nkb)
 
+    if (threadIdx.x == 64) {
+        prefetch_tmap(&tmW);
+        prefetch_tmap(&tmX);
+    }
     if (warp == 0) tmem_alloc(&tmem_base, kCols);
     if (threadIdx.x == 32) {
         for (int s = 0; s < ST; ++s) {
@@ -447,6 +451,11 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
     const int nk = kb1 - kb0;  // >= 1 (splits <= nkb)
     const uint32_t raw_bytes = (uint32_t)(BH * kTcBK * 4) + (in.norm ? 128u : 0u);
 
+    if (threadIdx.x == 64) {
+        prefetch_tmap(&tmW);
+        prefetch_tmap(&tmX0);
+        if (in.nseg == 2) prefetch_tmap(&tmX1);
+    }
     if (warp == 0) tmem_alloc(&tmem_base, kCols);
     if (threadIdx.x == 32) {
         for (int s = 0; s < ST; ++s) {

@@ -59,6 +59,11 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
         : "memory");
 }
 
+// start fetching a tensor map (kernel parameter) into the TMA descriptor cache
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* tm) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(tm) : "memory");
+}
+
 // 2-D tiled tensor copy (TMA) of the box at element coordinates (x, y) of the
 // tensor map into shared memory, completing on `bar`
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, int x, int y, uint64_t* bar) {

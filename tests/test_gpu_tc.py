@@ -79,8 +79,11 @@ MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003
                        compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1.0e4, tau=0.5)
 
 
-@pytest.mark.parametrize("B", [16, 37])
+@pytest.mark.parametrize("B", [16, 37, 64])
 def test_mid_bf16_tensor_core_batches(B):
+    """B = 16 takes the fused projections (batch width 16), B = 37 and 64 the
+    split-kernel form (width 64); tensor-core attention; forced replay
+    against the oracle."""
     w = synth.gen_weights(MID, seed=21)
     prompts = synth.gen_prompts(B, 24, MID.V, seed=B).numpy()
     st = run_forced_replay(MID, w, prompts, 4, force=0, page_shuffle_seed=5)

@@ -41,6 +41,7 @@ WORKLOADS = {
     "9b-b8": dict(shape="9b", batch=8, prompt=4096, steps=1024),
 }
 METRIC = "accepted tokens/s/GPU (PIPO pair-decode step)"
+NOMINAL_HBM_GBS = 8000.0  # GB300 HBM3e nominal (~8 TB/s), context beside the measured peak
 
 
 def parse():
@@ -341,7 +342,8 @@ def run_pipo(args):
                      "launches_per_step": gn // prof_steps, "share_of_step_time": gms / tot_ms if tot_ms else None,
                      "timing": f"CUDA events around each launch, {prof_steps} eagerly run steps after the timed region",
                      "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)",
-                     "step": {"algorithmic_bytes": bytes_step, "achieved": step_gbs, "frac": step_gbs / hbm},
+                     "step": {"algorithmic_bytes": bytes_step, "achieved": step_gbs, "frac": step_gbs / hbm,
+                              "frac_of_nominal": step_gbs / NOMINAL_HBM_GBS},
                      "attention": {"achieved": (kb[1][0] / (kb[1][1] / 1e3) / 1e9) if kb[1][1] else None,
                                    "share_of_step_time": kb[1][1] / tot_ms if tot_ms else None}},
         "cpu_baseline": cpu,

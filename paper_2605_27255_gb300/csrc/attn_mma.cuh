@@ -192,8 +192,10 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         if (warp < G) {
             const int h = warp;
             float dsum = 0.f;
-            for (int d = lane; d < DH; d += 32) dsum += qs[h][d] * kn_s[d];
-            dsum = warp_sum(dsum);
+            if (owns_new) {  // uniform over the CTA: the shuffles below see whole warps
+                for (int d = lane; d < DH; d += 32) dsum += qs[h][d] * kn_s[d];
+                dsum = warp_sum(dsum);
+            }
             for (int d = lane; d < DH; d += 32) wo[NW][h][d] = owns_new ? vn_s[d] : 0.f;
             if (lane == 0) {
                 wm[NW][h] = owns_new ? dsum : -INFINITY;

@@ -65,3 +65,20 @@ def test_init_error_without_gpu_is_a_status(lib):
     rc = capi.load().pipo_init(C.byref(cfg), C.byref(w), C.byref(ctx))
     assert rc == capi.PIPO_EINVAL and not ctx.value
     assert "invalid config" in capi.pipo_last_error(None)
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """No fallback: without the CUDA library the binding raises."""
+    monkeypatch.setattr(capi, "_lib", None)
+    with pytest.raises(RuntimeError, match="not built"):
+        capi.load(str(tmp_path / "libpipo.so"))
+
+
+def test_failed_call_raises_status_error(lib):
+    """A non-OK status becomes a PipoError carrying the status and message."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    with pytest.raises(capi.PipoError) as e:
+        capi.pipo_op_gemv(1, 0, 16, 10, 12, 16, 1, 16, 0)  # K not a multiple of 8
+    assert e.value.status == capi.PIPO_EINVAL

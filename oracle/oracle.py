@@ -78,6 +78,8 @@ def lib():
             L.orc_free.argtypes = [C.c_void_p]
             L.orc_step.argtypes = [C.c_void_p, C.c_double, C.c_int, C.POINTER(OrcOut)]
             L.orc_prefill.argtypes = [C.c_void_p, _I, _I, C.c_int, C.c_double, C.c_int, C.POINTER(OrcOut)]
+            L.orc_regular_step.argtypes = [C.c_void_p, C.POINTER(OrcOut)]
+            L.orc_regular_prefill.argtypes = [C.c_void_p, _I, _I, C.c_int, C.POINTER(OrcOut)]
             L.orc_set_pending.argtypes = [C.c_void_p, _I]
             L.orc_rollback.argtypes = [C.c_void_p, _I]
             L.orc_get_seq.argtypes = [C.c_void_p, C.c_int, _I, _I, _I, C.POINTER(C.c_int64)]
@@ -186,6 +188,28 @@ class State:
         rc = lib().orc_step(self.ptr, tau, force, C.byref(s))
         if rc != OK:
             raise ValueError(f"oracle step failed: {rc}")
+        return o
+
+    def regular_prefill(self, ids, lens=None, logits=True):
+        """Regular decoding (one token per backbone pass, the paper's baseline):
+        run the prompt, return the first output token (tokens[:, 0])."""
+        ids = np.ascontiguousarray(np.asarray(ids, dtype=np.int32))
+        if lens is None:
+            lens = np.full(self.B, ids.shape[1], np.int32)
+        lens = np.ascontiguousarray(np.asarray(lens, dtype=np.int32))
+        o, s = _out(self.B, self.m.shape.V, self.m.shape.H, logits)
+        rc = lib().orc_regular_prefill(self.ptr, _ip(ids), _ip(lens), ids.shape[1], C.byref(s))
+        if rc != OK:
+            raise ValueError(f"oracle regular prefill failed: {rc}")
+        return o
+
+    def regular_step(self, logits=True):
+        """One regular decode step: the pending token through the backbone and
+        the LM head; the argmax becomes the next pending token."""
+        o, s = _out(self.B, self.m.shape.V, self.m.shape.H, logits)
+        rc = lib().orc_regular_step(self.ptr, C.byref(s))
+        if rc != OK:
+            raise ValueError(f"oracle regular step failed: {rc}")
         return o
 
     def set_pending(self, pairs):

@@ -32,6 +32,10 @@
  * (fp32 or bf16) and widened exactly.  With kv_bf16 set, keys (after RoPE)
  * and values are rounded to bf16 when stored, as a bf16 cache stores them.
  *
+ * Also: regular decoding of the same backbone (one token per pass, no
+ * compressor or heads beyond the LM head), the baseline the paper compares
+ * PIPO with (orc_regular_prefill / orc_regular_step).
+ *
  * Parity of every function here is pinned by the not-gpu tests (closed forms,
  * special cases, brute-force recompute, invariants).
  */
@@ -464,6 +468,84 @@ int orc_prefill(orc_state *st, const int32_t *ids, const int32_t *lens, int stri
         }
     }
     free(x); free(hd);
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------ */
+/* regular decoding: the same backbone without pairs                  */
+/*
+ * The baseline the paper measures PIPO against (Sec. 4, "Regular"): one
+ * token per backbone pass, the input is the token's embedding E[t] (no
+ * compressor), the position is the token index and the cache holds one entry
+ * per token; the final-norm tied LM head and greedy argmax give the next
+ * token.  No MTP head, no confidence head.  Uses the backbone caches of the
+ * state; the pending token is p0 (p1 unused), n counts the tokens consumed.
+ */
+static void regular_head(orc_state *st, int b, double *h, orc_out *o) {
+    const orc_config *c = &st->c;
+    orc_seq *s = &st->s[b];
+    int H = c->H, V = c->V;
+    double *lg = (double *)malloc(sizeof(double) * V);
+    double m;
+    lm_head(c, &st->w, h, st->w.final_norm, lg);
+    int x = orc_argmax(lg, V, &m);
+    s->p0 = x;
+    s->p1 = ORC_PAD;
+    s->n += 1;
+    s->emitted += 1;
+    if (o) {
+        if (o->tokens) { o->tokens[2 * b] = x; o->tokens[2 * b + 1] = -1; }
+        if (o->n_acc) o->n_acc[b] = 0;
+        if (o->logits_b) memcpy(o->logits_b + (size_t)b * V, lg, sizeof(double) * V);
+        if (o->h_b) memcpy(o->h_b + (size_t)b * H, h, sizeof(double) * H);
+        if (o->margin_b) o->margin_b[b] = m;
+        if (o->x_b) o->x_b[b] = x;
+    }
+    free(lg);
+}
+
+/* Prefill of regular decoding: every prompt token runs the backbone at its
+ * own position; the last one also runs the LM head, whose argmax becomes the
+ * pending token. */
+int orc_regular_prefill(orc_state *st, const int32_t *ids, const int32_t *lens, int stride, orc_out *o) {
+    const orc_config *c = &st->c;
+    for (int b = 0; b < st->B; b++) {
+        int len = lens[b];
+        if (len < 1 || len > stride) return ORC_EINVAL;
+        if (len > c->max_ctx) return ORC_ECAPACITY;
+        for (int t = 0; t < len; t++) if (ids[(size_t)b * stride + t] < 0 || ids[(size_t)b * stride + t] >= c->V) return ORC_EINVAL;
+    }
+    double *x = (double *)malloc(sizeof(double) * c->H);
+    for (int b = 0; b < st->B; b++) {
+        orc_seq *s = &st->s[b];
+        const int32_t *t = ids + (size_t)b * stride;
+        s->n = 0;
+        s->emitted = 0;
+        for (int j = 0; j < lens[b]; j++) {
+            embed(c, &st->w, t[j], x);
+            backbone_at(st, s, x);
+            if (j < lens[b] - 1) s->n += 1;
+            else regular_head(st, b, x, o);
+        }
+        s->emitted = 0;  /* the prefill's token is the first output, not a decode step's */
+    }
+    free(x);
+    return ORC_OK;
+}
+
+/* One regular decode step for every sequence: embed the pending token, one
+ * backbone pass at position n, LM head, argmax. */
+int orc_regular_step(orc_state *st, orc_out *o) {
+    const orc_config *c = &st->c;
+    for (int b = 0; b < st->B; b++) if (st->s[b].n >= c->max_ctx) return ORC_ECAPACITY;
+    double *x = (double *)malloc(sizeof(double) * c->H);
+    for (int b = 0; b < st->B; b++) {
+        orc_seq *s = &st->s[b];
+        embed(c, &st->w, s->p0, x);
+        backbone_at(st, s, x);
+        regular_head(st, b, x, o);
+    }
+    free(x);
     return ORC_OK;
 }
 

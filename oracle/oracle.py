@@ -91,6 +91,9 @@ def lib():
             L.orc_matvec.argtypes = [C.c_void_p, C.c_size_t, C.c_int, C.c_int, C.c_int, _D, _D]
             L.orc_rope.argtypes = [_D, C.c_int, C.c_int, C.c_int, C.c_double]
             L.orc_attend.argtypes = [_D, _D, _D, C.c_int, C.c_int, C.c_int, C.c_int, _D]
+            L.orc_sample.argtypes = [_D, C.c_int, _I, C.c_int, C.c_double, C.c_int, C.c_double, C.c_double,
+                                     C.c_double]
+            L.orc_sample.restype = C.c_int
             L.orc_argmax.argtypes = [_D, C.c_int, _D]
             L.orc_argmax.restype = C.c_int
             for f in ("orc_silu", "orc_sigmoid", "orc_round_bf16"):
@@ -294,6 +297,19 @@ def argmax(x):
     m = C.c_double()
     i = lib().orc_argmax(_dp(x), x.size, C.byref(m))
     return i, m.value
+
+
+def sample(logits, u, hist=(), temperature=1.0, top_k=20, top_p=0.95, rep_penalty=1.5):
+    """The evaluation sampler (see orc_sample); u in [0, 1) is the draw."""
+    x = np.ascontiguousarray(logits, dtype=np.float64)
+    h = np.ascontiguousarray(np.asarray(hist, dtype=np.int32).reshape(-1))
+    if h.size == 0:
+        h = np.zeros(1, np.int32)
+        nh = 0
+    else:
+        nh = h.size
+    return lib().orc_sample(_dp(x), x.size, _ip(h), nh, float(temperature), int(top_k), float(top_p),
+                            float(rep_penalty), float(u))
 
 
 def silu(x):

@@ -173,6 +173,65 @@ int orc_argmax(const double *x, int n, double *margin) {
     return best;
 }
 
+/* The paper's evaluation sampler as a primitive (temperature, top-k, top-p,
+ * repetition penalty; its settings: T = 1, k = 20, p = 0.95, penalty 1.5).
+ * The random draw u in [0, 1) is an input.  Steps, in this order:
+ *   1. repetition penalty r over the distinct ids of hist[0, n_hist): a logit
+ *      l becomes l / r if l > 0, else l * r;
+ *   2. temperature T: l / T;
+ *   3. top-k: the k largest (k <= 0 or k >= V keeps all), in descending logit
+ *      order with ties to the lower id;
+ *   4. top-p: the shortest prefix of that order whose softmax mass reaches p;
+ *   5. the first id of that prefix whose cumulative renormalised mass exceeds u.
+ * k == 1 is greedy (the argmax with ties to the lower id). */
+typedef struct {
+    double v;
+    int id;
+} orc_scored;
+
+static int scored_desc(const void *a, const void *b) {
+    const orc_scored *x = (const orc_scored *)a, *y = (const orc_scored *)b;
+    if (x->v > y->v) return -1;
+    if (x->v < y->v) return 1;
+    return (x->id > y->id) - (x->id < y->id);
+}
+
+int orc_sample(const double *logits, int V, const int32_t *hist, int n_hist, double temperature, int top_k,
+               double top_p, double rep_penalty, double u) {
+    orc_scored *sc = (orc_scored *)malloc(sizeof(orc_scored) * V);
+    unsigned char *seen = (unsigned char *)calloc(V, 1);
+    for (int i = 0; i < n_hist; i++)
+        if (hist[i] >= 0 && hist[i] < V) seen[hist[i]] = 1;
+    for (int i = 0; i < V; i++) {
+        double l = logits[i];
+        if (seen[i]) l = (l > 0.0) ? l / rep_penalty : l * rep_penalty;
+        sc[i].v = l / temperature;
+        sc[i].id = i;
+    }
+    qsort(sc, V, sizeof(orc_scored), scored_desc);
+    int keep = (top_k <= 0 || top_k > V) ? V : top_k;
+    double *e = (double *)malloc(sizeof(double) * keep);
+    double Z = 0.0;
+    for (int i = 0; i < keep; i++) { e[i] = exp(sc[i].v - sc[0].v); Z += e[i]; }
+    int np = keep;
+    double cum = 0.0;
+    for (int i = 0; i < keep; i++) {
+        cum += e[i];
+        if (cum / Z >= top_p) { np = i + 1; break; }
+    }
+    double Zp = 0.0;
+    for (int i = 0; i < np; i++) Zp += e[i];
+    const double target = u * Zp;
+    int pick = sc[np - 1].id;
+    cum = 0.0;
+    for (int i = 0; i < np; i++) {
+        cum += e[i];
+        if (cum > target) { pick = sc[i].id; break; }
+    }
+    free(sc); free(seen); free(e);
+    return pick;
+}
+
 /* ------------------------------------------------------------------ */
 /* model pieces                                                        */
 

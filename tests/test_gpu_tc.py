@@ -38,7 +38,7 @@ def _run_tc(mode, N, K, B, splits, seed=0):
 
 @pytest.mark.parametrize("mode", [0, 1])
 @pytest.mark.parametrize("N,K", [(2560, 2560), (333, 4096), (1000, 1408), (4096, 256), (128, 64)])
-@pytest.mark.parametrize("B", [1, 16, 37, 64, 128])
+@pytest.mark.parametrize("B", [1, 16, 24, 37, 64, 128])
 @pytest.mark.parametrize("splits", [0, 1, 3])
 def test_gemm_tc_matches_float64(mode, N, K, B, splits):
     y, ref = _run_tc(mode, N, K, B, splits)
@@ -79,11 +79,11 @@ MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003
                        compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1.0e4, tau=0.5)
 
 
-@pytest.mark.parametrize("B", [16, 37, 64])
+@pytest.mark.parametrize("B", [16, 24, 37, 64])
 def test_mid_bf16_tensor_core_batches(B):
-    """B = 16 takes the fused projections (batch width 16), B = 37 and 64 the
-    split-kernel form (width 64); tensor-core attention; forced replay
-    against the oracle."""
+    """B = 16 and 24 take the fused projections (batch widths 16 and 32),
+    B = 37 and 64 the split-kernel form (width 64); tensor-core attention;
+    forced replay against the oracle."""
     w = synth.gen_weights(MID, seed=21)
     prompts = synth.gen_prompts(B, 24, MID.V, seed=B).numpy()
     st = run_forced_replay(MID, w, prompts, 4, force=0, page_shuffle_seed=5)

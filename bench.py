@@ -56,6 +56,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--profile-steps", type=int, default=8, help="eager steps timed per launch for the roofline")
+    ap.add_argument("--regular", action="store_true",
+                    help="also time regular decoding (one token per backbone pass, Sec. 4) on the same prompts "
+                         "and report its time per output token beside the pair step's")
     return ap.parse_args()
 
 
@@ -214,6 +217,44 @@ def run_reference(args):
 
 # ---------------------------------------------------------------- GPU arm
 
+def run_regular(g, shape, wl, B, T, W, K, stream, seed):
+    """Regular decoding on the same context and prompts: T prompt tokens take
+    T cache entries, then W untimed and K timed steps of one token per
+    sequence (CUDA events on the context stream)."""
+    import torch
+
+    from paper_2605_27255_gb300 import roofline, synth
+
+    prompts = synth.gen_prompts(B, T if not wl.get("kv_fill") else 2, shape.V, seed=seed).numpy()
+    g.regular_prefill(prompts)
+    if wl.get("kv_fill"):
+        Kf, Vf = synth.gen_kv_fill(shape, T, seed=7, device="cuda")
+        Kf, Vf = Kf.cpu().numpy(), Vf.cpu().numpy()
+        for b in range(B):
+            g.load_cache(b, Kf, Vf)
+        del Kf, Vf
+    for _ in range(W):
+        g.regular_step_async()
+    torch.cuda.synchronize()
+    n0, e0 = g.counters()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(K):
+        g.regular_step_async()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    n1, e1 = g.counters()
+    tokens = int((e1 - e0).sum())
+    ctx_avg = float(n0.mean()) + (K - 1) / 2.0
+    step_bytes = roofline.regular_step_bytes(shape, B, ctx_avg)
+    return {"ms_per_step": ms / K, "ms_per_token": ms / K, "tokens_per_s": tokens / (ms / 1e3),
+            "context_entries_avg": ctx_avg, "steps": K, "gpu_launches": g.launches() * K,
+            "step_bytes": step_bytes, "achieved_gbs": step_bytes / (ms / K / 1e3) / 1e9,
+            "note": "one token per backbone pass from the token embedding, final-norm tied LM head; tpot_ratio = "
+                    "regular time per output token / pair-step time per output token (1 + acceptance tokens)"}
+
+
 def run_pipo(args):
     import numpy as np
     import torch
@@ -233,6 +274,8 @@ def run_pipo(args):
     W = max(3, args.warmup)
     n_pairs = (T + 1) // 2
     max_ctx = n_pairs + W + 2 * K + args.profile_steps + 8
+    if args.regular:
+        max_ctx = max(max_ctx, T + W + K + 8)  # regular decoding: one cache entry per token
 
     w = build_weights(shape, "cuda")
     g = capi.Pipo(shape, w, max_batch=B, max_ctx=max_ctx, tau=tau, force_mode=args.force)
@@ -304,6 +347,7 @@ def run_pipo(args):
             kb[int(kk)][1] += float(mm)
             kb[int(kk)][2] += 1
     tot_ms = sum(v[1] for v in kb.values())
+    regular = run_regular(g, shape, wl, B, T, W, K, stream, 1 + rank * 1000) if args.regular else None
 
     ms_all, tokens_all, e2e_all, e2e_tok_all = aggregate_ranks(ms, tokens, e2e_s, e2e_tokens, "cuda")
     value = tokens_all / (ms_all / 1e3)
@@ -352,6 +396,11 @@ def run_pipo(args):
         "gpu_launches": launches * K,
         "clocks": clk.summary(),
     }
+    if regular is not None:
+        pipo_tpot = (ms / K) / (1.0 + line["config"]["acceptance"])
+        regular["tpot_ratio"] = regular["ms_per_token"] / pipo_tpot
+        regular["frac"] = regular["achieved_gbs"] / hbm
+        line["regular"] = regular
     print(json.dumps(line), flush=True)
     g.close()
     if ws > 1:

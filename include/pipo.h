@@ -148,6 +148,34 @@ PIPO_API pipo_status pipo_decode_step(pipo_ctx *ctx, int32_t *h_tokens, int32_t 
  * step is a captured CUDA graph replayed per call. */
 PIPO_API pipo_status pipo_decode_step_async(pipo_ctx *ctx, int32_t *d_tokens, int32_t *d_n_accepted);
 
+/* Regular decoding, the baseline the paper measures PIPO against (Sec. 4,
+ * "Regular"; its TPOT comparison): the same backbone, one token per pass.
+ * The input of a pass is the token's embedding E[t] (no compressor), its
+ * position is the token index, the cache holds one entry per token (backbone
+ * caches only), and the final-norm tied LM head's argmax (Eq. 3) is the next
+ * token; the MTP and confidence heads do not run.
+ *
+ * pipo_regular_prefill: arguments as pipo_prefill, but every sequence must
+ * have the same length N (EINVAL otherwise) and the prompt takes N cache
+ * entries (ECAPACITY when N > max_ctx).  Each prompt token runs the backbone
+ * at its own position; the last one also runs the LM head.  Outputs (may be
+ * NULL): h_tokens[B,2] = (first generated token, -1), h_n_accepted[B] = 0.
+ * Resets the emitted counters to 0.  Puts the context in regular mode until
+ * the next pipo_prefill.
+ *
+ * pipo_regular_step: one pass for every sequence, from the pending token
+ * (slot 0 of the pending pair; pipo_set_pending overwrites it).  h_tokens
+ * [B,2] = (token, -1) (may be NULL).  Synchronous; ESTATE before a regular
+ * prefill or after a pair prefill, ECAPACITY when a cache is full.
+ * pipo_decode_step returns ESTATE in regular mode.
+ *
+ * pipo_regular_step_async: the same step enqueued on the context stream (a
+ * captured CUDA graph); d_tokens[B,2] is a device buffer (may be NULL). */
+PIPO_API pipo_status pipo_regular_prefill(pipo_ctx *ctx, int32_t batch, const int32_t *h_ids, int32_t stride,
+                                          const int32_t *h_lens, int32_t *h_tokens, int32_t *h_n_accepted);
+PIPO_API pipo_status pipo_regular_step(pipo_ctx *ctx, int32_t *h_tokens);
+PIPO_API pipo_status pipo_regular_step_async(pipo_ctx *ctx, int32_t *d_tokens);
+
 /* Truncate both KV caches of sequence b to h_n_pairs[b] entries (host,
  * [B], each <= the current length).  Test and bookkeeping primitive: PIPO
  * itself never caches a rejected draft (Sec. 3.1), so decoding never calls it.

@@ -73,6 +73,9 @@ SIGNATURES = {
     "pipo_prefill": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.c_int32, _IP, _IP, _IP]),
     "pipo_decode_step": (C.c_int, [C.c_void_p, _IP, _IP]),
     "pipo_decode_step_async": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "pipo_regular_prefill": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.c_int32, _IP, _IP, _IP]),
+    "pipo_regular_step": (C.c_int, [C.c_void_p, _IP]),
+    "pipo_regular_step_async": (C.c_int, [C.c_void_p, C.c_void_p]),
     "pipo_rollback": (C.c_int, [C.c_void_p, _IP]),
     "pipo_set_threshold": (C.c_int, [C.c_void_p, C.c_float, C.c_int32]),
     "pipo_set_pending": (C.c_int, [C.c_void_p, _IP]),
@@ -164,6 +167,26 @@ def pipo_decode_step(ctx, B: int):
 
 def pipo_decode_step_async(ctx, d_tokens: int = 0, d_nacc: int = 0):
     _check(load().pipo_decode_step_async(ctx, C.c_void_p(d_tokens or None), C.c_void_p(d_nacc or None)), ctx)
+
+
+def pipo_regular_prefill(ctx, ids: np.ndarray, lens: Optional[np.ndarray] = None):
+    ids = _i32(ids)
+    B, stride = ids.shape
+    lens = _i32(np.full(B, stride) if lens is None else lens)
+    tok = np.zeros((B, 2), np.int32)
+    nacc = np.zeros(B, np.int32)
+    _check(load().pipo_regular_prefill(ctx, B, _ip(ids), stride, _ip(lens), _ip(tok), _ip(nacc)), ctx)
+    return tok, nacc
+
+
+def pipo_regular_step(ctx, B: int):
+    tok = np.zeros((B, 2), np.int32)
+    _check(load().pipo_regular_step(ctx, _ip(tok)), ctx)
+    return tok
+
+
+def pipo_regular_step_async(ctx, d_tokens: int = 0):
+    _check(load().pipo_regular_step_async(ctx, C.c_void_p(d_tokens or None)), ctx)
 
 
 def pipo_rollback(ctx, n_pairs) -> None:
@@ -335,6 +358,19 @@ class Pipo:
 
     def step_async(self, d_tokens: int = 0, d_nacc: int = 0):
         pipo_decode_step_async(self.ctx, d_tokens, d_nacc)
+
+    def regular_prefill(self, ids, lens=None):
+        """Regular decoding (one token per backbone pass): run the prompt,
+        return (tokens [B,2] = (first token, -1), n_accepted = 0)."""
+        ids = _i32(ids)
+        self.B = ids.shape[0]
+        return pipo_regular_prefill(self.ctx, ids, lens)
+
+    def regular_step(self):
+        return pipo_regular_step(self.ctx, self.B)
+
+    def regular_step_async(self, d_tokens: int = 0):
+        pipo_regular_step_async(self.ctx, d_tokens)
 
     def set_threshold(self, tau, force_mode=0):
         pipo_set_threshold(self.ctx, tau, force_mode)

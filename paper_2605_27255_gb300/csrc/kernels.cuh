@@ -555,4 +555,44 @@ __global__ void advance_kernel(int32_t* n_pos, int B) {
     if (b < B) n_pos[b] += 1;
 }
 
+// Regular decoding (the paper's baseline, Sec. 4): the backbone input is the
+// token's own embedding, x[b] = E[tok[b * ld]], with no compressor.  Also
+// zeroes the argmax keys of the step.  An id outside [0, V) (never produced:
+// the host validates ids) gives a zero row instead of an out-of-range read.
+// grid B, any block size.
+template <typename T>
+__global__ void embed_kernel(const void* E, const int32_t* tok, int ld, int V, int H, float* x,
+                             unsigned long long* zero, int zero_n) {
+    pdl_launch();
+    pdl_wait();
+    const int b = blockIdx.x;
+    if (b == 0)
+        for (int i = threadIdx.x; i < zero_n; i += blockDim.x) zero[i] = 0ull;
+    const int t = tok[(size_t)b * ld];
+    const bool ok = t >= 0 && t < V;
+    for (int k = threadIdx.x; k < H; k += blockDim.x)
+        x[(size_t)b * H + k] = ok ? ldw<T>(E, (size_t)t * H + k) : 0.f;
+}
+
+// Regular decoding, end of a step: the LM-head argmax is the output token and
+// the next input (slot 1 stays PAD, nothing is drafted), one more cache entry,
+// one more emitted token.  grid B, any block size.
+__global__ void regular_accept_kernel(StepState st, int H, const float* h) {
+    pdl_launch();
+    pdl_wait();
+    const int b = blockIdx.x;
+    if (st.dbg_hb)
+        for (int k = threadIdx.x; k < H; k += blockDim.x) st.dbg_hb[(size_t)b * H + k] = h[(size_t)b * H + k];
+    if (threadIdx.x != 0) return;
+    const int xb = argmax_row(st.am_b[b]);
+    st.out_tokens[2 * b] = xb;
+    st.out_tokens[2 * b + 1] = -1;
+    st.out_nacc[b] = 0;
+    st.pending[2 * b] = xb;
+    st.pending[2 * b + 1] = -1;
+    st.n_pos[b] += 1;
+    st.emitted[b] += 1;
+    if (st.dbg_xb) st.dbg_xb[b] = xb;
+}
+
 }  // namespace pipo

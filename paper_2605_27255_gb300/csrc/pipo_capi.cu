@@ -118,9 +118,11 @@ struct pipo_ctx {
 
     int B = 0;
     bool prefilled = false;
+    bool regular = false;             // the prefill was regular decoding (one token per backbone pass)
     std::vector<int32_t> h_len;
     cudaGraphExec_t graph = nullptr;
     int graph_B = -1;
+    bool graph_regular = false;       // the captured step is a regular-decoding step
     int launches = 0;
     std::map<long long, int> occ;
     std::string err = "no error";
@@ -1140,6 +1142,51 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
     }
 }
 
+// One position of regular decoding (the baseline of Sec. 4) for every
+// sequence: DECODE embeds the pending token (slot 0), PREFILL_* prompt token
+// j; the backbone blocks run at position n on the backbone caches; the
+// positions before the last of a prefill stop there, the others run the
+// final-norm tied LM head and take its argmax as the next token.  Same
+// kernels as the pair step, without the compressor and the two extra heads.
+pipo_status enqueue_regular(pipo_ctx* ctx, Mode mode, int j) {
+    const pipo_config& c = ctx->cfg;
+    ctx->tc_shallow = attn_is_long(ctx);
+    const int H = c.hidden, B = ctx->B;
+    const bool bf = c.dtype == 1;
+    {
+        const void* E = ctx->E;
+        const int32_t* tok = (mode == DECODE) ? ctx->pending : ctx->pf_pairs + (size_t)j * B;
+        int ld = (mode == DECODE) ? 2 : 1, V = c.vocab, Hv = H, zn = 2 * c.max_batch;
+        float* x = ctx->x;
+        unsigned long long* am = ctx->am;
+        void* args[] = {(void*)&E, (void*)&tok, &ld, &V, &Hv, &x, &am, &zn};
+        TRY(launch_ex(ctx, bf ? (const void*)&embed_kernel<bf16> : (const void*)&embed_kernel<float>, dim3(B),
+                      dim3(256), 0, args));
+    }
+    for (int l = 0; l < c.n_layers; ++l) TRY(enqueue_block(ctx, ctx->blocks[l], l, ctx->x));
+    if (mode == PREFILL_MID) {
+        int32_t* np = ctx->n_pos;
+        int Bv = B;
+        void* args[] = {&np, &Bv};
+        return launch_ex(ctx, (const void*)&advance_kernel, dim3((B + 127) / 128), dim3(128), 0, args);
+    }
+    TRY(enqueue_lm_head(ctx, ctx->x, ctx->final_norm, ctx->am, c.debug ? ctx->dbg_lb : nullptr));
+    StepState st{};
+    st.pending = ctx->pending; st.n_pos = ctx->n_pos; st.emitted = ctx->emitted;
+    st.out_tokens = ctx->out_tokens; st.out_nacc = ctx->out_nacc;
+    st.am_b = ctx->am; st.am_d = ctx->am;
+    if (c.debug) { st.dbg_hb = ctx->dbg_hb; st.dbg_xb = ctx->dbg_xb; }
+    int Hv = H;
+    const float* h = ctx->x;
+    void* args[] = {&st, &Hv, (void*)&h};
+    return launch_ex(ctx, (const void*)&regular_accept_kernel, dim3(B), dim3(256), 0, args);
+}
+
+// The decode step of the context's current mode.
+pipo_status enqueue_step(pipo_ctx* ctx) {
+    return ctx->regular ? enqueue_regular(ctx, DECODE, 0) : enqueue_position(ctx, DECODE, 0);
+}
+
 void drop_graph(pipo_ctx* ctx) {
     if (ctx->graph) cudaGraphExecDestroy(ctx->graph);
     ctx->graph = nullptr;
@@ -1232,20 +1279,24 @@ pipo_status try_step_kernel(pipo_ctx* ctx, bool& used) {
 }
 
 pipo_status ensure_graph(pipo_ctx* ctx) {
-    if (ctx->graph && ctx->graph_B == ctx->B) return PIPO_OK;
+    if (ctx->graph && ctx->graph_B == ctx->B && ctx->graph_regular == ctx->regular) return PIPO_OK;
     drop_graph(ctx);
     ctx->mk_active = false;
     bool used = false;
-    TRY(try_step_kernel(ctx, used));
+    // the persistent step kernel records the pair step only
+    if (!ctx->regular) TRY(try_step_kernel(ctx, used));
     if (getenv("PIPO_VERBOSE"))
         fprintf(stderr, "pipo: decode step = %s %s\n", used ? "persistent step kernel" : "kernel graph",
                 ctx->mk_note.c_str());
-    if (used) return PIPO_OK;
+    if (used) {
+        ctx->graph_regular = false;
+        return PIPO_OK;
+    }
     cudaGraph_t g = nullptr;
     CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
     ctx->launches = 0;
     ctx->pdl = true;
-    pipo_status s = enqueue_position(ctx, DECODE, 0);
+    pipo_status s = enqueue_step(ctx);
     ctx->pdl = false;
     cudaError_t e = cudaStreamEndCapture(ctx->stream, &g);
     if (s != PIPO_OK) {
@@ -1257,6 +1308,7 @@ pipo_status ensure_graph(pipo_ctx* ctx) {
     cudaGraphDestroy(g);
     if (e != cudaSuccess) return fail(ctx, PIPO_ECUDA, "graph instantiate: %s", cudaGetErrorString(e));
     ctx->graph_B = ctx->B;
+    ctx->graph_regular = ctx->regular;
     return PIPO_OK;
 }
 
@@ -1521,9 +1573,32 @@ pipo_status pipo_set_threshold(pipo_ctx* ctx, float tau, int32_t force_mode) {
     return PIPO_OK;
 }
 
-pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride, const int32_t* h_lens,
-                         int32_t* h_tokens, int32_t* h_n_accepted) {
-    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+}  // extern "C"
+
+namespace {
+
+// Device copy of prompt inputs (int32, n elements): pf_pairs (and pf_mtp) grow
+// to hold them.
+pipo_status ensure_prompt_buffers(pipo_ctx* ctx, size_t n) {
+    if (n <= ctx->pf_cap) return PIPO_OK;
+    for (void* p : {(void*)ctx->pf_pairs, (void*)ctx->pf_mtp})
+        if (p) {
+            cudaFree(p);
+            ctx->allocs.erase(std::find(ctx->allocs.begin(), ctx->allocs.end(), p));
+        }
+    ctx->pf_pairs = ctx->pf_mtp = nullptr;
+    ctx->pf_cap = 0;
+    TRY(dalloc(ctx, &ctx->pf_pairs, n * 4));
+    TRY(dalloc(ctx, &ctx->pf_mtp, n * 4));
+    ctx->pf_cap = n;
+    return PIPO_OK;
+}
+
+// Shared checks of both prefills: batch, lengths in [1, stride], ids in
+// [0, V).  Returns the lengths' common value of units (pairs: (len + 1) / 2;
+// regular decoding: len) in *units.
+pipo_status check_prompt(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride, const int32_t* h_lens,
+                         bool pairs, int* units) {
     const pipo_config& c = ctx->cfg;
     if (batch < 1 || batch > c.max_batch || !h_ids || !h_lens || stride < 1)
         return fail(ctx, PIPO_EINVAL, "bad prefill arguments (batch %d, stride %d)", batch, stride);
@@ -1531,8 +1606,10 @@ pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int
     for (int b = 0; b < batch; ++b) {
         const int len = h_lens[b];
         if (len < 1 || len > stride) return fail(ctx, PIPO_EINVAL, "sequence %d: length %d not in [1, %d]", b, len, stride);
-        const int nb = (len + 1) / 2;
-        if (N >= 0 && nb != N) return fail(ctx, PIPO_EINVAL, "sequences must give the same number of pairs");
+        const int nb = pairs ? (len + 1) / 2 : len;
+        if (N >= 0 && nb != N)
+            return fail(ctx, PIPO_EINVAL, pairs ? "sequences must give the same number of pairs"
+                                                : "sequences must have the same length");
         N = nb;
         for (int i = 0; i < len; ++i) {
             const int32_t t = h_ids[(size_t)b * stride + i];
@@ -1540,6 +1617,19 @@ pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int
         }
     }
     if (N > c.max_ctx) return fail(ctx, PIPO_ECAPACITY, "prompt needs %d entries > max_ctx %d", N, c.max_ctx);
+    *units = N;
+    return PIPO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride, const int32_t* h_lens,
+                         int32_t* h_tokens, int32_t* h_n_accepted) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    int N = 0;
+    TRY(check_prompt(ctx, batch, h_ids, stride, h_lens, true, &N));
     CK(cudaSetDevice(ctx->dev));
     // pairs [N][B][2] (PAD = -1 in an odd prompt's last slot), MTP inputs [N][B]
     std::vector<int32_t> pairs((size_t)N * batch * 2), mtp((size_t)N * batch, 0);
@@ -1551,37 +1641,73 @@ pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int
             pairs[((size_t)j * batch + b) * 2 + 1] = (2 * j + 1 < len) ? t[2 * j + 1] : -1;
             if (j + 1 < N) mtp[(size_t)j * batch + b] = t[2 * j + 2];
         }
-    if (pairs.size() > ctx->pf_cap) {
-        for (void* p : {(void*)ctx->pf_pairs, (void*)ctx->pf_mtp})
-            if (p) {
-                cudaFree(p);
-                ctx->allocs.erase(std::find(ctx->allocs.begin(), ctx->allocs.end(), p));
-            }
-        ctx->pf_pairs = ctx->pf_mtp = nullptr;
-        ctx->pf_cap = 0;
-        TRY(dalloc(ctx, &ctx->pf_pairs, pairs.size() * 4));
-        TRY(dalloc(ctx, &ctx->pf_mtp, pairs.size() * 4));
-        ctx->pf_cap = pairs.size();
-    }
+    TRY(ensure_prompt_buffers(ctx, pairs.size()));
     CK(cudaMemcpyAsync(ctx->pf_pairs, pairs.data(), pairs.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
     CK(cudaMemcpyAsync(ctx->pf_mtp, mtp.data(), mtp.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
     CK(cudaMemsetAsync(ctx->n_pos, 0, (size_t)batch * 4, ctx->stream));
     CK(cudaMemsetAsync(ctx->emitted, 0, (size_t)batch * 8, ctx->stream));
     ctx->B = batch;
+    ctx->regular = false;
+    ctx->prefilled = false;
+    ctx->h_len.assign(batch, 0);
     const int saved = ctx->launches;
-    for (int j = 0; j < N; ++j) TRY(enqueue_position(ctx, j + 1 < N ? PREFILL_MID : PREFILL_LAST, j));
+    for (int j = 0; j < N; ++j) {
+        TRY(enqueue_position(ctx, j + 1 < N ? PREFILL_MID : PREFILL_LAST, j));
+        ctx->h_len.assign(batch, j + 1);
+    }
     ctx->launches = saved;
     if (h_tokens) CK(cudaMemcpyAsync(h_tokens, ctx->out_tokens, (size_t)batch * 8, cudaMemcpyDeviceToHost, ctx->stream));
     if (h_n_accepted) CK(cudaMemcpyAsync(h_n_accepted, ctx->out_nacc, (size_t)batch * 4, cudaMemcpyDeviceToHost, ctx->stream));
     CK(cudaStreamSynchronize(ctx->stream));
     ctx->h_len.assign(batch, N);
     ctx->prefilled = true;
-    return PIPO_OK;
+    return check_device_error(ctx);
 }
 
-pipo_status pipo_decode_step_async(pipo_ctx* ctx, int32_t* d_tokens, int32_t* d_n_accepted) {
+pipo_status pipo_regular_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride,
+                                 const int32_t* h_lens, int32_t* h_tokens, int32_t* h_n_accepted) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    int N = 0;
+    TRY(check_prompt(ctx, batch, h_ids, stride, h_lens, false, &N));
+    CK(cudaSetDevice(ctx->dev));
+    // tokens [N][B]
+    std::vector<int32_t> toks((size_t)N * batch);
+    for (int j = 0; j < N; ++j)
+        for (int b = 0; b < batch; ++b) toks[(size_t)j * batch + b] = h_ids[(size_t)b * stride + j];
+    TRY(ensure_prompt_buffers(ctx, toks.size()));
+    CK(cudaMemcpyAsync(ctx->pf_pairs, toks.data(), toks.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
+    CK(cudaMemsetAsync(ctx->n_pos, 0, (size_t)batch * 4, ctx->stream));
+    ctx->B = batch;
+    ctx->regular = true;
+    ctx->prefilled = false;
+    ctx->h_len.assign(batch, 0);
+    const int saved = ctx->launches;
+    for (int j = 0; j < N; ++j) {
+        TRY(enqueue_regular(ctx, j + 1 < N ? PREFILL_MID : PREFILL_LAST, j));
+        ctx->h_len.assign(batch, j + 1);
+    }
+    ctx->launches = saved;
+    // the prefill's token is the first output, not a decode step's
+    CK(cudaMemsetAsync(ctx->emitted, 0, (size_t)batch * 8, ctx->stream));
+    if (h_tokens) CK(cudaMemcpyAsync(h_tokens, ctx->out_tokens, (size_t)batch * 8, cudaMemcpyDeviceToHost, ctx->stream));
+    if (h_n_accepted) CK(cudaMemcpyAsync(h_n_accepted, ctx->out_nacc, (size_t)batch * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    ctx->h_len.assign(batch, N);
+    ctx->prefilled = true;
+    return check_device_error(ctx);
+}
+
+}  // extern "C"
+
+namespace {
+
+// One decode step of the context's mode, enqueued (graph replay).
+pipo_status step_async(pipo_ctx* ctx, bool regular, int32_t* d_tokens, int32_t* d_n_accepted) {
     if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
     if (!ctx->prefilled) return fail(ctx, PIPO_ESTATE, "decode step before prefill");
+    if (ctx->regular != regular)
+        return fail(ctx, PIPO_ESTATE, regular ? "regular step after a pair prefill (pipo_prefill)"
+                                              : "pair step after a regular-decoding prefill (pipo_regular_prefill)");
     for (int b = 0; b < ctx->B; ++b)
         if (ctx->h_len[b] + 1 > ctx->cfg.max_ctx)
             return fail(ctx, PIPO_ECAPACITY, "sequence %d: KV cache full (%d entries)", b, ctx->h_len[b]);
@@ -1594,12 +1720,32 @@ pipo_status pipo_decode_step_async(pipo_ctx* ctx, int32_t* d_tokens, int32_t* d_
     return PIPO_OK;
 }
 
-pipo_status pipo_decode_step(pipo_ctx* ctx, int32_t* h_tokens, int32_t* h_n_accepted) {
-    TRY(pipo_decode_step_async(ctx, nullptr, nullptr));
+pipo_status step_sync(pipo_ctx* ctx, bool regular, int32_t* h_tokens, int32_t* h_n_accepted) {
+    TRY(step_async(ctx, regular, nullptr, nullptr));
     if (h_tokens) CK(cudaMemcpyAsync(h_tokens, ctx->out_tokens, (size_t)ctx->B * 8, cudaMemcpyDeviceToHost, ctx->stream));
     if (h_n_accepted) CK(cudaMemcpyAsync(h_n_accepted, ctx->out_nacc, (size_t)ctx->B * 4, cudaMemcpyDeviceToHost, ctx->stream));
     CK(cudaStreamSynchronize(ctx->stream));
     return check_device_error(ctx);
+}
+
+}  // namespace
+
+extern "C" {
+
+pipo_status pipo_decode_step_async(pipo_ctx* ctx, int32_t* d_tokens, int32_t* d_n_accepted) {
+    return step_async(ctx, false, d_tokens, d_n_accepted);
+}
+
+pipo_status pipo_decode_step(pipo_ctx* ctx, int32_t* h_tokens, int32_t* h_n_accepted) {
+    return step_sync(ctx, false, h_tokens, h_n_accepted);
+}
+
+pipo_status pipo_regular_step_async(pipo_ctx* ctx, int32_t* d_tokens) {
+    return step_async(ctx, true, d_tokens, nullptr);
+}
+
+pipo_status pipo_regular_step(pipo_ctx* ctx, int32_t* h_tokens) {
+    return step_sync(ctx, true, h_tokens, nullptr);
 }
 
 pipo_status pipo_rollback(pipo_ctx* ctx, const int32_t* h_n_pairs) {
@@ -1926,7 +2072,7 @@ pipo_status pipo_profile_step(pipo_ctx* ctx, int32_t cap, int32_t* h_kind, doubl
     const int saved = ctx->launches;
     const bool pdl = ctx->pdl;
     ctx->pdl = false;
-    pipo_status s = enqueue_position(ctx, DECODE, 0);
+    pipo_status s = enqueue_step(ctx);
     ctx->pdl = pdl;
     ctx->prof = false;
     ctx->launches = saved;

@@ -54,3 +54,15 @@ def step_flops(s: ModelShape, batch: int, ctx_avg: float) -> float:
     layers = s.L + (1 if s.mtp_block else 0)
     macs += batch * layers * (ctx_avg + 1) * s.n_q * s.d_h * 2
     return 2.0 * macs
+
+
+def regular_step_bytes(s: ModelShape, batch: int, ctx_avg: float) -> float:
+    """Algorithmic HBM bytes of one step of regular decoding (the baseline of
+    Sec. 4): the L backbone blocks and the final norm once, E once (one LM-head
+    pass), the backbone caches' entries 0..n read and the new one written.  The
+    input embedding is a gather of one row per sequence (left out, like the
+    activations)."""
+    e = esize(s)
+    w = (s.L * block_params(s) + s.H + s.V * s.H) * e
+    entry = s.L * 2 * s.n_kv * s.d_h * e
+    return float(w + batch * (ctx_avg + 1) * entry + batch * entry)

@@ -1,0 +1,145 @@
+"""Regular decoding on the GPU (the baseline of Sec. 4: one token per backbone
+pass, input E[t], position = token index, final-norm tied LM head) against the
+oracle's regular decoding, through the C ABI, with forced replay: after every
+step both sides continue from the oracle's token.
+
+Per step: LM-head logits max-abs <= 1e-4 (fp32) / 2e-2 (bf16), the token
+bit-exact where the oracle's top-1/top-2 margin > 1e-2, slot 1 always -1, no
+acceptance; the cache lengths and emitted counters after the run.
+
+Opt-in (PIPO_TEST_REGULAR=1) until the mode is part of the default suite.
+"""
+import os
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2605_27255_gb300 import capi, synth
+from parity_util import MARGIN, tol_for
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(os.environ.get("PIPO_TEST_REGULAR") != "1",
+                                 reason="regular-decoding GPU tests run with PIPO_TEST_REGULAR=1")]
+
+SMALL_BF16 = synth.ModelShape("reg-bf16", H=512, L=2, n_q=8, n_kv=2, d_h=128, F=1408, V=4096,
+                              compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1.0e6, tau=0.5)
+
+
+def _compare(shape, o, d, tok, nacc, where):
+    tol = tol_for(shape)
+    checked = 0
+    for b in range(tok.shape[0]):
+        e = float(np.abs(d["logits_b"][b] - o["logits_b"][b]).max())
+        assert e <= tol, f"{where} b={b}: logit error {e:.3g} > {tol}"
+        assert tok[b, 1] == -1 and nacc[b] == 0
+        if o["margin_b"][b] > MARGIN:
+            assert tok[b, 0] == o["tokens"][b, 0] == d["x_b"][b], f"{where} b={b}"
+            checked += 1
+    return checked
+
+
+def _run(shape, w, prompts, steps, max_ctx=None):
+    B, T = prompts.shape
+    max_ctx = max_ctx or T + steps + 1
+    gpu = capi.Pipo(shape, w, max_batch=B, max_ctx=max_ctx, debug=True)
+    try:
+        orc = O.State(O.Model(shape, w, max_ctx=max_ctx), B)
+        tok, nacc = gpu.regular_prefill(prompts)
+        o = orc.regular_prefill(prompts)
+        checked = _compare(shape, o, gpu.debug(), tok, nacc, "prefill")
+        for i in range(steps):
+            gpu.set_pending([[orc.seq(b)["p0"], -1] for b in range(B)])
+            tok = gpu.regular_step()
+            o = orc.regular_step()
+            checked += _compare(shape, o, gpu.debug(), tok, np.zeros(B, np.int32), f"step {i}")
+        n, e = gpu.counters()
+        assert list(n) == [orc.seq(b)["n"] for b in range(B)] == [T + steps] * B
+        assert list(e) == [orc.seq(b)["emitted"] for b in range(B)] == [steps] * B
+        return checked, B * (steps + 1)
+    finally:
+        gpu.close()
+
+
+def test_regular_tiny_fp32_matches_oracle():
+    s = synth.TINY
+    w = synth.gen_weights(s, seed=0)
+    prompts = synth.gen_prompts(1, 64, s.V, seed=1).numpy()
+    checked, total = _run(s, w, prompts, 16)
+    assert checked >= total // 2
+
+
+def test_regular_tiny_batch3_odd_length():
+    s = synth.TINY.with_(compressor="mlp")
+    w = synth.gen_weights(s, seed=2)
+    prompts = synth.gen_prompts(3, 37, s.V, seed=5).numpy()
+    checked, total = _run(s, w, prompts, 6)
+    assert checked >= total // 2
+
+
+@pytest.mark.parametrize("B", [1, 4, 16])
+def test_regular_bf16_matches_oracle(B):
+    """B = 1: CUDA-core GEMVs and the register-ring attention; B = 4, 16:
+    tcgen05 projections and the tensor-core attention (the pair step's
+    kernels at the same batch)."""
+    w = synth.gen_weights(SMALL_BF16, seed=3)
+    prompts = synth.gen_prompts(B, 40, SMALL_BF16.V, seed=2).numpy()
+    checked, total = _run(SMALL_BF16, w, prompts, 5)
+    assert checked >= total // 2
+
+
+def test_free_running_regular_tokens_follow_the_argmax():
+    """Without forced replay each step's input is the previous step's output
+    (the pending token is the device argmax)."""
+    s = synth.TINY
+    w = synth.gen_weights(s, seed=4)
+    prompts = synth.gen_prompts(2, 20, s.V, seed=6).numpy()
+    gpu = capi.Pipo(s, w, max_batch=2, max_ctx=32, debug=True)
+    try:
+        orc = O.State(O.Model(s, w, max_ctx=32), 2)
+        tok, _ = gpu.regular_prefill(prompts)
+        o = orc.regular_prefill(prompts)
+        for i in range(6):
+            if not np.array_equal(tok[:, 0], o["tokens"][:, 0]):
+                break  # a near tie decided differently: the histories part here
+            tok = gpu.regular_step()
+            o = orc.regular_step()
+            assert np.abs(gpu.debug()["logits_b"] - o["logits_b"]).max() <= tol_for(s)
+    finally:
+        gpu.close()
+
+
+def test_mode_errors_and_switching():
+    s = synth.TINY
+    w = synth.gen_weights(s, seed=0)
+    prompts = synth.gen_prompts(2, 16, s.V, seed=3).numpy()
+    gpu = capi.Pipo(s, w, max_batch=2, max_ctx=12, debug=True)
+    ref = capi.Pipo(s, w, max_batch=2, max_ctx=12, debug=True)
+    try:
+        with pytest.raises(capi.PipoError):
+            gpu.regular_step()  # before any prefill
+        with pytest.raises(capi.PipoError):
+            gpu.regular_prefill(prompts)  # 16 tokens > 12 entries
+        with pytest.raises(capi.PipoError):
+            gpu.regular_prefill(prompts, lens=[10, 9])  # unequal lengths
+        gpu.regular_prefill(prompts[:, :10])
+        with pytest.raises(capi.PipoError):
+            gpu.step()  # a pair step in regular mode
+        gpu.regular_step()
+        gpu.regular_step()
+        with pytest.raises(capi.PipoError):
+            gpu.regular_step()  # all 12 entries used
+        # back to pair decoding on the same context: the same results as a fresh one
+        a = gpu.prefill(prompts)
+        b = ref.prefill(prompts)
+        assert all(np.array_equal(x, y) for x, y in zip(a, b))
+        with pytest.raises(capi.PipoError):
+            gpu.regular_step()  # a regular step in pair mode
+        for _ in range(3):
+            a = gpu.step()
+            b = ref.step()
+            assert all(np.array_equal(x, y) for x, y in zip(a, b))
+            assert np.array_equal(gpu.debug()["logits_b"], ref.debug()["logits_b"])
+    finally:
+        gpu.close()
+        ref.close()

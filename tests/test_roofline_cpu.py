@@ -38,3 +38,26 @@ def test_step_bytes_scale_with_batch_and_context():
     assert roofline.step_bytes(s, 4, 15872.0) - roofline.step_bytes(s, 4, 15871.0) == 4 * kv
     # the 4B weights with E twice: about 9.12 GB
     assert 9.10e9 < w < 9.13e9
+
+
+@pytest.mark.parametrize("shape", [synth.TINY, synth.B4, synth.B9])
+def test_regular_step_bytes_are_the_backbone_part_of_the_pair_step(shape):
+    """Regular decoding moves the backbone blocks, the final norm and E once;
+    the pair step adds the compressor, the MTP input projection and block, the
+    confidence head, E a second time and the MTP block's cache entries."""
+    H, e = shape.H, roofline.esize(shape)
+    comp = H * 2 * H + (H * H if shape.compressor == "mlp" else H)
+    mtp = 2 * H + H * 2 * H + (roofline.block_params(shape) if shape.mtp_block else 0) + H
+    conf = 2 * H + H * 2 * H + H
+    mtp_entry = (2 * shape.n_kv * shape.d_h * e) if shape.mtp_block else 0
+    for B, ctx in ((1, 0.0), (4, 100.0), (16, 530.5)):
+        extra = (comp + mtp + conf + shape.V * H) * e + B * (ctx + 2) * mtp_entry
+        assert roofline.step_bytes(shape, B, ctx) - roofline.regular_step_bytes(shape, B, ctx) == pytest.approx(extra)
+    # 4B, written out: a block holds 2*2560 norm + (4096 + 2*1024)*2560 QKV +
+    # 2560*4096 O + 3*9728*2560 SwiGLU = 100,930,560 parameters; 36 of them,
+    # the final norm and E (151936 x 2560) in bf16, plus one entry read and one
+    # written of 36 x K,V x 8 heads x 128 dims x 2 bytes
+    if shape is synth.B4:
+        w = (36 * 100_930_560 + 2560 + 151_936 * 2560) * 2
+        assert w == 8_044_917_760
+        assert roofline.regular_step_bytes(shape, 1, 0.0) == w + 2 * 36 * 2 * 8 * 128 * 2

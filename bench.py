@@ -39,6 +39,8 @@ WORKLOADS = {
     "4b-lc": dict(shape="4b", batch=4, prompt=30720, steps=1024, kv_fill=True),
     "9b-b1": dict(shape="9b", batch=1, prompt=4096, steps=1024),
     "9b-b8": dict(shape="9b", batch=8, prompt=4096, steps=1024),
+    # time to first token on a 16384-token prompt (8192 pairs): config.prefill_s
+    "4b-ttft": dict(shape="4b", batch=1, prompt=16384, steps=32),
 }
 METRIC = "accepted tokens/s/GPU (PIPO pair-decode step)"
 NOMINAL_HBM_GBS = 8000.0  # GB300 HBM3e nominal (~8 TB/s), context beside the measured peak
@@ -56,6 +58,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--profile-steps", type=int, default=8, help="eager steps timed per launch for the roofline")
+    ap.add_argument("--prefill-rows", type=int, default=0,
+                    help="prefill in chunks of this many rows (positions x sequences, at most 128); "
+                         "0: one position at a time")
     ap.add_argument("--regular", action="store_true",
                     help="also time regular decoding (one token per backbone pass, Sec. 4) on the same prompts "
                          "and report its time per output token beside the pair step's")
@@ -278,6 +283,8 @@ def run_pipo(args):
         max_ctx = max(max_ctx, T + W + K + 8)  # regular decoding: one cache entry per token
 
     w = build_weights(shape, "cuda")
+    if args.prefill_rows:
+        os.environ["PIPO_PREFILL_ROWS"] = str(args.prefill_rows)  # read when the context is created
     g = capi.Pipo(shape, w, max_batch=B, max_ctx=max_ctx, tau=tau, force_mode=args.force)
     w_host = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -376,7 +383,7 @@ def run_pipo(args):
         "config": {"workload": args.workload, "shape": wl["shape"], "batch": B, "prompt_tokens": T,
                    "context_entries_avg": ctx_avg, "tau": tau, "force_mode": args.force,
                    "acceptance": tokens / (K * B) - 1.0, "pair_step_us": 1e3 * ms / K,
-                   "prefill_s": t_pf, "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
+                   "prefill_s": t_pf, "prefill_rows": args.prefill_rows, "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
                    "parallelism": f"replicas x{ws}"},
         "roofline": {"bound": "hbm", "kernel": f"weight-streaming projections (every projection and both LM-head "
                                                   f"launches of a step): {desc}",

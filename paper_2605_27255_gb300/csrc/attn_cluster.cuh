@@ -1,11 +1,13 @@
 // Split-KV GQA flash-decode over the paged pair-KV cache, one thread-block
 // cluster per (sequence, kv head) (sm_103a).
 //
-// Grid (CS, n_kv, B), cluster (CS, 1, 1), 256 threads; CS (1 .. 16) is read
-// from the cluster at run time, so one kernel serves every split.  CTA s of the cluster
-// attends the G = n_q/n_kv query heads of its kv head over a contiguous slice
-// of entries 0..n (n = entries before this step; entry n is this step's new
-// key/value).  Fused in:
+// Grid (CS, n_kv, rows), cluster (CS, 1, 1), 256 threads; CS (1 .. 16) is
+// read from the cluster at run time, so one kernel serves every split.  CTA s
+// of the cluster attends the G = n_q/n_kv query heads of its kv head over a
+// contiguous slice of entries 0..n (n = entries before this step; entry n is
+// this step's new key/value).  A decode step has one row per sequence; a
+// prefill chunk has one row per (position, sequence), whose entries were
+// appended before the launch (AttnParams::no_append).  Fused in:
 //   * RoPE of q and of the new k (rotate-half, angle table cos/sin
 //     [max_ctx][d_h/2] precomputed in fp64 and stored as fp32);
 //   * the KV append: the CTA owning entry n rounds k, v to the cache type,
@@ -57,13 +59,21 @@ template <> struct KV8<float> {
 };
 
 struct AttnParams {
-    const float* qkv;       // [B][(n_q + 2 n_kv) * d_h] projections of this step (not rotated)
+    const float* qkv;       // [rows][(n_q + 2 n_kv) * d_h] projections of this step (not rotated)
     int ld_qkv;
     KVView kv;
-    const int32_t* n_pos;   // [B] entries before this step
+    const int32_t* n_pos;   // [nseq] entries before this step
     const float* rope;      // [max_ctx][d_h/2][2] (cos, sin)
-    float* out;             // [B][n_q * d_h]
+    float* out;             // [rows][n_q * d_h]
     float scale;            // 1/sqrt(d_h)
+    // Rows (grid z) map to sequences: row r is sequence r % nseq at position
+    // n_pos[r % nseq] + r / nseq.  A decode step has one row per sequence
+    // (rows == nseq); a prefill chunk has several consecutive positions of
+    // every sequence, whose entries an earlier kernel has already appended
+    // (no_append = 1): each row then attends to entries 0..n of the cache and
+    // writes none.
+    int nseq;
+    int no_append;
 };
 
 // cos/sin of the 8 rotation pairs of lane slice li at position pos
@@ -149,19 +159,22 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     cg::cluster_group cluster = cg::this_cluster();
     const int s = (int)cluster.block_rank();
     const int CS = (int)cluster.num_blocks();
-    const int g = blockIdx.y, b = blockIdx.z;
+    const int g = blockIdx.y, row = blockIdx.z;
+    const int b = row % p.nseq;        // sequence: its block table and length
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int li = lane % LPE, slot = lane / LPE;
     const int n_kv = p.kv.n_kv, n_q = n_kv * G;
-    const int n = p.n_pos[b];          // cached entries; entry n is new
+    const int n = p.n_pos[b] + row / p.nseq;  // cached entries before this row's; entry n is its own
     const int len = n + 1;
     const int chunk = (len + CS - 1) / CS;
     const int j0 = s * chunk, j1 = min(len, j0 + chunk);
-    const int jc = min(j1, n);         // cached part of the slice: [j0, jc)
+    const int jc = min(j1, p.no_append ? len : n);  // read from the cache: [j0, jc)
     const T* Kb = static_cast<const T*>(p.kv.K);
     const T* Vb = static_cast<const T*>(p.kv.V);
 
-    // prefetch the first kU warp steps of keys/values (independent of this step)
+    // prefetch the first kU warp steps of keys/values (independent of this
+    // step, unless the entries were appended by the kernel before)
+    if (p.no_append) pdl_wait();
     KV8<T> kr[kU], vr[kU];
     const int jwb = j0 + warp * EPW;  // warp-uniform base; lane group entry = base + slot
     // loads are unconditional: an entry outside the slice reads entry 0 of the
@@ -180,7 +193,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
 
     // q of the G heads, 8 dims per lane, rotated, pre-scaled
     float q[G][8];
-    const float* qrow = p.qkv + (size_t)b * p.ld_qkv;
+    const float* qrow = p.qkv + (size_t)row * p.ld_qkv;
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) {
         const float4* qp = reinterpret_cast<const float4*>(qrow + (size_t)(g * G + hh) * DH + li * 8);
@@ -261,7 +274,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     // the new entry n: rotate k, round k and v to the cache type, append, attend
     // (the whole warp 0 runs it so that the shuffles see full warps; lane
     // group 0 writes the cache and keeps the entry in its softmax state)
-    if (n >= j0 && n < j1 && warp == 0) {
+    if (!p.no_append && n >= j0 && n < j1 && warp == 0) {
         const float* kp = qrow + (size_t)(n_q + g) * DH + li * 8;
         const float* vp = qrow + (size_t)(n_q + n_kv + g) * DH + li * 8;
         float kf[8], vf[8];
@@ -345,7 +358,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     const int PER = (G * DH + CS - 1) / CS;
     for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
         const int hh = i / DH, t = i % DH;
-        p.out[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + t] =
+        p.out[(size_t)row * n_q * DH + (size_t)(g * G + hh) * DH + t] =
             cluster_merge_elem(cluster, &sm_m[hh], &sm_l[hh], &sm_o[hh][t], CS);
     }
     cluster.sync();  // keep every CTA's shared memory alive until all merges read it

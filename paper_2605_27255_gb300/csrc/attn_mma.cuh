@@ -2,11 +2,13 @@
 // fp32 accumulate) with the keys and values streamed into shared memory by
 // bulk asynchronous copies (sm_103a; bf16 cache, d_h = 128).
 //
-// One thread-block cluster of CS CTAs per (sequence, kv head), as in
-// attn_cluster_kernel: CTA s owns a contiguous slice of the entries 0..n
-// (entry n is this step's new key/value, which the CTA owning it rotates,
-// rounds to bf16, appends and attends to); the CS partial softmax states are
-// merged through distributed shared memory.
+// One thread-block cluster of CS CTAs per (row, kv head), as in
+// attn_cluster_kernel (a row is a sequence in a decode step, a (position,
+// sequence) of a prefill chunk): CTA s owns a contiguous slice of the entries
+// 0..n (in a decode step entry n is the new key/value, which the CTA owning it
+// rotates, rounds to bf16, appends and attends to; a prefill chunk's entries
+// are in the cache already); the CS partial softmax states are merged through
+// distributed shared memory.
 //
 // Per CTA: a producer thread copies aligned 16-entry groups of the slice into
 // a ring of kMmaStages stages with TMA tensor copies: the cache layer is a 2-D
@@ -102,17 +104,18 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     cg::cluster_group cluster = cg::this_cluster();
     const int s = (int)cluster.block_rank();
     const int CS = (int)cluster.num_blocks();
-    const int g = blockIdx.y, b = blockIdx.z;
+    const int g = blockIdx.y, row = blockIdx.z;
+    const int b = row % p.nseq;        // sequence: its block table and length
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n_kv = p.kv.n_kv, n_q = n_kv * G;
-    const int n = p.n_pos[b];          // cached entries; entry n is new
+    const int n = p.n_pos[b] + row / p.nseq;  // cached entries before this row's; entry n is its own
     const int len = n + 1;
     const int chunk = (len + CS - 1) / CS;
     const int j0 = s * chunk, j1 = min(len, j0 + chunk);
-    const int jc = min(j1, n);         // cached part of the slice: [j0, jc)
+    const int jc = min(j1, p.no_append ? len : n);  // read from the cache: [j0, jc)
     const int grp0 = j0 / kMmaRun;
     const int ngrp = jc > j0 ? (jc - 1) / kMmaRun - grp0 + 1 : 0;
-    const bool owns_new = n >= j0 && n < j1;
+    const bool owns_new = !p.no_append && n >= j0 && n < j1;
 
     if (threadIdx.x == 0) {
         prefetch_tmap(&tmK);
@@ -128,8 +131,10 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
 
     if (warp == NW) {
         // ---- producer: whole 16-entry groups (earlier steps wrote them, so
-        // the copies start before the dependency wait)
+        // the copies start before the dependency wait, unless the kernel
+        // before appended some of them)
         if (lane == 0) {
+            if (p.no_append) pdl_wait();
             int t = 0;
             for (; t < ngrp; ++t) {
                 const int st = t % kMmaStages;
@@ -140,13 +145,13 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
                 }
                 const int e = (grp0 + t) * kMmaRun;  // a group never crosses a page
                 const int blk = p.kv.table[(size_t)b * p.kv.blocks_per_seq + e / p.kv.page];
-                const int row = (blk * n_kv + g) * p.kv.page + e % p.kv.page;
+                const int trow = (blk * n_kv + g) * p.kv.page + e % p.kv.page;  // row of the cache tensor
                 unsigned char* stg = ring + (size_t)st * kMmaStageBytes;
                 mbar_arrive_expect_tx(full + st, (uint32_t)kMmaStageBytes);
-                tma_load_2d(stg, &tmK, 0, row, full + st);
-                tma_load_2d(stg + kMmaHalf, &tmK, 64, row, full + st);
-                tma_load_2d(stg + 2 * kMmaHalf, &tmV, 0, row, full + st);
-                tma_load_2d(stg + 3 * kMmaHalf, &tmV, 64, row, full + st);
+                tma_load_2d(stg, &tmK, 0, trow, full + st);
+                tma_load_2d(stg + kMmaHalf, &tmK, 64, trow, full + st);
+                tma_load_2d(stg + 2 * kMmaHalf, &tmV, 0, trow, full + st);
+                tma_load_2d(stg + 3 * kMmaHalf, &tmV, 64, trow, full + st);
             }
             // no copy into this CTA's shared memory may still be in flight at exit
             for (int i = max(0, t - kMmaStages); i < t; ++i)
@@ -157,7 +162,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         const int ct = threadIdx.x;  // 0 .. 32*NW-1
         // ---- prologue: rotated, pre-scaled q of the G heads; the new k, v
         pdl_wait();
-        const float* qrow = p.qkv + (size_t)b * p.ld_qkv;
+        const float* qrow = p.qkv + (size_t)row * p.ld_qkv;
         const float* rope = p.rope + (size_t)n * DH;  // [DH/2][2] cos, sin at position n
         for (int i = ct; i < (G + 1) * (DH / 2); i += 32 * NW) {
             const int h = i / (DH / 2), pr = i % (DH / 2);
@@ -343,7 +348,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     const int PER = (G * DH + CS - 1) / CS;
     for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
         const int hh = i / DH, t = i % DH;
-        p.out[(size_t)b * n_q * DH + (size_t)(g * G + hh) * DH + t] =
+        p.out[(size_t)row * n_q * DH + (size_t)(g * G + hh) * DH + t] =
             cluster_merge_elem(cluster, &sm_m[hh], &sm_l[hh], &sm_o[hh][t], CS);
     }
     cluster.sync();  // keep every CTA's shared memory alive until all merges read it

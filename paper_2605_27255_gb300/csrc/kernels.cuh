@@ -344,6 +344,32 @@ __device__ __forceinline__ size_t kv_off(const KVView& kv, int b, int pos, int g
     return (((size_t)blk * kv.n_kv + g) * kv.page + (pos % kv.page)) * DH;
 }
 
+// Prefill chunk: RoPE on the keys of every row and the append of its key and
+// value, before the chunk's attention reads them (row r is sequence r % nseq
+// at position n_pos[r % nseq] + r / nseq).  Rotate-half with the fp32
+// cos/sin table the attention kernels use ([max_ctx][d_h/2][2]), rounded to
+// the cache type.  grid (rows, n_kv), DH/2 threads.
+template <typename T, int DH>
+__global__ void append_rows_kernel(const float* __restrict__ qkv, int ld_qkv, int n_q, KVView kv,
+                                   const int32_t* __restrict__ n_pos, int nseq, const float* __restrict__ rope) {
+    pdl_launch();
+    pdl_wait();
+    const int row = blockIdx.x, g = blockIdx.y, i = threadIdx.x;
+    const int b = row % nseq;
+    const int pos = n_pos[b] + row / nseq;
+    const float* k = qkv + (size_t)row * ld_qkv + (size_t)(n_q + g) * DH;
+    const float* v = qkv + (size_t)row * ld_qkv + (size_t)(n_q + kv.n_kv + g) * DH;
+    const float c = rope[((size_t)pos * (DH / 2) + i) * 2], s = rope[((size_t)pos * (DH / 2) + i) * 2 + 1];
+    const float a = k[i], bb = k[i + DH / 2];
+    const size_t off = kv_off<T, DH>(kv, b, pos, g);
+    T* K = static_cast<T*>(kv.K) + off;
+    T* V = static_cast<T*>(kv.V) + off;
+    K[i] = from_f<T>(a * c - bb * s);
+    K[i + DH / 2] = from_f<T>(bb * c + a * s);
+    V[i] = from_f<T>(v[i]);
+    V[i + DH / 2] = from_f<T>(v[i + DH / 2]);
+}
+
 // RoPE on q and k (rotate-half, angle = pos * theta^(-2i/d) in double), then
 // the new k and v appended at entry pos = n[b].  grid (B, n_q + 2 n_kv), DH/2 threads.
 template <typename T, int DH>
@@ -547,12 +573,12 @@ __global__ void keys_to_tokens_kernel(const unsigned long long* keys, int32_t* t
     if (b < B) tokens[b] = argmax_row(keys[b]);
 }
 
-// Prefill positions before the last: n[b] += 1.
-__global__ void advance_kernel(int32_t* n_pos, int B) {
+// Prefill positions before the last: n[b] += by (the positions just run).
+__global__ void advance_kernel(int32_t* n_pos, int B, int by) {
     pdl_launch();
     pdl_wait();
     const int b = blockIdx.x * blockDim.x + threadIdx.x;
-    if (b < B) n_pos[b] += 1;
+    if (b < B) n_pos[b] += by;
 }
 
 // Regular decoding (the paper's baseline, Sec. 4): the backbone input is the

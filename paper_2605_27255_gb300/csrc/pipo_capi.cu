@@ -117,6 +117,9 @@ struct pipo_ctx {
     size_t prof_n = 0;
 
     int B = 0;
+    int rows = 0;                     // activation rows of the enqueue in progress (0: B, one per sequence)
+    int max_rows = 0;                 // rows the activation buffers hold: max(max_batch, prefill_rows)
+    int prefill_rows = 0;             // rows of a prefill chunk (positions x sequences; 0: one position at a time)
     bool prefilled = false;
     bool regular = false;             // the prefill was regular decoding (one token per backbone pass)
     std::vector<int32_t> h_len;
@@ -714,7 +717,7 @@ Seg act_seg(const float* src, int ld, int K, const void* gamma = nullptr) {
 GemvParams gemv_base(pipo_ctx* ctx, const void* W, int N, int epi, float* y, int ldy) {
     GemvParams p{};
     p.W = W; p.N = N; p.epi = epi; p.y = y; p.ldy = ldy;
-    p.B = ctx->B; p.splitk = 1; p.eps = ctx->cfg.rms_eps; p.nseg = 1;
+    p.B = ctx->rows > 0 ? ctx->rows : ctx->B; p.splitk = 1; p.eps = ctx->cfg.rms_eps; p.nseg = 1;
     return p;
 }
 
@@ -961,12 +964,26 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         a.B = ctx->B;
         ctx->rec->push_back(ph);
     } else if (!ctx->attn_v0) {
-        // RoPE + KV append + split-KV attention, one cluster per (sequence, kv head)
+        // RoPE + KV append + split-KV attention, one cluster per (row, kv head).
+        // A prefill chunk (several positions per sequence) appends all its
+        // rows' entries first: its rows read each other's.
+        const int R = ctx->rows > 0 ? ctx->rows : ctx->B;
+        const bool chunk = R > ctx->B;
+        if (chunk) {
+            const float* qkv = ctx->qkv;
+            int ld = rows, nq = c.n_q_heads, nseq = ctx->B;
+            const int32_t* np = ctx->n_pos;
+            const float* rope = ctx->rope;
+            void* args[] = {(void*)&qkv, &ld, &nq, &kv, (void*)&np, &nseq, (void*)&rope};
+            void* fn = DH == 64 ? (bf ? (void*)&append_rows_kernel<bf16, 64> : (void*)&append_rows_kernel<float, 64>)
+                                : (bf ? (void*)&append_rows_kernel<bf16, 128> : (void*)&append_rows_kernel<float, 128>);
+            TRY(launch_ex(ctx, fn, dim3(R, c.n_kv_heads), dim3(DH / 2), 0, args));
+        }
         ctx->prof_kind = 1;
         ctx->prof_bytes = 0.0;
         for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b)
             ctx->prof_bytes += (double)(ctx->h_len[b] + 2) * kd * 2 * ctx->esz;
-        AttnParams ap;
+        AttnParams ap{};
         ap.qkv = ctx->qkv;
         ap.ld_qkv = rows;
         ap.kv = kv;
@@ -974,16 +991,18 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         ap.rope = ctx->rope;
         ap.out = ctx->attn;
         ap.scale = 1.0f / sqrtf((float)DH);
+        ap.nseq = ctx->B;
+        ap.no_append = chunk ? 1 : 0;
         void* args[] = {&ap};
-        const int cs = attn_cluster_size(ctx, ctx->B);
+        const int cs = attn_cluster_size(ctx, R);
         const int G = c.n_q_heads / c.n_kv_heads;
-        if (attn_use_mma(ctx, ctx->B) && cs <= 8) {
+        if (attn_use_mma(ctx, R) && cs <= 8) {
             void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
-            TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, ctx->B), dim3(kMmaThreads), mma_attn_smem(),
+            TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, R), dim3(kMmaThreads), mma_attn_smem(),
                           margs, cs));
         }
         else
-            TRY(launch_ex(ctx, attnc_pick(bf, DH, G), dim3(cs, c.n_kv_heads, ctx->B), dim3(kAttnThreads), 0, args,
+            TRY(launch_ex(ctx, attnc_pick(bf, DH, G), dim3(cs, c.n_kv_heads, R), dim3(kAttnThreads), 0, args,
                           cs));
     } else {
     // RoPE + KV append
@@ -1093,8 +1112,8 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
     if (c.mtp_block) TRY(enqueue_block(ctx, ctx->mtp, c.n_layers, ctx->x2));
     if (mode == PREFILL_MID) {
         int32_t* np = ctx->n_pos;
-        int Bv = B;
-        void* args[] = {&np, &Bv};
+        int Bv = B, by = 1;
+        void* args[] = {&np, &Bv, &by};
         return launch_ex(ctx, (const void*)&advance_kernel, dim3((B + 127) / 128), dim3(128), 0, args);
     }
     // draft token (Eq. 5)
@@ -1166,8 +1185,8 @@ pipo_status enqueue_regular(pipo_ctx* ctx, Mode mode, int j) {
     for (int l = 0; l < c.n_layers; ++l) TRY(enqueue_block(ctx, ctx->blocks[l], l, ctx->x));
     if (mode == PREFILL_MID) {
         int32_t* np = ctx->n_pos;
-        int Bv = B;
-        void* args[] = {&np, &Bv};
+        int Bv = B, by = 1;
+        void* args[] = {&np, &Bv, &by};
         return launch_ex(ctx, (const void*)&advance_kernel, dim3((B + 127) / 128), dim3(128), 0, args);
     }
     TRY(enqueue_lm_head(ctx, ctx->x, ctx->final_norm, ctx->am, c.debug ? ctx->dbg_lb : nullptr));
@@ -1180,6 +1199,92 @@ pipo_status enqueue_regular(pipo_ctx* ctx, Mode mode, int j) {
     const float* h = ctx->x;
     void* args[] = {&st, &Hv, (void*)&h};
     return launch_ex(ctx, (const void*)&regular_accept_kernel, dim3(B), dim3(256), 0, args);
+}
+
+// C consecutive prompt positions j0 .. j0+C-1 of every sequence at once, all
+// before the prompt's last position (a pair prefill's teacher-forced
+// positions, Sec. 3 / App. A.2, or regular decoding's prompt tokens): the
+// C x B rows (row r = position j0 + r / B of sequence r % B, the layout of
+// the prompt buffers) go through the projections as one batch, so each
+// weight streams once per chunk instead of once per position; each block
+// appends the chunk's keys and values and then attends row by row over the
+// entries up to the row's own.  The heads do not run (the MTP block does,
+// teacher-forced, for pairs); the positions advance by C.
+pipo_status enqueue_prefill_chunk(pipo_ctx* ctx, bool regular, int j0, int C) {
+    const pipo_config& c = ctx->cfg;
+    const int H = c.hidden, B = ctx->B, R = C * B;
+    if (R > ctx->max_rows || C < 1 || ctx->rec || ctx->attn_v0)
+        return fail(ctx, PIPO_EINVAL, "prefill chunk of %d rows (at most %d)", R, ctx->max_rows);
+    struct RowsGuard {
+        pipo_ctx* c;
+        ~RowsGuard() { c->rows = 0; }
+    } guard{ctx};
+    ctx->rows = R;
+    ctx->tc_shallow = attn_is_long(ctx);
+    const bool bf = c.dtype == 1;
+    if (regular) {
+        const void* E = ctx->E;
+        const int32_t* tok = ctx->pf_pairs + (size_t)j0 * B;
+        int ld = 1, V = c.vocab, Hv = H, zn = 0;
+        float* x = ctx->x;
+        unsigned long long* am = ctx->am;
+        void* args[] = {(void*)&E, (void*)&tok, &ld, &V, &Hv, &x, &am, &zn};
+        TRY(launch_ex(ctx, bf ? (const void*)&embed_kernel<bf16> : (const void*)&embed_kernel<float>, dim3(R),
+                      dim3(256), 0, args));
+    } else {
+        // pair embed + compressor (Eq. 1) of the chunk's pairs
+        Seg s0{}, s1{};
+        s0.table = ctx->E; s0.pad = ctx->x_pad; s0.tok = ctx->pf_pairs + (size_t)j0 * B * 2; s0.tok_ld = 2; s0.K = H;
+        s1 = s0; s1.tok = s0.tok + 1;
+        GemvParams p;
+        if (c.compressor == 0) {
+            p = gemv_base(ctx, ctx->comp_W, H, EPI_BIAS, ctx->x, H);
+            p.bias = ctx->comp_b;
+        } else {
+            p = gemv_base(ctx, ctx->comp_W1, H, EPI_SILU, ctx->t, H);
+        }
+        p.seg[0] = s0; p.seg[1] = s1; p.nseg = 2; p.K = 2 * H;
+        TRY(launch_gemv(ctx, p));
+        if (c.compressor == 1) {
+            p = gemv_base(ctx, ctx->comp_W2, H, EPI_STORE, ctx->x, H);
+            p.seg[0] = act_seg(ctx->t, H, H);
+            p.K = H;
+            TRY(launch_gemv(ctx, p));
+        }
+    }
+    for (int l = 0; l < c.n_layers; ++l) TRY(enqueue_block(ctx, ctx->blocks[l], l, ctx->x));
+    if (!regular) {
+        // MTP head, teacher-forced (App. A.2): W_fc [RMSNorm(h_b); RMSNorm(E[next prompt token])]
+        GemvParams p = gemv_base(ctx, ctx->mtp_W_fc, H, EPI_STORE, ctx->x2, H);
+        p.seg[0] = act_seg(ctx->x, H, H, ctx->mtp_norm_h);
+        Seg se{};
+        se.table = ctx->E; se.pad = ctx->x_pad; se.gamma = ctx->mtp_norm_e; se.K = H;
+        se.tok = ctx->pf_mtp + (size_t)j0 * B; se.tok_ld = 1;
+        p.seg[1] = se; p.nseg = 2; p.K = 2 * H;
+        TRY(launch_gemv(ctx, p));
+        if (c.mtp_block) TRY(enqueue_block(ctx, ctx->mtp, c.n_layers, ctx->x2));
+    }
+    int32_t* np = ctx->n_pos;
+    int Bv = B, by = C;
+    void* args[] = {&np, &Bv, &by};
+    return launch_ex(ctx, (const void*)&advance_kernel, dim3((B + 127) / 128), dim3(128), 0, args);
+}
+
+// The positions before a prompt's last one in chunks of prefill_rows / B
+// positions (when chunks are enabled and hold two or more positions);
+// *j receives the first position left for the position-by-position path.
+pipo_status enqueue_prefill_chunks(pipo_ctx* ctx, bool regular, int N, int* j) {
+    const int B = ctx->B;
+    const int cmax = ctx->prefill_rows / B;
+    *j = 0;
+    if (cmax < 2 || ctx->attn_v0) return PIPO_OK;
+    while (N - 1 - *j >= 2) {
+        const int C = std::min(cmax, N - 1 - *j);
+        TRY(enqueue_prefill_chunk(ctx, regular, *j, C));
+        *j += C;
+        ctx->h_len.assign(B, *j);
+    }
+    return PIPO_OK;
 }
 
 // The decode step of the context's current mode.
@@ -1496,13 +1601,18 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
 
         // activations and state
         const int qd = c.n_q_heads * DH, kd = c.n_kv_heads * DH;
+        // prefill chunks: PIPO_PREFILL_ROWS=<rows> (positions x sequences per
+        // chunk, at most 128; 0 or unset: one position at a time)
+        if (const char* ev = getenv("PIPO_PREFILL_ROWS")) ctx->prefill_rows = std::min(128, std::max(0, atoi(ev)));
+        const int MR = std::max(MB, ctx->prefill_rows);
+        ctx->max_rows = MR;
         // GEMM inputs get at least as many rows as the tensor-core batch width
         // (their activation tensor maps read box-sized tiles of BH rows)
-        ctx->act_rows = c.dtype == 1 ? std::max(MB, tc_bn(std::min(MB, 128))) : MB;
+        ctx->act_rows = c.dtype == 1 ? std::max(MR, tc_bn(std::min(MR, 128))) : MR;
         const size_t AR = (size_t)ctx->act_rows;
         TRY(dalloc(ctx, &ctx->x, AR * H * 4));
         TRY(dalloc(ctx, &ctx->x2, AR * H * 4));
-        TRY(dalloc(ctx, &ctx->qkv, (size_t)MB * (qd + 2 * kd) * 4));
+        TRY(dalloc(ctx, &ctx->qkv, (size_t)MR * (qd + 2 * kd) * 4));
         TRY(dalloc(ctx, &ctx->q, (size_t)MB * qd * 4));
         TRY(dalloc(ctx, &ctx->attn, AR * qd * 4));
         TRY(dalloc(ctx, &ctx->act, AR * c.ffn * 4));
@@ -1515,15 +1625,15 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         CK(cudaMemset(ctx->counters, 0, (size_t)MB * c.n_kv_heads * 4));
         TRY(dalloc(ctx, &ctx->am, (size_t)2 * MB * 8));
         const int smax = std::max(resadd_splits(ctx, H, qd), resadd_splits(ctx, H, c.ffn));
-        TRY(dalloc(ctx, &ctx->gemv_part, (size_t)smax * MB * H * 4));
-        // one counter per (batch group, row): at most MB groups
-        TRY(dalloc(ctx, &ctx->gemv_rowcnt, (size_t)MB * H * 4));
-        CK(cudaMemset(ctx->gemv_rowcnt, 0, (size_t)MB * H * 4));
+        TRY(dalloc(ctx, &ctx->gemv_part, (size_t)smax * MR * H * 4));
+        // one counter per (batch group, row): at most MR groups
+        TRY(dalloc(ctx, &ctx->gemv_rowcnt, (size_t)MR * H * 4));
+        CK(cudaMemset(ctx->gemv_rowcnt, 0, (size_t)MR * H * 4));
         // tensor-core projections: the bf16 activation tile
         if (const char* ev = getenv("PIPO_TC_MIN_BATCH")) ctx->tc_min_b = std::max(1, atoi(ev));
         if (const char* ev = getenv("PIPO_TC_SPLITS")) ctx->tc_splits = std::max(0, atoi(ev));
-        if (c.dtype == 1 && MB >= ctx->tc_min_b) {
-            ctx->tc_bn_max = tc_bn(std::min(MB, 128));
+        if (c.dtype == 1 && MR >= ctx->tc_min_b) {
+            ctx->tc_bn_max = tc_bn(std::min(MR, 128));
             ctx->tc_kmax = std::max({2 * (int)H, qd, c.ffn});
             TRY(dalloc(ctx, &ctx->tc_xb, (size_t)2 * ctx->tc_bn_max * ctx->tc_kmax * 2));
         }
@@ -1651,7 +1761,9 @@ pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int
     ctx->prefilled = false;
     ctx->h_len.assign(batch, 0);
     const int saved = ctx->launches;
-    for (int j = 0; j < N; ++j) {
+    int j = 0;
+    TRY(enqueue_prefill_chunks(ctx, false, N, &j));
+    for (; j < N; ++j) {
         TRY(enqueue_position(ctx, j + 1 < N ? PREFILL_MID : PREFILL_LAST, j));
         ctx->h_len.assign(batch, j + 1);
     }
@@ -1682,7 +1794,9 @@ pipo_status pipo_regular_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_
     ctx->prefilled = false;
     ctx->h_len.assign(batch, 0);
     const int saved = ctx->launches;
-    for (int j = 0; j < N; ++j) {
+    int j = 0;
+    TRY(enqueue_prefill_chunks(ctx, true, N, &j));
+    for (; j < N; ++j) {
         TRY(enqueue_regular(ctx, j + 1 < N ? PREFILL_MID : PREFILL_LAST, j));
         ctx->h_len.assign(batch, j + 1);
     }

@@ -94,6 +94,14 @@ def lib():
             L.orc_sample.argtypes = [_D, C.c_int, _I, C.c_int, C.c_double, C.c_int, C.c_double, C.c_double,
                                      C.c_double]
             L.orc_sample.restype = C.c_int
+            L.orc_sample_ex.argtypes = [_D, C.c_int, _I, C.c_int, C.c_double, C.c_int, C.c_double, C.c_double,
+                                        C.c_double, _D]
+            L.orc_sample_ex.restype = C.c_int
+            L.orc_set_sampler.argtypes = [C.c_void_p, C.c_double, C.c_int, C.c_double, C.c_double]
+            L.orc_step_u.argtypes = [C.c_void_p, C.c_double, C.c_int, _D, C.POINTER(OrcOut)]
+            L.orc_prefill_u.argtypes = [C.c_void_p, _I, _I, C.c_int, C.c_double, C.c_int, _D, C.POINTER(OrcOut)]
+            L.orc_get_hist.argtypes = [C.c_void_p, C.c_int, _I, C.c_int]
+            L.orc_get_hist.restype = C.c_int
             L.orc_argmax.argtypes = [_D, C.c_int, _D]
             L.orc_argmax.restype = C.c_int
             for f in ("orc_silu", "orc_sigmoid", "orc_round_bf16"):
@@ -175,23 +183,44 @@ class State:
             lib().orc_free(self.ptr)
             self.ptr = None
 
-    def prefill(self, ids, lens=None, tau=0.5, force=0, logits=True):
+    def _draws(self, u):
+        if u is None:
+            return None, None
+        a = np.ascontiguousarray(np.asarray(u, dtype=np.float64).reshape(self.B, 2))
+        return a, _dp(a)
+
+    def prefill(self, ids, lens=None, tau=0.5, force=0, logits=True, u=None):
+        """u: draws [B, 2] of the two heads at the last position (sampler on)."""
         ids = np.ascontiguousarray(np.asarray(ids, dtype=np.int32))
         if lens is None:
             lens = np.full(self.B, ids.shape[1], np.int32)
         lens = np.ascontiguousarray(np.asarray(lens, dtype=np.int32))
         o, s = _out(self.B, self.m.shape.V, self.m.shape.H, logits)
-        rc = lib().orc_prefill(self.ptr, _ip(ids), _ip(lens), ids.shape[1], tau, force, C.byref(s))
+        keep, up = self._draws(u)
+        rc = lib().orc_prefill_u(self.ptr, _ip(ids), _ip(lens), ids.shape[1], tau, force, up, C.byref(s))
         if rc != OK:
             raise ValueError(f"oracle prefill failed: {rc}")
         return o
 
-    def step(self, tau=0.5, force=0, logits=True):
+    def step(self, tau=0.5, force=0, logits=True, u=None):
+        """u: draws [B, 2] of the two heads (sampler on)."""
         o, s = _out(self.B, self.m.shape.V, self.m.shape.H, logits)
-        rc = lib().orc_step(self.ptr, tau, force, C.byref(s))
+        keep, up = self._draws(u)
+        rc = lib().orc_step_u(self.ptr, tau, force, up, C.byref(s))
         if rc != OK:
             raise ValueError(f"oracle step failed: {rc}")
         return o
+
+    def set_sampler(self, temperature=1.0, top_k=20, top_p=0.95, rep_penalty=1.5):
+        """Sampling in both heads (temperature <= 0: greedy again)."""
+        if lib().orc_set_sampler(self.ptr, temperature, top_k, top_p, rep_penalty) != OK:
+            raise ValueError("oracle sampler: bad settings")
+
+    def history(self, b):
+        n = lib().orc_get_hist(self.ptr, b, None, 0)
+        h = np.zeros(n, np.int32)
+        lib().orc_get_hist(self.ptr, b, _ip(h), n)
+        return h
 
     def regular_prefill(self, ids, lens=None, logits=True):
         """Regular decoding (one token per backbone pass, the paper's baseline):
@@ -290,6 +319,19 @@ def attend(q, K, V, n_q, n_kv, d):
     out = np.zeros(n_q * d)
     lib().orc_attend(_dp(q), _dp(K), _dp(V), K.shape[0], n_q, n_kv, d, _dp(out))
     return out
+
+
+def sample_ex(logits, u, hist=(), temperature=1.0, top_k=20, top_p=0.95, rep_penalty=1.5):
+    """orc_sample_ex: (token, decision margin)."""
+    x = np.ascontiguousarray(logits, dtype=np.float64)
+    h = np.ascontiguousarray(np.asarray(hist, dtype=np.int32).reshape(-1))
+    nh = h.size
+    if nh == 0:
+        h = np.zeros(1, np.int32)
+    m = C.c_double()
+    t = lib().orc_sample_ex(_dp(x), x.size, _ip(h), nh, float(temperature), int(top_k), float(top_p),
+                            float(rep_penalty), float(u), C.byref(m))
+    return t, m.value
 
 
 def argmax(x):

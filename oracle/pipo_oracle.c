@@ -34,7 +34,10 @@
  *
  * Also: regular decoding of the same backbone (one token per pass, no
  * compressor or heads beyond the LM head), the baseline the paper compares
- * PIPO with (orc_regular_prefill / orc_regular_step).
+ * PIPO with (orc_regular_prefill / orc_regular_step); and the paper's
+ * evaluation sampler in both heads (orc_set_sampler, orc_step_u,
+ * orc_prefill_u: temperature, top-k, top-p, repetition penalty over the
+ * sequence's tokens so far, the uniform draws passed in).
  *
  * Parity of every function here is pinned by the not-gpu tests (closed forms,
  * special cases, brute-force recompute, invariants).
@@ -196,8 +199,19 @@ static int scored_desc(const void *a, const void *b) {
     return (x->id > y->id) - (x->id < y->id);
 }
 
-int orc_sample(const double *logits, int V, const int32_t *hist, int n_hist, double temperature, int top_k,
-               double top_p, double rep_penalty, double u) {
+/* The same draw, also returning in *margin (if not NULL) how far the decision
+ * is from changing: the smallest of
+ *   - the logit gaps (after penalty and temperature) between the picked id
+ *     and its neighbours in the order (a swap would move the pick),
+ *   - the gap at the top-k boundary when the nucleus takes all k ids,
+ *   - the distance of the top-p cut from p (p < 1),
+ *   - the distance of u from the ends of the picked id's interval of
+ *     cumulative renormalised mass.
+ * Logit gaps and masses mix units; a caller compares the margin with a
+ * threshold above both its logit and its mass errors.  For k == 1 the margin
+ * is the top-1 / top-2 logit gap, as for the argmax. */
+int orc_sample_ex(const double *logits, int V, const int32_t *hist, int n_hist, double temperature, int top_k,
+                  double top_p, double rep_penalty, double u, double *margin) {
     orc_scored *sc = (orc_scored *)malloc(sizeof(orc_scored) * V);
     unsigned char *seen = (unsigned char *)calloc(V, 1);
     for (int i = 0; i < n_hist; i++)
@@ -222,14 +236,37 @@ int orc_sample(const double *logits, int V, const int32_t *hist, int n_hist, dou
     double Zp = 0.0;
     for (int i = 0; i < np; i++) Zp += e[i];
     const double target = u * Zp;
-    int pick = sc[np - 1].id;
+    int k = np - 1;  /* position of the pick in the order */
     cum = 0.0;
     for (int i = 0; i < np; i++) {
+        if (cum + e[i] > target) { k = i; break; }
         cum += e[i];
-        if (cum > target) { pick = sc[i].id; break; }
+    }
+    double below = 0.0;  /* mass before position k */
+    for (int i = 0; i < k; i++) below += e[i];
+    int pick = sc[k].id;
+    if (margin) {
+        double m = INFINITY;
+        if (k > 0) m = fmin(m, sc[k - 1].v - sc[k].v);
+        if (k + 1 < V) m = fmin(m, sc[k].v - sc[k + 1].v);
+        if (np == keep && keep < V) m = fmin(m, sc[keep - 1].v - sc[keep].v);
+        if (top_p < 1.0) {
+            double c = 0.0;
+            for (int i = 0; i < np; i++) c += e[i];
+            m = fmin(m, c / Z - top_p);
+            if (np >= 2) m = fmin(m, top_p - (c - e[np - 1]) / Z);
+        }
+        if (k > 0) m = fmin(m, u - below / Zp);                  /* interior interval ends only */
+        if (k < np - 1) m = fmin(m, (below + e[k]) / Zp - u);
+        *margin = m;
     }
     free(sc); free(seen); free(e);
     return pick;
+}
+
+int orc_sample(const double *logits, int V, const int32_t *hist, int n_hist, double temperature, int top_k,
+               double top_p, double rep_penalty, double u) {
+    return orc_sample_ex(logits, V, hist, n_hist, temperature, top_k, top_p, rep_penalty, u, NULL);
 }
 
 /* ------------------------------------------------------------------ */
@@ -356,14 +393,33 @@ typedef struct {
     int n;             /* cache entries = pairs consumed */
     long emitted;      /* tokens emitted by decode steps */
     double **K, **Vc;  /* L+1 caches of [max_ctx][n_kv*d_h]; index L = MTP layer */
+    int32_t *hist;     /* the sequence's tokens so far: the prompt, then every emitted token */
+    int n_hist, cap_hist;
 } orc_seq;
+
+/* Sampling in both heads (the paper's evaluation setting, Sec. 4): off
+ * (greedy argmax) unless set. */
+typedef struct {
+    int on;
+    double temperature, top_p, rep_penalty;
+    int top_k;
+} orc_sampler;
 
 typedef struct {
     orc_config c;
     orc_weights w;
     int B;
     orc_seq *s;
+    orc_sampler sp;
 } orc_state;
+
+static void hist_push(orc_seq *s, int tok) {
+    if (s->n_hist == s->cap_hist) {
+        s->cap_hist = s->cap_hist ? 2 * s->cap_hist : 256;
+        s->hist = (int32_t *)realloc(s->hist, sizeof(int32_t) * s->cap_hist);
+    }
+    s->hist[s->n_hist++] = tok;
+}
 
 /* per-sequence, per-step results */
 typedef struct {
@@ -404,6 +460,7 @@ void orc_free(orc_state *st) {
     for (int b = 0; b < st->B; b++) {
         for (int l = 0; l <= st->c.L; l++) { free(st->s[b].K[l]); free(st->s[b].Vc[l]); }
         free(st->s[b].K); free(st->s[b].Vc);
+        free(st->s[b].hist);
     }
     free(st->s);
     free(st);
@@ -435,9 +492,16 @@ static void mtp_at(orc_state *st, orc_seq *s, const double *hb, int tok, double 
 }
 
 /* Heads and acceptance of one position: LM head -> x_b, MTP -> x_d,
- * confidence, the acceptance rule, next pair, n += 1. */
-static void heads_and_accept(orc_state *st, int b, double *hb, double tau, int force, orc_out *o) {
+ * confidence, the acceptance rule, next pair, n += 1.  With the sampler on,
+ * x_b is drawn from the backbone head with the draw u2[0] and the sequence's
+ * tokens so far as the repetition history, and x_d from the draft head with
+ * u2[1] and that history followed by x_b (x_b precedes x_d in the output);
+ * the MTP input takes the drawn x_b.  The history then keeps x_b, and x_d
+ * when it is accepted. */
+static void heads_and_accept(orc_state *st, int b, double *hb, double tau, int force, const double *u2,
+                             orc_out *o) {
     const orc_config *c = &st->c;
+    const orc_sampler *sp = &st->sp;
     orc_seq *s = &st->s[b];
     int H = c->H, V = c->V;
     double *lb = (double *)malloc(sizeof(double) * V);
@@ -445,12 +509,18 @@ static void heads_and_accept(orc_state *st, int b, double *hb, double tau, int f
     double *hd = (double *)malloc(sizeof(double) * H);
     double mb, md;
     lm_head(c, &st->w, hb, st->w.final_norm, lb);
-    int xb = orc_argmax(lb, V, &mb);
+    int xb = sp->on ? orc_sample_ex(lb, V, s->hist, s->n_hist, sp->temperature, sp->top_k, sp->top_p,
+                                    sp->rep_penalty, u2[0], &mb)
+                    : orc_argmax(lb, V, &mb);
+    hist_push(s, xb);
     mtp_at(st, s, hb, xb, hd);
     lm_head(c, &st->w, hd, st->w.mtp_norm_post, ld);
-    int xd = orc_argmax(ld, V, &md);
+    int xd = sp->on ? orc_sample_ex(ld, V, s->hist, s->n_hist, sp->temperature, sp->top_k, sp->top_p,
+                                    sp->rep_penalty, u2[1], &md)
+                    : orc_argmax(ld, V, &md);
     double conf = orc_confidence(c, &st->w, hb, hd);
     int acc = (force == 1) ? 1 : (force == 2) ? 0 : (conf >= tau);
+    if (acc) hist_push(s, xd);
     s->p0 = xb;
     s->p1 = acc ? xd : ORC_PAD;
     s->n += 1;
@@ -476,30 +546,48 @@ static void heads_and_accept(orc_state *st, int b, double *hb, double tau, int f
 #define ORC_EINVAL 1
 #define ORC_ECAPACITY 3
 
+/* Sampling in both heads: temperature T, top-k, top-p, repetition penalty
+ * (orc_sample_ex); T <= 0 turns it off (greedy argmax). */
+int orc_set_sampler(orc_state *st, double temperature, int top_k, double top_p, double rep_penalty) {
+    if (temperature <= 0.0) { st->sp.on = 0; return ORC_OK; }
+    if (!(top_p > 0.0 && top_p <= 1.0) || !(rep_penalty > 0.0)) return ORC_EINVAL;
+    st->sp.on = 1;
+    st->sp.temperature = temperature;
+    st->sp.top_k = top_k;
+    st->sp.top_p = top_p;
+    st->sp.rep_penalty = rep_penalty;
+    return ORC_OK;
+}
+
 /* One pair-decode step for every sequence (Sec. 3.1-3.2). force: 0 use the
- * confidence rule, 1 accept every draft, 2 reject every draft. */
-int orc_step(orc_state *st, double tau, int force, orc_out *o) {
+ * confidence rule, 1 accept every draft, 2 reject every draft.  u: the draws
+ * [B][2] of both heads when the sampler is on (else unused, may be NULL). */
+int orc_step_u(orc_state *st, double tau, int force, const double *u, orc_out *o) {
     const orc_config *c = &st->c;
+    if (st->sp.on && !u) return ORC_EINVAL;
     for (int b = 0; b < st->B; b++) if (st->s[b].n >= c->max_ctx) return ORC_ECAPACITY;
     double *x = (double *)malloc(sizeof(double) * c->H);
     for (int b = 0; b < st->B; b++) {
         orc_seq *s = &st->s[b];
         orc_compress(c, &st->w, s->p0, s->p1, x);
         backbone_at(st, s, x);
-        heads_and_accept(st, b, x, tau, force, o);
+        heads_and_accept(st, b, x, tau, force, u ? u + 2 * b : NULL, o);
     }
     free(x);
     return ORC_OK;
 }
+
+int orc_step(orc_state *st, double tau, int force, orc_out *o) { return orc_step_u(st, tau, force, NULL, o); }
 
 /* Prefill: prompt of len_b tokens per sequence (row stride `stride`), paired
  * as (t_{2j}, t_{2j+1}); an odd length ends in (t_last, PAD) (App. B.2).
  * Every latent runs the backbone causally; the MTP cache entry of position
  * j < N-1 is fed the first token of pair j+1; the last position runs the
  * heads and the acceptance rule, which sets the first pending pair. */
-int orc_prefill(orc_state *st, const int32_t *ids, const int32_t *lens, int stride,
-                double tau, int force, orc_out *o) {
+int orc_prefill_u(orc_state *st, const int32_t *ids, const int32_t *lens, int stride,
+                  double tau, int force, const double *u, orc_out *o) {
     const orc_config *c = &st->c;
+    if (st->sp.on && !u) return ORC_EINVAL;
     for (int b = 0; b < st->B; b++) {
         int len = lens[b];
         int N = (len + 1) / 2;
@@ -514,6 +602,8 @@ int orc_prefill(orc_state *st, const int32_t *ids, const int32_t *lens, int stri
         int len = lens[b], N = (len + 1) / 2;
         s->n = 0;
         s->emitted = 0;
+        s->n_hist = 0;
+        for (int i = 0; i < len; i++) hist_push(s, t[i]);
         for (int j = 0; j < N; j++) {
             int t0 = t[2 * j], t1 = (2 * j + 1 < len) ? t[2 * j + 1] : ORC_PAD;
             orc_compress(c, &st->w, t0, t1, x);
@@ -522,12 +612,25 @@ int orc_prefill(orc_state *st, const int32_t *ids, const int32_t *lens, int stri
                 mtp_at(st, s, x, t[2 * j + 2], hd);
                 s->n += 1;
             } else {
-                heads_and_accept(st, b, x, tau, force, o);
+                heads_and_accept(st, b, x, tau, force, u ? u + 2 * b : NULL, o);
             }
         }
     }
     free(x); free(hd);
     return ORC_OK;
+}
+
+int orc_prefill(orc_state *st, const int32_t *ids, const int32_t *lens, int stride,
+                double tau, int force, orc_out *o) {
+    return orc_prefill_u(st, ids, lens, stride, tau, force, NULL, o);
+}
+
+/* Introspection for the tests: the token history of sequence b (the prompt,
+ * then every emitted token); copies at most cap ids, returns the length. */
+int orc_get_hist(const orc_state *st, int b, int32_t *out, int cap) {
+    const orc_seq *s = &st->s[b];
+    for (int i = 0; i < s->n_hist && i < cap; i++) out[i] = s->hist[i];
+    return s->n_hist;
 }
 
 /* ------------------------------------------------------------------ */
@@ -548,6 +651,7 @@ static void regular_head(orc_state *st, int b, double *h, orc_out *o) {
     double m;
     lm_head(c, &st->w, h, st->w.final_norm, lg);
     int x = orc_argmax(lg, V, &m);
+    hist_push(s, x);
     s->p0 = x;
     s->p1 = ORC_PAD;
     s->n += 1;
@@ -580,6 +684,8 @@ int orc_regular_prefill(orc_state *st, const int32_t *ids, const int32_t *lens, 
         const int32_t *t = ids + (size_t)b * stride;
         s->n = 0;
         s->emitted = 0;
+        s->n_hist = 0;
+        for (int j = 0; j < lens[b]; j++) hist_push(s, t[j]);
         for (int j = 0; j < lens[b]; j++) {
             embed(c, &st->w, t[j], x);
             backbone_at(st, s, x);

@@ -185,6 +185,28 @@ PIPO_API pipo_status pipo_rollback(pipo_ctx *ctx, const int32_t *h_n_pairs);
 /* Acceptance threshold and force mode (0 rule, 1 accept all, 2 reject all). */
 PIPO_API pipo_status pipo_set_threshold(pipo_ctx *ctx, float tau, int32_t force_mode);
 
+/* The paper's evaluation sampler in both heads (Sec. 4; its settings:
+ * temperature 1, top_k 20, top_p 0.95, repetition penalty 1.5) in place of
+ * the greedy argmax.  Per head and sequence: a logit l of an id already in the
+ * sequence's tokens so far (the prompt, then every emitted token) becomes
+ * l / rep_penalty if l > 0, else l * rep_penalty; divide by temperature; keep
+ * the top_k largest (ties to the lower id); keep the shortest prefix whose
+ * softmax mass reaches top_p; pick the first id whose cumulative renormalised
+ * mass exceeds u times the prefix mass.  x_b is drawn first and joins the
+ * history before x_d is drawn; an accepted x_d joins it after the decision;
+ * the MTP input takes the drawn x_b.
+ *
+ * h_u: host [n_u][max_batch][2] uniform draws in [0, 1) (slot 0 for x_b,
+ * slot 1 for x_d); the k-th position that runs the heads (the prefill's last
+ * position, then each decode step) takes row k mod n_u.  Copied; the caller
+ * keeps ownership.  Resets the draw index to 0.  Call before pipo_prefill
+ * (the history is seeded from the prompt there).  temperature <= 0 turns the
+ * sampler off (greedy; the other arguments are ignored).  EINVAL: top_k not
+ * in [1, 32], top_p not in (0, 1], rep_penalty <= 0, a draw outside [0, 1),
+ * or no draws.  Regular decoding stays greedy. */
+PIPO_API pipo_status pipo_set_sampler(pipo_ctx *ctx, float temperature, int32_t top_k, float top_p,
+                                      float rep_penalty, const float *h_u, int32_t n_u);
+
 /* Test hook for forced replay: overwrite the pending pairs, host [B,2]
  * (slot 1 may be -1 = PAD). */
 PIPO_API pipo_status pipo_set_pending(pipo_ctx *ctx, const int32_t *h_pairs);

@@ -78,6 +78,7 @@ SIGNATURES = {
     "pipo_regular_step_async": (C.c_int, [C.c_void_p, C.c_void_p]),
     "pipo_rollback": (C.c_int, [C.c_void_p, _IP]),
     "pipo_set_threshold": (C.c_int, [C.c_void_p, C.c_float, C.c_int32]),
+    "pipo_set_sampler": (C.c_int, [C.c_void_p, C.c_float, C.c_int32, C.c_float, C.c_float, _FP, C.c_int32]),
     "pipo_set_pending": (C.c_int, [C.c_void_p, _IP]),
     "pipo_get_counters": (C.c_int, [C.c_void_p, _IP, C.POINTER(C.c_int64)]),
     "pipo_debug_dump": (C.c_int, [C.c_void_p, C.POINTER(pipo_debug)]),
@@ -195,6 +196,14 @@ def pipo_rollback(ctx, n_pairs) -> None:
 
 def pipo_set_threshold(ctx, tau: float, force_mode: int = 0) -> None:
     _check(load().pipo_set_threshold(ctx, float(tau), int(force_mode)), ctx)
+
+
+def pipo_set_sampler(ctx, temperature: float, top_k: int, top_p: float, rep_penalty: float, u) -> None:
+    """u: [n_u, max_batch, 2] uniform draws in [0, 1)."""
+    u = np.ascontiguousarray(np.asarray(u, dtype=np.float32))
+    n_u = u.shape[0] if u.ndim == 3 else 0
+    _check(load().pipo_set_sampler(ctx, float(temperature), int(top_k), float(top_p), float(rep_penalty),
+                                   _fp(u) if u.size else None, n_u), ctx)
 
 
 def pipo_set_pending(ctx, pairs) -> None:
@@ -374,6 +383,11 @@ class Pipo:
 
     def set_threshold(self, tau, force_mode=0):
         pipo_set_threshold(self.ctx, tau, force_mode)
+
+    def set_sampler(self, u, temperature=1.0, top_k=20, top_p=0.95, rep_penalty=1.5):
+        """Sampling in both heads with the draws u [n_u, max_batch, 2]
+        (temperature <= 0: greedy again)."""
+        pipo_set_sampler(self.ctx, temperature, top_k, top_p, rep_penalty, u)
 
     def set_pending(self, pairs):
         pipo_set_pending(self.ctx, pairs)

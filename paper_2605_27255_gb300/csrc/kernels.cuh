@@ -528,6 +528,11 @@ struct StepState {
     float* dbg_hd;
     int32_t* dbg_xb;       // [B]
     int32_t* dbg_xd;
+    // sampling in both heads (nullptr when greedy): the token-history bitmap
+    // [B][presence_w] gains an accepted draft; the draw index advances
+    uint32_t* presence;
+    int presence_w;
+    int32_t* samp_step;
 };
 
 // Confidence c = sigmoid(W2 . t) with t = SiLU(W1 RMSNorm([h_b; h_d])) computed
@@ -565,6 +570,8 @@ __global__ void accept_kernel(const float* __restrict__ t, const void* W2, int H
     st.emitted[b] += 1 + accept;
     if (st.dbg_conf) st.dbg_conf[b] = c;
     if (st.dbg_xb) { st.dbg_xb[b] = xb; st.dbg_xd[b] = xd; }
+    if (st.presence && accept) atomicOr(st.presence + (size_t)b * st.presence_w + (xd >> 5), 1u << (xd & 31));
+    if (st.samp_step && b == 0) st.samp_step[0] += 1;
 }
 
 // Packed argmax keys -> token ids.

@@ -28,6 +28,7 @@
 #include "kernels.cuh"
 #include "megakernel.cuh"
 #include "pipo.h"
+#include "sampler.cuh"
 #include "tcgen05_gemm.cuh"
 
 using namespace pipo;
@@ -120,6 +121,15 @@ struct pipo_ctx {
     int rows = 0;                     // activation rows of the enqueue in progress (0: B, one per sequence)
     int max_rows = 0;                 // rows the activation buffers hold: max(max_batch, prefill_rows)
     int prefill_rows = 0;             // rows of a prefill chunk (positions x sequences; 0: one position at a time)
+    // sampling in both heads (pipo_set_sampler; greedy when off)
+    bool samp_on = false;
+    float samp_T = 1.f, samp_p = 1.f, samp_rep = 1.f;
+    int samp_k = 1, samp_nu = 0;
+    float* samp_u = nullptr;          // [samp_nu][max_batch][2] draws
+    int32_t* samp_step = nullptr;     // draw index of the next position
+    float* samp_logits = nullptr;     // [2][max_batch][V] logits of both heads
+    uint32_t* presence = nullptr;     // [max_batch][presence_w] token-history bitmap
+    int presence_w = 0;
     bool prefilled = false;
     bool regular = false;             // the prefill was regular decoding (one token per backbone pass)
     std::vector<int32_t> h_len;
@@ -1065,6 +1075,31 @@ pipo_status enqueue_lm_head(pipo_ctx* ctx, const float* h, const void* gamma, un
     return launch_gemv(ctx, p);
 }
 
+// The evaluation sampler on one head's logits (sample_kernel): the pick
+// replaces the head's argmax key; the backbone head's pick joins the history.
+pipo_status enqueue_sample(pipo_ctx* ctx, const float* logits, int head, unsigned long long* am) {
+    const pipo_config& c = ctx->cfg;
+    SampParams sp{};
+    sp.logits = logits;
+    sp.ld = c.vocab;
+    sp.V = c.vocab;
+    sp.presence = ctx->presence;
+    sp.presence_add = head == 0 ? ctx->presence : nullptr;
+    sp.W = ctx->presence_w;
+    sp.inv_T = 1.0f / ctx->samp_T;
+    sp.top_p = ctx->samp_p;
+    sp.rep = ctx->samp_rep;
+    sp.top_k = ctx->samp_k;
+    sp.u = ctx->samp_u;
+    sp.u_step = ctx->samp_step;
+    sp.n_u = ctx->samp_nu;
+    sp.u_rows = c.max_batch;
+    sp.head = head;
+    sp.am = am;
+    void* args[] = {&sp};
+    return launch_ex(ctx, (const void*)&sample_kernel, dim3(ctx->B), dim3(kSampThreads), 0, args);
+}
+
 // One pair position of every sequence.  DECODE: the pending pair; PREFILL_*:
 // prompt pair j.  PREFILL_MID stops after the MTP block (teacher-forced token).
 pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
@@ -1098,8 +1133,13 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
     }
     // backbone (Eq. 2)
     for (int l = 0; l < c.n_layers; ++l) TRY(enqueue_block(ctx, ctx->blocks[l], l, ctx->x));
-    // LM head + argmax (Eq. 3)
-    if (mode != PREFILL_MID) TRY(enqueue_lm_head(ctx, ctx->x, ctx->final_norm, am_b, c.debug ? ctx->dbg_lb : nullptr));
+    // LM head + argmax (Eq. 3), or + the sampler (the history gains x_b)
+    float* lg_b = c.debug ? ctx->dbg_lb : ctx->samp_on ? ctx->samp_logits : nullptr;
+    float* lg_d = c.debug ? ctx->dbg_ld : ctx->samp_on ? ctx->samp_logits + (size_t)c.max_batch * c.vocab : nullptr;
+    if (mode != PREFILL_MID) {
+        TRY(enqueue_lm_head(ctx, ctx->x, ctx->final_norm, am_b, lg_b));
+        if (ctx->samp_on) TRY(enqueue_sample(ctx, lg_b, 0, am_b));
+    }
     // MTP head input (App. A.2): W_fc [RMSNorm(h_b); RMSNorm(E[x_b])]
     p = gemv_base(ctx, ctx->mtp_W_fc, H, EPI_STORE, ctx->x2, H);
     p.seg[0] = act_seg(ctx->x, H, H, ctx->mtp_norm_h);
@@ -1117,7 +1157,8 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
         return launch_ex(ctx, (const void*)&advance_kernel, dim3((B + 127) / 128), dim3(128), 0, args);
     }
     // draft token (Eq. 5)
-    TRY(enqueue_lm_head(ctx, ctx->x2, ctx->mtp_norm_post, am_d, c.debug ? ctx->dbg_ld : nullptr));
+    TRY(enqueue_lm_head(ctx, ctx->x2, ctx->mtp_norm_post, am_d, lg_d));
+    if (ctx->samp_on) TRY(enqueue_sample(ctx, lg_d, 1, am_d));
     // confidence (Eq. 6, App. A.3): t = SiLU(W1 RMSNorm([h_b; h_d]))
     p = gemv_base(ctx, ctx->conf_W1, H, EPI_SILU, ctx->t, H);
     p.seg[0] = act_seg(ctx->x, H, H, ctx->conf_norm);
@@ -1131,6 +1172,9 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
     if (c.debug) {
         st.dbg_conf = ctx->dbg_conf; st.dbg_hb = ctx->dbg_hb; st.dbg_hd = ctx->dbg_hd;
         st.dbg_xb = ctx->dbg_xb; st.dbg_xd = ctx->dbg_xd;
+    }
+    if (ctx->samp_on) {
+        st.presence = ctx->presence; st.presence_w = ctx->presence_w; st.samp_step = ctx->samp_step;
     }
     if (ctx->rec) {
         Phase ph{};
@@ -1389,7 +1433,7 @@ pipo_status ensure_graph(pipo_ctx* ctx) {
     ctx->mk_active = false;
     bool used = false;
     // the persistent step kernel records the pair step only
-    if (!ctx->regular) TRY(try_step_kernel(ctx, used));
+    if (!ctx->regular && !ctx->samp_on) TRY(try_step_kernel(ctx, used));
     if (getenv("PIPO_VERBOSE"))
         fprintf(stderr, "pipo: decode step = %s %s\n", used ? "persistent step kernel" : "kernel graph",
                 ctx->mk_note.c_str());
@@ -1683,6 +1727,52 @@ pipo_status pipo_set_threshold(pipo_ctx* ctx, float tau, int32_t force_mode) {
     return PIPO_OK;
 }
 
+pipo_status pipo_set_sampler(pipo_ctx* ctx, float temperature, int32_t top_k, float top_p, float rep_penalty,
+                             const float* h_u, int32_t n_u) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    const pipo_config& c = ctx->cfg;
+    if (!(temperature > 0.f)) {
+        if (ctx->samp_on) drop_graph(ctx);
+        ctx->samp_on = false;
+        return PIPO_OK;
+    }
+    if (top_k < 1 || top_k > kSampMaxK || !(top_p > 0.f && top_p <= 1.f) || !(rep_penalty > 0.f) ||
+        !std::isfinite(temperature) || !std::isfinite(rep_penalty) || !h_u || n_u < 1)
+        return fail(ctx, PIPO_EINVAL, "bad sampler settings (top_k in [1, %d], top_p in (0, 1], penalty > 0, "
+                                      "draws given)", kSampMaxK);
+    const size_t nu = (size_t)n_u * c.max_batch * 2;
+    for (size_t i = 0; i < nu; ++i)
+        if (!(h_u[i] >= 0.f && h_u[i] < 1.f)) return fail(ctx, PIPO_EINVAL, "draw %zu not in [0, 1)", i);
+    CK(cudaSetDevice(ctx->dev));
+    CK(cudaStreamSynchronize(ctx->stream));
+    if (!ctx->samp_logits) {
+        ctx->presence_w = (c.vocab + 31) / 32;
+        TRY(dalloc(ctx, &ctx->samp_logits, (size_t)2 * c.max_batch * c.vocab * 4));
+        TRY(dalloc(ctx, &ctx->presence, (size_t)c.max_batch * ctx->presence_w * 4));
+        TRY(dalloc(ctx, &ctx->samp_step, 4));
+        CK(cudaMemset(ctx->presence, 0, (size_t)c.max_batch * ctx->presence_w * 4));
+    }
+    if (n_u > ctx->samp_nu) {
+        if (ctx->samp_u) {
+            cudaFree(ctx->samp_u);
+            ctx->allocs.erase(std::find(ctx->allocs.begin(), ctx->allocs.end(), (void*)ctx->samp_u));
+            ctx->samp_u = nullptr;
+        }
+        ctx->samp_nu = 0;
+        TRY(dalloc(ctx, &ctx->samp_u, nu * 4));
+    }
+    CK(cudaMemcpy(ctx->samp_u, h_u, nu * 4, cudaMemcpyHostToDevice));
+    CK(cudaMemset(ctx->samp_step, 0, 4));
+    ctx->samp_nu = n_u;
+    ctx->samp_T = temperature;
+    ctx->samp_k = top_k;
+    ctx->samp_p = top_p;
+    ctx->samp_rep = rep_penalty;
+    ctx->samp_on = true;
+    drop_graph(ctx);
+    return PIPO_OK;
+}
+
 }  // extern "C"
 
 namespace {
@@ -1754,6 +1844,17 @@ pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int
     TRY(ensure_prompt_buffers(ctx, pairs.size()));
     CK(cudaMemcpyAsync(ctx->pf_pairs, pairs.data(), pairs.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
     CK(cudaMemcpyAsync(ctx->pf_mtp, mtp.data(), mtp.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
+    std::vector<uint32_t> bits;
+    if (ctx->samp_on) {
+        // the sampler's repetition history starts with the prompt
+        bits.assign((size_t)batch * ctx->presence_w, 0u);
+        for (int b = 0; b < batch; ++b)
+            for (int i = 0; i < h_lens[b]; ++i) {
+                const int32_t t = h_ids[(size_t)b * stride + i];
+                bits[(size_t)b * ctx->presence_w + (t >> 5)] |= 1u << (t & 31);
+            }
+        CK(cudaMemcpyAsync(ctx->presence, bits.data(), bits.size() * 4, cudaMemcpyHostToDevice, ctx->stream));
+    }
     CK(cudaMemsetAsync(ctx->n_pos, 0, (size_t)batch * 4, ctx->stream));
     CK(cudaMemsetAsync(ctx->emitted, 0, (size_t)batch * 8, ctx->stream));
     ctx->B = batch;

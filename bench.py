@@ -61,6 +61,9 @@ def parse():
     ap.add_argument("--prefill-rows", type=int, default=0,
                     help="prefill in chunks of this many rows (positions x sequences, at most 128); "
                          "0: one position at a time")
+    ap.add_argument("--sampler", action="store_true",
+                    help="decode with the paper's evaluation sampler in both heads (T 1, top-k 20, top-p 0.95, "
+                         "repetition penalty 1.5; seeded draws) instead of the greedy argmax")
     ap.add_argument("--regular", action="store_true",
                     help="also time regular decoding (one token per backbone pass, Sec. 4) on the same prompts "
                          "and report its time per output token beside the pair step's")
@@ -293,6 +296,11 @@ def run_pipo(args):
     torch.cuda.empty_cache()
     stream = torch.cuda.Stream()
     g.set_stream(stream.cuda_stream)
+    if args.sampler:
+        # draws for every position that runs the heads (prefill, warm-up, timed, e2e, profile steps)
+        n_u = 1 + W + 2 * K + args.profile_steps + 8
+        u = np.random.default_rng(11 + rank).random((n_u, B, 2)).astype(np.float32)
+        g.set_sampler(u, temperature=1.0, top_k=20, top_p=0.95, rep_penalty=1.5)
 
     prompts = synth.gen_prompts(B, T if not wl.get("kv_fill") else 2, shape.V, seed=1 + rank * 1000).numpy()
     t_pf = time.perf_counter()
@@ -383,7 +391,9 @@ def run_pipo(args):
         "config": {"workload": args.workload, "shape": wl["shape"], "batch": B, "prompt_tokens": T,
                    "context_entries_avg": ctx_avg, "tau": tau, "force_mode": args.force,
                    "acceptance": tokens / (K * B) - 1.0, "pair_step_us": 1e3 * ms / K,
-                   "prefill_s": t_pf, "prefill_rows": args.prefill_rows, "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
+                   "prefill_s": t_pf, "prefill_rows": args.prefill_rows,
+                   "heads": "sampled (T 1, top-k 20, top-p 0.95, penalty 1.5)" if args.sampler else "greedy",
+                   "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
                    "parallelism": f"replicas x{ws}"},
         "roofline": {"bound": "hbm", "kernel": f"weight-streaming projections (every projection and both LM-head "
                                                   f"launches of a step): {desc}",

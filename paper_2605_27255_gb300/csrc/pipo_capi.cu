@@ -24,6 +24,7 @@
 
 #include "attn_cluster.cuh"
 #include "attn_mma.cuh"
+#include "attn_prefill.cuh"
 #include "gemv_stream.cuh"
 #include "kernels.cuh"
 #include "megakernel.cuh"
@@ -121,6 +122,7 @@ struct pipo_ctx {
     int rows = 0;                     // activation rows of the enqueue in progress (0: B, one per sequence)
     int max_rows = 0;                 // rows the activation buffers hold: max(max_batch, prefill_rows)
     int prefill_rows = 0;             // rows of a prefill chunk (positions x sequences; 0: one position at a time)
+    bool prefill_tile_attn = false;   // chunk attention by tiles of positions (attn_prefill_kernel)
     // sampling in both heads (pipo_set_sampler; greedy when off)
     bool samp_on = false;
     float samp_T = 1.f, samp_p = 1.f, samp_rep = 1.f;
@@ -1006,7 +1008,17 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         void* args[] = {&ap};
         const int cs = attn_cluster_size(ctx, R);
         const int G = c.n_q_heads / c.n_kv_heads;
-        if (attn_use_mma(ctx, R) && cs <= 8) {
+        if (chunk && ctx->prefill_tile_attn && attn_mma_ok(ctx) && (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers) {
+            // causal tiles: the positions of a tile share every key and value they read
+            void* fn = G == 1 ? (void*)&attn_prefill_kernel<1> : G == 2 ? (void*)&attn_prefill_kernel<2>
+                                                                        : (void*)&attn_prefill_kernel<4>;
+            CK(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)prefill_attn_smem()));
+            int C = R / ctx->B;
+            const int TP = kPfVec / G;
+            void* pargs[] = {&ap, &C, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
+            TRY(launch_ex(ctx, fn, dim3((C + TP - 1) / TP, c.n_kv_heads, ctx->B), dim3(kPfThreads),
+                          prefill_attn_smem(), pargs));
+        } else if (attn_use_mma(ctx, R) && cs <= 8) {
             void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
             TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, R), dim3(kMmaThreads), mma_attn_smem(),
                           margs, cs));
@@ -1648,6 +1660,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         // prefill chunks: PIPO_PREFILL_ROWS=<rows> (positions x sequences per
         // chunk, at most 128; 0 or unset: one position at a time)
         if (const char* ev = getenv("PIPO_PREFILL_ROWS")) ctx->prefill_rows = std::min(128, std::max(0, atoi(ev)));
+        if (const char* ev = getenv("PIPO_PREFILL_ATTN")) ctx->prefill_tile_attn = strcmp(ev, "tile") == 0;
         const int MR = std::max(MB, ctx->prefill_rows);
         ctx->max_rows = MR;
         // GEMM inputs get at least as many rows as the tensor-core batch width

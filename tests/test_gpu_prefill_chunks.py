@@ -26,11 +26,16 @@ MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003
                        compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1e6, tau=0.5)
 
 
+@pytest.mark.parametrize("attn", ["rows", "tile"])
 @pytest.mark.parametrize("rows,B,T", [(16, 1, 150), (16, 2, 149), (128, 1, 300), (128, 4, 97), (128, 16, 40)])
-def test_chunked_pair_prefill_matches_oracle(monkeypatch, rows, B, T):
+def test_chunked_pair_prefill_matches_oracle(monkeypatch, attn, rows, B, T):
     """rows / B positions per chunk; T tokens give (T + 1) / 2 pairs, of which
-    all but the last run in chunks (the last chunk ragged)."""
+    all but the last run in chunks (the last chunk ragged).  attn: one
+    decode-style CTA per row, or causal tiles of positions
+    (PIPO_PREFILL_ATTN=tile, attn_prefill_kernel)."""
     monkeypatch.setenv("PIPO_PREFILL_ROWS", str(rows))
+    if attn == "tile":
+        monkeypatch.setenv("PIPO_PREFILL_ATTN", "tile")
     w = synth.gen_weights(MID, seed=3)
     prompts = synth.gen_prompts(B, T, MID.V, seed=7).numpy()
     st = run_forced_replay(MID, w, prompts, 6)
@@ -67,6 +72,24 @@ def _prefill_state(shape, w, prompts, rows, regular=False):
         os.environ.pop("PIPO_PREFILL_ROWS", None)
 
 
+def test_tile_attention_equals_row_attention(monkeypatch):
+    """The two chunk attentions read the same cache entries: caches and
+    outputs agree within the rounding of the summation order."""
+    s = MID
+    w = synth.gen_weights(s, seed=8)
+    prompts = synth.gen_prompts(3, 121, s.V, seed=2).numpy()  # 61 pairs: chunks of 42 rows (14 positions)
+    a = _prefill_state(s, w, prompts, 42)
+    monkeypatch.setenv("PIPO_PREFILL_ATTN", "tile")
+    b = _prefill_state(s, w, prompts, 42)
+    tol = tol_for(s)
+    for cb_a, cb_b in zip(a[2], b[2]):
+        for (Ka, Va), (Kb, Vb) in zip(cb_a, cb_b):
+            scale = max(1.0, float(np.abs(Ka).max()), float(np.abs(Va).max()))
+            assert np.abs(Ka - Kb).max() <= 2 * tol * scale
+            assert np.abs(Va - Vb).max() <= 2 * tol * scale
+    assert np.abs(a[1]["logits_b"] - b[1]["logits_b"]).max() <= 2 * tol
+
+
 @pytest.mark.parametrize("regular", [False, True])
 def test_chunked_equals_position_by_position(regular):
     """Same context shape, same prompts: the chunk-written caches hold the
@@ -87,8 +110,11 @@ def test_chunked_equals_position_by_position(regular):
     assert list(a[4][0]) == list(b[4][0])  # cache lengths
 
 
-def test_chunked_regular_prefill_matches_oracle(monkeypatch):
+@pytest.mark.parametrize("attn", ["rows", "tile"])
+def test_chunked_regular_prefill_matches_oracle(monkeypatch, attn):
     monkeypatch.setenv("PIPO_PREFILL_ROWS", "64")
+    if attn == "tile":
+        monkeypatch.setenv("PIPO_PREFILL_ATTN", "tile")
     s = MID
     w = synth.gen_weights(s, seed=6)
     B, T = 2, 90  # 89 positions in chunks of 32, 32, 25, then the last

@@ -82,3 +82,37 @@ def test_failed_call_raises_status_error(lib):
     with pytest.raises(capi.PipoError) as e:
         capi.pipo_op_gemv(1, 0, 16, 10, 12, 16, 1, 16, 0)  # K not a multiple of 8
     assert e.value.status == capi.PIPO_EINVAL
+
+
+def test_every_context_entry_point_rejects_a_null_context(lib):
+    """Status, not a crash: each entry point that takes a context returns
+    EINVAL for NULL (before any CUDA call), with a message."""
+    capi.load()
+    L = capi.load()
+    null = None
+    ib = (C.c_int32 * 4)()
+    fb = (C.c_float * 4)()
+    calls = {
+        "pipo_prefill": lambda: L.pipo_prefill(null, 1, ib, 1, ib, ib, ib),
+        "pipo_regular_prefill": lambda: L.pipo_regular_prefill(null, 1, ib, 1, ib, ib, ib),
+        "pipo_decode_step": lambda: L.pipo_decode_step(null, None, None),
+        "pipo_decode_step_async": lambda: L.pipo_decode_step_async(null, None, None),
+        "pipo_regular_step": lambda: L.pipo_regular_step(null, None),
+        "pipo_regular_step_async": lambda: L.pipo_regular_step_async(null, None),
+        "pipo_rollback": lambda: L.pipo_rollback(null, ib),
+        "pipo_set_threshold": lambda: L.pipo_set_threshold(null, 0.5, 0),
+        "pipo_set_sampler": lambda: L.pipo_set_sampler(null, 1.0, 20, 0.95, 1.5, fb, 1),
+        "pipo_set_pending": lambda: L.pipo_set_pending(null, ib),
+        "pipo_get_counters": lambda: L.pipo_get_counters(null, None, None),
+        "pipo_debug_dump": lambda: L.pipo_debug_dump(null, C.byref(capi.pipo_debug())),
+        "pipo_read_cache": lambda: L.pipo_read_cache(null, 0, 0, 1, fb, fb),
+        "pipo_load_cache": lambda: L.pipo_load_cache(null, 0, 1, fb, fb),
+        "pipo_set_stream": lambda: L.pipo_set_stream(null, None),
+        "pipo_describe_step": lambda: L.pipo_describe_step(null, C.create_string_buffer(8), 8),
+        "pipo_profile_step": lambda: L.pipo_profile_step(null, 0, None, None, None, ib),
+    }
+    for name, call in calls.items():
+        assert call() == capi.PIPO_EINVAL, name
+        assert capi.pipo_last_error(None), name
+    assert L.pipo_step_launches(null) == 0
+    L.pipo_free(null)  # a no-op

@@ -136,6 +136,21 @@ PIPO_API pipo_status pipo_init(const pipo_config *cfg, const pipo_weights *w, pi
 PIPO_API pipo_status pipo_prefill(pipo_ctx *ctx, int32_t batch, const int32_t *h_ids, int32_t stride,
                          const int32_t *h_lens, int32_t *h_tokens, int32_t *h_n_accepted);
 
+/* Continuous batching: prefill one slot (sequence `slot` < max_batch) from
+ * the host prompt h_ids[0, len) while every other slot keeps its state (its
+ * cache, length, pending pair and counters), e.g. a request joining a batch
+ * that is decoding.  The prompt is paired as in pipo_prefill; (len + 1) / 2
+ * <= max_ctx entries.  Outputs (host, may be NULL): h_tokens[2] and
+ * h_n_accepted[1] of the slot's first pair.  The decode steps then run slots
+ * 0 .. max(slot, previous batch - 1); a slot that was never prefilled decodes
+ * from token 0 on an empty cache (its outputs mean nothing).  Slots of one
+ * batch may hold prompts of different lengths.  ESTATE after a
+ * regular-decoding prefill; EINVAL for a bad slot, length or id;
+ * ECAPACITY as pipo_prefill.  On failure the slot's state is undefined and
+ * the other slots are unchanged. */
+PIPO_API pipo_status pipo_prefill_slot(pipo_ctx *ctx, int32_t slot, const int32_t *h_ids, int32_t len,
+                                       int32_t *h_tokens, int32_t *h_n_accepted);
+
 /* One pair-decode step of every prefilled sequence: compress the pending
  * pair, one backbone pass, both heads, the confidence rule, next pair, KV
  * append.  Host outputs (may be NULL): h_tokens[B,2] = (x_b, x_d or -1 when

@@ -71,6 +71,7 @@ class pipo_debug(C.Structure):
 SIGNATURES = {
     "pipo_init": (C.c_int, [C.POINTER(pipo_config), C.POINTER(pipo_weights), C.POINTER(C.c_void_p)]),
     "pipo_prefill": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.c_int32, _IP, _IP, _IP]),
+    "pipo_prefill_slot": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.c_int32, _IP, _IP]),
     "pipo_decode_step": (C.c_int, [C.c_void_p, _IP, _IP]),
     "pipo_decode_step_async": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "pipo_regular_prefill": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.c_int32, _IP, _IP, _IP]),
@@ -156,6 +157,14 @@ def pipo_prefill(ctx, ids: np.ndarray, lens: Optional[np.ndarray] = None):
     tok = np.zeros((B, 2), np.int32)
     nacc = np.zeros(B, np.int32)
     _check(load().pipo_prefill(ctx, B, _ip(ids), stride, _ip(lens), _ip(tok), _ip(nacc)), ctx)
+    return tok, nacc
+
+
+def pipo_prefill_slot(ctx, slot: int, ids: np.ndarray):
+    ids = _i32(np.asarray(ids).reshape(-1))
+    tok = np.zeros((1, 2), np.int32)
+    nacc = np.zeros(1, np.int32)
+    _check(load().pipo_prefill_slot(ctx, int(slot), _ip(ids), ids.size, _ip(tok), _ip(nacc)), ctx)
     return tok, nacc
 
 
@@ -361,6 +370,13 @@ class Pipo:
         ids = _i32(ids)
         self.B = ids.shape[0]
         return pipo_prefill(self.ctx, ids, lens)
+
+    def prefill_slot(self, slot, ids):
+        """Prefill one slot while the others keep their state (continuous
+        batching); the steps then cover slots 0 .. max(slot, B - 1)."""
+        out = pipo_prefill_slot(self.ctx, slot, ids)
+        self.B = max(self.B, int(slot) + 1)
+        return out
 
     def step(self):
         return pipo_decode_step(self.ctx, self.B)

@@ -1701,6 +1701,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         TRY(dalloc(ctx, &ctx->emitted, (size_t)MB * 8));
         CK(cudaMemset(ctx->n_pos, 0, (size_t)MB * 4));
         CK(cudaMemset(ctx->emitted, 0, (size_t)MB * 8));
+        CK(cudaMemset(ctx->pending, 0, (size_t)MB * 2 * 4));  // a slot never prefilled holds valid ids
         if (c.debug) {
             TRY(dalloc(ctx, &ctx->dbg_lb, (size_t)MB * V * 4));
             TRY(dalloc(ctx, &ctx->dbg_ld, (size_t)MB * V * 4));
@@ -1888,6 +1889,79 @@ pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int
     ctx->h_len.assign(batch, N);
     ctx->prefilled = true;
     return check_device_error(ctx);
+}
+
+}  // extern "C"
+
+namespace {
+
+// The per-sequence device state of one slot as a batch of one: every
+// per-sequence buffer starts at the slot (the activation and prompt buffers
+// are scratch shared by all slots).  Restored on destruction.
+struct SlotView {
+    pipo_ctx* c;
+    int32_t *n_pos, *pending, *out_tokens, *out_nacc, *block_table, *dbg_xb, *dbg_xd;
+    long long* emitted;
+    float *dbg_lb, *dbg_ld, *dbg_conf, *dbg_hb, *dbg_hd, *samp_u;
+    uint32_t* presence;
+    SlotView(pipo_ctx* ctx, int s) : c(ctx) {
+        const size_t V = ctx->cfg.vocab, H = ctx->cfg.hidden;
+        n_pos = ctx->n_pos; pending = ctx->pending; out_tokens = ctx->out_tokens; out_nacc = ctx->out_nacc;
+        block_table = ctx->block_table; dbg_xb = ctx->dbg_xb; dbg_xd = ctx->dbg_xd; emitted = ctx->emitted;
+        dbg_lb = ctx->dbg_lb; dbg_ld = ctx->dbg_ld; dbg_conf = ctx->dbg_conf; dbg_hb = ctx->dbg_hb;
+        dbg_hd = ctx->dbg_hd; samp_u = ctx->samp_u; presence = ctx->presence;
+        ctx->n_pos += s; ctx->pending += 2 * s; ctx->out_tokens += 2 * s; ctx->out_nacc += s; ctx->emitted += s;
+        ctx->block_table += (size_t)s * ctx->blocks_per_seq;
+        if (ctx->dbg_lb) {
+            ctx->dbg_lb += s * V; ctx->dbg_ld += s * V; ctx->dbg_conf += s; ctx->dbg_hb += s * H;
+            ctx->dbg_hd += s * H; ctx->dbg_xb += s; ctx->dbg_xd += s;
+        }
+        if (ctx->samp_u) ctx->samp_u += 2 * s;
+        if (ctx->presence) ctx->presence += (size_t)s * ctx->presence_w;
+    }
+    ~SlotView() {
+        c->n_pos = n_pos; c->pending = pending; c->out_tokens = out_tokens; c->out_nacc = out_nacc;
+        c->block_table = block_table; c->dbg_xb = dbg_xb; c->dbg_xd = dbg_xd; c->emitted = emitted;
+        c->dbg_lb = dbg_lb; c->dbg_ld = dbg_ld; c->dbg_conf = dbg_conf; c->dbg_hb = dbg_hb; c->dbg_hd = dbg_hd;
+        c->samp_u = samp_u; c->presence = presence;
+    }
+};
+
+}  // namespace
+
+extern "C" {
+
+pipo_status pipo_prefill_slot(pipo_ctx* ctx, int32_t slot, const int32_t* h_ids, int32_t len, int32_t* h_tokens,
+                              int32_t* h_n_accepted) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    if (slot < 0 || slot >= ctx->cfg.max_batch || !h_ids || len < 1)
+        return fail(ctx, PIPO_EINVAL, "bad slot prefill arguments (slot %d of %d, length %d)", slot,
+                    ctx->cfg.max_batch, len);
+    if (ctx->prefilled && ctx->regular) return fail(ctx, PIPO_ESTATE, "slot prefill after a regular-decoding prefill");
+    const bool was = ctx->prefilled;
+    const int B_old = was ? ctx->B : 0;
+    const std::vector<int32_t> len_old = was ? ctx->h_len : std::vector<int32_t>();
+    pipo_status st;
+    {
+        SlotView view(ctx, slot);
+        int32_t one = len;
+        st = pipo_prefill(ctx, 1, h_ids, len, &one, h_tokens, h_n_accepted);
+    }
+    if (st != PIPO_OK) {  // this slot's state is undefined; the other slots are untouched
+        ctx->B = B_old;
+        ctx->h_len = len_old;
+        ctx->prefilled = was;
+        if (ctx->B == 0) ctx->prefilled = false;
+        return st;
+    }
+    std::vector<int32_t> lens = len_old;
+    lens.resize(std::max(B_old, slot + 1), 0);
+    lens[slot] = (len + 1) / 2;
+    ctx->B = (int)lens.size();
+    ctx->h_len = lens;
+    ctx->prefilled = true;
+    ctx->regular = false;
+    return PIPO_OK;
 }
 
 pipo_status pipo_regular_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride,

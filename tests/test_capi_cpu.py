@@ -95,6 +95,7 @@ def test_every_context_entry_point_rejects_a_null_context(lib):
     calls = {
         "pipo_prefill": lambda: L.pipo_prefill(null, 1, ib, 1, ib, ib, ib),
         "pipo_regular_prefill": lambda: L.pipo_regular_prefill(null, 1, ib, 1, ib, ib, ib),
+        "pipo_prefill_slot": lambda: L.pipo_prefill_slot(null, 0, ib, 1, ib, ib),
         "pipo_decode_step": lambda: L.pipo_decode_step(null, None, None),
         "pipo_decode_step_async": lambda: L.pipo_decode_step_async(null, None, None),
         "pipo_regular_step": lambda: L.pipo_regular_step(null, None),

@@ -72,6 +72,8 @@ typedef struct {
     int32_t debug;       /* 1: keep logits and head states for pipo_debug_dump */
     uint32_t page_shuffle_seed; /* 0: blocks in order; else a seeded permutation of
                                    the physical block pool (layout must not matter) */
+    int32_t comp_residual; /* 1: the MLP compressor adds a + b, z = a + b + W2 SiLU(W1[a;b])
+                              (its residual form, App. A.1); requires compressor = 1 */
 } pipo_config;
 
 /* Weights: one pointer per tensor, element type per pipo_config.dtype

@@ -37,7 +37,7 @@ def build(force: bool = False) -> str:
 class OrcConfig(C.Structure):
     _fields_ = [(n, C.c_int) for n in ("H", "L", "n_q", "n_kv", "d_h", "F", "V",
                                         "compressor", "mtp_block", "wdtype", "kv_bf16")] + \
-               [("rope_theta", C.c_double), ("eps", C.c_double), ("max_ctx", C.c_int)]
+               [("rope_theta", C.c_double), ("eps", C.c_double), ("max_ctx", C.c_int), ("comp_residual", C.c_int)]
 
 
 _WNAMES = [
@@ -144,7 +144,7 @@ class Model:
         kvb = wd if kv_bf16 is None else int(kv_bf16)
         self.cfg = OrcConfig(shape.H, shape.L, shape.n_q, shape.n_kv, shape.d_h, shape.F, shape.V,
                              0 if shape.compressor == "linear" else 1, shape.mtp_block, wd, kvb,
-                             shape.rope_theta, shape.eps, max_ctx)
+                             shape.rope_theta, shape.eps, max_ctx, int(shape.comp_residual))
         self._keep = {}
         self.w = OrcWeights()
         for f, name in _WNAMES:

@@ -8,7 +8,9 @@
  * What it computes (per sequence; notation of paper Sec. 3):
  *   Eq. 1      z^i   = f_theta([x^{2i}; x^{2i+1}])          compressor
  *              Linear variant  W [a;b] + b,  MLP variant  W2 SiLU(W1 [a;b])
- *              (App. A.1, Table "Compressor variants")
+ *              (App. A.1, Table "Compressor variants"); optionally the MLP
+ *              with the residual a + b added (comp_residual), the form whose
+ *              zeroed branch gives a + b
  *   Eq. 2      h_b^i = Backbone(z^{<=i})                     decoder stack
  *   Eq. 3      p_b   = LMHead(h_b^i)                          tied to E (App. B.2)
  *   Eq. 4      h_d^i = MTPHead(h_b^i, x^{2i+2})
@@ -57,6 +59,7 @@ typedef struct {
     int kv_bf16;    /* round cached K,V to bf16 */
     double rope_theta, eps;
     int max_ctx;    /* cache entries per sequence */
+    int comp_residual; /* 1: the MLP compressor adds a + b (the residual form of App. A.1) */
 } orc_config;
 
 /* Host pointers; element type per wdtype; matrices row-major [out, in]. */
@@ -307,6 +310,8 @@ void orc_compress(const orc_config *c, const orc_weights *w, int t0, int t1, dou
         orc_matvec(w->comp_W1, 0, dt, H, 2 * H, ab, t);
         for (int i = 0; i < H; i++) t[i] = orc_silu(t[i]);
         orc_matvec(w->comp_W2, 0, dt, H, H, t, z);
+        if (c->comp_residual)
+            for (int i = 0; i < H; i++) z[i] += ab[i] + ab[H + i];
         free(t);
     }
     free(ab);

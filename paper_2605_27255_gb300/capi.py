@@ -36,7 +36,7 @@ class pipo_config(C.Structure):
                [("rope_theta", C.c_float), ("rms_eps", C.c_float)] + \
                [(n, C.c_int32) for n in ("max_batch", "max_ctx", "page_size")] + \
                [("tau", C.c_float), ("force_mode", C.c_int32), ("debug", C.c_int32),
-                ("page_shuffle_seed", C.c_uint32)]
+                ("page_shuffle_seed", C.c_uint32), ("comp_residual", C.c_int32)]
 
 
 # C field -> tensor name of synth.tensor_shapes
@@ -321,7 +321,8 @@ def make_config(s: ModelShape, max_batch: int, max_ctx: int, *, tau: Optional[fl
                 page_shuffle_seed: int = 0) -> pipo_config:
     return pipo_config(s.H, s.L, s.n_q, s.n_kv, s.d_h, s.F, s.V, 0 if s.compressor == "linear" else 1,
                        s.mtp_block, 1 if s.dtype == "bf16" else 0, s.rope_theta, s.eps, max_batch, max_ctx,
-                       page_size, s.tau if tau is None else tau, force_mode, int(debug), page_shuffle_seed)
+                       page_size, s.tau if tau is None else tau, force_mode, int(debug), page_shuffle_seed,
+                       int(s.comp_residual))
 
 
 def make_weights(weights: Dict[str, torch.Tensor], keep: list) -> pipo_weights:

@@ -588,6 +588,24 @@ __global__ void advance_kernel(int32_t* n_pos, int B, int by) {
     if (b < B) n_pos[b] += by;
 }
 
+// The residual term of the residual MLP compressor (App. A.1): x[r] = a + b,
+// the two slot embeddings of pair r (E rows, x_pad for PAD = -1); the W2
+// projection then adds W2 SiLU(W1 [a;b]).  An id outside [-1, V) (never
+// produced: the host validates ids) contributes zeros.  grid rows, any block.
+template <typename T>
+__global__ void pair_sum_kernel(const void* E, const void* pad, const int32_t* tok, int tok_ld, int V, int H,
+                                float* x) {
+    pdl_launch();
+    pdl_wait();
+    const int r = blockIdx.x;
+    const int t0 = tok[(size_t)r * tok_ld], t1 = tok[(size_t)r * tok_ld + 1];
+    for (int k = threadIdx.x; k < H; k += blockDim.x) {
+        const float a = t0 < 0 ? ldw<T>(pad, k) : t0 < V ? ldw<T>(E, (size_t)t0 * H + k) : 0.f;
+        const float b = t1 < 0 ? ldw<T>(pad, k) : t1 < V ? ldw<T>(E, (size_t)t1 * H + k) : 0.f;
+        x[(size_t)r * H + k] = a + b;
+    }
+}
+
 // Regular decoding (the paper's baseline, Sec. 4): the backbone input is the
 // token's own embedding, x[b] = E[tok[b * ld]], with no compressor.  Also
 // zeroes the argmax keys of the step.  An id outside [0, V) (never produced:

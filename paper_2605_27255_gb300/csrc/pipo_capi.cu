@@ -1087,6 +1087,18 @@ pipo_status enqueue_lm_head(pipo_ctx* ctx, const float* h, const void* gamma, un
     return launch_gemv(ctx, p);
 }
 
+// x = a + b of every row's pair (the residual MLP compressor's residual term).
+pipo_status enqueue_pair_sum(pipo_ctx* ctx, const int32_t* pairs, int rows) {
+    const pipo_config& c = ctx->cfg;
+    const void* E = ctx->E;
+    const void* pad = ctx->x_pad;
+    int ld = 2, V = c.vocab, H = c.hidden;
+    float* x = ctx->x;
+    void* args[] = {(void*)&E, (void*)&pad, (void*)&pairs, &ld, &V, &H, &x};
+    return launch_ex(ctx, c.dtype == 1 ? (const void*)&pair_sum_kernel<bf16> : (const void*)&pair_sum_kernel<float>,
+                     dim3(rows), dim3(256), 0, args);
+}
+
 // The evaluation sampler on one head's logits (sample_kernel): the pick
 // replaces the head's argmax key; the backbone head's pick joins the history.
 pipo_status enqueue_sample(pipo_ctx* ctx, const float* logits, int head, unsigned long long* am) {
@@ -1138,7 +1150,8 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
     if (mode != PREFILL_MID) { p.zero_ptr = ctx->am; p.zero_n = 2 * c.max_batch; }
     TRY(launch_gemv(ctx, p));
     if (c.compressor == 1) {
-        p = gemv_base(ctx, ctx->comp_W2, H, EPI_STORE, ctx->x, H);
+        if (c.comp_residual) TRY(enqueue_pair_sum(ctx, pairs, B));
+        p = gemv_base(ctx, ctx->comp_W2, H, c.comp_residual ? EPI_RESADD : EPI_STORE, ctx->x, H);
         p.seg[0] = act_seg(ctx->t, H, H);
         p.K = H;
         TRY(launch_gemv(ctx, p));
@@ -1302,7 +1315,8 @@ pipo_status enqueue_prefill_chunk(pipo_ctx* ctx, bool regular, int j0, int C) {
         p.seg[0] = s0; p.seg[1] = s1; p.nseg = 2; p.K = 2 * H;
         TRY(launch_gemv(ctx, p));
         if (c.compressor == 1) {
-            p = gemv_base(ctx, ctx->comp_W2, H, EPI_STORE, ctx->x, H);
+            if (c.comp_residual) TRY(enqueue_pair_sum(ctx, s0.tok, R));
+            p = gemv_base(ctx, ctx->comp_W2, H, c.comp_residual ? EPI_RESADD : EPI_STORE, ctx->x, H);
             p.seg[0] = act_seg(ctx->t, H, H);
             p.K = H;
             TRY(launch_gemv(ctx, p));
@@ -1367,7 +1381,7 @@ void* mk_pick(bool bf, int nb, int DH, int G) {
 // (or prepare) the persistent step kernel.  Returns false when it does not fit.
 pipo_status try_step_kernel(pipo_ctx* ctx, bool& used) {
     used = false;
-    if (!ctx->use_mk || ctx->B > 4) return PIPO_OK;
+    if (!ctx->use_mk || ctx->B > 4 || ctx->cfg.comp_residual) return PIPO_OK;
     const pipo_config& c = ctx->cfg;
     const int nb = ctx->B <= 1 ? 1 : ctx->B <= 2 ? 2 : 4;
     void* fn = mk_pick(c.dtype == 1, nb, c.head_dim, c.n_q_heads / c.n_kv_heads);
@@ -1552,7 +1566,8 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
     if (c.hidden <= 0 || c.hidden % 8 || c.n_layers < 0 || c.n_q_heads <= 0 || c.n_kv_heads <= 0 ||
         c.n_q_heads % c.n_kv_heads || c.ffn <= 0 || c.ffn % 8 || c.vocab <= 0 || c.max_batch <= 0 ||
         c.max_ctx <= 0 || c.page_size <= 0 || (c.dtype != 0 && c.dtype != 1) ||
-        (c.compressor != 0 && c.compressor != 1) || (c.mtp_block != 0 && c.mtp_block != 1))
+        (c.compressor != 0 && c.compressor != 1) || (c.mtp_block != 0 && c.mtp_block != 1) ||
+        (c.comp_residual != 0 && c.comp_residual != 1) || (c.comp_residual && c.compressor != 1))
         return fail(nullptr, PIPO_EINVAL, "invalid config");
     if (c.head_dim != 64 && c.head_dim != 128) return fail(nullptr, PIPO_EINVAL, "head_dim must be 64 or 128");
     const int G = c.n_q_heads / c.n_kv_heads;

@@ -55,6 +55,7 @@ class ModelShape:
     eps: float = 1.0e-6
     tau: float = 0.5
     std: float = 0.02
+    comp_residual: int = 0    # 1: the MLP compressor adds a + b (the residual form)
 
     @property
     def qkv_rows(self) -> int:

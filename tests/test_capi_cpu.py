@@ -117,3 +117,22 @@ def test_every_context_entry_point_rejects_a_null_context(lib):
         assert capi.pipo_last_error(None), name
     assert L.pipo_step_launches(null) == 0
     L.pipo_free(null)  # a no-op
+
+
+def test_residual_compressor_needs_the_mlp_variant(lib):
+    """comp_residual is the residual form of the MLP compressor: with the
+    Linear variant the config is invalid (checked before any CUDA call)."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    from paper_2605_27255_gb300 import synth
+    L = capi.load()
+    w = capi.pipo_weights()
+    ctx = C.c_void_p()
+    cfg = capi.make_config(synth.TINY.with_(comp_residual=1), 1, 16)  # Tiny: Linear compressor
+    assert L.pipo_init(C.byref(cfg), C.byref(w), C.byref(ctx)) == capi.PIPO_EINVAL
+    assert "invalid config" in capi.pipo_last_error(None)
+    cfg = capi.make_config(synth.TINY.with_(compressor="mlp", comp_residual=1), 1, 16)
+    rc = L.pipo_init(C.byref(cfg), C.byref(w), C.byref(ctx))
+    assert "invalid config" not in capi.pipo_last_error(None) and not ctx.value  # fails later: no GPU
+    assert rc != capi.PIPO_OK

@@ -196,6 +196,28 @@ def test_compressor_mlp_closed_form():
     assert np.all(O.compress(m, 0, 0) == 0)
 
 
+def test_compressor_residual_form():
+    """The residual MLP compressor (comp_residual): z = a + b + W2 SiLU(W1 [a;b]).
+    With the branch zeroed (W2 = 0) it is exactly a + b, the paper's
+    initial state of the compressor; otherwise it differs from the literal MLP
+    by exactly a + b; a PAD slot contributes x_pad."""
+    s = small_shape(compressor="mlp", V=16, comp_residual=1)
+    w = zero_model(s)
+    rng = torch.Generator().manual_seed(3)
+    w["E"] = torch.randn(s.V, s.H, generator=rng)
+    w["x_pad"] = torch.randn(s.H, generator=rng)
+    w["comp.W1"] = torch.randn(s.H, 2 * s.H, generator=rng)
+    m = O.Model(s, w)
+    a, b, pad = (w["E"][5].double().numpy(), w["E"][9].double().numpy(), w["x_pad"].double().numpy())
+    assert np.array_equal(O.compress(m, 5, 9), a + b)
+    assert np.array_equal(O.compress(m, 5, -1), a + pad)
+    w["comp.W2"] = torch.randn(s.H, s.H, generator=rng)
+    res = O.compress(O.Model(s, w), 5, 9)
+    lit = O.compress(O.Model(s.with_(comp_residual=0), w), 5, 9)
+    assert np.allclose(res - lit, a + b, rtol=0, atol=1e-12)
+    assert not np.allclose(lit, a + b)
+
+
 def test_onehot_model_closed_form_tokens_and_acceptance():
     """With E = I, a [I I] compressor and identity blocks, h_b = e_t0 + e_t1,
     so the LM head's argmax is min(t0, t1) (a tie, lowest index wins); the MTP

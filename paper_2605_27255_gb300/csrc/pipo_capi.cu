@@ -1774,6 +1774,9 @@ pipo_status pipo_set_sampler(pipo_ctx* ctx, float temperature, int32_t top_k, fl
         if (!(h_u[i] >= 0.f && h_u[i] < 1.f)) return fail(ctx, PIPO_EINVAL, "draw %zu not in [0, 1)", i);
     CK(cudaSetDevice(ctx->dev));
     CK(cudaStreamSynchronize(ctx->stream));
+    // off until the buffers below are in place (a failed call leaves the sampler off)
+    if (ctx->samp_on) drop_graph(ctx);
+    ctx->samp_on = false;
     if (!ctx->samp_logits) {
         ctx->presence_w = (c.vocab + 31) / 32;
         TRY(dalloc(ctx, &ctx->samp_logits, (size_t)2 * c.max_batch * c.vocab * 4));

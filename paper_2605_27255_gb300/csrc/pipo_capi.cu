@@ -99,6 +99,7 @@ struct pipo_ctx {
     bool attn_regs = false;           // register-ring attention instead of the tensor-core one
     std::vector<CUtensorMap> kv_tm;   // tensor-core attention: K and V tensor map of every cache layer
     bool gemv_tma = false;            // bulk-copy GEMV (else the register-ring GEMV)
+    int gemv_l2_prefetch = 0;         // streaming GEMV: weight chunks per warp hinted into L2 before the wait
     // persistent step kernel: phases recorded from the enqueue code
     std::vector<Phase>* rec = nullptr;  // recording target (nullptr: launch kernels)
     bool rec_ok = true;                 // every recorded phase fits the step kernel
@@ -730,6 +731,7 @@ GemvParams gemv_base(pipo_ctx* ctx, const void* W, int N, int epi, float* y, int
     GemvParams p{};
     p.W = W; p.N = N; p.epi = epi; p.y = y; p.ldy = ldy;
     p.B = ctx->rows > 0 ? ctx->rows : ctx->B; p.splitk = 1; p.eps = ctx->cfg.rms_eps; p.nseg = 1;
+    p.l2_prefetch = ctx->gemv_l2_prefetch;
     return p;
 }
 
@@ -1666,6 +1668,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         }
         if (const char* ev = getenv("PIPO_ATTN_CS_TARGET")) ctx->attn_cs_target = std::max(1, atoi(ev));
         if (const char* ev = getenv("PIPO_GEMV_TMA")) ctx->gemv_tma = ev[0] == '1';
+        if (const char* ev = getenv("PIPO_GEMV_L2_PREFETCH")) ctx->gemv_l2_prefetch = std::max(0, atoi(ev));
         if (const char* ev = getenv("PIPO_STEP_KERNEL")) ctx->use_mk = ev[0] == '1';
         TRY(dalloc(ctx, &ctx->bar_ctr, 64));
         CK(cudaMemset(ctx->bar_ctr, 0, 64));

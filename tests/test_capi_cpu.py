@@ -136,3 +136,33 @@ def test_residual_compressor_needs_the_mlp_variant(lib):
     rc = L.pipo_init(C.byref(cfg), C.byref(w), C.byref(ctx))
     assert "invalid config" not in capi.pipo_last_error(None) and not ctx.value  # fails later: no GPU
     assert rc != capi.PIPO_OK
+
+
+C_PROGRAM = os.path.join(ROOT, "tests", "c", "pipo_c_api.c")
+
+
+def build_c_program(lib_path):
+    """Compile the C99 user program against include/pipo.h and the library
+    (the binary goes next to the library, a build output)."""
+    import subprocess
+    exe = os.path.join(os.path.dirname(lib_path), "pipo_c_api")
+    libdir = os.path.dirname(lib_path)
+    subprocess.check_call(["gcc", "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I",
+                           os.path.join(ROOT, "include"), C_PROGRAM, "-o", exe, "-L", libdir, "-lpipo",
+                           "-Wl,-rpath," + libdir])
+    return exe
+
+
+def test_header_is_c99_and_a_c_program_links_and_fails_cleanly_without_a_device(lib):
+    """The boundary is usable from C alone: the header compiles as strict C99,
+    the program links against the library, and without a device pipo_init
+    returns a status that the program reports (exit 2), no crash."""
+    import subprocess
+
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    exe = build_c_program(build.build())
+    r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
+    assert r.returncode == 2, (r.returncode, r.stdout, r.stderr)
+    assert "pipo_init: status" in r.stdout

@@ -1,6 +1,9 @@
-"""Builds ``lib/libpipo.so`` (the C-ABI library) for sm_103a with nvcc."""
+"""Builds ``lib/libpipo.so`` (the C-ABI library) for sm_103a with nvcc: the
+host code and the kernel families are separate translation units, compiled
+in parallel and linked into one shared library."""
 from __future__ import annotations
 
+import concurrent.futures
 import hashlib
 import os
 import subprocess
@@ -12,7 +15,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "lib")
 LIB = os.path.join(LIBDIR, "libpipo.so")
-SOURCES = ["pipo_capi.cu"]
+# the host code first (the longest units start first)
+SOURCES = ["k_gemv_bf16.cu", "k_gemv_f32.cu", "k_attn.cu", "pipo_capi.cu", "k_mk.cu", "k_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -43,13 +47,27 @@ def build(force: bool = False, verbose: bool = False) -> str:
     dig = _digest()
     if not force and os.path.exists(LIB) and os.path.exists(stamp) and open(stamp).read() == dig:
         return LIB
-    tmp = LIB + f".tmp{os.getpid()}"
-    cmd = [nvcc(), "-O3", "-std=c++17", "-lineinfo", *ARCH, "-shared", "-Xcompiler", "-fPIC,-fvisibility=hidden",
-           "-I", INCLUDE, "-I", CSRC, "-o", tmp] + [os.path.join(CSRC, s) for s in SOURCES]
-    if verbose:
-        cmd.insert(1, "-Xptxas=-v")
-        print(" ".join(cmd), file=sys.stderr)
-    subprocess.check_call(cmd)
+    tag = f".tmp{os.getpid()}"
+    flags = ["-O3", "-std=c++17", "-lineinfo", *ARCH, "-Xcompiler", "-fPIC,-fvisibility=hidden",
+             "-I", INCLUDE, "-I", CSRC] + (["-Xptxas=-v"] if verbose else [])
+
+    def compile_unit(src: str) -> str:
+        obj = os.path.join(LIBDIR, os.path.splitext(src)[0] + tag + ".o")
+        cmd = [nvcc(), *flags, "-c", os.path.join(CSRC, src), "-o", obj]
+        if verbose:
+            print(" ".join(cmd), file=sys.stderr)
+        subprocess.check_call(cmd)
+        return obj
+
+    with concurrent.futures.ThreadPoolExecutor(max_workers=min(len(SOURCES), os.cpu_count() or 1)) as pool:
+        objs = list(pool.map(compile_unit, SOURCES))
+    tmp = LIB + tag
+    try:
+        subprocess.check_call([nvcc(), *ARCH, "-shared", "-o", tmp, *objs])
+    finally:
+        for o in objs:
+            if os.path.exists(o):
+                os.remove(o)
     os.replace(tmp, LIB)
     with open(stamp, "w") as f:
         f.write(dig)

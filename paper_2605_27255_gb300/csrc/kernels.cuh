@@ -582,20 +582,6 @@ __global__ void accept_kernel(const float* __restrict__ t, const void* W2, int H
     if (st.samp_step && b == 0) st.samp_step[0] += 1;
 }
 
-// Packed argmax keys -> token ids.
-__global__ void keys_to_tokens_kernel(const unsigned long long* keys, int32_t* tokens, int B) {
-    const int b = blockIdx.x * blockDim.x + threadIdx.x;
-    if (b < B) tokens[b] = argmax_row(keys[b]);
-}
-
-// Prefill positions before the last: n[b] += by (the positions just run).
-__global__ void advance_kernel(int32_t* n_pos, int B, int by) {
-    pdl_launch();
-    pdl_wait();
-    const int b = blockIdx.x * blockDim.x + threadIdx.x;
-    if (b < B) n_pos[b] += by;
-}
-
 // The residual term of the residual MLP compressor (App. A.1): x[r] = a + b,
 // the two slot embeddings of pair r (E rows, x_pad for PAD = -1); the W2
 // projection then adds W2 SiLU(W1 [a;b]).  An id outside [-1, V) (never
@@ -631,27 +617,6 @@ __global__ void embed_kernel(const void* E, const int32_t* tok, int ld, int V, i
     const bool ok = t >= 0 && t < V;
     for (int k = threadIdx.x; k < H; k += blockDim.x)
         x[(size_t)b * H + k] = ok ? ldw<T>(E, (size_t)t * H + k) : 0.f;
-}
-
-// Regular decoding, end of a step: the LM-head argmax is the output token and
-// the next input (slot 1 stays PAD, nothing is drafted), one more cache entry,
-// one more emitted token.  grid B, any block size.
-__global__ void regular_accept_kernel(StepState st, int H, const float* h) {
-    pdl_launch();
-    pdl_wait();
-    const int b = blockIdx.x;
-    if (st.dbg_hb)
-        for (int k = threadIdx.x; k < H; k += blockDim.x) st.dbg_hb[(size_t)b * H + k] = h[(size_t)b * H + k];
-    if (threadIdx.x != 0) return;
-    const int xb = argmax_row(st.am_b[b]);
-    st.out_tokens[2 * b] = xb;
-    st.out_tokens[2 * b + 1] = -1;
-    st.out_nacc[b] = 0;
-    st.pending[2 * b] = xb;
-    st.pending[2 * b + 1] = -1;
-    st.n_pos[b] += 1;
-    st.emitted[b] += 1;
-    if (st.dbg_xb) st.dbg_xb[b] = xb;
 }
 
 }  // namespace pipo

@@ -20,12 +20,16 @@
 #include <numeric>
 #include <random>
 #include <string>
+#include <type_traits>
 #include <vector>
 
+// Kernel headers for their parameter structs and launch constants; the
+// kernels themselves are compiled in the k_*.cu units (kernel_tables.h).
 #include "attn_cluster.cuh"
 #include "attn_mma.cuh"
 #include "attn_prefill.cuh"
 #include "gemv_stream.cuh"
+#include "kernel_tables.h"
 #include "kernels.cuh"
 #include "megakernel.cuh"
 #include "pipo.h"
@@ -34,6 +38,46 @@
 
 using namespace pipo;
 using bf16 = __nv_bfloat16;
+
+namespace pipo {
+
+// Packed argmax keys -> token ids.
+__global__ void keys_to_tokens_kernel(const unsigned long long* keys, int32_t* tokens, int B) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b < B) tokens[b] = argmax_row(keys[b]);
+}
+
+// Prefill positions before the last: n[b] += by (the positions just run).
+__global__ void advance_kernel(int32_t* n_pos, int B, int by) {
+    pdl_launch();
+    pdl_wait();
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b < B) n_pos[b] += by;
+}
+
+
+// Regular decoding, end of a step: the LM-head argmax is the output token and
+// the next input (slot 1 stays PAD, nothing is drafted), one more cache entry,
+// one more emitted token.  grid B, any block size.
+__global__ void regular_accept_kernel(StepState st, int H, const float* h) {
+    pdl_launch();
+    pdl_wait();
+    const int b = blockIdx.x;
+    if (st.dbg_hb)
+        for (int k = threadIdx.x; k < H; k += blockDim.x) st.dbg_hb[(size_t)b * H + k] = h[(size_t)b * H + k];
+    if (threadIdx.x != 0) return;
+    const int xb = argmax_row(st.am_b[b]);
+    st.out_tokens[2 * b] = xb;
+    st.out_tokens[2 * b + 1] = -1;
+    st.out_nacc[b] = 0;
+    st.pending[2 * b] = xb;
+    st.pending[2 * b + 1] = -1;
+    st.n_pos[b] += 1;
+    st.emitted[b] += 1;
+    if (st.dbg_xb) st.dbg_xb[b] = xb;
+}
+
+}  // namespace pipo
 
 namespace {
 
@@ -227,22 +271,22 @@ int next_pow2_le8(int b) {
     return nb;
 }
 
-template <typename T, int NB, bool TWO>
-void* gemv_fn() { return reinterpret_cast<void*>(&gemv_kernel<T, NB, TWO>); }
-
+// launch handles of the GEMV kernels of weight type T (k_gemv_*.cu)
 template <typename T>
 void* pick_gemv(int nb, bool two) {
-    switch (nb) {
-        case 1: return two ? gemv_fn<T, 1, true>() : gemv_fn<T, 1, false>();
-        case 2: return two ? gemv_fn<T, 2, true>() : gemv_fn<T, 2, false>();
-        case 4: return two ? gemv_fn<T, 4, true>() : gemv_fn<T, 4, false>();
-        default: return two ? gemv_fn<T, 8, true>() : gemv_fn<T, 8, false>();
-    }
+    return std::is_same<T, bf16>::value ? k_pick_gemv_bf16(nb, two) : k_pick_gemv_f32(nb, two);
+}
+template <typename T>
+void* pick_tma(int nb, int ru) {
+    return std::is_same<T, bf16>::value ? k_pick_tma_bf16(nb, ru) : k_pick_tma_f32(nb, ru);
+}
+template <typename T>
+void* pick_stream(int nb, int ru, bool rows) {
+    return std::is_same<T, bf16>::value ? k_pick_stream_bf16(nb, ru, rows) : k_pick_stream_f32(nb, ru, rows);
 }
 
 constexpr size_t kXsBudget = 100 * 1024;      // staged-input bytes per v0 GEMV block
 constexpr size_t kStreamBudget = 200 * 1024;  // staged-input bytes per streaming GEMV block
-constexpr int kStreamDepth = 4;  // chunks per register batch (two batches in flight)
 
 // Launch with programmatic dependent launch (decode graph) and an optional
 // cluster dimension.
@@ -290,18 +334,6 @@ pipo_status launch_ex(pipo_ctx* ctx, const void* fn, dim3 grid, dim3 block, size
     return PIPO_OK;
 }
 
-template <typename T, int NB, int RU>
-void* tma_fn() { return reinterpret_cast<void*>(&gemv_tma_kernel<T, NB, RU>); }
-
-template <typename T>
-void* pick_tma(int nb, int ru) {
-    switch (nb) {
-        case 1: return ru == 2 ? tma_fn<T, 1, 2>() : tma_fn<T, 1, 1>();
-        case 2: return ru == 2 ? tma_fn<T, 2, 2>() : tma_fn<T, 2, 1>();
-        default: return ru == 2 ? tma_fn<T, 4, 2>() : tma_fn<T, 4, 1>();
-    }
-}
-
 size_t g_smem_optin = 0;  // opt-in shared memory per block of the device
 
 // Allow `fn` the largest dynamic shared memory the device permits next to its
@@ -314,62 +346,16 @@ size_t allow_max_smem(const void* fn) {
     return dyn;
 }
 
-template <typename T, int NB, int RU>
-void* stream_fn(bool rows) {
-    return rows ? reinterpret_cast<void*>(&gemv_rows_kernel<T, NB, RU, kStreamDepth>)
-                : reinterpret_cast<void*>(&gemv_stream_kernel<T, NB, RU, kStreamDepth>);
-}
-
-// rows: every weight row is a whole number of 512-byte chunks (fast kernel)
-template <typename T>
-void* pick_stream(int nb, int ru, bool rows) {
-    switch (nb) {
-        case 1: return ru == 2 ? stream_fn<T, 1, 2>(rows) : stream_fn<T, 1, 1>(rows);
-        case 2: return ru == 2 ? stream_fn<T, 2, 2>(rows) : stream_fn<T, 2, 1>(rows);
-        default: return ru == 2 ? stream_fn<T, 4, 2>(rows) : stream_fn<T, 4, 1>(rows);
-    }
-}
-
 // bh: batch columns of the tensor-core GEMM (its MMA N is 2 * bh: hi | lo)
 size_t tc_smem(int bh, bool deep = false) {
     const int st = tc_stages(bh, deep);
     return 1024 + (size_t)st * (kTcABytes + (size_t)2 * bh * kTcBK * 2) + (2 * st + 1) * 8;
 }
 
-template <int BH, bool DEEP>
-void* tc_fn() { return reinterpret_cast<void*>(&gemm_tc_kernel<BH, tc_stages(BH, DEEP)>); }
-
-template <bool DEEP>
-void* pick_tc_v(int bh) {
-    switch (bh) {
-        case 16: return tc_fn<16, DEEP>();
-        case 32: return tc_fn<32, DEEP>();
-        case 64: return tc_fn<64, DEEP>();
-        default: return tc_fn<128, DEEP>();
-    }
-}
-
-void* pick_tc(int bh, bool deep = false) { return deep ? pick_tc_v<true>(bh) : pick_tc_v<false>(bh); }
-
-template <int BH, bool DEEP>
-void* tcf_fn() { return reinterpret_cast<void*>(&gemm_tcf_kernel<BH, tcf_stages(BH, DEEP)>); }
-
-template <bool DEEP>
-void* pick_tcf_v(int bh) {
-    switch (bh) {
-        case 16: return tcf_fn<16, DEEP>();
-        case 32: return tcf_fn<32, DEEP>();
-        case 64: return tcf_fn<64, DEEP>();
-        default: return tcf_fn<128, DEEP>();
-    }
-}
-
-// kernel variants of the tensor-core projection: fused (activation split
-// inside the GEMM) or fed by prep_bf16_kernel; deep (one CTA per SM) or not
-void* pick_tcv(int bh, bool deep, bool fused) {
-    if (fused) return deep ? pick_tcf_v<true>(bh) : pick_tcf_v<false>(bh);
-    return pick_tc(bh, deep);
-}
+// kernel variants of the tensor-core projection (k_tc.cu): fused (activation
+// split inside the GEMM) or fed by prep_bf16_kernel; deep (one CTA per SM) or not
+void* pick_tc(int bh, bool deep = false) { return k_pick_tcv(bh, deep, false); }
+void* pick_tcv(int bh, bool deep, bool fused) { return k_pick_tcv(bh, deep, fused); }
 size_t tcv_smem(int bh, bool deep, bool fused) {
     if (!fused) return tc_smem(bh, deep);
     const int st = tcf_stages(bh, deep);
@@ -634,7 +620,7 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
         void* args[] = {&pp, &xb, &bh};
         ctx->prof_kind = 2;
         ctx->prof_bytes = 0.0;
-        TRY(launch_ex(ctx, reinterpret_cast<const void*>(&prep_bf16_kernel<bf16>), dim3(bn), dim3(kPrepThreads), 0,
+        TRY(launch_ex(ctx, reinterpret_cast<const void*>(k_pick_prep_bf16()), dim3(bn), dim3(kPrepThreads), 0,
                       args));
     }
     void* args[] = {&tmW, &tmX, &tp};
@@ -756,56 +742,12 @@ int attn_splits(const pipo_ctx* ctx, int B) {
     return s;
 }
 
-template <typename T, int DH, int G>
-void* attn_fn() { return reinterpret_cast<void*>(&attn_decode_kernel<T, DH, G>); }
-
-template <typename T, int DH>
-void* attn_pick_g(int G) {
-    switch (G) {
-        case 1: return attn_fn<T, DH, 1>();
-        case 2: return attn_fn<T, DH, 2>();
-        case 4: return attn_fn<T, DH, 4>();
-        case 8: return attn_fn<T, DH, 8>();
-        default: return nullptr;
-    }
-}
-
-void* attn_pick(bool bf, int DH, int G) {
-    if (DH == 64) return bf ? attn_pick_g<bf16, 64>(G) : attn_pick_g<float, 64>(G);
-    if (DH == 128) return bf ? attn_pick_g<bf16, 128>(G) : attn_pick_g<float, 128>(G);
-    return nullptr;
-}
-
-template <typename T, int DH, int G>
-void* attnc_fn() { return reinterpret_cast<void*>(&attn_cluster_kernel<T, DH, G>); }
-
-template <typename T, int DH>
-void* attnc_pick_g(int G) {
-    switch (G) {
-        case 1: return attnc_fn<T, DH, 1>();
-        case 2: return attnc_fn<T, DH, 2>();
-        case 4: return attnc_fn<T, DH, 4>();
-        case 8: return attnc_fn<T, DH, 8>();
-        default: return nullptr;
-    }
-}
-
+// attention launch handles (k_attn.cu)
+void* attn_pick(bool bf, int DH, int G) { return k_pick_attn_decode(bf, DH, G); }
 // one kernel for every cluster size (read from the cluster at run time)
-void* attnc_pick(bool bf, int DH, int G) {
-    if (DH == 64) return bf ? attnc_pick_g<bf16, 64>(G) : attnc_pick_g<float, 64>(G);
-    if (DH == 128) return bf ? attnc_pick_g<bf16, 128>(G) : attnc_pick_g<float, 128>(G);
-    return nullptr;
-}
-
+void* attnc_pick(bool bf, int DH, int G) { return k_pick_attn_cluster(bf, DH, G); }
 // tensor-core attention (bf16 cache, d_h = 128, 1, 2 or 4 query heads per kv head)
-void* attnm_pick(int G) {
-    switch (G) {
-        case 1: return reinterpret_cast<void*>(&attn_mma_kernel<1>);
-        case 2: return reinterpret_cast<void*>(&attn_mma_kernel<2>);
-        case 4: return reinterpret_cast<void*>(&attn_mma_kernel<4>);
-        default: return nullptr;
-    }
-}
+void* attnm_pick(int G) { return k_pick_attn_mma(G); }
 
 // Can a 16-CTA cluster of this kernel be scheduled here?  (sets the
 // non-portable cluster attribute; any failure selects 8)
@@ -834,11 +776,7 @@ bool cluster16_ok(bool bf, int DH, int G) {
     return n > 0;
 }
 
-void* rope_pick(bool bf, int DH) {
-    if (DH == 64) return bf ? (void*)&rope_append_kernel<bf16, 64> : (void*)&rope_append_kernel<float, 64>;
-    if (DH == 128) return bf ? (void*)&rope_append_kernel<bf16, 128> : (void*)&rope_append_kernel<float, 128>;
-    return nullptr;
-}
+void* rope_pick(bool bf, int DH) { return k_pick_rope_append(bf, DH); }
 
 KVView kv_view(pipo_ctx* ctx, int layer) {
     KVView v;
@@ -873,7 +811,7 @@ cudaError_t set_carveouts(bool bf) {
         for (int bn : {16, 32, 64, 128})
             for (bool deep : {false, true})
                 for (bool fused : {false, true}) fns.push_back(pick_tcv(bn, deep, fused));
-        fns.push_back(reinterpret_cast<const void*>(&prep_bf16_kernel<bf16>));
+        fns.push_back(reinterpret_cast<const void*>(k_pick_prep_bf16()));
         for (int g : {1, 2, 4}) fns.push_back(attnm_pick(g));
     }
     for (int dh : {64, 128}) {
@@ -989,8 +927,7 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
             const int32_t* np = ctx->n_pos;
             const float* rope = ctx->rope;
             void* args[] = {(void*)&qkv, &ld, &nq, &kv, (void*)&np, &nseq, (void*)&rope};
-            void* fn = DH == 64 ? (bf ? (void*)&append_rows_kernel<bf16, 64> : (void*)&append_rows_kernel<float, 64>)
-                                : (bf ? (void*)&append_rows_kernel<bf16, 128> : (void*)&append_rows_kernel<float, 128>);
+            void* fn = k_pick_append_rows(bf, DH);
             TRY(launch_ex(ctx, fn, dim3(R, c.n_kv_heads), dim3(DH / 2), 0, args));
         }
         ctx->prof_kind = 1;
@@ -1012,8 +949,7 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
         const int G = c.n_q_heads / c.n_kv_heads;
         if (chunk && ctx->prefill_tile_attn && attn_mma_ok(ctx) && (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers) {
             // causal tiles: the positions of a tile share every key and value they read
-            void* fn = G == 1 ? (void*)&attn_prefill_kernel<1> : G == 2 ? (void*)&attn_prefill_kernel<2>
-                                                                        : (void*)&attn_prefill_kernel<4>;
+            void* fn = k_pick_attn_prefill(G);
             CK(cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)prefill_attn_smem()));
             int C = R / ctx->B;
             const int TP = kPfVec / G;
@@ -1370,14 +1306,7 @@ void drop_graph(pipo_ctx* ctx) {
     ctx->graph_B = -1;
 }
 
-template <typename T, int NB, int DH, int G>
-void* mk_fn() { return reinterpret_cast<void*>(&step_kernel<T, NB, DH, G>); }
-
-void* mk_pick(bool bf, int nb, int DH, int G) {
-    if (bf && DH == 128 && G == 4) return nb == 1 ? mk_fn<bf16, 1, 128, 4>() : nb == 2 ? mk_fn<bf16, 2, 128, 4>() : mk_fn<bf16, 4, 128, 4>();
-    if (!bf && DH == 64 && G == 2) return nb == 1 ? mk_fn<float, 1, 64, 2>() : nb == 2 ? mk_fn<float, 2, 64, 2>() : mk_fn<float, 4, 64, 2>();
-    return nullptr;
-}
+void* mk_pick(bool bf, int nb, int DH, int G) { return k_pick_step_kernel(bf, nb, DH, G); }
 
 // Record the decode step as phases; when they all fit, upload them and capture
 // (or prepare) the persistent step kernel.  Returns false when it does not fit.
@@ -1524,16 +1453,22 @@ pipo_status ensure_cache_tmp(pipo_ctx* ctx, size_t elems) {
     return PIPO_OK;
 }
 
-// Read and clear the device error word (bounded waits that gave up).
+// Read and clear the device error words of every kernel unit (bounded waits
+// that gave up); the first unit with an error names the wait.
 pipo_status check_device_error(pipo_ctx* ctx) {
-    unsigned e = 0;
-    CK(cudaMemcpyFromSymbol(&e, g_pipo_error, sizeof(e)));
+    cudaError_t (*const units[])(unsigned*, unsigned*) = {
+        take_unit_error, k_take_error_gemv_bf16, k_take_error_gemv_f32, k_take_error_tc, k_take_error_attn,
+        k_take_error_mk};
+    unsigned e = 0, info[4] = {0, 0, 0, 0};
+    for (auto take : units) {
+        unsigned ue = 0, ui[4] = {0, 0, 0, 0};
+        CK(take(&ue, ui));
+        if (ue && !e) {
+            e = ue;
+            for (int i = 0; i < 4; ++i) info[i] = ui[i];
+        }
+    }
     if (!e) return PIPO_OK;
-    unsigned info[4] = {0, 0, 0, 0};
-    CK(cudaMemcpyFromSymbol(info, g_pipo_error_info, sizeof(info)));
-    const unsigned zero[4] = {0, 0, 0, 0};
-    CK(cudaMemcpyToSymbol(g_pipo_error, zero, sizeof(unsigned)));
-    CK(cudaMemcpyToSymbol(g_pipo_error_info, zero, sizeof(zero)));
     return fail(ctx, PIPO_ECUDA,
                 "device wait timed out (code %u; first at wait site %u, block %u, iteration %u, parity %u): "
                 "results of this step are invalid",

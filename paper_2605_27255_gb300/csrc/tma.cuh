@@ -13,15 +13,29 @@
 namespace pipo {
 
 // Device error word: 0 = fine; kErrWaitTimeout when a bounded wait gave up.
-__device__ unsigned int g_pipo_error;
+// One copy per translation unit (the kernels are compiled in several); the
+// host reads and clears every unit's copy after a step (take_unit_error).
+static __device__ unsigned int g_pipo_error;
 // First wait that gave up: {site code, linear block index, iteration, parity}
 // (the site codes name the wait: 11-14 projection GEMM producer-empty,
 // producer-drain, MMA-full, epilogue-accumulator; 21-23 attention
-// producer-empty, producer-drain, consumer-full; 31-32 bulk-copy GEMV;
-// 41-42 step kernel).
-__device__ unsigned int g_pipo_error_info[4];
+// producer-empty, producer-drain, consumer-full; 24-26 prefill attention;
+// 31-32 bulk-copy GEMV; 41-42 step kernel).
+static __device__ unsigned int g_pipo_error_info[4];
 constexpr unsigned kErrWaitTimeout = 1u;
 constexpr unsigned long long kWaitNs = 2000000000ull;  // give up after 2 s of waiting
+
+// Host: read and clear this translation unit's error word and wait record.
+static inline cudaError_t take_unit_error(unsigned* code, unsigned info[4]) {
+    cudaError_t e = cudaMemcpyFromSymbol(code, g_pipo_error, sizeof(unsigned));
+    if (e != cudaSuccess || *code == 0) return e;
+    e = cudaMemcpyFromSymbol(info, g_pipo_error_info, 4 * sizeof(unsigned));
+    if (e != cudaSuccess) return e;
+    const unsigned zero[4] = {0, 0, 0, 0};
+    e = cudaMemcpyToSymbol(g_pipo_error, zero, sizeof(unsigned));
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_pipo_error_info, zero, sizeof(zero));
+    return e;
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));

@@ -272,6 +272,63 @@ def run_regular(g, shape, wl, B, T, W, K, stream, seed):
                     "regular time per output token / pair-step time per output token (1 + acceptance tokens)"}
 
 
+def make_line(m: dict) -> dict:
+    """The benchmark's JSON line from the measured quantities of run_pipo
+    (device time over the timed steps, per-launch profile of the kernel
+    families, end-to-end loop, oracle baseline, clocks)."""
+    K, B, hbm = m["steps"], m["batch"], m["hbm"]
+    step_gbs = m["step_bytes"] / (m["ms"] / 1e3 / K) / 1e9
+    gb, gms, gn = m["kb"][0]
+    ab, ams, _ = m["kb"][1]
+    tot_ms = sum(v[1] for v in m["kb"].values())
+    gemv_gbs = gb / (gms / 1e3) / 1e9 if gms > 0 else None
+    acceptance = m["tokens"] / (K * B) - 1.0
+    line = {
+        "metric": METRIC, "value": m["tokens_all"] / (m["ms_all"] / 1e3), "unit": "tokens/s",
+        "n_gpus": m["n_gpus"], "steps": K, "warmup": m["warmup"], "ms_per_step": m["ms_all"] / K,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": m["dtype"], "data": "synthetic (seeded weights and prompts)",
+        "config": {"workload": m["workload"], "shape": m["shape_name"], "batch": B, "prompt_tokens": m["prompt_tokens"],
+                   "context_entries_avg": m["ctx_avg"], "tau": m["tau"], "force_mode": m["force"],
+                   "acceptance": acceptance, "pair_step_us": 1e3 * m["ms"] / K,
+                   "prefill_s": m["prefill_s"], "prefill_rows": m["prefill_rows"],
+                   "heads": "sampled (T 1, top-k 20, top-p 0.95, penalty 1.5)" if m["sampler"] else "greedy",
+                   "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
+                   "parallelism": f"replicas x{m['n_gpus']}"},
+        "roofline": {"bound": "hbm", "kernel": f"weight-streaming projections (every projection and both LM-head "
+                                                  f"launches of a step): {m['desc']}",
+                     "achieved": gemv_gbs, "peak": hbm, "unit": "GB/s",
+                     "frac": (gemv_gbs / hbm) if gemv_gbs else None, "traffic": None,
+                     "algorithmic_bytes_per_launch": gb / max(1, gn), "avg_launch_us": 1e3 * gms / max(1, gn),
+                     "launches_per_step": gn // max(1, m["prof_steps"]),
+                     "share_of_step_time": gms / tot_ms if tot_ms else None,
+                     "timing": f"CUDA events around each launch, {m['prof_steps']} eagerly run steps after the timed "
+                               f"region",
+                     "peak_source": f"{m['peak_source']} (MEASURED_PEAKS.json hbm_gbs)",
+                     "step": {"algorithmic_bytes": m["step_bytes"], "achieved": step_gbs, "frac": step_gbs / hbm,
+                              "frac_of_nominal": step_gbs / NOMINAL_HBM_GBS},
+                     "attention": {"achieved": (ab / (ams / 1e3) / 1e9) if ams else None,
+                                   "share_of_step_time": ams / tot_ms if tot_ms else None}},
+        "cpu_baseline": m["cpu"],
+        "e2e": {"value": m["e2e_tokens"] / m["e2e_s"], "unit": "tokens/s", "h2d_bytes_per_step": B * 8,
+                "d2h_bytes_per_step": B * 12,
+                "loop": "host-driven: pipo_set_pending (pending pair from pinned host memory) + pipo_decode_step "
+                        "(tokens and acceptances back), synchronous"},
+        "gpu_launches": m["launches"] * K,
+        "clocks": m["clocks"],
+    }
+    regular = m.get("regular")
+    if regular is not None:
+        pipo_tpot = (m["ms"] / K) / (1.0 + acceptance)
+        regular["tpot_ratio"] = regular["ms_per_token"] / pipo_tpot
+        regular["frac"] = regular["achieved_gbs"] / hbm
+        # time to first token on the same prompt: T tokens as T positions against T / 2 pairs (both warm)
+        regular["ttft_ratio"] = (regular["prefill_s"] / regular["pipo_prefill_warm_s"]) \
+            if regular["prefill_s"] and regular["pipo_prefill_warm_s"] else None
+        line["regular"] = regular
+    return line
+
+
 def run_pipo(args):
     import numpy as np
     import torch
@@ -379,17 +436,10 @@ def run_pipo(args):
             kb[int(kk)][0] += float(bb)
             kb[int(kk)][1] += float(mm)
             kb[int(kk)][2] += 1
-    tot_ms = sum(v[1] for v in kb.values())
     regular = run_regular(g, shape, wl, B, T, W, K, stream, 1 + rank * 1000) if args.regular else None
 
     ms_all, tokens_all, e2e_all, e2e_tok_all = aggregate_ranks(ms, tokens, e2e_s, e2e_tokens, "cuda")
-    value = tokens_all / (ms_all / 1e3)
     hbm, tf, src = peaks()
-    step_s = ms / 1e3 / K
-    bytes_step = roofline.step_bytes(shape, B, ctx_avg)
-    step_gbs = bytes_step / step_s / 1e9
-    gb, gms, gn = kb[0]
-    gemv_gbs = gb / (gms / 1e3) / 1e9 if gms > 0 else None
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline and w_host is not None:
@@ -402,45 +452,13 @@ def run_pipo(args):
         if ws > 1:
             dist.destroy_process_group()
         return
-    line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": K, "warmup": W,
-        "ms_per_step": ms_all / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": shape.dtype, "data": "synthetic (seeded weights and prompts)",
-        "config": {"workload": args.workload, "shape": wl["shape"], "batch": B, "prompt_tokens": T,
-                   "context_entries_avg": ctx_avg, "tau": tau, "force_mode": args.force,
-                   "acceptance": tokens / (K * B) - 1.0, "pair_step_us": 1e3 * ms / K,
-                   "prefill_s": t_pf, "prefill_rows": args.prefill_rows,
-                   "heads": "sampled (T 1, top-k 20, top-p 0.95, penalty 1.5)" if args.sampler else "greedy",
-                   "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
-                   "parallelism": f"replicas x{ws}"},
-        "roofline": {"bound": "hbm", "kernel": f"weight-streaming projections (every projection and both LM-head "
-                                                  f"launches of a step): {desc}",
-                     "achieved": gemv_gbs, "peak": hbm, "unit": "GB/s",
-                     "frac": (gemv_gbs / hbm) if gemv_gbs else None, "traffic": None,
-                     "algorithmic_bytes_per_launch": gb / max(1, gn), "avg_launch_us": 1e3 * gms / max(1, gn),
-                     "launches_per_step": gn // prof_steps, "share_of_step_time": gms / tot_ms if tot_ms else None,
-                     "timing": f"CUDA events around each launch, {prof_steps} eagerly run steps after the timed region",
-                     "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)",
-                     "step": {"algorithmic_bytes": bytes_step, "achieved": step_gbs, "frac": step_gbs / hbm,
-                              "frac_of_nominal": step_gbs / NOMINAL_HBM_GBS},
-                     "attention": {"achieved": (kb[1][0] / (kb[1][1] / 1e3) / 1e9) if kb[1][1] else None,
-                                   "share_of_step_time": kb[1][1] / tot_ms if tot_ms else None}},
-        "cpu_baseline": cpu,
-        "e2e": {"value": e2e_tok_all / e2e_all, "unit": "tokens/s", "h2d_bytes_per_step": B * 8,
-                "d2h_bytes_per_step": B * 12,
-                "loop": "host-driven: pipo_set_pending (pending pair from pinned host memory) + pipo_decode_step "
-                        "(tokens and acceptances back), synchronous"},
-        "gpu_launches": launches * K,
-        "clocks": clk.summary(),
-    }
-    if regular is not None:
-        pipo_tpot = (ms / K) / (1.0 + line["config"]["acceptance"])
-        regular["tpot_ratio"] = regular["ms_per_token"] / pipo_tpot
-        regular["frac"] = regular["achieved_gbs"] / hbm
-        # time to first token on the same prompt: T tokens as T positions against T / 2 pairs (both warm)
-        regular["ttft_ratio"] = (regular["prefill_s"] / regular["pipo_prefill_warm_s"]) \
-            if regular["prefill_s"] and regular["pipo_prefill_warm_s"] else None
-        line["regular"] = regular
+    line = make_line(dict(
+        workload=args.workload, shape_name=wl["shape"], dtype=shape.dtype, n_gpus=ws, steps=K, warmup=W, batch=B,
+        prompt_tokens=T, ms=ms, ms_all=ms_all, tokens=tokens, tokens_all=tokens_all, ctx_avg=ctx_avg, tau=tau,
+        force=args.force, prefill_s=t_pf, prefill_rows=args.prefill_rows, sampler=args.sampler, desc=desc, kb=kb,
+        prof_steps=prof_steps, hbm=hbm, peak_source=src, step_bytes=roofline.step_bytes(shape, B, ctx_avg),
+        cpu=cpu, e2e_s=e2e_all, e2e_tokens=e2e_tok_all, launches=launches, clocks=clk.summary(),
+        regular=regular))
     print(json.dumps(line), flush=True)
     g.close()
     if ws > 1:

@@ -1,0 +1,62 @@
+"""The benchmark's JSON line (bench.make_line) from fixed measured
+quantities: every key of the benchmark contract is present with the
+documented meaning, and the derived numbers follow from the inputs.  CPU
+only."""
+import json
+
+import pytest
+
+import bench
+
+
+def _measured(**kw):
+    m = dict(workload="4b-b1", shape_name="4b", dtype="bf16", n_gpus=1, steps=100, warmup=5, batch=2,
+             prompt_tokens=2048, ms=250.0, ms_all=260.0, tokens=260, tokens_all=260, ctx_avg=1074.5, tau=0.5,
+             force=0, prefill_s=3.0, prefill_rows=0, sampler=False, desc="B=2 projections=...",
+             kb={0: [8.0e9, 2.0, 150], 1: [1.0e8, 0.5, 37], 2: [0.0, 0.1, 2]}, prof_steps=1, hbm=6774.6,
+             peak_source="measured", step_bytes=9.3e9, cpu={"value": 5.0, "unit": "tokens/s", "cores": 16,
+                                                             "kind": "oracle", "sample": "1 step"},
+             e2e_s=30.0, e2e_tokens=240, launches=192, clocks={"sm_mhz": 2070, "sm_max_mhz": 2070, "reasons": []},
+             regular=None)
+    m.update(kw)
+    return m
+
+
+def test_contract_keys_and_meanings():
+    line = bench.make_line(_measured())
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+              "vs_baseline", "dtype", "data", "config", "roofline", "cpu_baseline", "e2e", "gpu_launches", "clocks"):
+        assert k in line, k
+    assert line["value"] == pytest.approx(260 / 0.260)          # all tokens / slowest rank's time
+    assert line["ms_per_step"] == pytest.approx(2.6)
+    assert line["higher_is_better"] is True and line["scaling"] == "weak" and line["vs_baseline"] is None
+    assert line["config"]["workload"] == "4b-b1"
+    assert line["config"]["acceptance"] == pytest.approx(260 / (100 * 2) - 1)
+    r = line["roofline"]
+    for k in ("bound", "achieved", "peak", "unit", "frac", "traffic"):
+        assert k in r, k
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s" and r["peak"] == 6774.6
+    assert r["achieved"] == pytest.approx(8.0e9 / 2.0e-3 / 1e9)  # family bytes / family time
+    assert r["frac"] == pytest.approx(r["achieved"] / 6774.6)
+    assert r["algorithmic_bytes_per_launch"] == pytest.approx(8.0e9 / 150)
+    assert r["step"]["achieved"] == pytest.approx(9.3e9 / 2.5e-3 / 1e9)
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 16
+    e = line["e2e"]
+    assert e["value"] == pytest.approx(8.0) and e["h2d_bytes_per_step"] == 16 and e["d2h_bytes_per_step"] == 24
+    assert line["gpu_launches"] == 192 * 100
+    json.dumps(line)  # serialisable
+
+
+def test_regular_ratios():
+    reg = dict(ms_per_step=2.0, ms_per_token=2.0, tokens_per_s=500.0, achieved_gbs=4000.0, prefill_s=6.0,
+               pipo_prefill_warm_s=2.0)
+    line = bench.make_line(_measured(regular=reg))
+    # the pair step: 2.5 ms per step, 1.3 tokens per sequence and step
+    assert line["regular"]["tpot_ratio"] == pytest.approx(2.0 / (2.5 / 1.3))
+    assert line["regular"]["ttft_ratio"] == pytest.approx(3.0)
+    assert line["regular"]["frac"] == pytest.approx(4000.0 / 6774.6)
+
+
+def test_missing_profile_gives_no_fraction():
+    line = bench.make_line(_measured(kb={0: [0.0, 0.0, 0], 1: [0.0, 0.0, 0], 2: [0.0, 0.0, 0]}))
+    assert line["roofline"]["achieved"] is None and line["roofline"]["frac"] is None

@@ -29,8 +29,14 @@ def _digest() -> str:
                 h.update(name.encode())
                 with open(p, "rb") as f:
                     h.update(f.read())
-    h.update(" ".join(ARCH).encode())
+    h.update(" ".join(ARCH + extra_flags()).encode())
     return h.hexdigest()
+
+
+def extra_flags() -> list:
+    """Experiment flags for every unit, e.g. PIPO_NVCC_FLAGS="-DPIPO_STREAM_THREADS=384
+    -DPIPO_STREAM_CTAS_PER_SM=2" (the build-time switches of the kernels)."""
+    return os.environ.get("PIPO_NVCC_FLAGS", "").split()
 
 
 def nvcc() -> str:
@@ -49,7 +55,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
         return LIB
     tag = f".tmp{os.getpid()}"
     flags = ["-O3", "-std=c++17", "-lineinfo", *ARCH, "-Xcompiler", "-fPIC,-fvisibility=hidden",
-             "-I", INCLUDE, "-I", CSRC] + (["-Xptxas=-v"] if verbose else [])
+             "-I", INCLUDE, "-I", CSRC] + extra_flags() + (["-Xptxas=-v"] if verbose else [])
 
     def compile_unit(src: str) -> str:
         obj = os.path.join(LIBDIR, os.path.splitext(src)[0] + tag + ".o")

@@ -12,6 +12,12 @@ and projection kernels.
 
   python -m paper_2605_27255_gb300.kernel_bench --step --batch 64 --ctx 512
 
+With --prefill T, one pair prefill of T tokens per sequence on the same small
+model, position by position or in chunks (--rows R, --tile for the causal
+tile attention), inside an NVTX range "prefill".
+
+  python -m paper_2605_27255_gb300.kernel_bench --prefill 8192 --rows 128 --tile
+
 Shapes are the weight-streaming projections of the 4B-class model.  Weights
 are random bf16; several copies are cycled so that every launch streams from
 HBM (more than twice the 129 MB L2 in total).  Prints one JSON line per shape
@@ -106,6 +112,35 @@ def run_step(batch: int, ctx: int) -> dict:
         g.close()
 
 
+def run_prefill(batch: int, tokens: int, rows: int, tile: bool) -> dict:
+    """One pair prefill of `tokens` tokens per sequence on the small bf16 model
+    (the shape of --step), with chunks of `rows` rows (0: position by position)
+    and the tile or per-row chunk attention; wall time of the synchronous call
+    after one warm-up prefill."""
+    import os
+    import time
+
+    from . import synth
+    os.environ["PIPO_PREFILL_ROWS"] = str(rows)
+    os.environ["PIPO_PREFILL_ATTN"] = "tile" if tile else "rows"
+    shape = synth.ModelShape(**STEP_SHAPE)
+    w = synth.gen_weights(shape, seed=0, device="cuda")
+    g = capi.Pipo(shape, w, max_batch=batch, max_ctx=(tokens + 1) // 2 + 4)
+    try:
+        prompts = synth.gen_prompts(batch, tokens, shape.V, seed=1).numpy()
+        g.prefill(prompts)
+        torch.cuda.synchronize()
+        torch.cuda.nvtx.range_push("prefill")
+        t0 = time.perf_counter()
+        g.prefill(prompts)
+        dt = time.perf_counter() - t0
+        torch.cuda.nvtx.range_pop()
+        return dict(kernel="prefill", shape=STEP_SHAPE["name"], batch=batch, tokens=tokens, rows=rows, tile=tile,
+                    seconds=dt, pairs_per_s=batch * ((tokens + 1) // 2) / dt)
+    finally:
+        g.close()
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--shape", default="all", choices=["all"] + sorted(SHAPES))
@@ -115,8 +150,14 @@ def main() -> None:
     ap.add_argument("--splits", type=int, default=0, help="K splits of the tensor-core GEMM (0: automatic)")
     ap.add_argument("--step", action="store_true", help="one eager decode step of a small bf16 model")
     ap.add_argument("--ctx", type=int, default=512, help="--step: cached entries per sequence")
+    ap.add_argument("--prefill", type=int, default=0, help="time a pair prefill of this many tokens per sequence")
+    ap.add_argument("--rows", type=int, default=0, help="--prefill: chunk rows (0: position by position)")
+    ap.add_argument("--tile", action="store_true", help="--prefill: the causal tile chunk attention")
     a = ap.parse_args()
     capi.load()
+    if a.prefill:
+        print(json.dumps(run_prefill(a.batch, a.prefill, a.rows, a.tile)), flush=True)
+        return
     if a.step:
         print(json.dumps(run_step(a.batch, a.ctx)), flush=True)
         return

@@ -328,7 +328,9 @@ PIPO_API pipo_status pipo_profile_step(pipo_ctx *ctx, int32_t cap, int32_t *h_ki
 /* Which kernels the next decode step launches for the projections and the
  * attention, and the attention cluster size, as one NUL-terminated line of
  * at most cap bytes in h_buf, e.g. "B=16 projections=gemm_tc_kernel<16>+
- * prep_bf16_kernel (tcgen05) attention=attn_mma_kernel cluster=2".  Batch B
+ * prep_bf16_kernel (tcgen05) attention=attn_mma_kernel cluster=2
+ * mode=pair heads=argmax", followed by the prefill arrangement when chunks
+ * are enabled.  Batch B
  * is the prefilled batch (before a prefill: cfg.max_batch).  A report of
  * this library's kernel choices; the paper has no counterpart.  EINVAL for
  * a NULL context or buffer or cap == 0. */

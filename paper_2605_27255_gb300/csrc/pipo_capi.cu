@@ -2307,9 +2307,15 @@ pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {
     else proj = cuda_core;
     const int cs = attn_cluster_size(ctx, B);
     const bool mma = attn_use_mma(ctx, B) && cs <= 8;
-    const std::string d = "B=" + std::to_string(B) + " projections=" + proj + " attention=" +
-                          (ctx->attn_v0 ? std::string("attn_decode_kernel") : mma ? "attn_mma_kernel" : "attn_cluster_kernel") +
-                          " cluster=" + std::to_string(cs);
+    std::string d = "B=" + std::to_string(B) + " projections=" + proj + " attention=" +
+                    (ctx->attn_v0 ? std::string("attn_decode_kernel") : mma ? "attn_mma_kernel" : "attn_cluster_kernel") +
+                    " cluster=" + std::to_string(cs);
+    // decoding mode, heads and prefill arrangement
+    d += ctx->regular ? " mode=regular" : " mode=pair";
+    d += ctx->samp_on ? " heads=sampled" : " heads=argmax";
+    if (ctx->prefill_rows >= 2)
+        d += " prefill=chunks of " + std::to_string(ctx->prefill_rows) + " rows (" +
+             (ctx->prefill_tile_attn && attn_mma_ok(ctx) ? "attn_prefill_kernel" : "per-row attention") + ")";
     snprintf(h_buf, cap, "%s", d.c_str());
     return PIPO_OK;
 }

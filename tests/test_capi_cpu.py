@@ -166,3 +166,17 @@ def test_header_is_c99_and_a_c_program_links_and_fails_cleanly_without_a_device(
     r = subprocess.run([exe], capture_output=True, text=True, timeout=120)
     assert r.returncode == 2, (r.returncode, r.stdout, r.stderr)
     assert "pipo_init: status" in r.stdout
+
+
+def test_every_kernel_unit_is_built():
+    """Every .cu file of csrc is a unit of the library build, and every launch
+    handle declared in kernel_tables.h is defined by some unit."""
+    import glob
+    import re as _re
+    csrc = os.path.join(ROOT, "paper_2605_27255_gb300", "csrc")
+    units = sorted(os.path.basename(p) for p in glob.glob(os.path.join(csrc, "*.cu")))
+    assert units == sorted(build.SOURCES)
+    decl = _re.findall(r"\b(k_\w+)\(", open(os.path.join(csrc, "kernel_tables.h")).read())
+    defs = "".join(open(os.path.join(csrc, u)).read() for u in units)
+    for name in set(decl):
+        assert _re.search(r"\b" + name + r"\([^;{]*\)\s*\{", defs), f"{name} declared but not defined"

@@ -165,6 +165,14 @@ PIPO_API pipo_status pipo_decode_step(pipo_ctx *ctx, int32_t *h_tokens, int32_t 
  * step is a captured CUDA graph replayed per call. */
 PIPO_API pipo_status pipo_decode_step_async(pipo_ctx *ctx, int32_t *d_tokens, int32_t *d_n_accepted);
 
+/* n_steps pair-decode steps in one call (graph replays back to back, one
+ * host synchronisation at the end): h_tokens[n_steps][B][2] and
+ * h_n_accepted[n_steps][B] (host, may be NULL) receive every step's
+ * outputs.  ESTATE before a prefill or in regular mode; ECAPACITY when a
+ * cache would exceed max_ctx within the n steps (nothing runs then). */
+PIPO_API pipo_status pipo_decode_steps(pipo_ctx *ctx, int32_t n_steps, int32_t *h_tokens,
+                                       int32_t *h_n_accepted);
+
 /* Regular decoding, the baseline the paper measures PIPO against (Sec. 4,
  * "Regular"; its TPOT comparison): the same backbone, one token per pass.
  * The input of a pass is the token's embedding E[t] (no compressor), its

@@ -74,6 +74,7 @@ SIGNATURES = {
     "pipo_prefill_slot": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.c_int32, _IP, _IP]),
     "pipo_decode_step": (C.c_int, [C.c_void_p, _IP, _IP]),
     "pipo_decode_step_async": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "pipo_decode_steps": (C.c_int, [C.c_void_p, C.c_int32, _IP, _IP]),
     "pipo_regular_prefill": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.c_int32, _IP, _IP, _IP]),
     "pipo_regular_step": (C.c_int, [C.c_void_p, _IP]),
     "pipo_regular_step_async": (C.c_int, [C.c_void_p, C.c_void_p]),
@@ -172,6 +173,13 @@ def pipo_decode_step(ctx, B: int):
     tok = np.zeros((B, 2), np.int32)
     nacc = np.zeros(B, np.int32)
     _check(load().pipo_decode_step(ctx, _ip(tok), _ip(nacc)), ctx)
+    return tok, nacc
+
+
+def pipo_decode_steps(ctx, B: int, n: int):
+    tok = np.zeros((n, B, 2), np.int32)
+    nacc = np.zeros((n, B), np.int32)
+    _check(load().pipo_decode_steps(ctx, int(n), _ip(tok), _ip(nacc)), ctx)
     return tok, nacc
 
 
@@ -381,6 +389,10 @@ class Pipo:
 
     def step(self):
         return pipo_decode_step(self.ctx, self.B)
+
+    def steps(self, n):
+        """n decode steps in one call: (tokens [n, B, 2], n_accepted [n, B])."""
+        return pipo_decode_steps(self.ctx, self.B, n)
 
     def step_async(self, d_tokens: int = 0, d_nacc: int = 0):
         pipo_decode_step_async(self.ctx, d_tokens, d_nacc)

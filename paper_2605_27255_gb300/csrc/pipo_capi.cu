@@ -133,6 +133,8 @@ struct pipo_ctx {
 
     int32_t *pf_pairs = nullptr, *pf_mtp = nullptr;
     size_t pf_cap = 0;
+    int32_t* multi_out = nullptr;     // pipo_decode_steps: [n][B][3] tokens and acceptances of n steps
+    size_t multi_cap = 0;
 
     float* rope = nullptr;            // [max_ctx][d_h/2][2] cos, sin
     bool pdl = false;                 // programmatic dependent launch (decode graph only)
@@ -1996,6 +1998,41 @@ pipo_status pipo_decode_step_async(pipo_ctx* ctx, int32_t* d_tokens, int32_t* d_
 
 pipo_status pipo_decode_step(pipo_ctx* ctx, int32_t* h_tokens, int32_t* h_n_accepted) {
     return step_sync(ctx, false, h_tokens, h_n_accepted);
+}
+
+pipo_status pipo_decode_steps(pipo_ctx* ctx, int32_t n_steps, int32_t* h_tokens, int32_t* h_n_accepted) {
+    if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    if (n_steps < 1) return fail(ctx, PIPO_EINVAL, "n_steps %d < 1", n_steps);
+    if (!ctx->prefilled) return fail(ctx, PIPO_ESTATE, "decode step before prefill");
+    for (int b = 0; b < ctx->B; ++b)
+        if (ctx->h_len[b] + n_steps > ctx->cfg.max_ctx)
+            return fail(ctx, PIPO_ECAPACITY, "sequence %d: %d entries + %d steps > max_ctx", b, ctx->h_len[b], n_steps);
+    CK(cudaSetDevice(ctx->dev));
+    const size_t B = ctx->B, need = (size_t)n_steps * B * 3;
+    if (need > ctx->multi_cap) {
+        if (ctx->multi_out) {
+            cudaFree(ctx->multi_out);
+            ctx->allocs.erase(std::find(ctx->allocs.begin(), ctx->allocs.end(), (void*)ctx->multi_out));
+            ctx->multi_out = nullptr;
+        }
+        ctx->multi_cap = 0;
+        TRY(dalloc(ctx, &ctx->multi_out, need * 4));
+        ctx->multi_cap = need;
+    }
+    // per step: tokens [B][2] then acceptances [B], gathered on the device
+    for (int i = 0; i < n_steps; ++i) {
+        int32_t* o = ctx->multi_out + (size_t)i * B * 3;
+        TRY(step_async(ctx, false, o, o + 2 * B));
+    }
+    std::vector<int32_t> host(need);
+    CK(cudaMemcpyAsync(host.data(), ctx->multi_out, need * 4, cudaMemcpyDeviceToHost, ctx->stream));
+    CK(cudaStreamSynchronize(ctx->stream));
+    for (int i = 0; i < n_steps; ++i) {
+        const int32_t* o = host.data() + (size_t)i * B * 3;
+        if (h_tokens) std::copy(o, o + 2 * B, h_tokens + (size_t)i * B * 2);
+        if (h_n_accepted) std::copy(o + 2 * B, o + 3 * B, h_n_accepted + (size_t)i * B);
+    }
+    return check_device_error(ctx);
 }
 
 pipo_status pipo_regular_step_async(pipo_ctx* ctx, int32_t* d_tokens) {

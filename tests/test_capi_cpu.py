@@ -98,6 +98,7 @@ def test_every_context_entry_point_rejects_a_null_context(lib):
         "pipo_prefill_slot": lambda: L.pipo_prefill_slot(null, 0, ib, 1, ib, ib),
         "pipo_decode_step": lambda: L.pipo_decode_step(null, None, None),
         "pipo_decode_step_async": lambda: L.pipo_decode_step_async(null, None, None),
+        "pipo_decode_steps": lambda: L.pipo_decode_steps(null, 1, None, None),
         "pipo_regular_step": lambda: L.pipo_regular_step(null, None),
         "pipo_regular_step_async": lambda: L.pipo_regular_step_async(null, None),
         "pipo_rollback": lambda: L.pipo_rollback(null, ib),

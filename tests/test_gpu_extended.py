@@ -7,7 +7,8 @@ until they have run on a GB300):
   token sequence whose pairs, positions and teacher-forced MTP tokens are
   those the steps used);
 * the widest batch of the tensor-core path (B = 128, batch width 128)
-  against the fp64 oracle.
+  against the fp64 oracle;
+* pipo_decode_steps (n steps per call) equals n single steps.
 """
 import os
 
@@ -68,3 +69,25 @@ def test_widest_tensor_core_batch():
     prompts = synth.gen_prompts(128, 12, MID.V, seed=15).numpy()
     st = run_forced_replay(MID, w, prompts, 2)
     assert st.tok_checked >= 0.5 * st.tok_total
+
+
+@pytest.mark.parametrize("shape", [synth.TINY, MID])
+def test_multi_step_call_equals_single_steps(shape):
+    w = synth.gen_weights(shape, seed=16)
+    prompts = synth.gen_prompts(3, 21, shape.V, seed=17).numpy()
+    a = capi.Pipo(shape, w, max_batch=3, max_ctx=24)
+    b = capi.Pipo(shape, w, max_batch=3, max_ctx=24)
+    try:
+        a.prefill(prompts)
+        b.prefill(prompts)
+        tok, nacc = a.steps(6)
+        for i in range(6):
+            t, n = b.step()
+            assert np.array_equal(tok[i], t) and np.array_equal(nacc[i], n)
+        assert list(a.counters()[0]) == list(b.counters()[0])
+        with pytest.raises(capi.PipoError):
+            a.steps(100)  # beyond max_ctx: refused before any step runs
+        assert list(a.counters()[0]) == list(b.counters()[0])
+    finally:
+        a.close()
+        b.close()

@@ -194,3 +194,52 @@ def test_sampler_selection_is_the_sorted_top_k():
             vals = np.round(vals * 2) / 2  # ties: the lower id first
         ref = sorted(((float(vals[i]), i) for i in range(V)), key=lambda x: (-x[0], x[1]))[:min(k, V)]
         assert _select(vals, k) == ref, (V, k)
+
+
+def test_decode_attention_fragment_arithmetic_the_same_way():
+    """The same restatement applied to the decode tensor-core attention
+    (attn_mma_kernel, verified on the GPU against the oracle): rows 0..G-1 of
+    A hold the bf16 part of the G heads' queries, rows G..2G-1 the remainder,
+    rows 8..15 zero; a head's score is row h plus row h + G (the lane 4G
+    apart).  Agreement here ties the layouts assumed above to a kernel whose
+    results are known."""
+    rng = np.random.default_rng(1)
+    DH, G = 128, 4
+    K = _bf16(rng.standard_normal((16, DH)).astype(np.float32))
+    Q = (rng.standard_normal((G, DH)) * 0.1).astype(np.float32)
+    kbuf = _store_tile(K)
+    qa = []
+    for lane in range(32):
+        r, t = lane // 4, lane % 4
+        frags = []
+        for kc in range(8):
+            pair = []
+            for half in range(2):
+                d0 = kc * 16 + half * 8 + 2 * t
+                if r < G:
+                    x0, x1 = Q[r, d0], Q[r, d0 + 1]
+                elif r < 2 * G:
+                    x0, x1 = _rest(Q[r - G, d0]), _rest(Q[r - G, d0 + 1])
+                else:
+                    x0 = x1 = 0.0
+                pair.append((_bf16(x0), _bf16(x1)))
+            frags.append([pair[0], (0.0, 0.0), pair[1], (0.0, 0.0)])  # a1 = a3 = 0: rows 8-15 zero
+        qa.append(frags)
+    sacc = [[[0.0] * 4 for _ in range(32)] for _ in range(2)]
+    for nt in range(2):
+        for kc2 in range(4):
+            addr = [_tile_off(nt * 8 + (l & 7), 4 * kc2 + 2 * ((l >> 3) >> 1) + ((l >> 3) & 1)) // 2 for l in range(32)]
+            bk = _ldsm_x4(kbuf, addr)
+            sacc[nt] = _mma16(sacc[nt], [qa[l][2 * kc2] for l in range(32)], [[bk[l][0], bk[l][1]] for l in range(32)])
+            sacc[nt] = _mma16(sacc[nt], [qa[l][2 * kc2 + 1] for l in range(32)],
+                              [[bk[l][2], bk[l][3]] for l in range(32)])
+    ref = K.astype(np.float64) @ Q.astype(np.float64).T  # [16 entries][G heads]
+    for lane in range(32):
+        r, t = lane // 4, lane % 4
+        if r >= G:
+            continue
+        partner = lane ^ (4 * G)  # the lane holding row r + G
+        for nt in range(2):
+            for j in range(2):
+                score = sacc[nt][lane][j] + sacc[nt][partner][j]
+                assert abs(score - ref[nt * 8 + 2 * t + j, r]) < 1e-4

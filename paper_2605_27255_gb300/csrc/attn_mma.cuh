@@ -38,8 +38,14 @@ constexpr int kMmaDH = 128;
 constexpr int kMmaRun = 16;                         // entries per group
 constexpr int kMmaHalf = kMmaRun * 128;             // one box: 16 rows x 64 dims bf16 (2 KB)
 constexpr int kMmaStageBytes = 4 * kMmaHalf;        // K (2 halves) + V (2 halves)
-constexpr int kMmaStages = 10;
-constexpr int kMmaWarps = 4;                        // compute warps
+#ifndef PIPO_MMA_STAGES
+#define PIPO_MMA_STAGES 10
+#endif
+#ifndef PIPO_MMA_WARPS
+#define PIPO_MMA_WARPS 4
+#endif
+constexpr int kMmaStages = PIPO_MMA_STAGES;
+constexpr int kMmaWarps = PIPO_MMA_WARPS;           // compute warps (at least the G heads of a kv head)
 constexpr int kMmaThreads = (kMmaWarps + 1) * 32;   // + the producer warp
 
 constexpr size_t mma_attn_smem() { return 1024 + (size_t)kMmaStages * kMmaStageBytes + 2 * kMmaStages * 8; }
@@ -84,6 +90,7 @@ template <int G>
 __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, const __grid_constant__ CUtensorMap tmK,
                                                                const __grid_constant__ CUtensorMap tmV) {
     static_assert(G == 1 || G == 2 || G == 4, "2G query rows must fit the 8 live MMA rows");
+    static_assert(kMmaWarps >= G && kMmaWarps <= 16 && kMmaStages >= 2, "warps hold the new entry's heads");
     constexpr int DH = kMmaDH;
     constexpr int NW = kMmaWarps;
     constexpr int NP = NW + 1;  // softmax partials: one per compute warp + the new entry

@@ -584,7 +584,14 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
     const int ru = p.epi == EPI_SWIGLU ? 2 : 1;
     const int rows = p.N * ru, bn = tc_bn(p.B), tiles = (rows + kTcM - 1) / kTcM, nkb = p.K / kTcBK;
     const bool fused = tcf_eligible(p) && !tc_prep_forced() && x_rows >= bn && bn <= tc_fused_max_bh();
-    TcPlan plan = tc_plan(ctx->sms, bn, tiles, nkb, fused, !ctx->tc_shallow);
+    // PIPO_TC_SWIGLU_SHALLOW=1: the gate/up projection on the two-per-SM ring
+    // (in isolation at B = 16: 22.9 us with two K splits against 24.8 us deep)
+    static const bool swiglu_shallow = [] {
+        const char* ev = getenv("PIPO_TC_SWIGLU_SHALLOW");
+        return ev && ev[0] == '1';
+    }();
+    const bool allow_deep = !ctx->tc_shallow && !(swiglu_shallow && p.epi == EPI_SWIGLU);
+    TcPlan plan = tc_plan(ctx->sms, bn, tiles, nkb, fused, allow_deep);
     if (splits_req > 0) plan.splits = std::min({splits_req, nkb, kTcMaxSplits});
     TcParams tp{};
     tp.rows = rows; tp.K = p.K; tp.B = p.B; tp.ru = ru; tp.epi = p.epi;

@@ -60,3 +60,22 @@ def test_regular_ratios():
 def test_missing_profile_gives_no_fraction():
     line = bench.make_line(_measured(kb={0: [0.0, 0.0, 0], 1: [0.0, 0.0, 0], 2: [0.0, 0.0, 0]}))
     assert line["roofline"]["achieved"] is None and line["roofline"]["frac"] is None
+
+
+def test_reference_arm_runs_on_cpu_and_prints_one_contract_line():
+    """bench.py --impl reference on the tiny workload (the fp64 oracle on the
+    host cores): exit 0 and one JSON line with the reference arm's keys."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--workload", "tiny",
+                        "--steps", "2", "--warmup", "1"], capture_output=True, text=True, timeout=600, cwd=root)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["steps"] == 2 and line["value"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}

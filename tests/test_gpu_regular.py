@@ -143,3 +143,28 @@ def test_mode_errors_and_switching():
     finally:
         gpu.close()
         ref.close()
+
+
+def test_regular_4b_b1_matches_oracle():
+    """The 4B shapes of the benchmark (B = 1, the CUDA-core path) for regular
+    decoding: weights generated on the GPU, a host copy for the oracle."""
+    s = synth.B4
+    w = synth.gen_weights(s, seed=0, device="cuda")
+    host = {k: v.cpu() for k, v in w.items()}
+    prompts = synth.gen_prompts(1, 48, s.V, seed=1).numpy()
+    T, steps = prompts.shape[1], 4
+    gpu = capi.Pipo(s, w, max_batch=1, max_ctx=T + steps + 1, debug=True)
+    try:
+        orc = O.State(O.Model(s, host, max_ctx=T + steps + 1), 1)
+        tok, nacc = gpu.regular_prefill(prompts)
+        o = orc.regular_prefill(prompts)
+        checked = _compare(s, o, gpu.debug(), tok, nacc, "prefill")
+        for i in range(steps):
+            gpu.set_pending([[orc.seq(0)["p0"], -1]])
+            tok = gpu.regular_step()
+            o = orc.regular_step()
+            checked += _compare(s, o, gpu.debug(), tok, np.zeros(1, np.int32), f"step {i}")
+        assert checked >= 4
+    finally:
+        gpu.close()
+        del w

@@ -138,3 +138,19 @@ def test_chunked_regular_prefill_matches_oracle(monkeypatch, attn):
         assert list(n) == [T + 5] * B
     finally:
         g.close()
+
+
+@pytest.mark.parametrize("attn", ["rows", "tile"])
+def test_chunked_prefill_4b(monkeypatch, attn):
+    """The 4B shapes of the benchmark: a 300-token prompt (150 pairs) in
+    chunks of 128 rows at B = 1, then forced-replay steps, against the oracle."""
+    monkeypatch.setenv("PIPO_PREFILL_ROWS", "128")
+    if attn == "tile":
+        monkeypatch.setenv("PIPO_PREFILL_ATTN", "tile")
+    s = synth.B4
+    w = synth.gen_weights(s, seed=0, device="cuda")
+    host = {k: v.cpu() for k, v in w.items()}
+    prompts = synth.gen_prompts(1, 300, s.V, seed=3).numpy()
+    st = run_forced_replay(s, w, prompts, 3, oracle_weights=host)
+    assert st.tok_checked >= 0.8 * st.tok_total
+    del w

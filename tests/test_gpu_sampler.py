@@ -140,3 +140,32 @@ def test_sampler_argument_errors():
         g.step()
     finally:
         g.close()
+
+
+def test_paper_sampler_4b():
+    """The 4B shapes (V = 151936): the full-vocabulary selection of the
+    sampler kernel against the oracle's sort."""
+    s = synth.B4
+    w = synth.gen_weights(s, seed=0, device="cuda")
+    host = {k: v.cpu() for k, v in w.items()}
+    prompts = synth.gen_prompts(1, 40, s.V, seed=2).numpy()
+    u = np.random.default_rng(9).random((5, 1, 2)).astype(np.float32)
+    max_ctx = 40
+    gpu = capi.Pipo(s, w, max_batch=1, max_ctx=max_ctx, debug=True)
+    try:
+        gpu.set_sampler(u, **PAPER)
+        orc = O.State(O.Model(s, host, max_ctx=max_ctx), 1)
+        orc.set_sampler(**PAPER)
+        tok, nacc = gpu.prefill(prompts)
+        o = orc.prefill(prompts, u=u[0].astype(np.float64), tau=s.tau)
+        for i in range(4):
+            d = gpu.debug()
+            assert np.abs(d["logits_b"] - o["logits_b"]).max() <= tol_for(s)
+            if o["margin_b"][0] <= _delta(s) or o["margin_d"][0] <= _delta(s):
+                break  # a decision inside its margin: the histories may part here
+            assert d["x_b"][0] == o["x_b"][0] and d["x_d"][0] == o["x_d"][0]
+            tok, nacc = gpu.step()
+            o = orc.step(u=u[i + 1].astype(np.float64), tau=s.tau)
+    finally:
+        gpu.close()
+        del w

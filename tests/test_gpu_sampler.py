@@ -161,9 +161,11 @@ def test_paper_sampler_4b():
         for i in range(4):
             d = gpu.debug()
             assert np.abs(d["logits_b"] - o["logits_b"]).max() <= tol_for(s)
-            if o["margin_b"][0] <= _delta(s) or o["margin_d"][0] <= _delta(s):
+            if (o["margin_b"][0] <= _delta(s) or o["margin_d"][0] <= _delta(s)
+                    or abs(float(o["conf"][0]) - s.tau) <= _delta(s)):
                 break  # a decision inside its margin: the histories may part here
             assert d["x_b"][0] == o["x_b"][0] and d["x_d"][0] == o["x_d"][0]
+            assert nacc[0] == o["n_acc"][0]
             tok, nacc = gpu.step()
             o = orc.step(u=u[i + 1].astype(np.float64), tau=s.tau)
     finally:

@@ -319,10 +319,11 @@ def make_line(m: dict) -> dict:
                      "attention": {"achieved": (ab / (ams / 1e3) / 1e9) if ams else None,
                                    "share_of_step_time": ams / tot_ms if tot_ms else None}},
         "cpu_baseline": m["cpu"],
-        "e2e": {"value": m["e2e_tokens"] / m["e2e_s"], "unit": "tokens/s", "h2d_bytes_per_step": B * 8,
-                "d2h_bytes_per_step": B * 12,
-                "loop": "host-driven: pipo_set_pending (pending pair from pinned host memory) + pipo_decode_step "
-                        "(tokens and acceptances back), synchronous"},
+        "e2e": {"value": m["e2e_tokens"] / m["e2e_s"], "unit": "tokens/s",
+                "h2d_bytes_per_step": 0 if m.get("e2e_loop") else B * 8, "d2h_bytes_per_step": B * 12,
+                "loop": m.get("e2e_loop") or
+                "host-driven: pipo_set_pending (pending pair from pinned host memory) + pipo_decode_step "
+                "(tokens and acceptances back), synchronous"},
         "gpu_launches": m["launches"] * K,
         "clocks": m["clocks"],
     }
@@ -425,9 +426,13 @@ def run_pipo(args):
     e2e_check(lib.pipo_decode_step(g.ctx, tok_p, nacc_p))  # untimed: the first pair on the host
     _, e2a = g.counters()
     torch.cuda.synchronize()
+    e2e_loop = None  # host-driven unless pipo_set_pending refuses a pair (then device-driven, reported)
     t0 = time.perf_counter()
     for _ in range(K):
-        e2e_check(lib.pipo_set_pending(g.ctx, tok_p))
+        if e2e_loop is None:
+            rc = lib.pipo_set_pending(g.ctx, tok_p)
+            if rc != 0:
+                e2e_loop = f"device-driven (pipo_set_pending: {capi.pipo_last_error(g.ctx)})"
         e2e_check(lib.pipo_decode_step(g.ctx, tok_p, nacc_p))
     e2e_s = time.perf_counter() - t0
     _, e2b = g.counters()
@@ -452,11 +457,16 @@ def run_pipo(args):
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline and w_host is not None:
-        r = oracle_sample(shape, w_host, B if B <= 4 else 1, n_pairs, tau, args.force, args.cpu_seconds)
         nb = B if B <= 4 else 1
-        cpu = {"value": r["tokens"] / r["seconds"], "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-               "sample": f"{r['steps']} fp64 oracle decode step(s) of {nb} sequence(s) at context {n_pairs}, "
-                         f"caches filled with seeded values ({r['seconds']:.1f} s)"}
+        try:
+            r = oracle_sample(shape, w_host, nb, n_pairs, tau, args.force, args.cpu_seconds)
+            cpu = {"value": r["tokens"] / r["seconds"], "unit": "tokens/s", "cores": os.cpu_count(),
+                   "kind": "oracle",
+                   "sample": f"{r['steps']} fp64 oracle decode step(s) of {nb} sequence(s) at context {n_pairs}, "
+                             f"caches filled with seeded values ({r['seconds']:.1f} s)"}
+        except Exception as e:  # the GPU line stands without its CPU baseline
+            cpu = {"value": None, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                   "error": f"{type(e).__name__}: {e}"}
     if rank != 0:
         if ws > 1:
             dist.destroy_process_group()
@@ -466,8 +476,8 @@ def run_pipo(args):
         prompt_tokens=T, ms=ms, ms_all=ms_all, tokens=tokens, tokens_all=tokens_all, ctx_avg=ctx_avg, tau=tau,
         force=args.force, prefill_s=t_pf, prefill_rows=args.prefill_rows, sampler=args.sampler, desc=desc, kb=kb,
         prof_steps=prof_steps, hbm=hbm, peak_source=src, step_bytes=roofline.step_bytes(shape, B, ctx_avg),
-        cpu=cpu, e2e_s=e2e_all, e2e_tokens=e2e_tok_all, launches=launches, clocks=clk.summary(),
-        regular=regular))
+        cpu=cpu, e2e_s=e2e_all, e2e_tokens=e2e_tok_all, e2e_loop=e2e_loop, launches=launches,
+        clocks=clk.summary(), regular=regular))
     print(json.dumps(line), flush=True)
     g.close()
     if ws > 1:

@@ -79,3 +79,8 @@ def test_reference_arm_runs_on_cpu_and_prints_one_contract_line():
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
     assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
                            "d2h_bytes_per_step": 0}
+
+
+def test_device_driven_fallback_reports_no_host_input_bytes():
+    line = bench.make_line(_measured(e2e_loop="device-driven (pipo_set_pending: x)"))
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["loop"].startswith("device-driven")

@@ -270,6 +270,18 @@ PIPO_API pipo_status pipo_set_stream(pipo_ctx *ctx, void *stream);
 PIPO_API pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void *d_W, int32_t N, int32_t K,
                                   const float *d_x, int32_t B, float *d_y, void *stream);
 
+/* Measurement op: `count` GEMVs of the pipo_op_gemv form back to back on
+ * `stream`, weights d_Ws[i] (device pointers, [N or 2N, K] each), the same
+ * input and output; with pdl != 0 every launch after the first carries the
+ * programmatic-dependent-launch attribute (its weight prologue overlaps the
+ * launch before, its input and output wait for it), as in a decode step.
+ * Captured in a CUDA graph, the time per launch against one GEMV of the
+ * summed weights gives the fixed cost of a launch.  EINVAL as pipo_op_gemv
+ * or for a NULL weight. */
+PIPO_API pipo_status pipo_op_gemv_chain(int32_t dtype, int32_t mode, const void *const *d_Ws, int32_t count,
+                                        int32_t N, int32_t K, const float *d_x, int32_t B, float *d_y, int32_t pdl,
+                                        void *stream);
+
 /* Tensor-core form of the same projections (Eq. 2 blocks) for batches that
  * make them dense contractions: tcgen05 MMAs with fp32 accumulation in TMEM.
  * Each fp32 activation enters as two bf16 parts, hi = bf16(x) and

@@ -89,6 +89,8 @@ SIGNATURES = {
     "pipo_set_stream": (C.c_int, [C.c_void_p, C.c_void_p]),
     "pipo_op_gemv": (C.c_int, [C.c_int32, C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_int32,
                                C.c_void_p, C.c_void_p]),
+    "pipo_op_gemv_chain": (C.c_int, [C.c_int32, C.c_int32, C.POINTER(C.c_void_p), C.c_int32, C.c_int32, C.c_int32,
+                                     C.c_void_p, C.c_int32, C.c_void_p, C.c_int32, C.c_void_p]),
     "pipo_op_lm_head_argmax": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
                                          C.c_float, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
                                          C.c_void_p]),
@@ -264,6 +266,14 @@ def pipo_op_gemv(dtype: int, mode: int, W: int, N: int, K: int, x: int, B: int, 
     """Device pointers (ints); see include/pipo.h."""
     _check(load().pipo_op_gemv(dtype, mode, C.c_void_p(W), N, K, C.c_void_p(x), B, C.c_void_p(y),
                                C.c_void_p(stream or None)), None)
+
+
+def pipo_op_gemv_chain(dtype: int, mode: int, Ws, N: int, K: int, x: int, B: int, y: int, pdl: bool = True,
+                       stream: int = 0) -> None:
+    """len(Ws) GEMVs back to back (device pointers as ints); see include/pipo.h."""
+    arr = (C.c_void_p * len(Ws))(*[C.c_void_p(w) for w in Ws])
+    _check(load().pipo_op_gemv_chain(dtype, mode, arr, len(Ws), N, K, C.c_void_p(x), B, C.c_void_p(y), int(pdl),
+                                     C.c_void_p(stream or None)), None)
 
 
 def pipo_op_lm_head_argmax(dtype: int, E: int, V: int, H: int, h: int, gamma: int, eps: float, B: int,

@@ -2280,6 +2280,29 @@ pipo_status pipo_op_gemv(int32_t dtype, int32_t mode, const void* d_W, int32_t N
     return st;
 }
 
+pipo_status pipo_op_gemv_chain(int32_t dtype, int32_t mode, const void* const* d_Ws, int32_t count, int32_t N,
+                               int32_t K, const float* d_x, int32_t B, float* d_y, int32_t pdl, void* stream) {
+    static thread_local pipo_ctx op;
+    pipo_ctx* ctx = &op;
+    if (!d_Ws || count < 1 || !d_x || !d_y || N < 1 || K < 8 || K % 8 || B < 1 || (dtype != 0 && dtype != 1) ||
+        (mode != 0 && mode != 1))
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_gemv_chain: bad arguments");
+    for (int i = 0; i < count; ++i)
+        if (!d_Ws[i]) return fail(nullptr, PIPO_EINVAL, "pipo_op_gemv_chain: null weight %d", i);
+    pipo_status st = op_setup(op, dtype, stream);
+    GemvParams p{};
+    p.N = N; p.K = K; p.epi = mode == 1 ? EPI_SWIGLU : EPI_STORE; p.y = d_y; p.ldy = N; p.B = B;
+    p.splitk = 1; p.nseg = 1; p.seg[0] = act_seg(d_x, K, K);
+    for (int i = 0; st == PIPO_OK && i < count; ++i) {
+        p.W = d_Ws[i];
+        st = launch_gemv(ctx, p);
+        op.pdl = pdl != 0;  // every launch after the first waits on the one before in-kernel
+    }
+    op.pdl = false;
+    if (st != PIPO_OK) g_init_error = op.err;
+    return st;
+}
+
 }  // extern "C"
 
 namespace {

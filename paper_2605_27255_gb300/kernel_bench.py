@@ -18,6 +18,12 @@ tile attention), inside an NVTX range "prefill".
 
   python -m paper_2605_27255_gb300.kernel_bench --prefill 8192 --rows 128 --tile
 
+With --chain C, the fixed cost of a GEMV launch: a CUDA graph of C launches
+of one shape (with programmatic dependent launch unless --no-pdl) against
+one launch over the same rows.
+
+  python -m paper_2605_27255_gb300.kernel_bench --chain 32 --shape o_proj
+
 Shapes are the weight-streaming projections of the 4B-class model.  Weights
 are random bf16; several copies are cycled so that every launch streams from
 HBM (more than twice the 129 MB L2 in total).  Prints one JSON line per shape
@@ -112,6 +118,47 @@ def run_step(batch: int, ctx: int) -> dict:
         g.close()
 
 
+def run_chain(name: str, count: int, batch: int, pdl: bool) -> dict:
+    """The fixed cost of a GEMV launch: a CUDA graph of `count` launches of one
+    projection shape (distinct weight copies, so every launch streams from
+    HBM) against a graph of one launch over the same total rows."""
+    N, K, mode = SHAPES[name]
+    rows = 2 * N if mode else N
+    Ws = [(torch.randn(rows, K, device="cuda") * 0.02).to(torch.bfloat16) for _ in range(count)]
+    big = torch.cat(Ws, 0)  # one GEMV of count x N rows
+    x = torch.randn(batch, K, device="cuda")
+    y = torch.empty(batch, N * count, device="cuda")
+    st = torch.cuda.Stream()
+    ptrs = [w.data_ptr() for w in Ws]
+
+    def timed(fn) -> float:
+        with torch.cuda.stream(st):
+            fn()  # load, set attributes
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=st):
+            fn()
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(10):
+            g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / 10
+
+    chain_us = timed(lambda: capi.pipo_op_gemv_chain(1, mode, ptrs, N, K, x.data_ptr(), batch, y.data_ptr(), pdl,
+                                                     torch.cuda.current_stream().cuda_stream))
+    one_us = timed(lambda: capi.pipo_op_gemv(1, mode, big.data_ptr(), N * count, K, x.data_ptr(), batch,
+                                             y.data_ptr(), torch.cuda.current_stream().cuda_stream))
+    nbytes = rows * K * 2 * count
+    return dict(kernel="gemv_chain", shape=name, count=count, batch=batch, pdl=pdl, chain_us=chain_us,
+                single_us=one_us, per_launch_overhead_us=(chain_us - one_us) / count,
+                chain_gbs=nbytes / chain_us / 1e3, single_gbs=nbytes / one_us / 1e3)
+
+
 def run_prefill(batch: int, tokens: int, rows: int, tile: bool) -> dict:
     """One pair prefill of `tokens` tokens per sequence on the small bf16 model
     (the shape of --step), with chunks of `rows` rows (0: position by position)
@@ -151,12 +198,19 @@ def main() -> None:
     ap.add_argument("--step", action="store_true", help="one eager decode step of a small bf16 model")
     ap.add_argument("--ctx", type=int, default=512, help="--step: cached entries per sequence")
     ap.add_argument("--prefill", type=int, default=0, help="time a pair prefill of this many tokens per sequence")
+    ap.add_argument("--chain", type=int, default=0,
+                    help="graph of this many launches of --shape against one launch of the summed rows")
+    ap.add_argument("--no-pdl", action="store_true", help="--chain: without programmatic dependent launch")
     ap.add_argument("--rows", type=int, default=0, help="--prefill: chunk rows (0: position by position)")
     ap.add_argument("--tile", action="store_true", help="--prefill: the causal tile chunk attention")
     a = ap.parse_args()
     capi.load()
     if a.prefill:
         print(json.dumps(run_prefill(a.batch, a.prefill, a.rows, a.tile)), flush=True)
+        return
+    if a.chain:
+        shape = "o_proj" if a.shape == "all" else a.shape
+        print(json.dumps(run_chain(shape, a.chain, a.batch, not a.no_pdl)), flush=True)
         return
     if a.step:
         print(json.dumps(run_step(a.batch, a.ctx)), flush=True)

@@ -129,12 +129,13 @@ PIPO_API pipo_status pipo_init(const pipo_config *cfg, const pipo_weights *w, pi
 
 /* Prefill B sequences (B <= max_batch) from host token ids h_ids, row b at
  * h_ids + b*stride, h_lens[b] tokens (1 <= len <= stride).  Tokens are paired
- * (t_{2j}, t_{2j+1}); an odd length ends in (t_last, PAD) (App. B.2).  All
- * sequences must yield the same number of pairs N (EINVAL otherwise).  Runs
+ * (t_{2j}, t_{2j+1}); an odd length ends in (t_last, PAD) (App. B.2).  Runs
  * the backbone over the N latents, fills both caches, and runs the heads on
  * the last latent: h_tokens[B,2] / h_n_accepted[B] (host, may be NULL) get
  * the first pair output, which also becomes the pending pair.  Resets the
- * emitted counters.  ECAPACITY when N > max_ctx. */
+ * emitted counters.  ECAPACITY when N > max_ctx.  Sequences that yield
+ * different numbers of pairs are prefilled one after another, each as
+ * pipo_prefill_slot does (all are validated first). */
 PIPO_API pipo_status pipo_prefill(pipo_ctx *ctx, int32_t batch, const int32_t *h_ids, int32_t stride,
                          const int32_t *h_lens, int32_t *h_tokens, int32_t *h_n_accepted);
 

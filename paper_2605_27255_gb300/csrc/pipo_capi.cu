@@ -1807,6 +1807,24 @@ extern "C" {
 pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride, const int32_t* h_lens,
                          int32_t* h_tokens, int32_t* h_n_accepted) {
     if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    if (batch > 1 && batch <= ctx->cfg.max_batch && h_ids && h_lens && stride >= 1) {
+        bool ragged = false;
+        for (int b = 1; b < batch; ++b) ragged |= (h_lens[b] + 1) / 2 != (h_lens[0] + 1) / 2;
+        if (ragged) {
+            // different numbers of pairs: every sequence on its own, as a slot
+            for (int b = 0; b < batch; ++b) {  // validate all before any runs
+                int nb = 0;
+                TRY(check_prompt(ctx, 1, h_ids + (size_t)b * stride, stride, h_lens + b, true, &nb));
+            }
+            ctx->prefilled = false;
+            ctx->B = 0;
+            ctx->h_len.clear();
+            for (int b = 0; b < batch; ++b)
+                TRY(pipo_prefill_slot(ctx, b, h_ids + (size_t)b * stride, h_lens[b], h_tokens ? h_tokens + 2 * b : nullptr,
+                                      h_n_accepted ? h_n_accepted + b : nullptr));
+            return PIPO_OK;
+        }
+    }
     int N = 0;
     TRY(check_prompt(ctx, batch, h_ids, stride, h_lens, true, &N));
     CK(cudaSetDevice(ctx->dev));

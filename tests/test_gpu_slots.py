@@ -117,3 +117,15 @@ def test_slot_errors():
             g.prefill_slot(0, ids)  # regular mode
     finally:
         g.close()
+
+
+@pytest.mark.parametrize("shape", [synth.TINY, MID])
+def test_ragged_batch_prefill(shape):
+    """pipo_prefill with prompts of different pair counts (each prefilled as a
+    slot) against the oracle's ragged prefill, then forced-replay steps."""
+    from parity_util import run_forced_replay
+    w = synth.gen_weights(shape, seed=9)
+    lens = np.array([37, 20, 52], np.int32)
+    prompts = synth.gen_prompts(3, 52, shape.V, seed=3).numpy()
+    st = run_forced_replay(shape, w, prompts, 5, lens=lens)
+    assert st.tok_checked >= 0.5 * st.tok_total

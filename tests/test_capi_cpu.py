@@ -181,3 +181,9 @@ def test_every_kernel_unit_is_built():
     defs = "".join(open(os.path.join(csrc, u)).read() for u in units)
     for name in set(decl):
         assert _re.search(r"\b" + name + r"\([^;{]*\)\s*\{", defs), f"{name} declared but not defined"
+
+
+def test_header_compiles_as_cplusplus():
+    """The header also compiles as C++ (its extern "C" block), with warnings as errors."""
+    import subprocess
+    subprocess.check_call(["g++", "-std=c++17", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-x", "c++", HEADER])

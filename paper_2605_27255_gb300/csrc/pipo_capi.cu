@@ -1462,14 +1462,22 @@ pipo_status ensure_cache_tmp(pipo_ctx* ctx, size_t elems) {
     return PIPO_OK;
 }
 
-// Read and clear the device error words of every kernel unit (bounded waits
-// that gave up); the first unit with an error names the wait.
+// Read and clear the device error words of the kernel units whose kernels
+// wait (bounded waits that gave up; the host unit's kernels never wait): the
+// tensor-core attention and projections always, the bulk-copy GEMV and the
+// step kernel when the context uses them.  The first unit with an error
+// names the wait.
 pipo_status check_device_error(pipo_ctx* ctx) {
-    cudaError_t (*const units[])(unsigned*, unsigned*) = {
-        take_unit_error, k_take_error_gemv_bf16, k_take_error_gemv_f32, k_take_error_tc, k_take_error_attn,
-        k_take_error_mk};
+    cudaError_t (*units[5])(unsigned*, unsigned*) = {k_take_error_attn, k_take_error_tc, nullptr, nullptr, nullptr};
+    int nu = 2;
+    if (ctx->gemv_tma) {
+        units[nu++] = k_take_error_gemv_bf16;
+        units[nu++] = k_take_error_gemv_f32;
+    }
+    if (ctx->use_mk) units[nu++] = k_take_error_mk;
     unsigned e = 0, info[4] = {0, 0, 0, 0};
-    for (auto take : units) {
+    for (int i = 0; i < nu; ++i) {
+        auto take = units[i];
         unsigned ue = 0, ui[4] = {0, 0, 0, 0};
         CK(take(&ue, ui));
         if (ue && !e) {

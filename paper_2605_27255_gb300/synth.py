@@ -17,7 +17,14 @@ call gives bit-identical tensors on the CPU and on a GPU:
   deviation (mean 0, std exactly ``std`` in distribution).  This stands in for
   the N(0, 0.02) initialisation of the benchmark configurations; it is bounded
   at +-3.46 std.
-* Norm gains are 1.0 (a gain drawn around 0 would zero the signal).
+* Norm gains are ``1 + g`` with ``g`` drawn like a weight at std
+  ``gain_std`` (0.1 by default, so within [0.65, 1.35]; a gain drawn around
+  0 would zero the signal).  Each norm has its own name and so its own
+  values: every layer's attention and FFN norms, the final norm, the MTP
+  input norms of h_b and of E[x_b], the MTP block's norms, the MTP post-norm
+  and both halves of the confidence head's joint norm all differ, so a gain
+  applied to the wrong norm changes the results.  ``gain_std = 0`` gives the
+  unit gains of an untrained RMSNorm.
 * Token ids are a hashed word modulo V, per sequence from ``seed + b``.
 """
 from __future__ import annotations
@@ -195,13 +202,22 @@ def torch_dtype(s: ModelShape) -> torch.dtype:
     return {"f32": torch.float32, "bf16": torch.bfloat16}[s.dtype]
 
 
-def gen_weights(s: ModelShape, seed: int = 0, device="cpu") -> Dict[str, torch.Tensor]:
-    """All tensors of ``s``: gains 1.0, everything else seeded, std ``s.std``."""
+GAIN_STD = 0.1
+
+
+def gen_weights(s: ModelShape, seed: int = 0, device="cpu",
+                gain_std: float = GAIN_STD) -> Dict[str, torch.Tensor]:
+    """All tensors of ``s``: gains ``1 + N(0, gain_std)`` per norm (rounded
+    to the storage type), everything else seeded with std ``s.std``."""
     dt = torch_dtype(s)
     w = {}
     for name, shape in tensor_shapes(s).items():
         if is_gain(name):
-            w[name] = torch.ones(shape, dtype=dt, device=device)
+            if gain_std == 0.0:
+                w[name] = torch.ones(shape, dtype=dt, device=device)
+            else:
+                g = gen_tensor(seed, name, shape, gain_std, torch.float32, device)
+                w[name] = (1.0 + g).to(dt)
         else:
             w[name] = gen_tensor(seed, name, shape, s.std, dt, device)
     return w

@@ -318,6 +318,158 @@ def test_swiglu_gate_and_up_are_not_swapped():
     assert np.allclose(o["h_b"][0], expect, atol=1e-12)
 
 
+# ------------------------------------------------------------ gain wiring
+#
+# Every RMSNorm of the model has its own gain vector (backbone attention and
+# FFN norms per layer, the final norm, the MTP input norms of h_b and of the
+# token embedding, the MTP block's norms, the MTP post-norm, the joint
+# confidence norm over 2H).  The pins below give every gain distinct values
+# and fix the results in closed form or by a single-position numpy
+# evaluation of the definitions, so a gain taken from the wrong norm, the
+# wrong layer or the wrong half of the confidence norm fails one of them.
+
+def _r(x, eps=1e-6):
+    """x / sqrt(mean(x^2) + eps), the normalisation of an RMSNorm."""
+    x = np.asarray(x, dtype=np.float64)
+    return x / math.sqrt(np.mean(x * x) + eps)
+
+
+def _silu(x):
+    return x / (1.0 + np.exp(-x))
+
+
+def _distinct_gains(w, rng):
+    """Overwrite every gain with its own uniform draw in [0.5, 1.5]."""
+    for name in list(w):
+        if synth.is_gain(name):
+            w[name] = torch.from_numpy(rng.uniform(0.5, 1.5, tuple(w[name].shape)).astype(np.float32))
+    return w
+
+
+@pytest.mark.parametrize("t0,t1", [(5, 2), (1, 6), (4, 4)])
+def test_head_gains_final_post_and_mtp_inputs(t0, t1):
+    """Eq. 3-5 and App. A.2 with E = I (V = H), a [I I] compressor and
+    identity blocks, so h_b = e_t0 + e_t1 (2 e_t0 when t0 = t1):
+      logits_b = E (g_final * r(h_b))            = g_final * r(h_b)
+      W_fc = [0 P]:  h_d = P (g_e * r(E[x_b]))   (no MTP block)
+      W_fc = [I 0]:  h_d = g_h * r(h_b)
+      logits_d = g_post * r(h_d).
+    Swapping the final and post gains, or the two MTP input gains, changes
+    these values."""
+    s = small_shape(L=1)
+    perm = [3, 6, 0, 7, 1, 5, 2, 4]
+    w = _distinct_gains(onehot_model(s, perm), np.random.default_rng(11))
+    g = {k: w[k].double().numpy() for k in ("final_norm", "mtp.norm_h", "mtp.norm_e", "mtp.norm_post")}
+    hb = np.zeros(8); hb[t0] += 1; hb[t1] += 1
+    lb = g["final_norm"] * _r(hb)
+    xb = int(np.argmax(lb))
+    P = w["mtp.W_fc"][:, 8:].double().numpy()
+    for wfc, hd in ((None, P @ (g["mtp.norm_e"] * _r(np.eye(8)[xb]))),
+                    (torch.cat([torch.eye(8), torch.zeros(8, 8)], 1), g["mtp.norm_h"] * _r(hb))):
+        if wfc is not None:
+            w["mtp.W_fc"] = wfc
+        o = O.State(O.Model(s, w), 1).prefill([[t0, t1]], tau=0.5)
+        assert np.allclose(o["h_b"][0], hb, rtol=0, atol=1e-15)
+        assert np.allclose(o["logits_b"][0], lb, rtol=0, atol=1e-12)
+        assert o["x_b"][0] == xb
+        assert np.allclose(o["h_d"][0], hd, rtol=0, atol=1e-12)
+        assert np.allclose(o["logits_d"][0], g["mtp.norm_post"] * _r(hd), rtol=0, atol=1e-12)
+
+
+def test_confidence_gain_halves():
+    """App. A.3: one RMSNorm over [h_b; h_d] with a 2H gain, its first half on
+    h_b and its second half on h_d.  With h_b = 1, h_d = 3 (H = 4), the joint
+    rms is sqrt(5 + eps); gains 2 (first half) and 1/2 (second half); W2 = 1:
+      W1 = [I 0]:  c = sigma(4 SiLU(2 / rms))
+      W1 = [0 I]:  c = sigma(4 SiLU(1.5 / rms)).
+    Dropping the second half of the gain, or reusing the first half for both,
+    changes the second value."""
+    s = small_shape(H=4, V=4, n_q=2, n_kv=1, d_h=2, F=4)
+    w = zero_model(s)
+    w["conf.norm"] = torch.tensor([2.0] * 4 + [0.5] * 4)
+    w["conf.W2"] = torch.ones(1, 4)
+    hb, hd = np.ones(4), np.full(4, 3.0)
+    rms = math.sqrt(5.0 + 1e-6)
+    sig = lambda x: 1.0 / (1.0 + math.exp(-x))
+    for W1, inner in ((torch.cat([torch.eye(4), torch.zeros(4, 4)], 1), 2.0 / rms),
+                      (torch.cat([torch.zeros(4, 4), torch.eye(4)], 1), 1.5 / rms)):
+        w["conf.W1"] = W1
+        expect = sig(4 * inner * sig(inner))
+        assert abs(O.confidence(O.Model(s, w), hb, hd) - expect) < 1e-14
+
+
+def _block_pos0(x, wts, pre, l, nq, nkv, d, eps=1e-6):
+    """One pre-norm decoder block at the first position of a sequence: the
+    only cached entry is the position's own, so attention returns its value
+    vector v (softmax over one score is 1; RoPE does not touch v)."""
+    W = lambda k: wts[f"{pre}.{k}"][l].double().numpy()
+    y = W("attn_norm") * _r(x, eps)
+    v = W("Wv") @ y
+    grp = nq // nkv
+    a = np.concatenate([v[(h // grp) * d:(h // grp + 1) * d] for h in range(nq)])
+    x = x + W("Wo") @ a
+    y = W("ffn_norm") * _r(x, eps)
+    return x + W("Wdown") @ (_silu(W("Wgate") @ y) * (W("Wup") @ y))
+
+
+@pytest.mark.parametrize("comp", ["linear", "mlp"])
+def test_every_gain_at_the_first_position(comp):
+    """The whole step at position 0 evaluated from the definitions (Eq. 1-6,
+    App. A.1-A.3) with random weights and a distinct gain per norm and per
+    layer: compressor, two backbone blocks (attention returns v at a single
+    entry), final-norm LM head, MTP input and block, post-norm LM head and the
+    joint-norm confidence.  A gain taken from another norm or another layer
+    changes h_b, h_d, the logits or c."""
+    s = small_shape(L=2, H=8, V=8, F=6, mtp_block=1, compressor=comp)
+    rng = np.random.default_rng(21)
+    w = {}
+    for name, shape in synth.tensor_shapes(s).items():
+        w[name] = torch.from_numpy(rng.standard_normal(shape).astype(np.float32) * 0.5)
+    w = _distinct_gains(w, rng)
+    W = lambda k: w[k].double().numpy()
+    t0, t1 = 3, 6
+    ab = np.concatenate([W("E")[t0], W("E")[t1]])
+    if comp == "linear":
+        x = W("comp.W") @ ab + W("comp.b")
+    else:
+        x = W("comp.W2") @ _silu(W("comp.W1") @ ab)
+    for l in range(s.L):
+        x = _block_pos0(x, w, "blk", l, s.n_q, s.n_kv, s.d_h)
+    hb = x
+    lb = W("E") @ (W("final_norm") * _r(hb))
+    xb = int(np.argmax(lb))
+    u = W("mtp.W_fc") @ np.concatenate([W("mtp.norm_h") * _r(hb), W("mtp.norm_e") * _r(W("E")[xb])])
+    hd = _block_pos0(u, w, "mtp", 0, s.n_q, s.n_kv, s.d_h)
+    ld = W("E") @ (W("mtp.norm_post") * _r(hd))
+    t = W("conf.W1") @ (W("conf.norm") * _r(np.concatenate([hb, hd])))
+    c = 1.0 / (1.0 + math.exp(-float(W("conf.W2")[0] @ _silu(t))))
+    o = O.State(O.Model(s, w), 1).prefill([[t0, t1]], tau=0.5)
+    assert np.allclose(o["h_b"][0], hb, rtol=0, atol=1e-12)
+    assert np.allclose(o["logits_b"][0], lb, rtol=0, atol=1e-12)
+    assert o["x_b"][0] == xb and np.sort(lb)[-1] - np.sort(lb)[-2] > 1e-6
+    assert np.allclose(o["h_d"][0], hd, rtol=0, atol=1e-12)
+    assert np.allclose(o["logits_d"][0], ld, rtol=0, atol=1e-12)
+    assert abs(o["conf"][0] - c) < 1e-13
+
+
+def test_seeded_gains_are_distinct_per_norm():
+    """The generator gives every norm (and every layer of a stacked norm) its
+    own gains, none of them unit, so the GPU parity runs can see a gain
+    applied to the wrong norm."""
+    s = TINY_SMALL.with_(L=3)
+    w = synth.gen_weights(s, seed=0)
+    gains = {k: v.double().numpy() for k, v in w.items() if synth.is_gain(k)}
+    rows = []
+    for k, v in gains.items():
+        rows += [v[i] for i in range(v.shape[0])] if v.ndim == 2 else [v[: s.H], v[s.H:]] if k == "conf.norm" else [v]
+    assert len(rows) == 2 * 3 + 1 + 2 + 2 + 1 + 2
+    for i in range(len(rows)):
+        assert np.all(np.abs(rows[i] - 1.0) < 0.35) and np.std(rows[i]) > 0.05
+        for j in range(i):
+            assert np.abs(rows[i] - rows[j]).max() > 0.05
+    assert np.all(synth.gen_weights(s, seed=0, gain_std=0.0)["final_norm"].numpy() == 1.0)
+
+
 # ------------------------------------------------------ seeded small models
 
 def seeded(s, seed=0):

@@ -6,6 +6,16 @@ pair, so each step is compared from identical history.  Per step:
     (2e-2 for bf16 models, 1e-4 for fp32 models);
   * x_b / x_d bit-exact wherever the oracle's top-1/top-2 logit margin > 1e-2;
   * the accept decision bit-exact wherever |c - tau| > 1e-2.
+
+Where the oracle's backbone top-1/top-2 margin is within 1e-2, both argmax
+results are correct, and the GPU may feed the other token to the MTP head.
+The test then checks that the GPU's choice is within the margin under the
+oracle's logits.  From there on it compares none of that sequence's
+draft-side outputs: the draft logits, the draft token, the confidence and
+the accept decision.  Those depend on the token the MTP head consumed, and
+the MTP cache keeps that entry for the rest of the run.  Backbone outputs
+are still compared, because forced replay gives the backbone identical
+inputs.
 """
 import numpy as np
 
@@ -26,23 +36,33 @@ class Stats:
         self.acc_checked = 0
         self.max_logit_err = 0.0
         self.max_conf_err = 0.0
+        self.mtp_diverged = set()  # sequences whose MTP head took the other side of an x_b near-tie
 
 
 def compare(shape, tau, o, d, tok, nacc, force, stats, tol, where=""):
     B = tok.shape[0]
     for b in range(B):
         eb = float(np.abs(d["logits_b"][b] - o["logits_b"][b]).max())
-        ed = float(np.abs(d["logits_d"][b] - o["logits_d"][b]).max())
-        ec = abs(float(d["conf"][b]) - float(o["conf"][b]))
-        stats.max_logit_err = max(stats.max_logit_err, eb, ed)
-        stats.max_conf_err = max(stats.max_conf_err, ec)
-        assert eb <= tol and ed <= tol, f"{where} b={b}: logit error {eb:.3g}/{ed:.3g} > {tol}"
-        assert ec <= tol, f"{where} b={b}: confidence error {ec:.3g} > {tol}"
+        stats.max_logit_err = max(stats.max_logit_err, eb)
+        assert eb <= tol, f"{where} b={b}: logit error {eb:.3g} > {tol}"
         stats.tok_total += 2
         if o["margin_b"][b] > MARGIN:
             assert d["x_b"][b] == o["x_b"][b], f"{where} b={b}: x_b {d['x_b'][b]} != {o['x_b'][b]}"
             assert tok[b, 0] == o["tokens"][b, 0]
             stats.tok_checked += 1
+        elif d["x_b"][b] != o["x_b"][b]:
+            # a near-tie taken the other way: valid if within the margin under the oracle's logits
+            gap = float(o["logits_b"][b][o["x_b"][b]] - o["logits_b"][b][d["x_b"][b]])
+            assert 0.0 <= gap <= MARGIN, f"{where} b={b}: x_b {d['x_b'][b]} is {gap:.3g} below the top"
+            stats.mtp_diverged.add(b)
+        if b in stats.mtp_diverged:
+            continue
+        ed = float(np.abs(d["logits_d"][b] - o["logits_d"][b]).max())
+        ec = abs(float(d["conf"][b]) - float(o["conf"][b]))
+        stats.max_logit_err = max(stats.max_logit_err, ed)
+        stats.max_conf_err = max(stats.max_conf_err, ec)
+        assert ed <= tol, f"{where} b={b}: draft logit error {ed:.3g} > {tol}"
+        assert ec <= tol, f"{where} b={b}: confidence error {ec:.3g} > {tol}"
         if o["margin_d"][b] > MARGIN:
             assert d["x_d"][b] == o["x_d"][b], f"{where} b={b}: x_d {d['x_d'][b]} != {o['x_d'][b]}"
             stats.tok_checked += 1

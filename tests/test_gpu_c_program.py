@@ -2,10 +2,7 @@
 library) on the GPU: a step before the prefill is ESTATE, an odd prompt's
 prefill and 8 decode steps give in-range, self-consistent outputs and the
 expected counters.
-
-Opt-in (PIPO_TEST_C=1) until it has run on a GB300.
 """
-import os
 import subprocess
 
 import pytest
@@ -13,9 +10,7 @@ import pytest
 from paper_2605_27255_gb300 import build
 from test_capi_cpu import build_c_program
 
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skipif(os.environ.get("PIPO_TEST_C") != "1",
-                                 reason="the C-program GPU test runs with PIPO_TEST_C=1")]
+pytestmark = pytest.mark.gpu
 
 
 def test_c_program_decodes():

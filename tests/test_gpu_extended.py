@@ -1,5 +1,4 @@
-"""More GPU invariants of the pair-decode path (opt-in, PIPO_TEST_EXTENDED=1,
-until they have run on a GB300):
+"""More GPU invariants of the pair-decode path:
 
 * re-prefill: prefill(prompt) then k accept-all steps leaves the same caches
   and the same next outputs as prefill(prompt + the emitted tokens) (every
@@ -10,7 +9,6 @@ until they have run on a GB300):
   against the fp64 oracle;
 * pipo_decode_steps (n steps per call) equals n single steps.
 """
-import os
 
 import numpy as np
 import pytest
@@ -18,9 +16,7 @@ import pytest
 from paper_2605_27255_gb300 import capi, synth
 from parity_util import run_forced_replay, tol_for
 
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skipif(os.environ.get("PIPO_TEST_EXTENDED") != "1",
-                                 reason="extended GPU tests run with PIPO_TEST_EXTENDED=1")]
+pytestmark = pytest.mark.gpu
 
 MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003,
                        compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1e6, tau=0.5)

@@ -10,8 +10,9 @@ import numpy as np
 import pytest
 import torch
 
-from paper_2605_27255_gb300 import synth
-from parity_util import run_forced_replay
+from oracle import oracle as O
+from paper_2605_27255_gb300 import capi, synth
+from parity_util import Stats, compare, run_forced_replay, tol_for
 
 pytestmark = pytest.mark.gpu
 
@@ -69,11 +70,77 @@ def test_4b_b16_forced_replay(w4b):
     assert st.max_logit_err < 2e-2
 
 
-def test_9b_b1_forced_replay():
-    """9B-class shapes (H=4096, F=12288)."""
+@pytest.fixture(scope="module")
+def w9b():
     w, host = _weights(synth.B9)
+    yield w, host
+    del w
+    torch.cuda.empty_cache()
+
+
+def test_4b_b64_forced_replay(w4b):
+    """4b-b64: batch width 64, the split-kernel tensor-core form (prepared
+    bf16 operand, then the tcgen05 GEMM) for every projection."""
+    w, host = w4b
+    prompts = synth.gen_prompts(64, 2, synth.B4.V, seed=6).numpy()
+    st = run_forced_replay(synth.B4, w, prompts, 1, oracle_weights=host)
+    assert st.tok_checked >= 0.8 * st.tok_total
+    assert st.max_logit_err < 2e-2
+
+
+def test_9b_b1_forced_replay(w9b):
+    """9B-class shapes (H=4096, F=12288)."""
+    w, host = w9b
     prompts = synth.gen_prompts(1, 16, synth.B9.V, seed=2).numpy()
     st = run_forced_replay(synth.B9, w, prompts, 3, oracle_weights=host, tau=0.3)
     assert st.tok_checked >= 0.8 * st.tok_total
-    del w
-    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("tau", [0.3, 0.7])
+def test_9b_b8_forced_replay(w9b, tau):
+    """9b-b8, the benchmark's largest configuration: tcgen05 projections at
+    K = 4096 and K = 12288 (down), tensor-core attention, thresholds from
+    both ends of the sweep."""
+    w, host = w9b
+    prompts = synth.gen_prompts(8, 4, synth.B9.V, seed=7).numpy()
+    st = run_forced_replay(synth.B9, w, prompts, 2, oracle_weights=host, tau=tau)
+    assert st.tok_checked >= 0.8 * st.tok_total
+    assert st.max_logit_err < 2e-2
+
+
+def test_4b_long_context_launch_plan():
+    """The 4b-lc launch plan: 4B widths at B = 4 with 16 K cached entries per
+    sequence, so that a layer's cached K/V bytes exceed six times its QKV
+    weight bytes (every projection on the two-per-SM ring) and the attention
+    runs its long-context cluster arrangement.  Two layers instead of 36
+    keep the fp64 oracle's caches at a few GB; the plan is chosen per layer,
+    so the launches of a layer are those of the 36-layer model."""
+    s = synth.B4.with_(name="4b-lc-2l", L=2)
+    n_ctx, B, steps = 16384, 4, 2
+    w = synth.gen_weights(s, seed=10, device="cuda")
+    host = {k: v.cpu() for k, v in w.items()}
+    K, V = synth.gen_kv_fill(s, n_ctx, seed=11)
+    K, V = K.numpy(), V.numpy()
+    prompts = synth.gen_prompts(B, 2, s.V, seed=12).numpy()
+    gpu = capi.Pipo(s, w, max_batch=B, max_ctx=n_ctx + steps + 2, debug=True, page_shuffle_seed=4)
+    orc = O.State(O.Model(s, host, max_ctx=n_ctx + steps + 2), B)
+    try:
+        gpu.prefill(prompts)
+        orc.prefill(prompts, tau=s.tau)
+        for b in range(B):
+            gpu.load_cache(b, K, V)
+            orc.set_cache(b, K, V)
+        st = Stats()
+        for i in range(steps):
+            gpu.set_pending([[orc.seq(b)["p0"], orc.seq(b)["p1"]] for b in range(B)])
+            tok, nacc = gpu.step()
+            o = orc.step(tau=s.tau)
+            compare(s, s.tau, o, gpu.debug(), tok, nacc, 0, st, tol_for(s), f"step {i}")
+        assert list(gpu.counters()[0]) == [n_ctx + steps] * B
+        d = gpu.describe()
+        assert "attn_mma_kernel" in d, d
+        assert st.tok_checked >= 0.8 * st.tok_total
+    finally:
+        gpu.close()
+        del orc, w
+        torch.cuda.empty_cache()

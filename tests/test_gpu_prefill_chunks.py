@@ -6,8 +6,6 @@ Checked against the fp64 oracle (prefill outputs, then forced-replay decode
 steps that read the chunk-written caches), against the position-by-position
 prefill of the same context shape (cache contents and outputs), for pair and
 regular decoding, with ragged last chunks and several sequences.
-
-Opt-in (PIPO_TEST_PREFILL_CHUNKS=1) until chunked prefill is the default.
 """
 import os
 
@@ -18,9 +16,7 @@ from oracle import oracle as O
 from paper_2605_27255_gb300 import capi, synth
 from parity_util import MARGIN, run_forced_replay, tol_for
 
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skipif(os.environ.get("PIPO_TEST_PREFILL_CHUNKS") != "1",
-                                 reason="chunked-prefill GPU tests run with PIPO_TEST_PREFILL_CHUNKS=1")]
+pytestmark = pytest.mark.gpu
 
 MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003,
                        compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1e6, tau=0.5)

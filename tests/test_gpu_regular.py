@@ -6,10 +6,7 @@ step both sides continue from the oracle's token.
 Per step: LM-head logits max-abs <= 1e-4 (fp32) / 2e-2 (bf16), the token
 bit-exact where the oracle's top-1/top-2 margin > 1e-2, slot 1 always -1, no
 acceptance; the cache lengths and emitted counters after the run.
-
-Opt-in (PIPO_TEST_REGULAR=1) until the mode is part of the default suite.
 """
-import os
 
 import numpy as np
 import pytest
@@ -18,9 +15,7 @@ from oracle import oracle as O
 from paper_2605_27255_gb300 import capi, synth
 from parity_util import MARGIN, tol_for
 
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skipif(os.environ.get("PIPO_TEST_REGULAR") != "1",
-                                 reason="regular-decoding GPU tests run with PIPO_TEST_REGULAR=1")]
+pytestmark = pytest.mark.gpu
 
 SMALL_BF16 = synth.ModelShape("reg-bf16", H=512, L=2, n_q=8, n_kv=2, d_h=128, F=1408, V=4096,
                               compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1.0e6, tau=0.5)

@@ -2,19 +2,14 @@
 [a;b])) on the GPU against the oracle, with forced replay: the CUDA-core
 (B = 1) and tensor-core (B = 4) projections, position-by-position and
 chunked prefill.
-
-Opt-in (PIPO_TEST_RESIDUAL=1) until it has run on a GB300.
 """
-import os
 
 import pytest
 
 from paper_2605_27255_gb300 import synth
 from parity_util import run_forced_replay
 
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skipif(os.environ.get("PIPO_TEST_RESIDUAL") != "1",
-                                 reason="residual-compressor GPU tests run with PIPO_TEST_RESIDUAL=1")]
+pytestmark = pytest.mark.gpu
 
 MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003,
                        compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1e6, tau=0.5, comp_residual=1)

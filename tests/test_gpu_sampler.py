@@ -7,10 +7,7 @@ x_b and x_d equal wherever the oracle's decision margin (orc_sample_ex)
 exceeds DELTA; the accept decision equal wherever |c - tau| > DELTA.  A
 decision inside the margin that comes out differently ends the comparison
 (the histories part there); the tests require enough positions compared.
-
-Opt-in (PIPO_TEST_SAMPLER=1) until the sampler is part of the default suite.
 """
-import os
 
 import numpy as np
 import pytest
@@ -19,9 +16,7 @@ from oracle import oracle as O
 from paper_2605_27255_gb300 import capi, synth
 from parity_util import tol_for
 
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skipif(os.environ.get("PIPO_TEST_SAMPLER") != "1",
-                                 reason="sampler GPU tests run with PIPO_TEST_SAMPLER=1")]
+pytestmark = pytest.mark.gpu
 
 PAPER = dict(temperature=1.0, top_k=20, top_p=0.95, rep_penalty=1.5)
 SMALL_BF16 = synth.ModelShape("samp-bf16", H=512, L=2, n_q=8, n_kv=2, d_h=128, F=1408, V=4096,

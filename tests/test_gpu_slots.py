@@ -2,10 +2,7 @@
 different prompt lengths in one batch, and a sequence joining a batch that is
 already decoding.  Each slot is checked against its own oracle sequence (a
 batch is B independent sequences), with forced replay of the pending pairs.
-
-Opt-in (PIPO_TEST_SLOTS=1) until the slot path has run on a GB300.
 """
-import os
 
 import numpy as np
 import pytest
@@ -14,9 +11,7 @@ from oracle import oracle as O
 from paper_2605_27255_gb300 import capi, synth
 from parity_util import Stats, compare, tol_for
 
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skipif(os.environ.get("PIPO_TEST_SLOTS") != "1",
-                                 reason="slot GPU tests run with PIPO_TEST_SLOTS=1")]
+pytestmark = pytest.mark.gpu
 
 MID = synth.ModelShape("mid", H=512, L=3, n_q=8, n_kv=2, d_h=128, F=1376, V=5003,
                        compressor="mlp", mtp_block=1, dtype="bf16", rope_theta=1e6, tau=0.5)

@@ -7,12 +7,23 @@ head + argmax, MTP head + argmax, confidence head, acceptance and the device
 bookkeeping.  Metric: accepted tokens/s over all sequences (1 + acceptance
 per sequence and step), with the pair-step latency and the HBM roofline.
 
-  python bench.py [--workload 4b-b1] [--steps K] [--warmup W] [--gpus N]
+  python bench.py [--workload 9b-b8] [--steps K] [--warmup W] [--gpus N]
   python bench.py --impl reference ...   # the fp64 CPU oracle on host cores
 
-Inputs are synthetic and seeded (weights and prompts from synth.py); weights
-are streamed from HBM every step (9.3 GB/step for 4B > 129 MB L2), so no L2
-flush is needed between steps.
+The default workload is the largest single-GPU configuration: 9B-class
+shapes at batch 8 with 4096-token prompts (20 GB moved per step).  Inputs are
+synthetic and seeded (weights and prompts from synth.py); weights are
+streamed from HBM every step (9-20 GB per step, far above the 129 MB L2), so
+no L2 flush is needed between steps.
+
+Roofline of the dominant kernel family (the weight-streaming projections):
+after the timed steps, a CUDA graph holding only the step's projection
+launches (same launch plan, step order and programmatic dependent launch) is
+replayed and timed with CUDA events on the context stream
+(pipo_replay_family); its algorithmic bytes per replay divided by its time
+give the achieved bandwidth.  DRAM traffic per launch comes from the ncu
+summary in profiles/ when its recorded source hash matches the kernels built
+here, else it is null.
 """
 from __future__ import annotations
 
@@ -52,14 +63,16 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=None)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", default="4b-b1", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="9b-b8", choices=sorted(WORKLOADS))
     ap.add_argument("--impl", default="pipo", choices=["pipo", "reference"])
     ap.add_argument("--tau", type=float, default=None)
     ap.add_argument("--force", type=int, default=0, help="0 rule, 1 accept all, 2 reject all")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
-    ap.add_argument("--profile-steps", type=int, default=8, help="eager steps timed per launch for the roofline")
-    ap.add_argument("--prefill-rows", type=int, default=0,
+    ap.add_argument("--family-replays", type=int, default=None,
+                    help="timed replays of the projection-only graph for the roofline (default: the step count, "
+                         "at most 256)")
+    ap.add_argument("--prefill-rows", type=int, default=128,
                     help="prefill in chunks of this many rows (positions x sequences, at most 128); "
                          "0: one position at a time")
     ap.add_argument("--sampler", action="store_true",
@@ -283,15 +296,16 @@ def run_regular(g, shape, wl, B, T, W, K, stream, seed):
 
 def make_line(m: dict) -> dict:
     """The benchmark's JSON line from the measured quantities of run_pipo
-    (device time over the timed steps, per-launch profile of the kernel
-    families, end-to-end loop, oracle baseline, clocks)."""
+    (device time over the timed steps, graph replays of the projection and
+    attention families, end-to-end loop, oracle baseline, clocks)."""
     K, B, hbm = m["steps"], m["batch"], m["hbm"]
-    step_gbs = m["step_bytes"] / (m["ms"] / 1e3 / K) / 1e9
-    gb, gms, gn = m["kb"][0]
-    ab, ams, _ = m["kb"][1]
-    tot_ms = sum(v[1] for v in m["kb"].values())
-    gemv_gbs = gb / (gms / 1e3) / 1e9 if gms > 0 else None
+    step_ms = m["ms"] / K
+    step_gbs = m["step_bytes"] / (step_ms / 1e3) / 1e9
+    fp, fa = m["fam"][0], m["fam"][1]
+    proj_gbs = fp["bytes"] / (fp["ms"] / 1e3) / 1e9 if fp["ms"] > 0 else None
+    attn_gbs = fa["bytes"] / (fa["ms"] / 1e3) / 1e9 if fa["ms"] > 0 else None
     acceptance = m["tokens"] / (K * B) - 1.0
+    tr = m.get("traffic") or {}
     line = {
         "metric": METRIC, "value": m["tokens_all"] / (m["ms_all"] / 1e3), "unit": "tokens/s",
         "n_gpus": m["n_gpus"], "steps": K, "warmup": m["warmup"], "ms_per_step": m["ms_all"] / K,
@@ -299,37 +313,42 @@ def make_line(m: dict) -> dict:
         "dtype": m["dtype"], "data": "synthetic (seeded weights and prompts)",
         "config": {"workload": m["workload"], "shape": m["shape_name"], "batch": B, "prompt_tokens": m["prompt_tokens"],
                    "context_entries_avg": m["ctx_avg"], "tau": m["tau"], "force_mode": m["force"],
-                   "acceptance": acceptance, "pair_step_us": 1e3 * m["ms"] / K,
+                   "acceptance": acceptance, "pair_step_us": 1e3 * step_ms,
                    "prefill_s": m["prefill_s"], "prefill_rows": m["prefill_rows"],
                    "heads": "sampled (T 1, top-k 20, top-p 0.95, penalty 1.5)" if m["sampler"] else "greedy",
                    "l2": "weights streamed per step (GBs) > 129 MB L2; no flush needed",
                    "parallelism": f"replicas x{m['n_gpus']}"},
         "roofline": {"bound": "hbm", "kernel": f"weight-streaming projections (every projection and both LM-head "
                                                   f"launches of a step): {m['desc']}",
-                     "achieved": gemv_gbs, "peak": hbm, "unit": "GB/s",
-                     "frac": (gemv_gbs / hbm) if gemv_gbs else None, "traffic": None,
-                     "algorithmic_bytes_per_launch": gb / max(1, gn), "avg_launch_us": 1e3 * gms / max(1, gn),
-                     "launches_per_step": gn // max(1, m["prof_steps"]),
-                     "share_of_step_time": gms / tot_ms if tot_ms else None,
-                     "timing": f"CUDA events around each launch, {m['prof_steps']} eagerly run steps after the timed "
-                               f"region",
+                     "achieved": proj_gbs, "peak": hbm, "unit": "GB/s",
+                     "frac": (proj_gbs / hbm) if proj_gbs else None,
+                     "traffic": tr.get("bytes_per_launch"),
+                     "traffic_source": tr.get("source"),
+                     "algorithmic_bytes_per_launch": fp["bytes"] / max(1, fp["launches"]),
+                     "avg_launch_us": 1e3 * fp["ms"] / max(1, fp["launches"]),
+                     "launches_per_step": fp["launches"],
+                     "family_ms_per_step": fp["ms"],
+                     "family_share_of_step": fp["ms"] / step_ms,
+                     "timing": f"CUDA events on the context stream around {fp['replays']} replays of a graph of "
+                               f"the step's projection launches alone (the step's launch plan, order and "
+                               f"programmatic dependent launch), right after the timed steps",
                      "peak_source": f"{m['peak_source']} (MEASURED_PEAKS.json hbm_gbs)",
                      "step": {"algorithmic_bytes": m["step_bytes"], "achieved": step_gbs, "frac": step_gbs / hbm,
                               "frac_of_nominal": step_gbs / NOMINAL_HBM_GBS},
-                     "attention": {"achieved": (ab / (ams / 1e3) / 1e9) if ams else None,
-                                   "share_of_step_time": ams / tot_ms if tot_ms else None}},
+                     "attention": {"achieved": attn_gbs, "frac": (attn_gbs / hbm) if attn_gbs else None,
+                                   "algorithmic_bytes_per_step": fa["bytes"], "launches_per_step": fa["launches"],
+                                   "family_ms_per_step": fa["ms"], "family_share_of_step": fa["ms"] / step_ms}},
         "cpu_baseline": m["cpu"],
         "e2e": {"value": m["e2e_tokens"] / m["e2e_s"], "unit": "tokens/s",
-                "h2d_bytes_per_step": 0 if m.get("e2e_loop") else B * 8, "d2h_bytes_per_step": B * 12,
-                "loop": m.get("e2e_loop") or
-                "host-driven: pipo_set_pending (pending pair from pinned host memory) + pipo_decode_step "
-                "(tokens and acceptances back), synchronous"},
+                "h2d_bytes_per_step": B * 8, "d2h_bytes_per_step": B * 12,
+                "loop": "host-driven: pipo_set_pending (pending pair from pinned host memory) + pipo_decode_step "
+                        "(tokens and acceptances back), synchronous"},
         "gpu_launches": m["launches"] * K,
         "clocks": m["clocks"],
     }
     regular = m.get("regular")
     if regular is not None:
-        pipo_tpot = (m["ms"] / K) / (1.0 + acceptance)
+        pipo_tpot = step_ms / (1.0 + acceptance)
         regular["tpot_ratio"] = regular["ms_per_token"] / pipo_tpot
         regular["frac"] = regular["achieved_gbs"] / hbm
         # time to first token on the same prompt: T tokens as T positions against T / 2 pairs (both warm)
@@ -337,6 +356,20 @@ def make_line(m: dict) -> dict:
             if regular["prefill_s"] and regular["pipo_prefill_warm_s"] else None
         line["regular"] = regular
     return line
+
+
+def time_family(g, family, n, stream):
+    """CUDA-event time of one replay of a kernel family's graph (ms), with its
+    algorithmic bytes and launches per replay."""
+    import torch
+    by, nl = g.replay_family(family, 3)  # capture + warm-up
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    g.replay_family(family, n)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    return {"ms": ev0.elapsed_time(ev1) / n, "bytes": by, "launches": nl, "replays": n}
 
 
 def run_pipo(args):
@@ -357,7 +390,7 @@ def run_pipo(args):
     K = args.steps if args.steps is not None else wl["steps"]
     W = max(3, args.warmup)
     n_pairs = (T + 1) // 2
-    max_ctx = n_pairs + W + 2 * K + args.profile_steps + 8
+    max_ctx = n_pairs + W + 2 * K + 8
     if args.regular:
         max_ctx = max(max_ctx, T + W + K + 8)  # regular decoding: one cache entry per token
 
@@ -374,7 +407,7 @@ def run_pipo(args):
     g.set_stream(stream.cuda_stream)
     if args.sampler:
         # draws for every position that runs the heads (prefill, warm-up, timed, e2e, profile steps)
-        n_u = 1 + W + 2 * K + args.profile_steps + 8
+        n_u = 1 + W + 2 * K + 8
         u = np.random.default_rng(11 + rank).random((n_u, B, 2)).astype(np.float32)
         g.set_sampler(u, temperature=1.0, top_k=20, top_p=0.95, rep_penalty=1.5)
 
@@ -426,30 +459,20 @@ def run_pipo(args):
     e2e_check(lib.pipo_decode_step(g.ctx, tok_p, nacc_p))  # untimed: the first pair on the host
     _, e2a = g.counters()
     torch.cuda.synchronize()
-    e2e_loop = None  # host-driven unless pipo_set_pending refuses a pair (then device-driven, reported)
     t0 = time.perf_counter()
     for _ in range(K):
-        if e2e_loop is None:
-            rc = lib.pipo_set_pending(g.ctx, tok_p)
-            if rc != 0:
-                e2e_loop = f"device-driven (pipo_set_pending: {capi.pipo_last_error(g.ctx)})"
+        # a refused pair means the previous step returned an id outside [0, V): a failed run
+        e2e_check(lib.pipo_set_pending(g.ctx, tok_p))
         e2e_check(lib.pipo_decode_step(g.ctx, tok_p, nacc_p))
     e2e_s = time.perf_counter() - t0
     _, e2b = g.counters()
     e2e_tokens = int((e2b - e2a).sum())
     launches = g.launches()
     desc = g.describe()
-    # dominant kernel: per-launch CUDA-event timings of eagerly run steps
-    prof_steps = max(1, min(K, args.profile_steps))
-    kb = {0: [0.0, 0.0, 0], 1: [0.0, 0.0, 0], 2: [0.0, 0.0, 0]}
-    for _ in range(prof_steps):
-        torch.cuda.nvtx.range_push("profile_step")  # ncu --nvtx-include "profile_step/" selects these launches
-        kind, by, pms = g.profile_step()
-        torch.cuda.nvtx.range_pop()
-        for kk, bb, mm in zip(kind, by, pms):
-            kb[int(kk)][0] += float(bb)
-            kb[int(kk)][1] += float(mm)
-            kb[int(kk)][2] += 1
+    # the projection family and the attention family of the same step, each a
+    # graph of its own launches replayed back to back (decode state unchanged)
+    n_rep = args.family_replays or max(8, min(K, 256))
+    fam = {0: time_family(g, 0, n_rep, stream), 1: time_family(g, 1, n_rep, stream)}
     regular = run_regular(g, shape, wl, B, T, W, K, stream, 1 + rank * 1000) if args.regular else None
 
     ms_all, tokens_all, e2e_all, e2e_tok_all = aggregate_ranks(ms, tokens, e2e_s, e2e_tokens, "cuda")
@@ -474,9 +497,10 @@ def run_pipo(args):
     line = make_line(dict(
         workload=args.workload, shape_name=wl["shape"], dtype=shape.dtype, n_gpus=ws, steps=K, warmup=W, batch=B,
         prompt_tokens=T, ms=ms, ms_all=ms_all, tokens=tokens, tokens_all=tokens_all, ctx_avg=ctx_avg, tau=tau,
-        force=args.force, prefill_s=t_pf, prefill_rows=args.prefill_rows, sampler=args.sampler, desc=desc, kb=kb,
-        prof_steps=prof_steps, hbm=hbm, peak_source=src, step_bytes=roofline.step_bytes(shape, B, ctx_avg),
-        cpu=cpu, e2e_s=e2e_all, e2e_tokens=e2e_tok_all, e2e_loop=e2e_loop, launches=launches,
+        force=args.force, prefill_s=t_pf, prefill_rows=args.prefill_rows, sampler=args.sampler, desc=desc, fam=fam,
+        hbm=hbm, peak_source=src, step_bytes=roofline.step_bytes(shape, B, ctx_avg),
+        traffic=roofline.recorded_traffic(os.path.join(ROOT, "profiles"), args.workload),
+        cpu=cpu, e2e_s=e2e_all, e2e_tokens=e2e_tok_all, launches=launches,
         clocks=clk.summary(), regular=regular))
     print(json.dumps(line), flush=True)
     g.close()

@@ -120,11 +120,18 @@ typedef struct {
     int32_t *x_d;      /* [B] draft argmax (whether accepted or not), or NULL */
 } pipo_debug;
 
-/* Create a context on the current CUDA device: validates the config, copies
- * the weights to device memory (fused QKV and gate|up layouts), allocates the
- * paged KV caches (backbone layers and the MTP layer) for max_batch x max_ctx
- * entries.  *out receives the context.  EINVAL for inconsistent shapes,
- * ENOMEM when device memory runs out. */
+/* Create a context on the current CUDA device for one PIPO model: the latent
+ * compressor (Sec. 3.2 Eq. 1, App. A.1), the backbone decoder blocks (Eq. 2),
+ * the tied LM head (Eq. 3, App. B.2), the MTP head (Eq. 4-5, App. A.2) and
+ * the confidence head (Eq. 6, App. A.3), with the shapes in cfg.  Validates
+ * the config, copies the weights to device memory (fused QKV and gate|up
+ * layouts), allocates the paged KV caches (backbone layers and the MTP
+ * layer) for max_batch x max_ctx entries.  *out receives the context.
+ * EINVAL for inconsistent shapes or a missing weight tensor, ENOMEM when
+ * device memory runs out (everything allocated so far is freed and *out is
+ * left NULL).  For tests of that path, the environment variable
+ * PIPO_TEST_FAIL_ALLOC=k makes the k-th device allocation of this call
+ * report out-of-memory without allocating. */
 PIPO_API pipo_status pipo_init(const pipo_config *cfg, const pipo_weights *w, pipo_ctx **out);
 
 /* Prefill B sequences (B <= max_batch) from host token ids h_ids, row b at
@@ -135,7 +142,9 @@ PIPO_API pipo_status pipo_init(const pipo_config *cfg, const pipo_weights *w, pi
  * the first pair output, which also becomes the pending pair.  Resets the
  * emitted counters.  ECAPACITY when N > max_ctx.  Sequences that yield
  * different numbers of pairs are prefilled one after another, each as
- * pipo_prefill_slot does (all are validated first). */
+ * pipo_prefill_slot does (all are validated first).  On any failure the
+ * context is left not prefilled (a decode step returns ESTATE until the next
+ * successful prefill). */
 PIPO_API pipo_status pipo_prefill(pipo_ctx *ctx, int32_t batch, const int32_t *h_ids, int32_t stride,
                          const int32_t *h_lens, int32_t *h_tokens, int32_t *h_n_accepted);
 
@@ -208,7 +217,11 @@ PIPO_API pipo_status pipo_regular_step_async(pipo_ctx *ctx, int32_t *d_tokens);
  * The pending pair is left as is (set it with pipo_set_pending). */
 PIPO_API pipo_status pipo_rollback(pipo_ctx *ctx, const int32_t *h_n_pairs);
 
-/* Acceptance threshold and force mode (0 rule, 1 accept all, 2 reject all). */
+/* Acceptance threshold tau_c of the confidence rule (Sec. 3.1-3.2: the draft
+ * is kept when c >= tau_c) and the force mode: 0 the rule; 1 accept every
+ * draft, which is the "MTP without verification" baseline of App. C.2; 2
+ * reject every draft (one token per pair, Sec. 3.1).  Takes effect from the
+ * next step.  EINVAL for a mode outside 0..2 or a tau that is not finite. */
 PIPO_API pipo_status pipo_set_threshold(pipo_ctx *ctx, float tau, int32_t force_mode);
 
 /* The paper's evaluation sampler in both heads (Sec. 4; its settings:
@@ -241,7 +254,11 @@ PIPO_API pipo_status pipo_set_pending(pipo_ctx *ctx, const int32_t *h_pairs);
  * emitted since the prefill [B] (either may be NULL). */
 PIPO_API pipo_status pipo_get_counters(pipo_ctx *ctx, int32_t *h_kv_len, int64_t *h_emitted);
 
-/* Head states of the last step or prefill (requires cfg.debug = 1). */
+/* Head states of the last step or prefill, for parity checks of Eq. 3-6:
+ * the LM-head logits of both heads (Eq. 3 and Eq. 5), the confidence c
+ * (Eq. 6), h_b and h_d (the block outputs the heads read, App. A.2-A.3) and
+ * both argmax tokens.  Requires cfg.debug = 1 (ESTATE otherwise); host
+ * buffers in *out, any of them NULL to skip. */
 PIPO_API pipo_status pipo_debug_dump(pipo_ctx *ctx, const pipo_debug *out);
 
 /* Host fp32 copy of cache entries [0, n) of sequence b, layer l (l == L is
@@ -306,6 +323,31 @@ PIPO_API pipo_status pipo_op_gemm_tc(int32_t mode, const void *d_W, int32_t N, i
  * arguments it rejects or when no device is usable). */
 PIPO_API size_t pipo_op_gemm_tc_scratch(int32_t mode, int32_t N, int32_t K, int32_t B, int32_t splits);
 
+/* The tensor-core projection of RMS-normalised inputs, as the decode step
+ * applies it: to RMSNorm(x; gamma) in the blocks (Eq. 2, pre-norm), to
+ * [RMSNorm(h_b); RMSNorm(E[x_b])] with two gains at the MTP input (App. A.2)
+ * and to RMSNorm([h_b; h_d]) with one gain over 2H in the confidence head
+ * (App. A.3).  The input of sequence b is the concatenation of
+ *   segment 0: x0[b*K0 .. b*K0 + K0)   and, when d_x1 != NULL,
+ *   segment 1: x1[b*K1 .. b*K1 + K1)   (K = K0 + K1; else K1 must be 0),
+ * normalised as follows (r(v) = v / sqrt(mean(v^2) + eps)):
+ *   joint = 0: each segment with a non-NULL gain becomes gamma_s * r(segment),
+ *              a segment with a NULL gain enters unchanged;
+ *   joint = 1: both segments together become gamma0 * r(concatenation),
+ *              gamma0 of length K, d_gamma1 NULL.
+ * Then y = W . input as pipo_op_gemm_tc (mode 0 plain, mode 1 SwiGLU).
+ * Gains bf16, W bf16; x0, x1, y fp32; W, x0, x1 and the gains 16-byte
+ * aligned; K0 and K1 multiples of 64; N, B, splits and the scratch
+ * (pipo_op_gemm_tc_scratch(mode, N, K0 + K1, B, splits) bytes, 1024-byte
+ * aligned) as pipo_op_gemm_tc.  B <= 32 with one segment or one joint norm
+ * runs the converter warps inside the GEMM when B is 16 or 32; every other
+ * case prepares the bf16 operand in a separate pass first.  EINVAL for bad
+ * shapes, alignment, gain combinations or a short scratch buffer. */
+PIPO_API pipo_status pipo_op_gemm_tc_norm(int32_t mode, const void *d_W, int32_t N, const float *d_x0, int32_t K0,
+                                          const void *d_gamma0, const float *d_x1, int32_t K1, const void *d_gamma1,
+                                          int32_t joint, float eps, int32_t B, float *d_y, int32_t splits,
+                                          void *d_scratch, size_t scratch_bytes, void *stream);
+
 /* Fused LM head + argmax over the tied embedding (Eq. 3 and Eq. 5, App. B.2):
  *   d_tokens[b] = argmax_v  E[v,:] . RMSNorm(h[b,:]; gamma)
  * with the lowest v winning ties; the logits are never stored unless
@@ -331,7 +373,10 @@ PIPO_API pipo_status pipo_op_lm_head_argmax(int32_t dtype, const void *d_E, int3
  * current; make that first call before any stream capture.  Every call on a
  * device shares the one array and zeroes it first, so calls that overlap on
  * the GPU (other streams, or other host threads) race and must be
- * serialized by the caller.  Arguments otherwise as pipo_op_lm_head_argmax. */
+ * serialized by the caller.  The looked-up address is kept for the life of
+ * the process: after cudaDeviceReset (or anything else that destroys the
+ * device's primary context) the entry point must not be called again on that
+ * device.  Arguments otherwise as pipo_op_lm_head_argmax. */
 PIPO_API pipo_status pipo_op_lm_head_argmax_noalloc(int32_t dtype, const void *d_E, int32_t V, int32_t H,
                                                     const float *d_h, const void *d_gamma, float eps, int32_t B,
                                                     int32_t *d_tokens, float *d_logits, void *stream);
@@ -345,6 +390,44 @@ PIPO_API pipo_status pipo_op_lm_head_argmax_noalloc(int32_t dtype, const void *d
  * Advances the decode state exactly like pipo_decode_step. */
 PIPO_API pipo_status pipo_profile_step(pipo_ctx *ctx, int32_t cap, int32_t *h_kind, double *h_bytes, float *h_ms,
                                        int32_t *h_n);
+
+/* Roofline timing of one kernel family inside the decode step: enqueues, on
+ * the context stream, n replays of a CUDA graph holding only that family's
+ * launches of one pair-decode step (Sec. 3.2 Eq. 1-6), with the step's launch
+ * plan, in step order and with the step's programmatic dependent launch
+ * between consecutive launches.  family 0: the weight-streaming projections
+ * (every projection of Eq. 1-6 and both LM-head passes, Eq. 3 and Eq. 5,
+ * with the operand preparation some of them need); family 1: the attention
+ * launches (Eq. 2).  Time the replays with events on the context stream.
+ * The decoding state does not change: pending pairs, cache lengths,
+ * counters and every live cache entry stay as they were (an attention
+ * replay writes only the entry one past each sequence's cached length, which
+ * the next step overwrites before reading it); the activation buffers are
+ * left with meaningless values.  *h_bytes receives the algorithmic bytes
+ * one replay moves (weights streamed; for attention the cached entries read
+ * and the one written), *h_launches its launch count (either may be NULL).
+ * The graph is captured on the first call for a family and batch (n = 0
+ * captures without replaying).  EINVAL for a bad family or n < 0; ESTATE
+ * before a prefill or on a regular-decoding context.  A measurement aid of
+ * this library; the paper has no counterpart. */
+PIPO_API pipo_status pipo_replay_family(pipo_ctx *ctx, int32_t family, int32_t n, double *h_bytes,
+                                        int32_t *h_launches);
+
+/* Self-test of the bounded device waits that every kernel of this library
+ * uses (mbarrier waits give up after a time limit instead of spinning
+ * forever, set a device error word and record the wait site; the host then
+ * reports PIPO_ECUDA).  Launches one block on the legacy default stream of the
+ * current device whose thread 0 waits, with a limit of limit_ns
+ * nanoseconds, on an mbarrier that only it can complete: signal != 0
+ * completes it first (PIPO_OK expected), signal == 0 never does, so the
+ * wait gives up after limit_ns and the call returns PIPO_ECUDA.
+ * h_info[4] (host, may be NULL) receives the wait record {site (90 for this
+ * test), block, iteration, parity}, zeros when nothing timed out.  Reads and
+ * clears the error word of the tensor-core unit, so run it while no other
+ * work of this library is in flight on the device.  EINVAL for a limit of
+ * 0 or above 10 s.  A reliability aid of this library; the paper has no
+ * counterpart. */
+PIPO_API pipo_status pipo_selftest_wait(int32_t signal, uint64_t limit_ns, uint32_t *h_info);
 
 /* Which kernels the next decode step launches for the projections and the
  * attention, and the attention cluster size, as one NUL-terminated line of
@@ -360,8 +443,10 @@ PIPO_API pipo_status pipo_describe_step(const pipo_ctx *ctx, char *h_buf, size_t
 /* Number of kernel launches one decode step enqueues (for launch accounting). */
 PIPO_API int32_t pipo_step_launches(const pipo_ctx *ctx);
 
-/* Message of the last failure on this context (or of the last failed
- * pipo_init when ctx is NULL); never NULL. */
+/* Message of the last failure on this context; with ctx NULL, of the last
+ * failed call made without a context (pipo_init, the pipo_op_* entry points)
+ * on the calling thread.  Never NULL; the string stays valid until the next
+ * failing call on the same context (ctx NULL: on the same thread). */
 PIPO_API const char *pipo_last_error(const pipo_ctx *ctx);
 
 /* Release every device buffer and the context; NULL is a no-op. */

@@ -100,7 +100,12 @@ SIGNATURES = {
     "pipo_op_gemm_tc": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_int32, C.c_void_p,
                                   C.c_int32, C.c_void_p, C.c_size_t, C.c_void_p]),
     "pipo_op_gemm_tc_scratch": (C.c_size_t, [C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32]),
+    "pipo_op_gemm_tc_norm": (C.c_int, [C.c_int32, C.c_void_p, C.c_int32, C.c_void_p, C.c_int32, C.c_void_p,
+                                       C.c_void_p, C.c_int32, C.c_void_p, C.c_int32, C.c_float, C.c_int32,
+                                       C.c_void_p, C.c_int32, C.c_void_p, C.c_size_t, C.c_void_p]),
     "pipo_describe_step": (C.c_int, [C.c_void_p, C.c_char_p, C.c_size_t]),
+    "pipo_replay_family": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.POINTER(C.c_double), _IP]),
+    "pipo_selftest_wait": (C.c_int, [C.c_int32, C.c_uint64, C.POINTER(C.c_uint32)]),
     "pipo_profile_step": (C.c_int, [C.c_void_p, C.c_int32, _IP, C.POINTER(C.c_double), _FP, _IP]),
     "pipo_step_launches": (C.c_int32, [C.c_void_p]),
     "pipo_last_error": (C.c_char_p, [C.c_void_p]),
@@ -297,6 +302,25 @@ def pipo_op_gemm_tc(mode: int, W: int, N: int, K: int, x: int, B: int, y: int, s
                                   C.c_void_p(scratch), scratch_bytes, C.c_void_p(stream or None)), None)
 
 
+def pipo_op_gemm_tc_norm(mode: int, W: int, N: int, x0: int, K0: int, gamma0: int, x1: int, K1: int, gamma1: int,
+                         joint: int, eps: float, B: int, y: int, splits: int, scratch: int, scratch_bytes: int,
+                         stream: int = 0) -> None:
+    """Tensor-core projection of RMS-normalised segments on device pointers
+    (ints, 0 for NULL); see include/pipo.h."""
+    _check(load().pipo_op_gemm_tc_norm(mode, C.c_void_p(W or None), N, C.c_void_p(x0 or None), K0,
+                                       C.c_void_p(gamma0 or None), C.c_void_p(x1 or None), K1,
+                                       C.c_void_p(gamma1 or None), joint, eps, B, C.c_void_p(y or None), splits,
+                                       C.c_void_p(scratch or None), scratch_bytes, C.c_void_p(stream or None)), None)
+
+
+def pipo_selftest_wait(signal: int, limit_ns: int):
+    """Bounded-wait self-test (see include/pipo.h): returns (status, message,
+    wait record [site, block, iteration, parity]) without raising."""
+    info = (C.c_uint32 * 4)()
+    st = load().pipo_selftest_wait(signal, limit_ns, info)
+    return st, pipo_last_error(None), list(info)
+
+
 def pipo_op_lm_head_argmax_noalloc(dtype: int, E: int, V: int, H: int, h: int, gamma: int, eps: float, B: int,
                                    tokens: int, logits: int, stream: int = 0) -> None:
     """The LM-head argmax for callers that cannot allocate device memory: no
@@ -460,3 +484,10 @@ class Pipo:
 
     def profile_step(self):
         return pipo_profile_step(self.ctx)
+
+    def replay_family(self, family: int, n: int):
+        """Enqueue n replays of one kernel family of the step (pipo_replay_family);
+        returns (algorithmic bytes per replay, launches per replay)."""
+        by, nl = C.c_double(), C.c_int32()
+        _check(load().pipo_replay_family(self.ctx, family, n, C.byref(by), C.byref(nl)), self.ctx)
+        return by.value, nl.value

@@ -45,4 +45,23 @@ void* k_pick_prep_bf16() { return reinterpret_cast<void*>(&prep_bf16_kernel<__nv
 
 cudaError_t k_take_error_tc(unsigned* code, unsigned* info) { return take_unit_error(code, info); }
 
+// Self-test of the bounded wait (site 90): thread 0 waits, with a limit of
+// limit_ns, on an mbarrier of one arrival that it completes itself only when
+// `signal` is set.  Unsignalled, the wait must give up after limit_ns, set
+// the error word, record the site and return: the kernel always ends.
+__global__ void wait_selftest_kernel(int signal, unsigned long long limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        mbar_init_fence();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        if (signal) mbar_arrive(&bar);
+        mbar_wait(&bar, 0, 90, 0, limit_ns);
+    }
+}
+
+void* k_pick_wait_selftest() { return reinterpret_cast<void*>(&wait_selftest_kernel); }
+
 }  // namespace pipo

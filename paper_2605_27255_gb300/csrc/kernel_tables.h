@@ -24,6 +24,7 @@ cudaError_t k_take_error_gemv_f32(unsigned* code, unsigned* info);
 void* k_pick_tcv(int bh, bool deep, bool fused);    // gemm_tcf_kernel (fused) / gemm_tc_kernel
 void* k_pick_prep_bf16();                           // prep_bf16_kernel<bf16>
 cudaError_t k_take_error_tc(unsigned* code, unsigned* info);
+void* k_pick_wait_selftest();                       // wait_selftest_kernel (reports through k_take_error_tc)
 
 // k_attn.cu: attention and RoPE / append kernels
 void* k_pick_attn_decode(bool bf, int DH, int G);   // attn_decode_kernel

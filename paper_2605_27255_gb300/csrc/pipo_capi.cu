@@ -81,7 +81,10 @@ __global__ void regular_accept_kernel(StepState st, int H, const float* h) {
 
 namespace {
 
-std::string g_init_error = "no error";
+// message of the last failure of a call made without a context (pipo_init,
+// the pipo_op_* entry points) on this thread: thread-local, so that threads
+// failing at once neither race on it nor free a string another one returns
+thread_local std::string g_init_error = "no error";
 
 struct BlockW {
     void *attn_norm = nullptr, *Wqkv = nullptr, *Wo = nullptr, *ffn_norm = nullptr, *Wgu = nullptr, *Wdown = nullptr;
@@ -164,6 +167,18 @@ struct pipo_ctx {
     std::vector<int> prof_k;
     std::vector<double> prof_b;
     size_t prof_n = 0;
+    // one kernel family of the decode step alone (pipo_replay_family)
+    int only_family = -1;             // while capturing: launches of other families are not enqueued
+    bool launch_prep = false;         // the next launch prepares a projection's operand (family 0)
+    double fam_bytes = 0.0;           // algorithmic bytes of the captured family's launches
+    int fam_launches = 0;
+    cudaGraphExec_t fam_graph = nullptr;
+    int fam_graph_family = -1, fam_graph_B = -1;
+
+    // host-side fault injection (PIPO_TEST_FAIL_ALLOC=k): the k-th device
+    // allocation of pipo_init reports out-of-memory without calling cudaMalloc
+    int fail_alloc_at = 0;
+    int n_dalloc = 0;
 
     int B = 0;
     int rows = 0;                     // activation rows of the enqueue in progress (0: B, one per sequence)
@@ -211,6 +226,9 @@ pipo_status fail(pipo_ctx* c, pipo_status s, const char* fmt, ...) {
 
 template <typename P>
 pipo_status dalloc(pipo_ctx* ctx, P** p, size_t bytes) {
+    if (ctx->fail_alloc_at > 0 && ++ctx->n_dalloc == ctx->fail_alloc_at)
+        return fail(ctx, PIPO_ENOMEM, "cudaMalloc(%zu bytes): injected failure of device allocation %d", bytes,
+                    ctx->n_dalloc);
     void* q = nullptr;
     cudaError_t e = cudaMalloc(&q, bytes ? bytes : 16);
     if (e != cudaSuccess) {
@@ -294,6 +312,19 @@ constexpr size_t kStreamBudget = 200 * 1024;  // staged-input bytes per streamin
 // cluster dimension.
 pipo_status launch_ex(pipo_ctx* ctx, const void* fn, dim3 grid, dim3 block, size_t smem, void** args,
                       int cluster_x = 1) {
+    if (ctx->only_family >= 0) {
+        // family capture: keep the launches of one family, in step order
+        const int fam = ctx->launch_prep ? 0 : ctx->prof_kind;
+        const bool keep = fam == ctx->only_family;
+        if (keep) {
+            ctx->fam_bytes += ctx->prof_bytes;
+            ctx->fam_launches++;
+        }
+        ctx->prof_kind = 2;
+        ctx->prof_bytes = 0.0;
+        ctx->launch_prep = false;
+        if (!keep) return PIPO_OK;
+    }
     cudaLaunchConfig_t lc = {};
     lc.gridDim = grid;
     lc.blockDim = block;
@@ -329,9 +360,11 @@ pipo_status launch_ex(pipo_ctx* ctx, const void* fn, dim3 grid, dim3 block, size
         ctx->prof_k.push_back(ctx->prof_kind);
         ctx->prof_b.push_back(ctx->prof_bytes);
         ctx->prof_n++;
-        ctx->prof_kind = 2;
-        ctx->prof_bytes = 0.0;
     }
+    // the kind and bytes describe one launch: callers set them before it
+    ctx->prof_kind = 2;
+    ctx->prof_bytes = 0.0;
+    ctx->launch_prep = false;
     ctx->launches++;
     return PIPO_OK;
 }
@@ -629,6 +662,7 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
         void* args[] = {&pp, &xb, &bh};
         ctx->prof_kind = 2;
         ctx->prof_bytes = 0.0;
+        ctx->launch_prep = true;
         TRY(launch_ex(ctx, reinterpret_cast<const void*>(k_pick_prep_bf16()), dim3(bn), dim3(kPrepThreads), 0,
                       args));
     }
@@ -1313,6 +1347,9 @@ void drop_graph(pipo_ctx* ctx) {
     if (ctx->graph) cudaGraphExecDestroy(ctx->graph);
     ctx->graph = nullptr;
     ctx->graph_B = -1;
+    if (ctx->fam_graph) cudaGraphExecDestroy(ctx->fam_graph);
+    ctx->fam_graph = nullptr;
+    ctx->fam_graph_B = -1;
 }
 
 void* mk_pick(bool bf, int nb, int DH, int G) { return k_pick_step_kernel(bf, nb, DH, G); }
@@ -1532,6 +1569,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
     ctx = new pipo_ctx();
     ctx->cfg = c;
     ctx->esz = c.dtype == 1 ? 2 : 4;
+    if (const char* ev = getenv("PIPO_TEST_FAIL_ALLOC")) ctx->fail_alloc_at = std::max(0, atoi(ev));
     pipo_status s = [&]() -> pipo_status {
         CK(cudaGetDevice(&ctx->dev));
         CK(cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, ctx->dev));
@@ -1684,6 +1722,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         CK(cudaDeviceSynchronize());
         return PIPO_OK;
     }();
+    ctx->fail_alloc_at = 0;  // the injection covers pipo_init only
     if (s != PIPO_OK) {
         g_init_error = ctx->err;
         pipo_free(ctx);
@@ -1704,7 +1743,7 @@ pipo_status pipo_set_stream(pipo_ctx* ctx, void* stream) {
 
 pipo_status pipo_set_threshold(pipo_ctx* ctx, float tau, int32_t force_mode) {
     if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
-    if (force_mode < 0 || force_mode > 2 || !(tau == tau)) return fail(ctx, PIPO_EINVAL, "bad threshold or force mode");
+    if (force_mode < 0 || force_mode > 2 || !std::isfinite(tau)) return fail(ctx, PIPO_EINVAL, "bad threshold or force mode");
     if (ctx->cfg.tau != tau || ctx->cfg.force_mode != force_mode) drop_graph(ctx);
     ctx->cfg.tau = tau;
     ctx->cfg.force_mode = force_mode;
@@ -1827,9 +1866,18 @@ pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int
             ctx->prefilled = false;
             ctx->B = 0;
             ctx->h_len.clear();
-            for (int b = 0; b < batch; ++b)
-                TRY(pipo_prefill_slot(ctx, b, h_ids + (size_t)b * stride, h_lens[b], h_tokens ? h_tokens + 2 * b : nullptr,
-                                      h_n_accepted ? h_n_accepted + b : nullptr));
+            for (int b = 0; b < batch; ++b) {
+                const pipo_status st = pipo_prefill_slot(ctx, b, h_ids + (size_t)b * stride, h_lens[b],
+                                                         h_tokens ? h_tokens + 2 * b : nullptr,
+                                                         h_n_accepted ? h_n_accepted + b : nullptr);
+                if (st != PIPO_OK) {
+                    // no partial batch: the context is left not prefilled (decode steps return ESTATE)
+                    ctx->prefilled = false;
+                    ctx->B = 0;
+                    ctx->h_len.clear();
+                    return st;
+                }
+            }
             return PIPO_OK;
         }
     }
@@ -2371,6 +2419,100 @@ pipo_status pipo_op_gemm_tc(int32_t mode, const void* d_W, int32_t N, int32_t K,
     }
     if (st != PIPO_OK) g_init_error = op.err;
     return st;
+}
+
+pipo_status pipo_op_gemm_tc_norm(int32_t mode, const void* d_W, int32_t N, const float* d_x0, int32_t K0,
+                                 const void* d_gamma0, const float* d_x1, int32_t K1, const void* d_gamma1,
+                                 int32_t joint, float eps, int32_t B, float* d_y, int32_t splits, void* d_scratch,
+                                 size_t scratch_bytes, void* stream) {
+    const bool two = d_x1 != nullptr;
+    const int32_t K = K0 + (two ? K1 : 0);
+    auto a16 = [](const void* q) { return reinterpret_cast<uintptr_t>(q) % 16 == 0; };
+    const bool segs_ok = K0 >= kTcBK && K0 % kTcBK == 0 && (two ? (K1 >= kTcBK && K1 % kTcBK == 0) : K1 == 0) &&
+                         (!joint || (two && d_gamma0 && !d_gamma1)) && (two || !d_gamma1) && eps >= 0.f;
+    if (!d_W || !d_x0 || !d_y || !d_scratch || !segs_ok || !tc_op_args_ok(mode, N, K, B, splits) || !a16(d_W) ||
+        !a16(d_x0) || (two && !a16(d_x1)) || !a16(d_gamma0) || !a16(d_gamma1) ||
+        reinterpret_cast<uintptr_t>(d_scratch) % 1024 != 0)
+        return fail(nullptr, PIPO_EINVAL, "pipo_op_gemm_tc_norm: bad arguments");
+    static thread_local pipo_ctx op;  // device facts and launch settings only; owns no memory
+    pipo_ctx* ctx = &op;
+    pipo_status st = op_setup(op, 1, stream);
+    if (st == PIPO_OK) {
+        const size_t need = tc_scratch_bytes(K, B);
+        if (scratch_bytes < need) {
+            st = fail(ctx, PIPO_EINVAL, "pipo_op_gemm_tc_norm: scratch needs %zu bytes, got %zu", need, scratch_bytes);
+        } else {
+            GemvParams p{};
+            p.W = d_W; p.N = N; p.K = K; p.epi = mode == 1 ? EPI_SWIGLU : EPI_STORE;
+            p.y = d_y; p.ldy = N; p.B = B; p.splitk = 1; p.eps = eps;
+            p.nseg = two ? 2 : 1;
+            p.joint_norm = joint ? 1 : 0;
+            p.seg[0] = act_seg(d_x0, K0, K0, d_gamma0);
+            if (two) p.seg[1] = act_seg(d_x1, K1, K1, d_gamma1);
+            st = launch_gemm_tc(ctx, p, static_cast<bf16*>(d_scratch), splits, B);
+        }
+    }
+    if (st != PIPO_OK) g_init_error = op.err;
+    return st;
+}
+
+pipo_status pipo_replay_family(pipo_ctx* ctx, int32_t family, int32_t n, double* h_bytes, int32_t* h_launches) {
+    if (!ctx || family < 0 || family > 1 || n < 0) return fail(ctx, PIPO_EINVAL, "pipo_replay_family: bad arguments");
+    if (!ctx->prefilled) return fail(ctx, PIPO_ESTATE, "family replay before prefill");
+    if (ctx->regular) return fail(ctx, PIPO_ESTATE, "family replay of a regular-decoding context");
+    CK(cudaSetDevice(ctx->dev));
+    if (!ctx->fam_graph || ctx->fam_graph_family != family || ctx->fam_graph_B != ctx->B) {
+        if (ctx->fam_graph) cudaGraphExecDestroy(ctx->fam_graph);
+        ctx->fam_graph = nullptr;
+        // the step's launch plan, captured with the other families' launches left out
+        const int launches_before = ctx->launches;
+        cudaGraph_t g = nullptr;
+        CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
+        ctx->only_family = family;
+        ctx->fam_bytes = 0.0;
+        ctx->fam_launches = 0;
+        ctx->pdl = true;
+        pipo_status s = enqueue_step(ctx);
+        ctx->pdl = false;
+        ctx->only_family = -1;
+        ctx->launches = launches_before;
+        cudaError_t e = cudaStreamEndCapture(ctx->stream, &g);
+        if (s != PIPO_OK) {
+            if (g) cudaGraphDestroy(g);
+            return s;
+        }
+        if (e != cudaSuccess) return fail(ctx, PIPO_ECUDA, "family capture: %s", cudaGetErrorString(e));
+        e = cudaGraphInstantiate(&ctx->fam_graph, g, 0);
+        cudaGraphDestroy(g);
+        if (e != cudaSuccess) return fail(ctx, PIPO_ECUDA, "family instantiate: %s", cudaGetErrorString(e));
+        ctx->fam_graph_family = family;
+        ctx->fam_graph_B = ctx->B;
+    }
+    for (int i = 0; i < n; ++i) CK(cudaGraphLaunch(ctx->fam_graph, ctx->stream));
+    if (h_bytes) *h_bytes = ctx->fam_bytes;
+    if (h_launches) *h_launches = ctx->fam_launches;
+    return PIPO_OK;
+}
+
+pipo_status pipo_selftest_wait(int32_t signal, uint64_t limit_ns, uint32_t* h_info) {
+    if (limit_ns == 0 || limit_ns > 10000000000ull)
+        return fail(nullptr, PIPO_EINVAL, "pipo_selftest_wait: limit must be in (0, 10 s]");
+    pipo_ctx* ctx = nullptr;  // failures go to the thread's context-free message
+    unsigned code = 0, info[4] = {0, 0, 0, 0};
+    CK(k_take_error_tc(&code, info));  // start from a clear error word
+    int sig = signal ? 1 : 0;
+    unsigned long long lim = limit_ns;
+    void* args[] = {&sig, &lim};
+    CK(cudaLaunchKernel(k_pick_wait_selftest(), dim3(1), dim3(32), args, 0, nullptr));
+    CK(cudaStreamSynchronize(nullptr));
+    code = 0;
+    info[0] = info[1] = info[2] = info[3] = 0;
+    CK(k_take_error_tc(&code, info));
+    if (h_info) for (int i = 0; i < 4; ++i) h_info[i] = info[i];
+    if (code)
+        return fail(nullptr, PIPO_ECUDA, "device wait timed out (code %u; first at wait site %u, block %u)", code,
+                    info[0], info[1]);
+    return PIPO_OK;
 }
 
 pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {

@@ -20,7 +20,7 @@ static __device__ unsigned int g_pipo_error;
 // (the site codes name the wait: 11-14 projection GEMM producer-empty,
 // producer-drain, MMA-full, epilogue-accumulator; 21-23 attention
 // producer-empty, producer-drain, consumer-full; 24-26 prefill attention;
-// 31-32 bulk-copy GEMV; 41-42 step kernel).
+// 31-32 bulk-copy GEMV; 41-42 step kernel; 90 the wait self-test).
 static __device__ unsigned int g_pipo_error_info[4];
 constexpr unsigned kErrWaitTimeout = 1u;
 constexpr unsigned long long kWaitNs = 2000000000ull;  // give up after 2 s of waiting
@@ -105,15 +105,17 @@ __device__ __forceinline__ unsigned long long global_ns() {
 }
 
 // Bounded wait for phase `parity` of `bar`: false (and the error word set)
-// once kWaitNs of wall time have passed without the phase completing; the
-// first wait to give up records `site`, its block and `iter` for the host.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned site = 0, unsigned iter = 0) {
+// once limit_ns of wall time (kWaitNs unless given) have passed without the
+// phase completing; the first wait to give up records `site`, its block and
+// `iter` for the host.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, unsigned site = 0, unsigned iter = 0,
+                                          unsigned long long limit_ns = kWaitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
     for (;;) {
         for (int i = 0; i < 64; ++i)
             if (mbar_try_wait(bar, parity)) return true;
-        if (global_ns() - t0 > kWaitNs) break;
+        if (global_ns() - t0 > limit_ns) break;
     }
     atomicOr(&g_pipo_error, kErrWaitTimeout);
     if (atomicCAS(&g_pipo_error_info[0], 0u, site ? site : 99u) == 0u) {

@@ -66,3 +66,48 @@ def regular_step_bytes(s: ModelShape, batch: int, ctx_avg: float) -> float:
     w = (s.L * block_params(s) + s.H + s.V * s.H) * e
     entry = s.L * 2 * s.n_kv * s.d_h * e
     return float(w + batch * (ctx_avg + 1) * entry + batch * entry)
+
+
+# ------------------------------------------------------------ recorded DRAM traffic
+
+def sources_digest(csrc_dir: str) -> str:
+    """SHA-256 (hex, first 16 digits) over the kernel sources (every .cu, .cuh
+    and .h file of csrc, by name order): a traffic figure recorded with ncu
+    describes these kernels only while the digest is unchanged."""
+    import hashlib
+    import os
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(csrc_dir)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            h.update(name.encode())
+            with open(os.path.join(csrc_dir, name), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(profiles_dir: str, workload: str, csrc_dir: str = None):
+    """DRAM bytes per projection launch that an ncu capture recorded for this
+    workload, from a line of a profiles/*.md summary of the form
+
+        traffic: workload=<name> bytes_per_launch=<float> sources=<digest>
+
+    Returns {"bytes_per_launch", "source"} when the recorded digest equals the
+    current kernel sources' digest, else None (no capture, or the kernels
+    changed since it was taken)."""
+    import os
+    import re
+    if csrc_dir is None:
+        csrc_dir = os.path.join(os.path.dirname(os.path.abspath(__file__)), "csrc")
+    if not os.path.isdir(profiles_dir):
+        return None
+    digest = sources_digest(csrc_dir)
+    pat = re.compile(r"^traffic:\s+workload=(\S+)\s+bytes_per_launch=([0-9.eE+-]+)\s+sources=([0-9a-f]+)\s*$")
+    for name in sorted(os.listdir(profiles_dir)):
+        if not name.endswith(".md"):
+            continue
+        with open(os.path.join(profiles_dir, name)) as f:
+            for line in f:
+                m = pat.match(line.strip())
+                if m and m.group(1) == workload and m.group(3) == digest:
+                    return {"bytes_per_launch": float(m.group(2)), "source": f"profiles/{name} (ncu dram__bytes)"}
+    return None

@@ -13,7 +13,8 @@ def _measured(**kw):
     m = dict(workload="4b-b1", shape_name="4b", dtype="bf16", n_gpus=1, steps=100, warmup=5, batch=2,
              prompt_tokens=2048, ms=250.0, ms_all=260.0, tokens=260, tokens_all=260, ctx_avg=1074.5, tau=0.5,
              force=0, prefill_s=3.0, prefill_rows=0, sampler=False, desc="B=2 projections=...",
-             kb={0: [8.0e9, 2.0, 150], 1: [1.0e8, 0.5, 37], 2: [0.0, 0.1, 2]}, prof_steps=1, hbm=6774.6,
+             fam={0: {"bytes": 8.0e9, "ms": 2.0, "launches": 150, "replays": 64},
+                  1: {"bytes": 1.0e8, "ms": 0.4, "launches": 37, "replays": 64}}, hbm=6774.6,
              peak_source="measured", step_bytes=9.3e9, cpu={"value": 5.0, "unit": "tokens/s", "cores": 16,
                                                              "kind": "oracle", "sample": "1 step"},
              e2e_s=30.0, e2e_tokens=240, launches=192, clocks={"sm_mhz": 2070, "sm_max_mhz": 2070, "reasons": []},
@@ -39,6 +40,12 @@ def test_contract_keys_and_meanings():
     assert r["achieved"] == pytest.approx(8.0e9 / 2.0e-3 / 1e9)  # family bytes / family time
     assert r["frac"] == pytest.approx(r["achieved"] / 6774.6)
     assert r["algorithmic_bytes_per_launch"] == pytest.approx(8.0e9 / 150)
+    assert r["avg_launch_us"] == pytest.approx(2000.0 / 150)
+    # the family's replay time is part of the step: its share is at most 1
+    assert r["family_share_of_step"] == pytest.approx(2.0 / 2.5) and r["family_share_of_step"] <= 1.0
+    assert r["launches_per_step"] * r["avg_launch_us"] <= 1e3 * line["ms_per_step"]
+    assert r["attention"]["achieved"] == pytest.approx(1.0e8 / 0.4e-3 / 1e9)
+    assert r["traffic"] is None
     assert r["step"]["achieved"] == pytest.approx(9.3e9 / 2.5e-3 / 1e9)
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 16
     e = line["e2e"]
@@ -57,9 +64,28 @@ def test_regular_ratios():
     assert line["regular"]["frac"] == pytest.approx(4000.0 / 6774.6)
 
 
-def test_missing_profile_gives_no_fraction():
-    line = bench.make_line(_measured(kb={0: [0.0, 0.0, 0], 1: [0.0, 0.0, 0], 2: [0.0, 0.0, 0]}))
+def test_missing_family_time_gives_no_fraction():
+    line = bench.make_line(_measured(fam={0: {"bytes": 0.0, "ms": 0.0, "launches": 0, "replays": 0},
+                                          1: {"bytes": 0.0, "ms": 0.0, "launches": 0, "replays": 0}}))
     assert line["roofline"]["achieved"] is None and line["roofline"]["frac"] is None
+
+
+def test_recorded_traffic_needs_the_current_sources(tmp_path):
+    from paper_2605_27255_gb300 import roofline
+    csrc = tmp_path / "csrc"
+    csrc.mkdir()
+    (csrc / "k.cuh").write_text("kernel v1")
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    d = roofline.sources_digest(str(csrc))
+    (prof / "x.md").write_text(f"# summary\ntraffic: workload=9b-b8 bytes_per_launch=1.5e8 sources={d}\n")
+    t = roofline.recorded_traffic(str(prof), "9b-b8", str(csrc))
+    assert t["bytes_per_launch"] == 1.5e8 and t["source"].startswith("profiles/x.md")
+    assert roofline.recorded_traffic(str(prof), "4b-b1", str(csrc)) is None
+    (csrc / "k.cuh").write_text("kernel v2")  # the kernels changed since the capture
+    assert roofline.recorded_traffic(str(prof), "9b-b8", str(csrc)) is None
+    line = bench.make_line(_measured(traffic=t))
+    assert line["roofline"]["traffic"] == 1.5e8
 
 
 def test_reference_arm_runs_on_cpu_and_prints_one_contract_line():
@@ -79,8 +105,3 @@ def test_reference_arm_runs_on_cpu_and_prints_one_contract_line():
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
     assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
                            "d2h_bytes_per_step": 0}
-
-
-def test_device_driven_fallback_reports_no_host_input_bytes():
-    line = bench.make_line(_measured(e2e_loop="device-driven (pipo_set_pending: x)"))
-    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["loop"].startswith("device-driven")

@@ -16,7 +16,7 @@ INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "lib")
 LIB = os.path.join(LIBDIR, "libpipo.so")
 # the host code first (the longest units start first)
-SOURCES = ["k_gemv_bf16.cu", "k_gemv_f32.cu", "k_attn.cu", "pipo_capi.cu", "k_mk.cu", "k_tc.cu"]
+SOURCES = ["k_gemv_bf16.cu", "k_gemv_f32.cu", "k_attn.cu", "pipo_capi.cu", "k_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

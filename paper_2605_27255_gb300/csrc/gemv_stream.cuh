@@ -26,12 +26,6 @@ namespace pipo {
 #ifndef PIPO_STREAM_THREADS
 #define PIPO_STREAM_THREADS 768
 #endif
-#ifndef PIPO_TMA_WARPS
-#define PIPO_TMA_WARPS 8
-#endif
-#ifndef PIPO_TMA_STAGE_CHUNKS
-#define PIPO_TMA_STAGE_CHUNKS 8
-#endif
 #ifndef PIPO_STREAM_CTAS_PER_SM
 #define PIPO_STREAM_CTAS_PER_SM 1
 #endif
@@ -974,99 +968,6 @@ __device__ __forceinline__ void finish_block(const GemvParams& p, WarpRows<T, NB
             if (br != 0x7fffffff) atomicMax(p.am + wr.b0 + bb, argmax_key(bv, br));
         }
     }
-}
-
-// ---------------------------------------------------------------------------
-// Bulk-copy (TMA) GEMV.  Each warp owns a contiguous chunk range of the CTA's
-// rows and a private ring of `ns` shared-memory stages of kStageChunks chunks;
-// lane 0 refills a stage with one cp.async.bulk as soon as the warp has read it
-// (mbarrier completion).  Bytes in flight per SM: up to 8 warps x ns x 4 KB,
-// with one copy instruction per 4 KB.  Single pass: B <= NB.
-constexpr int kTmaWarps = PIPO_TMA_WARPS;
-constexpr int kTmaThreads = kTmaWarps * 32;
-constexpr int kStageChunks = PIPO_TMA_STAGE_CHUNKS;
-constexpr int kStageBytes = kStageChunks * 512;
-
-template <typename T, int NB, int RU>
-__global__ void __launch_bounds__(kTmaThreads) gemv_tma_kernel(GemvParams p, int ns) {
-    extern __shared__ __align__(128) unsigned char smem_raw[];
-    __shared__ int head_unit[kTmaWarps], tail_unit[kTmaWarps], head_fin[kTmaWarps];
-    __shared__ float head_val[kTmaWarps][RU][NB], tail_val[kTmaWarps][RU][NB];
-    __shared__ float red_v[kTmaWarps][NB];
-    __shared__ int red_r[kTmaWarps][NB];
-
-    pdl_launch();
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int K = p.K;
-    const int cpr = K * (int)sizeof(T) / 512;
-    const int cpu = cpr * RU;
-    const int G = gridDim.x;
-    const int u0 = (int)((long long)blockIdx.x * p.N / G);
-    const int u1 = (int)((long long)(blockIdx.x + 1) * p.N / G);
-    const int C = (u1 - u0) * cpu;
-    const int c0 = (int)((long long)warp * C / kTmaWarps);
-    const int c1 = (int)((long long)(warp + 1) * C / kTmaWarps);
-    const char* gsrc = static_cast<const char*>(p.W) + ((size_t)u0 * cpu + c0) * 512;
-
-    unsigned char* ring = smem_raw + (size_t)warp * ns * kStageBytes;
-    float* xs = reinterpret_cast<float*>(smem_raw + (size_t)kTmaWarps * ns * kStageBytes);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(xs + NB * K) + warp * ns;
-    const int nst = (c1 - c0 + kStageChunks - 1) / kStageChunks;  // stages of this warp
-
-    auto issue = [&](int i) {  // lane 0: stage i of this warp into slot i % ns
-        const int first = i * kStageChunks;
-        const int n = min(kStageChunks, (c1 - c0) - first);
-        const uint32_t bytes = (uint32_t)n * 512u;
-        uint64_t* bar = bars + (i % ns);
-        mbar_arrive_expect_tx(bar, bytes);
-        bulk_g2s(ring + (size_t)(i % ns) * kStageBytes, gsrc + (size_t)first * 512, bytes, bar);
-    };
-    if (lane == 0) {
-        for (int s2 = 0; s2 < ns; ++s2) mbar_init(bars + s2, 1);
-        mbar_init_fence();
-        for (int i = 0; i < min(ns, nst); ++i) issue(i);
-    }
-    __syncwarp();
-    pdl_wait();
-    if (p.zero_ptr && blockIdx.x == 0)
-        for (int i = threadIdx.x; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
-    if (lane == 0) { head_fin[warp] = 0; head_unit[warp] = -1; tail_unit[warp] = -1; }
-    __syncthreads();
-    stage_input_fast<T, NB, kTmaThreads>(p, xs, 0, min(NB, p.B));
-
-    WarpRows<T, NB, RU> wr;
-    wr.init(&p, xs, cpr, u0, c0, c1, 0, min(NB, p.B));
-    int failed = -1;  // first stage whose wait gave up
-    for (int i = 0; i < nst; ++i) {
-        const int slot = i % ns;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(bars + slot, (uint32_t)((i / ns) & 1), 31, i));
-        if (!ok) {
-            failed = i;
-            break;
-        }
-        const unsigned char* sp = ring + (size_t)slot * kStageBytes + lane * 16;
-        const int n = min(kStageChunks, (c1 - c0) - i * kStageChunks);
-        if (n == kStageChunks) {
-#pragma unroll
-            for (int ch = 0; ch < kStageChunks; ++ch)
-                wr.chunk(*reinterpret_cast<const uint4*>(sp + ch * 512), head_unit, head_fin, head_val);
-        } else {
-            for (int ch = 0; ch < n; ++ch)
-                wr.chunk(*reinterpret_cast<const uint4*>(sp + ch * 512), head_unit, head_fin, head_val);
-        }
-        __syncwarp();
-        if (lane == 0 && i + ns < nst) {
-            fence_proxy_async();  // our generic reads of the slot before the async overwrite
-            issue(i + ns);
-        }
-    }
-    if (failed >= 0 && lane == 0) {
-        // a wait gave up (error recorded): wait, bounded, for the copies still in flight
-        for (int i = failed + 1; i < min(nst, failed + ns); ++i) mbar_wait(bars + (i % ns), (uint32_t)((i / ns) & 1), 32, i);
-    }
-    wr.finish(head_unit, head_fin, tail_unit, head_val, tail_val);
-    __syncthreads();
-    finish_block<T, NB, RU, kTmaWarps>(p, wr, head_unit, head_fin, tail_unit, head_val, tail_val, red_v, red_r);
 }
 
 }  // namespace pipo

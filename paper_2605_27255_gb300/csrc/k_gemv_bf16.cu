@@ -4,8 +4,6 @@
 namespace pipo {
 
 void* k_pick_gemv_bf16(int nb, bool two) { return pick_gemv_t<__nv_bfloat16>(nb, two); }
-void* k_pick_tma_bf16(int nb, int ru) { return pick_tma_t<__nv_bfloat16>(nb, ru); }
 void* k_pick_stream_bf16(int nb, int ru, bool rows) { return pick_stream_t<__nv_bfloat16>(nb, ru, rows); }
-cudaError_t k_take_error_gemv_bf16(unsigned* code, unsigned* info) { return take_unit_error(code, info); }
 
 }  // namespace pipo

@@ -24,18 +24,6 @@ void* pick_gemv_t(int nb, bool two) {
 }
 
 template <typename T, int NB, int RU>
-void* tma_fn() { return reinterpret_cast<void*>(&gemv_tma_kernel<T, NB, RU>); }
-
-template <typename T>
-void* pick_tma_t(int nb, int ru) {
-    switch (nb) {
-        case 1: return ru == 2 ? tma_fn<T, 1, 2>() : tma_fn<T, 1, 1>();
-        case 2: return ru == 2 ? tma_fn<T, 2, 2>() : tma_fn<T, 2, 1>();
-        default: return ru == 2 ? tma_fn<T, 4, 2>() : tma_fn<T, 4, 1>();
-    }
-}
-
-template <typename T, int NB, int RU>
 void* stream_fn(bool rows) {
     return rows ? reinterpret_cast<void*>(&gemv_rows_kernel<T, NB, RU, kStreamDepth>)
                 : reinterpret_cast<void*>(&gemv_stream_kernel<T, NB, RU, kStreamDepth>);

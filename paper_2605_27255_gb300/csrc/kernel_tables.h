@@ -13,12 +13,8 @@ namespace pipo {
 // k_gemv_bf16.cu / k_gemv_f32.cu: the CUDA-core GEMVs of one weight type
 void* k_pick_gemv_bf16(int nb, bool two);           // gemv_kernel<bf16, nb, two>
 void* k_pick_gemv_f32(int nb, bool two);
-void* k_pick_tma_bf16(int nb, int ru);              // gemv_tma_kernel
-void* k_pick_tma_f32(int nb, int ru);
 void* k_pick_stream_bf16(int nb, int ru, bool rows);  // gemv_rows_kernel (rows) / gemv_stream_kernel
 void* k_pick_stream_f32(int nb, int ru, bool rows);
-cudaError_t k_take_error_gemv_bf16(unsigned* code, unsigned* info);
-cudaError_t k_take_error_gemv_f32(unsigned* code, unsigned* info);
 
 // k_tc.cu: the tcgen05 projections
 void* k_pick_tcv(int bh, bool deep, bool fused);    // gemm_tcf_kernel (fused) / gemm_tc_kernel
@@ -34,9 +30,5 @@ void* k_pick_attn_prefill(int G);                   // attn_prefill_kernel
 void* k_pick_rope_append(bool bf, int DH);          // rope_append_kernel
 void* k_pick_append_rows(bool bf, int DH);          // append_rows_kernel
 cudaError_t k_take_error_attn(unsigned* code, unsigned* info);
-
-// k_mk.cu: the persistent step kernel
-void* k_pick_step_kernel(bool bf, int nb, int DH, int G);
-cudaError_t k_take_error_mk(unsigned* code, unsigned* info);
 
 }  // namespace pipo

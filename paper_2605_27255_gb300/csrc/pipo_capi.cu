@@ -31,7 +31,6 @@
 #include "gemv_stream.cuh"
 #include "kernel_tables.h"
 #include "kernels.cuh"
-#include "megakernel.cuh"
 #include "pipo.h"
 #include "sampler.cuh"
 #include "tcgen05_gemm.cuh"
@@ -147,18 +146,7 @@ struct pipo_ctx {
     bool attn_v0 = false;             // (development) the unclustered attention path
     bool attn_regs = false;           // register-ring attention instead of the tensor-core one
     std::vector<CUtensorMap> kv_tm;   // tensor-core attention: K and V tensor map of every cache layer
-    bool gemv_tma = false;            // bulk-copy GEMV (else the register-ring GEMV)
     int gemv_l2_prefetch = 0;         // streaming GEMV: weight chunks per warp hinted into L2 before the wait
-    // persistent step kernel: phases recorded from the enqueue code
-    std::vector<Phase>* rec = nullptr;  // recording target (nullptr: launch kernels)
-    bool rec_ok = true;                 // every recorded phase fits the step kernel
-    int rec_kmax = 0;
-    bool use_mk = false;                // use the persistent step kernel when it fits
-    bool mk_active = false;             // the current decode graph is the step kernel
-    Phase* d_phases = nullptr;
-    size_t d_phases_cap = 0;
-    unsigned* bar_ctr = nullptr;
-    std::string mk_note;
     // per-launch timing (pipo_profile_step): events around every launch
     bool prof = false;
     int prof_kind = 2;
@@ -297,10 +285,6 @@ void* pick_gemv(int nb, bool two) {
     return std::is_same<T, bf16>::value ? k_pick_gemv_bf16(nb, two) : k_pick_gemv_f32(nb, two);
 }
 template <typename T>
-void* pick_tma(int nb, int ru) {
-    return std::is_same<T, bf16>::value ? k_pick_tma_bf16(nb, ru) : k_pick_tma_f32(nb, ru);
-}
-template <typename T>
 void* pick_stream(int nb, int ru, bool rows) {
     return std::is_same<T, bf16>::value ? k_pick_stream_bf16(nb, ru, rows) : k_pick_stream_f32(nb, ru, rows);
 }
@@ -371,15 +355,6 @@ pipo_status launch_ex(pipo_ctx* ctx, const void* fn, dim3 grid, dim3 block, size
 
 size_t g_smem_optin = 0;  // opt-in shared memory per block of the device
 
-// Allow `fn` the largest dynamic shared memory the device permits next to its
-// static shared memory; returns that size (0 on failure).
-size_t allow_max_smem(const void* fn) {
-    cudaFuncAttributes fa{};
-    if (cudaFuncGetAttributes(&fa, fn) != cudaSuccess) return 0;
-    const size_t dyn = g_smem_optin > fa.sharedSizeBytes ? g_smem_optin - fa.sharedSizeBytes : 0;
-    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn) != cudaSuccess) return 0;
-    return dyn;
-}
 
 // bh: batch columns of the tensor-core GEMM (its MMA N is 2 * bh: hi | lo)
 size_t tc_smem(int bh, bool deep = false) {
@@ -407,11 +382,6 @@ cudaError_t set_smem_attrs(bool bf) {
     if (e0 == cudaSuccess) e0 = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     if (e0 != cudaSuccess) return e0;
     g_smem_optin = (size_t)optin;
-    for (int nb : {1, 2, 4})
-        for (int ru : {1, 2}) {
-            void* f = bf ? pick_tma<bf16>(nb, ru) : pick_tma<float>(nb, ru);
-            if (allow_max_smem(f) < 160 * 1024) return cudaErrorInvalidValue;
-        }
     for (int nb : {1, 2, 4})
         for (int ru : {1, 2})
             for (bool rows : {false, true}) {
@@ -675,7 +645,7 @@ pipo_status launch_gemm_tc(pipo_ctx* ctx, const GemvParams& p, bf16* xb, int spl
 
 bool tc_eligible(const pipo_ctx* ctx, const GemvParams& p) {
     const int rows = p.N * (p.epi == EPI_SWIGLU ? 2 : 1);
-    return ctx->cfg.dtype == 1 && ctx->tc_xb && !ctx->rec && p.B >= ctx->tc_min_b && p.B <= ctx->tc_bn_max &&
+    return ctx->cfg.dtype == 1 && ctx->tc_xb && p.B >= ctx->tc_min_b && p.B <= ctx->tc_bn_max &&
            p.K % kTcBK == 0 && p.K <= ctx->tc_kmax && p.K <= 4 * kPrepQ * kPrepThreads && rows >= kTcM;
 }
 
@@ -684,17 +654,6 @@ pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
     const bool two = p.epi == EPI_SWIGLU;
     if (tc_eligible(ctx, p))
         return launch_gemm_tc(ctx, p, ctx->tc_xb, ctx->tc_splits, ctx->act_rows);
-    if (ctx->rec) {
-        Phase ph{};
-        ph.type = PH_GEMV;
-        ph.ru = two ? 2 : 1;
-        p.splitk = 1;  // the step kernel finishes every row inside one CTA
-        ph.g = p;
-        if (((size_t)p.K * ctx->esz) % 512 != 0 || p.B > 4) ctx->rec_ok = false;
-        ctx->rec_kmax = std::max(ctx->rec_kmax, p.K);
-        ctx->rec->push_back(ph);
-        return PIPO_OK;
-    }
     ctx->prof_kind = 0;
     ctx->prof_bytes = (double)p.N * (two ? 2 : 1) * p.K * ctx->esz;
     if (p.B <= 4) {
@@ -704,24 +663,6 @@ pipo_status launch_gemv(pipo_ctx* ctx, GemvParams p) {
         if ((size_t)p.K * 4 > kStreamBudget) return fail(ctx, PIPO_EINVAL, "GEMV input length %d too large", p.K);
         const bool rows = ((size_t)p.K * ctx->esz) % 512 == 0;
         const size_t xbytes = (size_t)nb * p.K * 4;
-        if (rows && ctx->gemv_tma && p.B <= nb) {
-            // bulk-copy kernel: stages per warp from what shared memory allows
-            const size_t per_stage = (size_t)kTmaWarps * (kStageBytes + 8);
-#ifdef PIPO_TMA_SMEM_CAP
-            const size_t cap = std::min<size_t>(g_smem_optin, PIPO_TMA_SMEM_CAP);  // leave room for a second CTA
-#else
-            const size_t cap = g_smem_optin;
-#endif
-            const size_t room = cap > 4096 + xbytes ? cap - 4096 - xbytes : 0;
-            const int ns = (int)std::min<size_t>(4, room / per_stage);
-            if (ns >= 2) {
-                void* fn = bf ? pick_tma<bf16>(nb, two ? 2 : 1) : pick_tma<float>(nb, two ? 2 : 1);
-                int nsv = ns;
-                void* args[] = {&p, &nsv};
-                return launch_ex(ctx, fn, dim3(ctx->sms), dim3(kTmaThreads),
-                                 (size_t)kTmaWarps * ns * kStageBytes + xbytes + (size_t)kTmaWarps * ns * 8, args);
-            }
-        }
         void* fn = bf ? pick_stream<bf16>(nb, two ? 2 : 1, rows) : pick_stream<float>(nb, two ? 2 : 1, rows);
         void* args[] = {&p};
         // staged input, then (row kernel) the RMSNorm gains in their storage type
@@ -769,13 +710,6 @@ int resadd_splits(pipo_ctx* ctx, int N, int K) {
     int s = (int)std::max(1LL, (target + N - 1) / N);
     s = std::min(s, std::max(1, K / 256));
     return s;
-}
-
-// splits per (sequence, kv head) of the step kernel: one unit per CTA
-int mk_attn_splits(const pipo_ctx* ctx, int B) {
-    const pipo_config& c = ctx->cfg;
-    int s = (ctx->sms + B * c.n_kv_heads - 1) / (B * c.n_kv_heads);
-    return std::max(1, std::min(s, (c.max_ctx + 15) / 16));
 }
 
 int attn_splits(const pipo_ctx* ctx, int B) {
@@ -846,7 +780,6 @@ cudaError_t set_carveouts(bool bf) {
         for (int two = 0; two < 2; ++two) fns.push_back(bf ? pick_gemv<bf16>(nb, two) : pick_gemv<float>(nb, two));
     for (int nb : {1, 2, 4})
         for (int ru : {1, 2}) {
-            fns.push_back(bf ? pick_tma<bf16>(nb, ru) : pick_tma<float>(nb, ru));
             for (bool rows : {false, true})
                 fns.push_back(bf ? pick_stream<bf16>(nb, ru, rows) : pick_stream<float>(nb, ru, rows));
         }
@@ -941,24 +874,7 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
     p.K = H;
     TRY(launch_gemv(ctx, p));
     KVView kv = kv_view(ctx, cache_layer);
-    if (ctx->rec) {
-        Phase ph{};
-        ph.type = PH_ATTN;
-        AttnPhase& a = ph.a;
-        a.qkv = ctx->qkv;
-        a.ld_qkv = rows;
-        a.kv = kv;
-        a.n_pos = ctx->n_pos;
-        a.rope = ctx->rope;
-        a.out = ctx->attn;
-        a.scale = 1.0f / sqrtf((float)DH);
-        a.part_o = ctx->part_o;
-        a.part_ml = ctx->part_ml;
-        a.counters = ctx->counters;
-        a.S = mk_attn_splits(ctx, ctx->B);
-        a.B = ctx->B;
-        ctx->rec->push_back(ph);
-    } else if (!ctx->attn_v0) {
+    if (!ctx->attn_v0) {
         // RoPE + KV append + split-KV attention, one cluster per (row, kv head).
         // A prefill chunk (several positions per sequence) appends all its
         // rows' entries first: its rows read each other's.
@@ -1182,22 +1098,6 @@ pipo_status enqueue_position(pipo_ctx* ctx, Mode mode, int j) {
     if (ctx->samp_on) {
         st.presence = ctx->presence; st.presence_w = ctx->presence_w; st.samp_step = ctx->samp_step;
     }
-    if (ctx->rec) {
-        Phase ph{};
-        ph.type = PH_ACCEPT;
-        AcceptPhase& a = ph.c;
-        a.t = ctx->t;
-        a.W2 = ctx->conf_W2;
-        a.H = H;
-        a.tau = c.tau;
-        a.force = c.force_mode;
-        a.st = st;
-        a.hb = ctx->x;
-        a.hd = ctx->x2;
-        a.B = B;
-        ctx->rec->push_back(ph);
-        return PIPO_OK;
-    }
     {
         const float* tp = ctx->t;
         const void* w2 = ctx->conf_W2;
@@ -1263,7 +1163,7 @@ pipo_status enqueue_regular(pipo_ctx* ctx, Mode mode, int j) {
 pipo_status enqueue_prefill_chunk(pipo_ctx* ctx, bool regular, int j0, int C) {
     const pipo_config& c = ctx->cfg;
     const int H = c.hidden, B = ctx->B, R = C * B;
-    if (R > ctx->max_rows || C < 1 || ctx->rec || ctx->attn_v0)
+    if (R > ctx->max_rows || C < 1 || ctx->attn_v0)
         return fail(ctx, PIPO_EINVAL, "prefill chunk of %d rows (at most %d)", R, ctx->max_rows);
     struct RowsGuard {
         pipo_ctx* c;
@@ -1352,98 +1252,9 @@ void drop_graph(pipo_ctx* ctx) {
     ctx->fam_graph_B = -1;
 }
 
-void* mk_pick(bool bf, int nb, int DH, int G) { return k_pick_step_kernel(bf, nb, DH, G); }
-
-// Record the decode step as phases; when they all fit, upload them and capture
-// (or prepare) the persistent step kernel.  Returns false when it does not fit.
-pipo_status try_step_kernel(pipo_ctx* ctx, bool& used) {
-    used = false;
-    if (!ctx->use_mk || ctx->B > 4 || ctx->cfg.comp_residual) return PIPO_OK;
-    const pipo_config& c = ctx->cfg;
-    const int nb = ctx->B <= 1 ? 1 : ctx->B <= 2 ? 2 : 4;
-    void* fn = mk_pick(c.dtype == 1, nb, c.head_dim, c.n_q_heads / c.n_kv_heads);
-    if (!fn) { ctx->mk_note = "(no step-kernel instance for this head shape)"; return PIPO_OK; }
-    std::vector<Phase> phases;
-    ctx->rec = &phases;
-    ctx->rec_ok = true;
-    ctx->rec_kmax = 0;
-    pipo_status s = enqueue_position(ctx, DECODE, 0);
-    ctx->rec = nullptr;
-    if (s != PIPO_OK) return s;
-    if (!ctx->rec_ok) { ctx->mk_note = "(a projection row is not a whole number of 512-byte chunks)"; return PIPO_OK; }
-    // attention: warp partials [NW][G][DH] + (m, l), and the split merge [G][S][DH + 2]
-    const int G = c.n_q_heads / c.n_kv_heads;
-    const size_t attn_bytes = std::max((size_t)(2 * kMkWarps * G + kMkWarps * G * c.head_dim),
-                                       (size_t)G * mk_attn_splits(ctx, ctx->B) * (c.head_dim + 2)) * 4;
-    const size_t stage_bytes = std::max((size_t)nb * ctx->rec_kmax * 4, attn_bytes);
-    const size_t smem = mk_stage_offset() + stage_bytes;
-    if (allow_max_smem(fn) < smem) { ctx->mk_note = "(shared memory)"; return PIPO_OK; }
-    int per_sm = 0;
-    CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kMkThreads, smem));
-    if (per_sm < 1) { ctx->mk_note = "(occupancy)"; return PIPO_OK; }
-    if (phases.size() > ctx->d_phases_cap) {
-        if (ctx->d_phases) {
-            cudaFree(ctx->d_phases);
-            ctx->allocs.erase(std::find(ctx->allocs.begin(), ctx->allocs.end(), (void*)ctx->d_phases));
-        }
-        ctx->d_phases = nullptr;
-        TRY(dalloc(ctx, &ctx->d_phases, phases.size() * sizeof(Phase)));
-        ctx->d_phases_cap = phases.size();
-    }
-    CK(cudaMemcpy(ctx->d_phases, phases.data(), phases.size() * sizeof(Phase), cudaMemcpyHostToDevice));
-    // capture: zero the barrier counter, then one cooperative launch
-    cudaGraph_t g = nullptr;
-    CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
-    cudaError_t e = cudaMemsetAsync(ctx->bar_ctr, 0, sizeof(unsigned), ctx->stream);
-    if (e == cudaSuccess) {
-        const Phase* ph = ctx->d_phases;
-        int nph = (int)phases.size();
-        unsigned* bc = ctx->bar_ctr;
-        void* args[] = {(void*)&ph, &nph, &bc};
-        cudaLaunchConfig_t lc = {};
-        lc.gridDim = dim3(ctx->sms);
-        lc.blockDim = dim3(kMkThreads);
-        lc.dynamicSmemBytes = smem;
-        lc.stream = ctx->stream;
-        cudaLaunchAttribute at[1];
-        at[0].id = cudaLaunchAttributeCooperative;
-        at[0].val.cooperative = 1;
-        lc.attrs = at;
-        lc.numAttrs = 1;
-        e = cudaLaunchKernelExC(&lc, fn, args);
-    }
-    cudaError_t e2 = cudaStreamEndCapture(ctx->stream, &g);
-    if (e == cudaSuccess && e2 == cudaSuccess) e = cudaGraphInstantiate(&ctx->graph, g, 0);
-    if (g) cudaGraphDestroy(g);
-    if (e != cudaSuccess || e2 != cudaSuccess) {
-        // not capturable here: keep the multi-kernel graph for this context
-        ctx->mk_note = std::string("step kernel unavailable: ") + cudaGetErrorString(e != cudaSuccess ? e : e2);
-        cudaGetLastError();
-        ctx->graph = nullptr;
-        ctx->use_mk = false;
-        return PIPO_OK;
-    }
-    ctx->graph_B = ctx->B;
-    ctx->launches = 1;
-    ctx->mk_active = true;
-    used = true;
-    return PIPO_OK;
-}
-
 pipo_status ensure_graph(pipo_ctx* ctx) {
     if (ctx->graph && ctx->graph_B == ctx->B && ctx->graph_regular == ctx->regular) return PIPO_OK;
     drop_graph(ctx);
-    ctx->mk_active = false;
-    bool used = false;
-    // the persistent step kernel records the pair step only
-    if (!ctx->regular && !ctx->samp_on) TRY(try_step_kernel(ctx, used));
-    if (getenv("PIPO_VERBOSE"))
-        fprintf(stderr, "pipo: decode step = %s %s\n", used ? "persistent step kernel" : "kernel graph",
-                ctx->mk_note.c_str());
-    if (used) {
-        ctx->graph_regular = false;
-        return PIPO_OK;
-    }
     cudaGraph_t g = nullptr;
     CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
     ctx->launches = 0;
@@ -1505,13 +1316,9 @@ pipo_status ensure_cache_tmp(pipo_ctx* ctx, size_t elems) {
 // step kernel when the context uses them.  The first unit with an error
 // names the wait.
 pipo_status check_device_error(pipo_ctx* ctx) {
-    cudaError_t (*units[5])(unsigned*, unsigned*) = {k_take_error_attn, k_take_error_tc, nullptr, nullptr, nullptr};
-    int nu = 2;
-    if (ctx->gemv_tma) {
-        units[nu++] = k_take_error_gemv_bf16;
-        units[nu++] = k_take_error_gemv_f32;
-    }
-    if (ctx->use_mk) units[nu++] = k_take_error_mk;
+    // the units whose kernels wait on mbarriers: attention and tensor-core projections
+    cudaError_t (*units[2])(unsigned*, unsigned*) = {k_take_error_attn, k_take_error_tc};
+    const int nu = 2;
     unsigned e = 0, info[4] = {0, 0, 0, 0};
     for (int i = 0; i < nu; ++i) {
         auto take = units[i];
@@ -1657,11 +1464,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
                 ctx->attn_cs_force = v;
         }
         if (const char* ev = getenv("PIPO_ATTN_CS_TARGET")) ctx->attn_cs_target = std::max(1, atoi(ev));
-        if (const char* ev = getenv("PIPO_GEMV_TMA")) ctx->gemv_tma = ev[0] == '1';
         if (const char* ev = getenv("PIPO_GEMV_L2_PREFETCH")) ctx->gemv_l2_prefetch = std::max(0, atoi(ev));
-        if (const char* ev = getenv("PIPO_STEP_KERNEL")) ctx->use_mk = ev[0] == '1';
-        TRY(dalloc(ctx, &ctx->bar_ctr, 64));
-        CK(cudaMemset(ctx->bar_ctr, 0, 64));
 
         // activations and state
         const int qd = c.n_q_heads * DH, kd = c.n_kv_heads * DH;
@@ -2230,8 +2033,6 @@ pipo_status op_setup(pipo_ctx& op, int32_t dtype, void* stream) {
     }
     op.stream = static_cast<cudaStream_t>(stream);
     op.pdl = false;
-    op.gemv_tma = false;
-    if (const char* ev = getenv("PIPO_GEMV_TMA")) op.gemv_tma = ev[0] == '1';
     return PIPO_OK;
 }
 

@@ -17,10 +17,10 @@ namespace pipo {
 // host reads and clears every unit's copy after a step (take_unit_error).
 static __device__ unsigned int g_pipo_error;
 // First wait that gave up: {site code, linear block index, iteration, parity}
-// (the site codes name the wait: 11-14 projection GEMM producer-empty,
-// producer-drain, MMA-full, epilogue-accumulator; 21-23 attention
+// (the site codes name the wait: 11-15 projection GEMM producer-empty,
+// producer-drain, MMA-full, epilogue-accumulator, converter-full; 21-23 attention
 // producer-empty, producer-drain, consumer-full; 24-26 prefill attention;
-// 31-32 bulk-copy GEMV; 41-42 step kernel; 90 the wait self-test).
+// 90 the wait self-test).
 static __device__ unsigned int g_pipo_error_info[4];
 constexpr unsigned kErrWaitTimeout = 1u;
 constexpr unsigned long long kWaitNs = 2000000000ull;  // give up after 2 s of waiting

@@ -96,14 +96,29 @@ def test_9b_b1_forced_replay(w9b):
     assert st.tok_checked >= 0.8 * st.tok_total
 
 
+@pytest.fixture(scope="module")
+def w9b_4l():
+    s = synth.B9.with_(name="9b-4l", L=4)
+    w = synth.gen_weights(s, seed=0, device="cuda")
+    yield s, w, {k: v.cpu() for k, v in w.items()}
+    del w
+    torch.cuda.empty_cache()
+
+
 @pytest.mark.parametrize("tau", [0.3, 0.7])
-def test_9b_b8_forced_replay(w9b, tau):
-    """9b-b8, the benchmark's largest configuration: tcgen05 projections at
-    K = 4096 and K = 12288 (down), tensor-core attention, thresholds from
-    both ends of the sweep."""
-    w, host = w9b
-    prompts = synth.gen_prompts(8, 4, synth.B9.V, seed=7).numpy()
-    st = run_forced_replay(synth.B9, w, prompts, 2, oracle_weights=host, tau=tau)
+def test_9b_b8_forced_replay(w9b_4l, tau):
+    """The 9b-b8 launch plan: 9B widths at B = 8, tcgen05 projections at
+    K = 4096 and K = 12288 (down), tensor-core attention, thresholds from both
+    ends of the sweep.  Four layers: every layer launches the same kernels
+    with the same shapes as in the 36-layer model, and at four layers the
+    bf16 cache-rounding cascade (test_bf16_cache_rounding_cascade) has not yet
+    grown to the ulp level.  At 36 layers two independently rounded
+    computations of this model differ by about 0.02 in the 9B logits, the
+    size of the bar itself; the fp64 oracle against itself, seeded with a
+    1e-6 relative change, differs by 0.011 at the 4B shapes."""
+    s, w, host = w9b_4l
+    prompts = synth.gen_prompts(8, 4, s.V, seed=7).numpy()
+    st = run_forced_replay(s, w, prompts, 2, oracle_weights=host, tau=tau)
     assert st.tok_checked >= 0.8 * st.tok_total
     assert st.max_logit_err < 2e-2
 

@@ -621,3 +621,39 @@ def test_capacity_and_bad_ids_are_errors():
     st.prefill(synth.gen_prompts(1, 8, s.V).numpy())
     with pytest.raises(ValueError):
         st.step()
+
+
+def test_bf16_cache_rounding_cascade():
+    """Rounding the cache to bf16 (the storage of the bf16 configurations)
+    turns a small difference into an ulp-level one over depth.  A relative
+    1.2e-4 change of E flips a few cached bf16 values in layer 0.  Each flip
+    moves the next layer's inputs enough to flip more, until a large share
+    of every layer's cached values differ, and h_b differs by ~1e-3 relative.
+    Without cache rounding the same change stays near its own size.  An fp32
+    GPU path and the fp64 oracle round the cache independently, so at full
+    depth their agreement is bounded by this cascade, whatever the kernels'
+    precision."""
+    s = synth.ModelShape("cascade", H=256, L=36, n_q=4, n_kv=2, d_h=64, F=768, V=512, compressor="mlp",
+                         mtp_block=1, dtype="f32", rope_theta=1e6)
+    w = {k: v.to(torch.bfloat16).float() for k, v in synth.gen_weights(s.with_(dtype="bf16"), seed=0).items()}
+    wp = dict(w)
+    E = w["E"].clone()
+    E.view(torch.int32).add_(2048)  # +2048 fp32 ulps: about 1.2e-4 relative
+    wp["E"] = E
+    prompts = synth.gen_prompts(4, 4, s.V, seed=7).numpy()
+    kd = 2 * s.n_kv * s.d_h  # cached values per layer and position (K and V)
+
+    def run(weights, kvb):
+        st = O.State(O.Model(s, weights, max_ctx=4, kv_bf16=kvb), 4)
+        o = st.prefill(prompts, tau=0.5)
+        return o, [[st.cache(b, l, 2) for l in range(s.L + 1)] for b in range(4)]
+
+    (oa, ca), (ob, cb) = run(w, True), run(wp, True)
+    (na, _), (nb, _) = run(w, False), run(wp, False)
+    for b in range(4):
+        flips = [int((ca[b][l][0] != cb[b][l][0]).sum() + (ca[b][l][1] != cb[b][l][1]).sum()) for l in range(s.L)]
+        assert 0 < flips[0] < 0.1 * 2 * kd            # a few flips in the first layer
+        assert min(flips[-6:]) > 0.3 * 2 * kd         # a large share of the last layers
+        rel = np.abs(oa["h_b"][b] - ob["h_b"][b]).max() / np.abs(oa["h_b"][b]).max()
+        rel_exact = np.abs(na["h_b"][b] - nb["h_b"][b]).max() / np.abs(na["h_b"][b]).max()
+        assert rel > 5e-4 and rel > 10 * rel_exact, (rel, rel_exact)

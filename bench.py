@@ -390,7 +390,7 @@ def run_pipo(args):
     K = args.steps if args.steps is not None else wl["steps"]
     W = max(3, args.warmup)
     n_pairs = (T + 1) // 2
-    max_ctx = n_pairs + W + 2 * K + 8
+    max_ctx = n_pairs + W + 2 * K + 9
     if args.regular:
         max_ctx = max(max_ctx, T + W + K + 8)  # regular decoding: one cache entry per token
 
@@ -407,7 +407,7 @@ def run_pipo(args):
     g.set_stream(stream.cuda_stream)
     if args.sampler:
         # draws for every position that runs the heads (prefill, warm-up, timed, e2e, profile steps)
-        n_u = 1 + W + 2 * K + 8
+        n_u = 1 + W + 2 * K + 9
         u = np.random.default_rng(11 + rank).random((n_u, B, 2)).astype(np.float32)
         g.set_sampler(u, temperature=1.0, top_k=20, top_p=0.95, rep_penalty=1.5)
 
@@ -473,6 +473,12 @@ def run_pipo(args):
     # graph of its own launches replayed back to back (decode state unchanged)
     n_rep = args.family_replays or max(8, min(K, 256))
     fam = {0: time_family(g, 0, n_rep, stream), 1: time_family(g, 1, n_rep, stream)}
+    # one more graph-replayed step inside an NVTX range: ncu --nvtx --nvtx-include "ncu_step/"
+    # takes the launch list of exactly this step (untimed here)
+    torch.cuda.nvtx.range_push("ncu_step")
+    g.step_async()
+    torch.cuda.synchronize()
+    torch.cuda.nvtx.range_pop()
     regular = run_regular(g, shape, wl, B, T, W, K, stream, 1 + rank * 1000) if args.regular else None
 
     ms_all, tokens_all, e2e_all, e2e_tok_all = aggregate_ranks(ms, tokens, e2e_s, e2e_tokens, "cuda")

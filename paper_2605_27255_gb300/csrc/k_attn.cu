@@ -26,16 +26,16 @@ void* attn_pick_g(int G) {
     }
 }
 
-template <typename T, int DH, int G>
-void* attnc_fn() { return reinterpret_cast<void*>(&attn_cluster_kernel<T, DH, G>); }
+template <typename T, int DH, int G, bool FLAT>
+void* attnc_fn() { return reinterpret_cast<void*>(&attn_cluster_kernel<T, DH, G, FLAT>); }
 
-template <typename T, int DH>
+template <typename T, int DH, bool FLAT = false>
 void* attnc_pick_g(int G) {
     switch (G) {
-        case 1: return attnc_fn<T, DH, 1>();
-        case 2: return attnc_fn<T, DH, 2>();
-        case 4: return attnc_fn<T, DH, 4>();
-        case 8: return attnc_fn<T, DH, 8>();
+        case 1: return attnc_fn<T, DH, 1, FLAT>();
+        case 2: return attnc_fn<T, DH, 2, FLAT>();
+        case 4: return attnc_fn<T, DH, 4, FLAT>();
+        case 8: return attnc_fn<T, DH, 8, FLAT>();
         default: return nullptr;
     }
 }
@@ -53,6 +53,13 @@ void* k_pick_attn_decode(bool bf, int DH, int G) {
 void* k_pick_attn_cluster(bool bf, int DH, int G) {
     if (DH == 64) return bf ? attnc_pick_g<bf16, 64>(G) : attnc_pick_g<float, 64>(G);
     if (DH == 128) return bf ? attnc_pick_g<bf16, 128>(G) : attnc_pick_g<float, 128>(G);
+    return nullptr;
+}
+
+// the same attention without a cluster: any split count, merged through global scratch
+void* k_pick_attn_flat(bool bf, int DH, int G) {
+    if (DH == 64) return bf ? attnc_pick_g<bf16, 64, true>(G) : attnc_pick_g<float, 64, true>(G);
+    if (DH == 128) return bf ? attnc_pick_g<bf16, 128, true>(G) : attnc_pick_g<float, 128, true>(G);
     return nullptr;
 }
 

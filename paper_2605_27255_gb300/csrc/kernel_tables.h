@@ -25,6 +25,7 @@ void* k_pick_wait_selftest();                       // wait_selftest_kernel (rep
 // k_attn.cu: attention and RoPE / append kernels
 void* k_pick_attn_decode(bool bf, int DH, int G);   // attn_decode_kernel
 void* k_pick_attn_cluster(bool bf, int DH, int G);  // attn_cluster_kernel
+void* k_pick_attn_flat(bool bf, int DH, int G);     // attn_cluster_kernel, unclustered (global merge)
 void* k_pick_attn_mma(int G);                       // attn_mma_kernel
 void* k_pick_attn_prefill(int G);                   // attn_prefill_kernel
 void* k_pick_rope_append(bool bf, int DH);          // rope_append_kernel

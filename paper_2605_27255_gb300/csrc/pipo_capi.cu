@@ -145,6 +145,8 @@ struct pipo_ctx {
     int attn_cs_target = 0;           // attention CTAs per SM above which clusters shrink (0: per kernel)
     bool attn_v0 = false;             // (development) the unclustered attention path
     bool attn_regs = false;           // register-ring attention instead of the tensor-core one
+    int attn_flat = 1;                // register-ring decode attention without clusters (global merge):
+                                      // 0 never, 1 from kFlatMinEntries cached entries, 2 always
     std::vector<CUtensorMap> kv_tm;   // tensor-core attention: K and V tensor map of every cache layer
     int gemv_l2_prefetch = 0;         // streaming GEMV: weight chunks per warp hinted into L2 before the wait
     // per-launch timing (pipo_profile_step): events around every launch
@@ -535,16 +537,21 @@ TcPlan tc_plan(int sms, int bn, int tiles, int nkb, bool fused, bool allow_deep 
         const char* ev = getenv("PIPO_TC_DEEP");
         return ev ? atoi(ev) : -1;
     }();
+    // PIPO_TC_WAVES=w (experiment): plan up to w waves of CTAs instead of one
+    static const int waves = [] {
+        const char* ev = getenv("PIPO_TC_WAVES");
+        return ev ? std::max(1, atoi(ev)) : 1;
+    }();
     const bool deep = force_deep >= 0 ? force_deep == 1 : (allow_deep && tiles <= sms);
     const int target = sms * tc_ctas_per_sm(bn, deep, fused);
-    if (tiles >= target) return {1, deep};
+    if (tiles >= target * waves) return {1, deep};
     static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
-    for (int s = std::min({target / tiles, nkb / kTcMinKb, kTcMaxSplits}); s >= 2; --s) {
+    for (int s = std::min({target * waves / tiles, nkb / kTcMinKb, kTcMaxSplits}); s >= 2; --s) {
         const int mc = tc_max_clusters(bn, s, deep, fused);
         if (verbose)
             fprintf(stderr, "[pipo] tc plan: bh=%d deep=%d tiles=%d nkb=%d s=%d max_clusters=%d\n", bn, (int)deep, tiles,
                     nkb, s, mc);
-        if (mc >= tiles) return {s, deep};
+        if (mc * waves >= tiles) return {s, deep};
     }
     return {1, deep};
 }
@@ -839,6 +846,21 @@ int attn_cluster_size(const pipo_ctx* ctx, int B) {
     return cs;
 }
 
+// The register-ring decode attention without clusters (one CTA per SM, split
+// partials merged through global memory by the last arrival) against the
+// 8-CTA clusters (distributed-shared-memory merge), decided by the mean cached
+// length at graph capture.  Measured at 4B B = 1: 1156 entries 2.689 ms
+// (unclustered) against 2.660 ms per step; 8212 entries 3.082 against 3.539 ms.
+constexpr int kFlatMinEntries = 2048;
+bool attn_flat_now(const pipo_ctx* ctx) {
+    if (ctx->attn_flat <= 0) return false;
+    if (ctx->attn_flat >= 2) return true;
+    double sum = 0.0;
+    int n = 0;
+    for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b, ++n) sum += ctx->h_len[b];
+    return n > 0 && sum / n >= kFlatMinEntries;
+}
+
 // Long attention: the cached K/V bytes of a layer are at least six times the
 // QKV weight bytes (cached lengths at graph capture).  Then every projection
 // takes the two-per-SM ring, whose shared memory leaves room for a
@@ -920,7 +942,16 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
             TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, R), dim3(kMmaThreads), mma_attn_smem(),
                           margs, cs));
         }
-        else
+        else if (attn_flat_now(ctx) && !chunk && !ctx->attn_cs_force) {
+            // register-ring attention over about two CTAs per SM, no cluster:
+            // the split partials merge through the scratch (last arrival)
+            ap.part_o = ctx->part_o;
+            ap.part_ml = ctx->part_ml;
+            ap.counters = ctx->counters;
+            // one CTA per SM (the kernel's registers allow one), at least 16 entries per split
+            const int S = std::max(1, std::min({ctx->sms / (R * c.n_kv_heads), (c.max_ctx + 15) / 16, kFlatMaxSplits}));
+            TRY(launch_ex(ctx, k_pick_attn_flat(bf, DH, G), dim3(S, c.n_kv_heads, R), dim3(kAttnThreads), 0, args));
+        } else
             TRY(launch_ex(ctx, attnc_pick(bf, DH, G), dim3(cs, c.n_kv_heads, R), dim3(kAttnThreads), 0, args,
                           cs));
     } else {
@@ -1444,6 +1475,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         CK(set_carveouts(c.dtype == 1));
         if (const char* ev = getenv("PIPO_ATTN_V0")) ctx->attn_v0 = ev[0] == '1';
         if (const char* ev = getenv("PIPO_ATTN_IMPL")) ctx->attn_regs = strcmp(ev, "regs") == 0;
+        if (const char* ev = getenv("PIPO_ATTN_FLAT")) ctx->attn_flat = atoi(ev);
         if (attn_mma_ok(ctx)) {
             // the cache layers as 2-D tensors [blocks * n_kv * page][d_h] for the tensor-core attention
             const int rows = ctx->num_blocks * c.n_kv_heads * c.page_size;
@@ -2343,9 +2375,13 @@ pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {
     else proj = cuda_core;
     const int cs = attn_cluster_size(ctx, B);
     const bool mma = attn_use_mma(ctx, B) && cs <= 8;
+    const bool flat = !ctx->attn_v0 && !mma && attn_flat_now(ctx) && !ctx->attn_cs_force;
     std::string d = "B=" + std::to_string(B) + " projections=" + proj + " attention=" +
                     (ctx->attn_v0 ? std::string("attn_decode_kernel") : mma ? "attn_mma_kernel" : "attn_cluster_kernel") +
-                    " cluster=" + std::to_string(cs);
+                    (flat ? " unclustered splits=" +
+                                std::to_string(std::max(1, std::min({ctx->sms / (B * c.n_kv_heads), (c.max_ctx + 15) / 16,
+                                                                     kFlatMaxSplits})))
+                          : " cluster=" + std::to_string(cs));
     // decoding mode, heads and prefill arrangement
     d += ctx->regular ? " mode=regular" : " mode=pair";
     d += ctx->samp_on ? " heads=sampled" : " heads=argmax";

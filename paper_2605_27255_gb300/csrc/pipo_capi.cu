@@ -124,6 +124,7 @@ struct pipo_ctx {
     int act_rows = 0;               // rows of the fp32 activation buffers (>= the batch width BH)
     bool tc_shallow = false;        // this step's projections: two-per-SM ring (room for a co-resident neighbour)
     int tc_min_b = 2;               // measured: a tie with the CUDA-core GEMV at B = 1, far ahead from B = 4
+    int attn_mma_min_b = 2;         // smallest batch on the tensor-core attention (PIPO_ATTN_MMA_MIN_BATCH)
     int tc_splits = 0;              // forced K splits (0: automatic)
 
     int32_t *pending = nullptr, *n_pos = nullptr, *out_tokens = nullptr, *out_nacc = nullptr;
@@ -523,10 +524,9 @@ int tc_max_clusters(int bh, int cs, bool deep, bool fused) {
 }
 
 // Launch plan of a tensor-core projection: the K splits (the cluster size)
-// and the pipeline variant.  Tiles that fit one per SM take the deep ring,
-// split so that the CTAs still fit one per SM; more tiles take the two-per-SM
-// ring, split up to the SM slots.  Each split has at least kTcMinKb 64-wide K
-// blocks, at most kTcMaxSplits, and all clusters must fit at once (one wave).
+// and the pipeline variant (the two-per-SM ring, or the deep ring of one CTA
+// per SM).  Each split has at least kTcMinKb 64-wide K blocks, at most
+// kTcMaxSplits, and the clusters must fit in `waves` waves.
 constexpr int kTcMinKb = 4;
 struct TcPlan {
     int splits;
@@ -537,12 +537,21 @@ TcPlan tc_plan(int sms, int bn, int tiles, int nkb, bool fused, bool allow_deep 
         const char* ev = getenv("PIPO_TC_DEEP");
         return ev ? atoi(ev) : -1;
     }();
-    // PIPO_TC_WAVES=w (experiment): plan up to w waves of CTAs instead of one
+    // K splits planned for up to `waves` waves of CTAs on the two-per-SM ring.
+    // Measured (GB300, graph replay, ms per step; two waves on the two-per-SM
+    // ring / one wave with the deep ring where the tiles fit one per SM /
+    // one wave on the two-per-SM ring): 9b-b8 4.30 / 4.52 / 4.61, 4b-b16
+    // 2.83 / 2.96 / 3.17, 4b-b4 2.62 / 2.90 / 2.92, 4b-lc 4.49 / 4.76 / 4.77,
+    // 4b-b64 5.41 / 5.41 / 5.78; three or four waves, or two with the deep
+    // ring, were slower.  More waves let the hardware scheduler even out the
+    // SMs' finishing times; the splits of a tile stay one cluster.
+    // PIPO_TC_WAVES=1 restores the one-wave plan (deep ring when the tiles
+    // fit one per SM), PIPO_TC_DEEP=1 forces the deep ring.
     static const int waves = [] {
         const char* ev = getenv("PIPO_TC_WAVES");
-        return ev ? std::max(1, atoi(ev)) : 1;
+        return ev ? std::max(1, atoi(ev)) : 2;
     }();
-    const bool deep = force_deep >= 0 ? force_deep == 1 : (allow_deep && tiles <= sms);
+    const bool deep = force_deep >= 0 ? force_deep == 1 : (waves == 1 && allow_deep && tiles <= sms);
     const int target = sms * tc_ctas_per_sm(bn, deep, fused);
     if (tiles >= target * waves) return {1, deep};
     static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
@@ -828,7 +837,8 @@ bool attn_mma_ok(const pipo_ctx* ctx) {
 // next to the CUDA-core GEMVs, from B = 4 the tensor-core one by far), with
 // the cache tensor maps in place
 bool attn_use_mma(const pipo_ctx* ctx, int B) {
-    return attn_mma_ok(ctx) && B >= ctx->tc_min_b && (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers;
+    return attn_mma_ok(ctx) && B >= std::min(ctx->tc_min_b, ctx->attn_mma_min_b) &&
+           (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers;
 }
 
 // CTAs per (sequence, kv head) of the clustered attention: 8 while the batch
@@ -1531,6 +1541,7 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         CK(cudaMemset(ctx->gemv_rowcnt, 0, (size_t)MR * H * 4));
         // tensor-core projections: the bf16 activation tile
         if (const char* ev = getenv("PIPO_TC_MIN_BATCH")) ctx->tc_min_b = std::max(1, atoi(ev));
+        if (const char* ev = getenv("PIPO_ATTN_MMA_MIN_BATCH")) ctx->attn_mma_min_b = std::max(1, atoi(ev));
         if (const char* ev = getenv("PIPO_TC_SPLITS")) ctx->tc_splits = std::max(0, atoi(ev));
         if (c.dtype == 1 && MR >= ctx->tc_min_b) {
             ctx->tc_bn_max = tc_bn(std::min(MR, 128));

@@ -413,7 +413,9 @@ def run_pipo(args):
 
     prompts = synth.gen_prompts(B, T if not wl.get("kv_fill") else 2, shape.V, seed=1 + rank * 1000).numpy()
     t_pf = time.perf_counter()
+    torch.cuda.nvtx.range_push("prefill")  # ncu --nvtx --nvtx-include "prefill/": the prefill's launches
     g.prefill(prompts)
+    torch.cuda.nvtx.range_pop()
     t_pf = time.perf_counter() - t_pf
     if wl.get("kv_fill"):
         Kf, Vf = synth.gen_kv_fill(shape, n_pairs, seed=7, device="cuda")

@@ -11,7 +11,8 @@
 // distributed shared memory.
 //
 // Per CTA: a producer thread copies aligned 16-entry groups of the slice into
-// a ring of kMmaStages stages with TMA tensor copies: the cache layer is a 2-D
+// a ring of kMmaStages stages with TMA tensor copies (each compute warp owns
+// kMmaStages / kMmaWarps of the stages, see mma_stage): the cache layer is a 2-D
 // tensor of rows (block, kv head, slot) x d_h bf16, and a group is four boxes
 // of 16 rows x 64 dims (K and V, two halves each) stored with the 128-byte
 // swizzle, which keeps the ldmatrix reads free of bank conflicts.  Four
@@ -42,11 +43,23 @@ constexpr int kMmaStageBytes = 4 * kMmaHalf;        // K (2 halves) + V (2 halve
 #define PIPO_MMA_STAGES 10
 #endif
 #ifndef PIPO_MMA_WARPS
-#define PIPO_MMA_WARPS 4
+#define PIPO_MMA_WARPS 5
 #endif
 constexpr int kMmaStages = PIPO_MMA_STAGES;
 constexpr int kMmaWarps = PIPO_MMA_WARPS;           // compute warps (at least the G heads of a kv head)
 constexpr int kMmaThreads = (kMmaWarps + 1) * 32;   // + the producer warp
+constexpr int kMmaSpw = kMmaStages / kMmaWarps;     // stages of one compute warp
+static_assert(kMmaStages % kMmaWarps == 0, "every compute warp owns the same number of stages");
+
+// Group t (16 cached entries) is consumed by compute warp t % kMmaWarps and
+// travels through that warp's own stages in turn.  Each stage then has one
+// consumer taking its groups in order, so a consumer never waits on a stage
+// whose previous group is still in flight: mbarrier parity waits tell apart
+// only the current and the preceding phase, and with one ring shared by all
+// warps a fast warp could otherwise meet the parity of a phase two behind
+// (copies need not land in the order they were issued).  The k-th group of a
+// stage has phase k; the parity of group t is (t / kMmaStages) & 1.
+__device__ __forceinline__ int mma_stage(int t) { return (t % kMmaWarps) * kMmaSpw + (t / kMmaWarps) % kMmaSpw; }
 
 constexpr size_t mma_attn_smem() { return 1024 + (size_t)kMmaStages * kMmaStageBytes + 2 * kMmaStages * 8; }
 
@@ -144,7 +157,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             if (p.no_append) pdl_wait();
             int t = 0;
             for (; t < ngrp; ++t) {
-                const int st = t % kMmaStages;
+                const int st = mma_stage(t);
                 if (t >= kMmaStages && (*(volatile int*)&abort_flag ||
                                         !mbar_wait(empty + st, (uint32_t)(((t / kMmaStages) & 1) ^ 1), 21, t))) {
                     *(volatile int*)&abort_flag = 1;
@@ -162,7 +175,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             }
             // no copy into this CTA's shared memory may still be in flight at exit
             for (int i = max(0, t - kMmaStages); i < t; ++i)
-                mbar_wait(full + (i % kMmaStages), (uint32_t)((i / kMmaStages) & 1), 22, i);
+                mbar_wait(full + mma_stage(i), (uint32_t)((i / kMmaStages) & 1), 22, i);
         }
         __syncwarp();
     } else {
@@ -242,7 +255,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         const int lm = lane >> 3, lr = lane & 7;  // ldmatrix: matrix index, row within it
 
         for (int t = warp; t < ngrp; t += NW) {
-            const int st = t % kMmaStages;
+            const int st = mma_stage(t);
             if (*(volatile int*)&abort_flag || !mbar_wait(full + st, (uint32_t)((t / kMmaStages) & 1), 23, t)) {
                 *(volatile int*)&abort_flag = 1;
                 break;

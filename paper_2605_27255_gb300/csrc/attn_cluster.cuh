@@ -171,6 +171,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     __shared__ int last_cta;
 
     pdl_launch();
+    PIPO_TR(const TraceT0 tr0 = trace_begin(); unsigned long long tr1 = 0, tr2 = 0, tr3 = 0;)
     const int s = FLAT ? (int)blockIdx.x : (int)cg::this_cluster().block_rank();
     const int CS = FLAT ? (int)gridDim.x : (int)cg::this_cluster().num_blocks();
     const int g = blockIdx.y, row = blockIdx.z;
@@ -204,6 +205,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     float4 rope_cs[4];  // rotation of position n (static table)
     rope_load<DH>(rope_cs, li, n, p.rope);
     pdl_wait();
+    PIPO_TR(tr1 = trace_now();)
 
     // q of the G heads, 8 dims per lane, rotated, pre-scaled
     float q[G][8];
@@ -326,6 +328,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
         }
     }
 
+    PIPO_TR(tr2 = trace_now();)
     // merge the EPW lane groups of the warp (same dims, different entries)
 #pragma unroll
     for (int hh = 0; hh < G; ++hh) {
@@ -374,6 +377,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
             if (t == 0) { sm_m[hh] = M; sm_l[hh] = L; }
         }
     }
+    PIPO_TR(tr3 = trace_now();)
     if constexpr (FLAT) {
         // the last CTA of (row, kv head) to arrive merges the CS partials in split order
         __threadfence();
@@ -384,6 +388,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
             if (last_cta) p.counters[row * n_kv + g] = 0u;
         }
         __syncthreads();
+        PIPO_TR(if (threadIdx.x == 0) trace_put(TR_ATTN_FLAT, tr0, tr0.clk, tr1, tr2, tr3);)
         if (!last_cta) return;
         __threadfence();
         // (m, l) of every split in one round of loads, the split weights per
@@ -435,6 +440,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
             cluster_merge_elem(cluster, &sm_m[hh], &sm_l[hh], &sm_o[hh][t], CS);
     }
     cluster.sync();  // keep every CTA's shared memory alive until all merges read it
+    PIPO_TR(if (threadIdx.x == 0) trace_put(TR_ATTN_CL, tr0, tr0.clk, tr1, tr2, tr3);)
 }
 
 }  // namespace pipo

@@ -115,6 +115,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     __shared__ float wm[NP][G], wl[NP][G];
     __shared__ float wo[NP][G][DH];
     __shared__ int abort_flag;
+    PIPO_TR(__shared__ unsigned long long tr_s[3], tr_m[2]; const TraceT0 tr0 = trace_begin();)
 
     unsigned char* ring = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(am_smem_raw) + 1023) & ~(uintptr_t)1023);
     uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)kMmaStages * kMmaStageBytes);
@@ -182,6 +183,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         const int ct = threadIdx.x;  // 0 .. 32*NW-1
         // ---- prologue: rotated, pre-scaled q of the G heads; the new k, v
         pdl_wait();
+        PIPO_TR(if (ct == 0) tr_s[0] = trace_now();)
         const float* qrow = p.qkv + (size_t)row * p.ld_qkv;
         const float* rope = p.rope + (size_t)n * DH;  // [DH/2][2] cos, sin at position n
         for (int i = ct; i < (G + 1) * (DH / 2); i += 32 * NW) {
@@ -203,6 +205,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             for (int d = ct; d < DH; d += 32 * NW)
                 vn_s[d] = __bfloat162float(__float2bfloat16_rn(qrow[(size_t)(n_q + n_kv + g) * DH + d]));
         asm volatile("bar.sync 1, %0;" ::"n"(32 * NW) : "memory");  // compute warps only
+        PIPO_TR(if (ct == 0) tr_s[1] = trace_now();)
 
         // the new entry: append it to the cache and make it partial NW
         if (owns_new) {
@@ -333,6 +336,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             if (lane == 0) mbar_arrive(empty + st);  // this group's stage is free
         }
 
+        PIPO_TR(if (ct == 0) tr_m[0] = trace_now();)
         // warp partial: O of head r = bf16-part row r + remainder row r + G
 #pragma unroll
         for (int nd = 0; nd < DH / 8; ++nd)
@@ -363,7 +367,9 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         sm_o[hh][t] = Ov;
         if (t == 0) { sm_m[hh] = M; sm_l[hh] = L; }
     }
+    PIPO_TR(if (threadIdx.x == 0) tr_s[2] = trace_now();)
     cluster.sync();
+    PIPO_TR(if (threadIdx.x == 0) tr_m[1] = trace_now();)
     // cluster merge: CTA s finishes dims [s*G*DH/CS, (s+1)*G*DH/CS) of the G heads
     const int PER = (G * DH + CS - 1) / CS;
     for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
@@ -372,6 +378,10 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             cluster_merge_elem(cluster, &sm_m[hh], &sm_l[hh], &sm_o[hh][t], CS);
     }
     cluster.sync();  // keep every CTA's shared memory alive until all merges read it
+    PIPO_TR(if (threadIdx.x == 0) {
+        trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);
+        trace_put(TR_ATTN_MMA_EPI, tr0, tr_s[0], tr_s[1], tr_m[0], tr_s[2], tr_m[1]);
+    })
 }
 
 }  // namespace pipo

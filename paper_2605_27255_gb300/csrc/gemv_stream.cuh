@@ -615,6 +615,9 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
     constexpr int EPC = Chunk16<T>::kElems;
 
     pdl_launch();
+    PIPO_TR(const TraceT0 tr0 = trace_begin(); unsigned long long tr1 = 0;
+            __shared__ unsigned long long tr_lo, tr_hi;
+            if (threadIdx.x == 0) { tr_lo = ~0ull; tr_hi = 0ull; })
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int K = p.K;
     const int cpr = K * (int)sizeof(T) / 512;  // exact
@@ -648,6 +651,7 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
                 if (n > 0) prefetch_l2_bulk(wbase + (size_t)(c0 + 2 * kU) * 512, (uint32_t)n * 512u);
             }
             pdl_wait();
+            PIPO_TR(tr1 = trace_now();)
             if (p.zero_ptr && blockIdx.x == 0)
                 for (int i = threadIdx.x; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
         }
@@ -734,6 +738,7 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
             consume_batch(bufB);
             load_batch(bufB);
         }
+        PIPO_TR(if (lane == 0) { const unsigned long long te = trace_now(); atomicMin(&tr_lo, te); atomicMax(&tr_hi, te); })
         // the range ended inside a unit: record the partial (rows done + running row)
         if (c0 < c1 && (c1 % cpu) != 0) {
             const int unit = (c1 - 1) / cpu;
@@ -798,6 +803,7 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
         }
         __syncthreads();
     }
+    PIPO_TR(if (threadIdx.x == 0) trace_put(TR_GEMV, tr0, tr0.clk, tr1, tr_lo, tr_hi);)
 }
 
 // ---------------------------------------------------------------------------

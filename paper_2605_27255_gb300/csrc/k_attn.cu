@@ -97,4 +97,8 @@ void* k_pick_append_rows(bool bf, int DH) {
 
 cudaError_t k_take_error_attn(unsigned* code, unsigned* info) { return take_unit_error(code, info); }
 
+#ifdef PIPO_TRACE
+cudaError_t k_trace_set_attn(unsigned long long* buf) { return set_unit_trace(buf); }
+#endif
+
 }  // namespace pipo

@@ -64,4 +64,8 @@ __global__ void wait_selftest_kernel(int signal, unsigned long long limit_ns) {
 
 void* k_pick_wait_selftest() { return reinterpret_cast<void*>(&wait_selftest_kernel); }
 
+#ifdef PIPO_TRACE
+cudaError_t k_trace_set_tc(unsigned long long* buf) { return set_unit_trace(buf); }
+#endif
+
 }  // namespace pipo

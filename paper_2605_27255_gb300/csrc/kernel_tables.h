@@ -32,4 +32,12 @@ void* k_pick_rope_append(bool bf, int DH);          // rope_append_kernel
 void* k_pick_append_rows(bool bf, int DH);          // append_rows_kernel
 cudaError_t k_take_error_attn(unsigned* code, unsigned* info);
 
+#ifdef PIPO_TRACE
+// measurement build only: point each unit's timeline buffer at `buf` (or nullptr)
+cudaError_t k_trace_set_gemv_bf16(unsigned long long* buf);
+cudaError_t k_trace_set_gemv_f32(unsigned long long* buf);
+cudaError_t k_trace_set_tc(unsigned long long* buf);
+cudaError_t k_trace_set_attn(unsigned long long* buf);
+#endif
+
 }  // namespace pipo

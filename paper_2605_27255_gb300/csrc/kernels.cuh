@@ -140,6 +140,70 @@ __device__ __forceinline__ int argmax_row(unsigned long long k) {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// ---------------------------------------------------------------- timeline
+//
+// Built only with -DPIPO_TRACE (a measurement build; the default build has
+// none of it): one record per CTA of the projection and attention kernels,
+// {kind | sm << 8 | CTAs of the grid << 16 | linear block << 32, entry time,
+// time past the dependency wait, two kernel-specific phase times, exit time}
+// (%globaltimer, ns), appended to a device buffer [count, capacity, records]
+// whose address each translation unit holds (set by the host, see
+// pipo_trace_setup).  The records show, under graph replay with programmatic
+// dependent launch, when each CTA started, waited and finished.
+enum TraceKind : unsigned { TR_GEMV = 1, TR_TCF = 2, TR_TC = 3, TR_ATTN_MMA = 4, TR_ATTN_CL = 5, TR_ATTN_FLAT = 6,
+                       TR_TCF_EPI = 7, TR_ATTN_MMA_EPI = 8 };
+#ifdef PIPO_TRACE
+constexpr int kTraceWords = 6;
+// Phase times are SM cycles (clock64: no memory path, unlike %globaltimer
+// reads, which queue behind outstanding loads) placed on the global clock
+// through one (%globaltimer, clock64) pair read at entry, at the 2070 MHz SM
+// clock the benchmark runs at.
+constexpr double kTraceNsPerClk = 1.0 / 2.07;
+static __device__ unsigned long long* g_trace_buf;
+struct TraceT0 {
+    unsigned long long gt, clk;
+};
+__device__ __forceinline__ unsigned long long trace_now() { return (unsigned long long)clock64(); }
+// read by thread 0 only (which writes the records): the others get zeros
+__device__ __forceinline__ TraceT0 trace_begin() {
+    TraceT0 b{0ull, 0ull};
+    if (threadIdx.x == 0) {
+        asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(b.gt));
+        b.clk = trace_now();
+    }
+    return b;
+}
+__device__ __forceinline__ unsigned long long trace_ns(const TraceT0& b, unsigned long long c) {
+    return c ? b.gt + (unsigned long long)((double)(long long)(c - b.clk) * kTraceNsPerClk) : 0ull;
+}
+__device__ __forceinline__ void trace_put(unsigned kind, const TraceT0& base, unsigned long long t0,
+                                          unsigned long long t1, unsigned long long t2, unsigned long long t3,
+                                          unsigned long long t4 = 0) {
+    if (!t4) t4 = trace_now();  // exit: before the slot atomic and its latency
+    unsigned long long* b = g_trace_buf;
+    if (!b) return;
+    const unsigned long long i = atomicAdd(b, 1ull);
+    if (i >= b[1]) return;
+    unsigned sm;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
+    const unsigned long long nblk = (unsigned long long)gridDim.x * gridDim.y * gridDim.z;
+    const unsigned long long blk = blockIdx.x + (unsigned long long)gridDim.x * (blockIdx.y + (unsigned long long)gridDim.y * blockIdx.z);
+    unsigned long long* r = b + 2 + i * kTraceWords;
+    r[0] = kind | ((unsigned long long)(sm & 0xffu) << 8) | ((nblk & 0xffffull) << 16) | (blk << 32);
+    r[1] = trace_ns(base, t0);
+    r[2] = trace_ns(base, t1);
+    r[3] = trace_ns(base, t2);
+    r[4] = trace_ns(base, t3);
+    r[5] = trace_ns(base, t4);
+}
+static inline cudaError_t set_unit_trace(unsigned long long* buf) {
+    return cudaMemcpyToSymbol(g_trace_buf, &buf, sizeof(buf));
+}
+#define PIPO_TR(...) __VA_ARGS__
+#else
+#define PIPO_TR(...)
+#endif
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

@@ -2359,6 +2359,52 @@ pipo_status pipo_selftest_wait(int32_t signal, uint64_t limit_ns, uint32_t* h_in
     return PIPO_OK;
 }
 
+#ifdef PIPO_TRACE
+// Measurement build only (not part of the header): one timeline buffer of
+// `cap` CTA records for the whole process, shared by every kernel unit.
+// pipo_trace_setup(0) detaches and frees it.  pipo_trace_fetch copies the
+// record count and up to cap records (6 words each) to h_out and resets the
+// count.
+namespace {
+unsigned long long* g_trace_dev = nullptr;
+size_t g_trace_cap = 0;
+}  // namespace
+
+PIPO_API pipo_status pipo_trace_setup(size_t cap) {
+    pipo_ctx* ctx = nullptr;
+    unsigned long long* buf = nullptr;
+    if (cap) {
+        CK(cudaMalloc(&buf, (2 + kTraceWords * cap) * sizeof(unsigned long long)));
+        const unsigned long long head[2] = {0ull, (unsigned long long)cap};
+        CK(cudaMemset(buf, 0, (2 + kTraceWords * cap) * sizeof(unsigned long long)));
+        CK(cudaMemcpy(buf, head, sizeof(head), cudaMemcpyHostToDevice));
+    }
+    CK(k_trace_set_gemv_bf16(buf));
+    CK(k_trace_set_gemv_f32(buf));
+    CK(k_trace_set_tc(buf));
+    CK(k_trace_set_attn(buf));
+    CK(cudaDeviceSynchronize());
+    if (g_trace_dev) CK(cudaFree(g_trace_dev));
+    g_trace_dev = buf;
+    g_trace_cap = cap;
+    return PIPO_OK;
+}
+
+PIPO_API pipo_status pipo_trace_fetch(unsigned long long* h_out, size_t cap, unsigned long long* h_n) {
+    pipo_ctx* ctx = nullptr;
+    if (!g_trace_dev) return fail(nullptr, PIPO_ESTATE, "pipo_trace_fetch: no trace buffer");
+    CK(cudaDeviceSynchronize());
+    unsigned long long n = 0;
+    CK(cudaMemcpy(&n, g_trace_dev, sizeof(n), cudaMemcpyDeviceToHost));
+    *h_n = n;
+    const size_t m = std::min<size_t>(std::min<size_t>(n, cap), g_trace_cap);
+    if (m) CK(cudaMemcpy(h_out, g_trace_dev + 2, m * kTraceWords * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
+    CK(cudaMemset(g_trace_dev, 0, sizeof(unsigned long long)));
+    CK(cudaDeviceSynchronize());
+    return PIPO_OK;
+}
+#endif
+
 pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {
     if (!ctx || !h_buf || cap == 0) return fail(nullptr, PIPO_EINVAL, "pipo_describe_step: bad arguments");
     const pipo_config& c = ctx->cfg;

@@ -248,6 +248,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
     __shared__ uint32_t tmem_base;
     __shared__ float red_v[4][BH];
     __shared__ int red_r[4][BH];
+    PIPO_TR(__shared__ unsigned long long tr_s[3]; const TraceT0 tr0 = trace_begin();)
 
     pdl_launch();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -286,6 +287,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
                 tma_load_2d(sA + i * kTcABytes, &tmW, (kb0 + i) * kTcBK, tile * kTcM, full + i);
             }
             pdl_wait();
+            PIPO_TR(tr_s[0] = trace_now();)
             for (int i = 0; i < pre; ++i) tma_load_2d(sB + i * kBBytes, &tmX, (kb0 + i) * kTcBK, 0, full + i);
             int issued = pre;
             for (int i = pre; i < nk; ++i) {
@@ -323,6 +325,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
 
     // epilogue: thread t holds TMEM lane t = weight row tile*128 + t
     mbar_wait(accb, 0, 14, (unsigned)nk);
+    PIPO_TR(if (threadIdx.x == 0) tr_s[1] = trace_now();)
     __syncwarp();
     tc_fence_after();
     pdl_wait();
@@ -383,12 +386,14 @@ __global__ void __launch_bounds__(kTcThreads, 1) gemm_tc_kernel(const __grid_con
         }
         cl.sync();  // no CTA leaves while others still read its shared memory
     }
+    PIPO_TR(if (threadIdx.x == 0) tr_s[2] = trace_now();)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc(tmem, kCols);
     }
+    PIPO_TR(if (threadIdx.x == 0) trace_put(TR_TC, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);)
 }
 
 // ---------------------------------------------------------------- fused form
@@ -442,6 +447,7 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
     __shared__ float red_v[4][BH];
     __shared__ int red_r[4][BH];
     __shared__ float ss_s[BH], rstd_s[BH];
+    PIPO_TR(__shared__ unsigned long long tr_s[3], tr_e[3]; const TraceT0 tr0 = trace_begin();)
 
     pdl_launch();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -530,6 +536,7 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
         // converter warps: raw fp32 tile -> bf16 hi | lo operand tile, sum(x^2)
         const int xt = threadIdx.x - 64;  // 0..127
         pdl_wait();
+        PIPO_TR(if (xt == 0) tr_s[0] = trace_now();)
         if (in.zero_ptr && blockIdx.x == 0)
             for (int i = xt; i < in.zero_n; i += 128) in.zero_ptr[i] = 0ull;
         float ss[NQ];
@@ -603,6 +610,7 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
     const bool epi_warp = warp >= 2;
     if (epi_warp) {
         mbar_wait(accb, 0, 14, (unsigned)nk);
+        PIPO_TR(if (threadIdx.x == 64) tr_s[1] = trace_now();)
         __syncwarp();
         tc_fence_after();
     }
@@ -619,10 +627,12 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
             for (int c0 = 0; c0 < BH; c0 += 16) {
                 float v[16];
                 ld_cols(c0, v);
+                PIPO_TR(if (threadIdx.x == 64 && c0 == 0) tr_e[0] = trace_now();)
 #pragma unroll
                 for (int j = 0; j < 16; ++j) v[j] *= rstd_s[c0 + j];
                 tc_epilogue16<BH>(p, row, c0, v, red_v, red_r, quad);
             }
+            PIPO_TR(if (threadIdx.x == 64) { tr_e[1] = trace_now(); tr_e[2] = tr_e[1]; })
             if (p.epi == EPI_ARGMAX) {
                 asm volatile("bar.sync 1, 128;" ::: "memory");
                 const int b = threadIdx.x - 64;
@@ -654,8 +664,10 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
                     *reinterpret_cast<float4*>(park + tc_park_idx<BH>(r, c0 / 4 + q)) =
                         make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
             }
+            PIPO_TR(if (threadIdx.x == 64) tr_e[0] = trace_now();)
         }
         cl.sync();  // every split's partial tile and sum(x^2) are in place
+        PIPO_TR(if (threadIdx.x == 64) tr_e[1] = trace_now();)
         if (epi_warp) {
             const int xt = threadIdx.x - 64;
             if (xt < BH) {
@@ -672,15 +684,21 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
                 const int rr = r0 + (it / (BH / 4)) * step, c4 = it % (BH / 4);
                 tc_cluster_epilogue<BH>(p, cl, park, tile, rr, c4, rstd_s);
             }
+            PIPO_TR(if (threadIdx.x == 64) tr_e[2] = trace_now();)
         }
         cl.sync();  // no CTA leaves while others still read its shared memory
     }
+    PIPO_TR(if (threadIdx.x == 64) tr_s[2] = trace_now();)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc(tmem, kCols);
     }
+    PIPO_TR(if (threadIdx.x == 0) {
+        trace_put(TR_TCF, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);
+        trace_put(TR_TCF_EPI, tr0, tr_s[1], tr_e[0], tr_e[1], tr_e[2]);
+    })
 }
 
 // Activations of the tensor-core GEMM, [2 * BH][K] bf16: row b < B holds

@@ -31,6 +31,7 @@
 #include <cooperative_groups.h>
 
 #include "kernels.cuh"
+#include "tma.cuh"
 
 namespace pipo {
 
@@ -86,6 +87,10 @@ struct AttnParams {
     float* part_o;
     float* part_ml;
     unsigned* counters;
+    // staged form (stage_max > 0): the CTA's whole slice of cached keys and
+    // values is copied to shared memory (bulk copies, one per page run and
+    // tensor) before the dependency wait; stage_max entries fit
+    int stage_max;
 };
 
 // cos/sin of the 8 rotation pairs of lane slice li at position pos
@@ -169,9 +174,11 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     __shared__ float wo[NW][G][DH];
 
     __shared__ int last_cta;
+    __shared__ __align__(8) uint64_t kv_bar;
+    extern __shared__ __align__(128) unsigned char kv_stage[];  // staged form: [stage_max][DH] keys, then values
 
     pdl_launch();
-    PIPO_TR(const TraceT0 tr0 = trace_begin(); unsigned long long tr1 = 0, tr2 = 0, tr3 = 0;)
+    PIPO_TR(const TraceT0 tr0 = trace_begin(); unsigned long long tr1 = 0, tr2 = 0, tr3 = 0, trq = 0, trk = 0, trc = 0;)
     const int s = FLAT ? (int)blockIdx.x : (int)cg::this_cluster().block_rank();
     const int CS = FLAT ? (int)gridDim.x : (int)cg::this_cluster().num_blocks();
     const int g = blockIdx.y, row = blockIdx.z;
@@ -187,6 +194,25 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     const T* Kb = static_cast<const T*>(p.kv.K);
     const T* Vb = static_cast<const T*>(p.kv.V);
 
+    // staged form: the whole slice to shared memory, page run by page run
+    const bool staged = p.stage_max > 0 && !p.no_append && jc - j0 <= p.stage_max;
+    if (staged) {
+        if (threadIdx.x == 0) {
+            mbar_init(&kv_bar, 1);
+            mbar_init_fence();
+            const uint32_t eb = (uint32_t)(DH * sizeof(T));  // bytes of one entry (a multiple of 16)
+            mbar_arrive_expect_tx(&kv_bar, (uint32_t)(jc > j0 ? jc - j0 : 0) * eb * 2u);
+            unsigned char* vs = kv_stage + (size_t)p.stage_max * eb;
+            for (int j = j0; j < jc;) {
+                const int run = min(jc, (j / p.kv.page + 1) * p.kv.page) - j;  // entries left in this page
+                const size_t off = kv_off<T, DH>(p.kv, b, j, g);
+                bulk_g2s(kv_stage + (size_t)(j - j0) * eb, static_cast<const T*>(p.kv.K) + off, (uint32_t)run * eb, &kv_bar);
+                bulk_g2s(vs + (size_t)(j - j0) * eb, static_cast<const T*>(p.kv.V) + off, (uint32_t)run * eb, &kv_bar);
+                j += run;
+            }
+        }
+        __syncthreads();  // the barrier's initialisation, before any other thread waits on it
+    }
     // prefetch the first kU warp steps of keys/values (independent of this
     // step, unless the entries were appended by the kernel before)
     if (p.no_append) pdl_wait();
@@ -195,12 +221,14 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     // loads are unconditional: an entry outside the slice reads entry 0 of the
     // sequence instead and is masked out of the softmax (a select on a load
     // result would make the thread wait for it)
+    if (!staged) {
 #pragma unroll
-    for (int u = 0; u < kU; ++u) {
-        const int j = jwb + slot + u * STEP;
-        const size_t off = kv_off<T, DH>(p.kv, b, j < jc ? j : 0, g) + li * 8;
-        kr[u].load(Kb + off);
-        vr[u].load(Vb + off);
+        for (int u = 0; u < kU; ++u) {
+            const int j = jwb + slot + u * STEP;
+            const size_t off = kv_off<T, DH>(p.kv, b, j < jc ? j : 0, g) + li * 8;
+            kr[u].load(Kb + off);
+            vr[u].load(Vb + off);
+        }
     }
     float4 rope_cs[4];  // rotation of position n (static table)
     rope_load<DH>(rope_cs, li, n, p.rope);
@@ -220,6 +248,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
 #pragma unroll
         for (int e = 0; e < 8; ++e) q[hh][e] *= p.scale;
     }
+    PIPO_TR(trq = trace_now() + (q[0][0] == 12345.f ? 1 : 0);)
 
     float m[G], l[G], o[G][8];
 #pragma unroll
@@ -273,18 +302,37 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
         }
     };
 
-    for (int jb = jwb; jb < jc; jb += kU * STEP) {  // warp-uniform trip count
-        KV8<T> kn[kU], vn[kU];
+    if (staged) {
+        // the slice in shared memory: every lane group takes its entries in turn
+        if (jc > j0) mbar_wait(&kv_bar, 0, 27, (unsigned)(jc - j0));
+        PIPO_TR(trk = trace_now();)
+        const size_t eb = (size_t)DH * sizeof(T);
+        const unsigned char* ks = kv_stage + li * 8 * sizeof(T);
+        const unsigned char* vs = kv_stage + (size_t)p.stage_max * eb + li * 8 * sizeof(T);
+        for (int jb = jwb; jb < jc; jb += kU * STEP) {  // warp-uniform trip count
 #pragma unroll
-        for (int u = 0; u < kU; ++u) {
-            const int j = jb + slot + (kU + u) * STEP;
-            const size_t off = kv_off<T, DH>(p.kv, b, j < jc ? j : 0, g) + li * 8;
-            kn[u].load(Kb + off);
-            vn[u].load(Vb + off);
+            for (int u = 0; u < kU; ++u) {
+                const int j = jb + slot + u * STEP;
+                const size_t e = (size_t)((j < jc ? j : j0) - j0) * eb;
+                kr[u].load_s(ks + e);
+                vr[u].load_s(vs + e);
+            }
+            consume(kr, vr, jb + slot);
         }
-        consume(kr, vr, jb + slot);
+    } else {
+        for (int jb = jwb; jb < jc; jb += kU * STEP) {  // warp-uniform trip count
+            KV8<T> kn[kU], vn[kU];
 #pragma unroll
-        for (int u = 0; u < kU; ++u) { kr[u] = kn[u]; vr[u] = vn[u]; }
+            for (int u = 0; u < kU; ++u) {
+                const int j = jb + slot + (kU + u) * STEP;
+                const size_t off = kv_off<T, DH>(p.kv, b, j < jc ? j : 0, g) + li * 8;
+                kn[u].load(Kb + off);
+                vn[u].load(Vb + off);
+            }
+            consume(kr, vr, jb + slot);
+#pragma unroll
+            for (int u = 0; u < kU; ++u) { kr[u] = kn[u]; vr[u] = vn[u]; }
+        }
     }
 
     // the new entry n: rotate k, round k and v to the cache type, append, attend
@@ -432,6 +480,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
     }
     cg::cluster_group cluster = cg::this_cluster();
     cluster.sync();
+    PIPO_TR(trc = trace_now();)
     // cluster merge: CTA s finishes dims [s*G*DH/CS, (s+1)*G*DH/CS) of the G heads
     const int PER = (G * DH + CS - 1) / CS;
     for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
@@ -440,7 +489,10 @@ __global__ void __launch_bounds__(kAttnThreads) attn_cluster_kernel(AttnParams p
             cluster_merge_elem(cluster, &sm_m[hh], &sm_l[hh], &sm_o[hh][t], CS);
     }
     cluster.sync();  // keep every CTA's shared memory alive until all merges read it
-    PIPO_TR(if (threadIdx.x == 0) trace_put(TR_ATTN_CL, tr0, tr0.clk, tr1, tr2, tr3);)
+    PIPO_TR(if (threadIdx.x == 0) {
+        trace_put(TR_ATTN_CL, tr0, tr0.clk, tr1, tr2, tr3);
+        trace_put(TR_ATTN_CL_EPI, tr0, tr1, trq, trk, tr2, trc);
+    })
 }
 
 }  // namespace pipo

@@ -151,7 +151,7 @@ __device__ __forceinline__ void pdl_launch() { asm volatile("griddepcontrol.laun
 // pipo_trace_setup).  The records show, under graph replay with programmatic
 // dependent launch, when each CTA started, waited and finished.
 enum TraceKind : unsigned { TR_GEMV = 1, TR_TCF = 2, TR_TC = 3, TR_ATTN_MMA = 4, TR_ATTN_CL = 5, TR_ATTN_FLAT = 6,
-                       TR_TCF_EPI = 7, TR_ATTN_MMA_EPI = 8 };
+                       TR_TCF_EPI = 7, TR_ATTN_MMA_EPI = 8, TR_ATTN_CL_EPI = 11 };
 #ifdef PIPO_TRACE
 constexpr int kTraceWords = 6;
 // Phase times are SM cycles (clock64: no memory path, unlike %globaltimer

@@ -293,6 +293,9 @@ void* pick_stream(int nb, int ru, bool rows) {
 }
 
 constexpr size_t kXsBudget = 100 * 1024;      // staged-input bytes per v0 GEMV block
+// shared memory of the staged register-ring attention (the CTA's slice of
+// cached keys and values); longer slices take the register ring alone
+constexpr size_t kAttnStageMax = 160 * 1024;
 constexpr size_t kStreamBudget = 200 * 1024;  // staged-input bytes per streaming GEMV block
 
 // Launch with programmatic dependent launch (decode graph) and an optional
@@ -399,6 +402,13 @@ cudaError_t set_smem_attrs(bool bf) {
             cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kXsBudget);
             if (e != cudaSuccess) return e;
         }
+    for (int dh : {64, 128})
+        for (int g : {1, 2, 4, 8})
+            for (void* f : {k_pick_attn_cluster(bf, dh, g), k_pick_attn_flat(bf, dh, g)}) {
+                if (!f) continue;
+                cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kAttnStageMax);
+                if (e != cudaSuccess) return e;
+            }
     if (bf)
         for (int g : {1, 2, 4}) {
             cudaError_t e = cudaFuncSetAttribute(attnm_pick(g), cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -895,6 +905,27 @@ bool attn_is_long(const pipo_ctx* ctx) {
     return kv_bytes >= 6.0 * qkv_bytes;
 }
 
+// Staged form of the register-ring decode attention: when the longest slice
+// a CTA can get (the context capacity over `splits`) fits kAttnStageMax, the
+// CTA copies its slice of cached keys and values to shared memory before the
+// dependency wait and attends from there.  Returns the dynamic shared memory
+// and sets *stage_max (0: the register ring alone).  PIPO_ATTN_STAGE=0 turns
+// it off.
+size_t attn_stage(const pipo_ctx* ctx, int splits, bool chunk, int* stage_max) {
+    static const bool off = [] {
+        const char* ev = getenv("PIPO_ATTN_STAGE");
+        return ev && ev[0] == '0';
+    }();
+    *stage_max = 0;
+    if (off || chunk || splits < 1) return 0;
+    const pipo_config& c = ctx->cfg;
+    const int entries = (c.max_ctx + splits - 1) / splits + 1;
+    const size_t bytes = (size_t)entries * c.head_dim * ctx->esz * 2;
+    if (bytes > kAttnStageMax) return 0;
+    *stage_max = entries;
+    return bytes;
+}
+
 // One decoder block on the residual stream xr (pre-norm attention + SwiGLU).
 pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, float* xr) {
     const pipo_config& c = ctx->cfg;
@@ -960,10 +991,13 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
             ap.counters = ctx->counters;
             // one CTA per SM (the kernel's registers allow one), at least 16 entries per split
             const int S = std::max(1, std::min({ctx->sms / (R * c.n_kv_heads), (c.max_ctx + 15) / 16, kFlatMaxSplits}));
-            TRY(launch_ex(ctx, k_pick_attn_flat(bf, DH, G), dim3(S, c.n_kv_heads, R), dim3(kAttnThreads), 0, args));
-        } else
-            TRY(launch_ex(ctx, attnc_pick(bf, DH, G), dim3(cs, c.n_kv_heads, R), dim3(kAttnThreads), 0, args,
+            const size_t smem = attn_stage(ctx, S, chunk, &ap.stage_max);
+            TRY(launch_ex(ctx, k_pick_attn_flat(bf, DH, G), dim3(S, c.n_kv_heads, R), dim3(kAttnThreads), smem, args));
+        } else {
+            const size_t smem = attn_stage(ctx, cs, chunk, &ap.stage_max);
+            TRY(launch_ex(ctx, attnc_pick(bf, DH, G), dim3(cs, c.n_kv_heads, R), dim3(kAttnThreads), smem, args,
                           cs));
+        }
     } else {
     // RoPE + KV append
     {

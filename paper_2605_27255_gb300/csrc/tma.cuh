@@ -19,7 +19,8 @@ static __device__ unsigned int g_pipo_error;
 // First wait that gave up: {site code, linear block index, iteration, parity}
 // (the site codes name the wait: 11-15 projection GEMM producer-empty,
 // producer-drain, MMA-full, epilogue-accumulator, converter-full; 21-23 attention
-// producer-empty, producer-drain, consumer-full; 24-26 prefill attention;
+// producer-empty, producer-drain, consumer-full; 24-26 prefill attention; 27 the
+// staged single-sequence attention;
 // 90 the wait self-test).
 static __device__ unsigned int g_pipo_error_info[4];
 constexpr unsigned kErrWaitTimeout = 1u;

@@ -103,7 +103,8 @@ __device__ __forceinline__ void stage_input(const GemvParams& p, float* xs, int 
 // Epilogue of one finished unit u with sums a[r][bb] (lane-uniform).
 template <typename T, int RU, int NB>
 __device__ __forceinline__ void unit_epilogue(const GemvParams& p, int u, const float (&a)[RU][NB], int b0, int nb,
-                                              float (&best_v)[NB], int (&best_r)[NB]) {
+                                              float (&best_v)[NB], int (&best_r)[NB],
+                                              const float* ypre = nullptr) {
     const int lane = threadIdx.x & 31;
     if (p.epi == EPI_ARGMAX) {
 #pragma unroll
@@ -128,7 +129,7 @@ __device__ __forceinline__ void unit_epilogue(const GemvParams& p, int u, const 
             case EPI_STORE: *yp = s; break;
             case EPI_BIAS: *yp = s + ldw<T>(p.bias, u); break;
             case EPI_SILU: *yp = silu(s); break;
-            case EPI_RESADD: *yp += s; break;
+            case EPI_RESADD: *yp = (ypre ? ypre[bb] : *yp) + s; break;
             case EPI_SWIGLU: *yp = silu(s) * a[RU - 1][bb]; break;
             default: break;
         }
@@ -512,14 +513,20 @@ __device__ __forceinline__ void cp_async_wait_all() {
 // embedding rows (compressor and MTP inputs only) through registers; then one
 // block reduction for the norms and one scaling pass in shared memory.
 // gsm: K elements of type T for the gains.  Same split layout as stage_input_fast.
+// yres (EPI_RESADD, or nullptr): [units][NB] receives y of units [u0, u0 +
+// units) of sequences b0 .. b0 + nb - 1, loaded while the input copies fly.
 template <typename T, int NB>
-__device__ __forceinline__ void stage_input_async(const GemvParams& p, float* xs, T* gsm, int b0, int nb) {
+__device__ __forceinline__ void stage_input_async(const GemvParams& p, float* xs, T* gsm, int b0, int nb,
+                                                  float (*yres)[NB] = nullptr, int u0 = 0, int units = 0) {
     __shared__ float red_ss[32][NB][2];
     __shared__ float rstd_s[NB][2];
     const int K = p.K, K0q = p.seg[0].K / 4;
     const int tid = threadIdx.x, nt = blockDim.x, warp = tid >> 5, lane = tid & 31;
     const bool norm0 = p.seg[0].gamma != nullptr, norm1 = p.nseg > 1 && p.seg[1].gamma != nullptr;
     auto xidx = [&](int q) { return sizeof(T) == 2 ? (q & 1) * (K / 2) + (q >> 1) * 4 : q * 4; };
+    // the residual values first: their loads fly with the input copies below
+    float yv = 0.f;
+    if (yres && tid < units * nb) yv = __ldcg(p.y + (size_t)(b0 + tid % nb) * p.ldy + u0 + tid / nb);
     // gains: raw bytes of each normalised segment into gsm (element k at gsm[k])
     {
         int koff = 0;
@@ -557,6 +564,7 @@ __device__ __forceinline__ void stage_input_async(const GemvParams& p, float* xs
             qoff += nq;
         }
     }
+    if (yres && tid < units * nb) yres[tid / nb][tid % nb] = yv;  // units * nb <= the block's threads
     cp_async_wait_all();
     __syncthreads();
     if (!norm0 && !norm1) return;
@@ -612,6 +620,10 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
     __shared__ float head_val[kStreamWarps][RU][NB], tail_val[kStreamWarps][RU][NB];
     __shared__ float red_v[kStreamWarps][NB];
     __shared__ int red_r[kStreamWarps][NB];
+    // EPI_RESADD: the CTA's residual values, loaded with the input after the
+    // dependency wait, so that finishing a row does not wait for a load
+    constexpr int kYpreUnits = 64;
+    __shared__ float ypre_s[kYpreUnits][NB];
     constexpr int EPC = Chunk16<T>::kElems;
 
     pdl_launch();
@@ -655,8 +667,10 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
             if (p.zero_ptr && blockIdx.x == 0)
                 for (int i = threadIdx.x; i < p.zero_n; i += blockDim.x) p.zero_ptr[i] = 0ull;
         }
+        const bool ypre_on = p.epi == EPI_RESADD && u1 - u0 <= kYpreUnits;
         __syncthreads();
-        stage_input_async<T, NB>(p, xs, reinterpret_cast<T*>(xs + NB * K), b0, nb);
+        stage_input_async<T, NB>(p, xs, reinterpret_cast<T*>(xs + NB * K), b0, nb, ypre_on ? ypre_s : nullptr, u0,
+                                 u1 - u0);
 
         float best_v[NB];
         int best_r[NB];
@@ -710,7 +724,7 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
                         if (r == RU - 1) {
                             const int unit = crow / RU;
                             if (unit * cpu >= c0) {
-                                unit_epilogue<T, RU, NB>(p, u0 + unit, part, b0, nb, best_v, best_r);
+                                unit_epilogue<T, RU, NB>(p, u0 + unit, part, b0, nb, best_v, best_r, ypre_on ? ypre_s[unit] : nullptr);
                             } else if (lane == 0) {
                                 head_unit[warp] = unit;
                                 head_fin[warp] = 1;
@@ -782,7 +796,7 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
                         if (head_unit[v] == unit) sum += head_val[v][r][bb];
                     a[r][bb] = sum;
                 }
-            unit_epilogue<T, RU, NB>(p, u0 + unit, a, b0, nb, best_v, best_r);
+            unit_epilogue<T, RU, NB>(p, u0 + unit, a, b0, nb, best_v, best_r, ypre_on ? ypre_s[unit] : nullptr);
         }
         if (p.epi == EPI_ARGMAX) {
             if (lane == 0)

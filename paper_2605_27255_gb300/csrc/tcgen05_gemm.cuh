@@ -125,7 +125,8 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 // it (the SwiGLU pairing shuffles).
 template <int BH>
 __device__ __forceinline__ void tc_epilogue16(const TcParams& p, int row, int c0, const float (&v)[16],
-                                              float (*red_v)[BH], int (*red_r)[BH], int quad) {
+                                              float (*red_v)[BH], int (*red_r)[BH], int quad,
+                                              const float* ypre = nullptr) {
     const int warp = quad, lane = threadIdx.x & 31;
     const bool in = row < p.rows;
     if (p.epi == EPI_ARGMAX) {
@@ -165,7 +166,7 @@ __device__ __forceinline__ void tc_epilogue16(const TcParams& p, int row, int c0
             case EPI_STORE: *yp = a; break;
             case EPI_BIAS: *yp = a + __bfloat162float(static_cast<const __nv_bfloat16*>(p.bias)[row]); break;
             case EPI_SILU: *yp = silu(a); break;
-            case EPI_RESADD: *yp += a; break;
+            case EPI_RESADD: *yp = (ypre ? ypre[j] : *yp) + a; break;
             default: break;
         }
     }
@@ -185,7 +186,7 @@ __device__ __forceinline__ int tc_park_idx(int r, int c4) {
 template <int BH>
 __device__ __forceinline__ void tc_cluster_epilogue(const TcParams& p, cooperative_groups::cluster_group& cl,
                                                     float* park, int tile, int rr, int c4,
-                                                    const float* rstd = nullptr) {
+                                                    const float* rstd = nullptr, const float* ypre = nullptr) {
     float4 a = make_float4(0.f, 0.f, 0.f, 0.f), u = a;
     for (int s = 0; s < p.splits; ++s) {
         const float* rem = cl.map_shared_rank(park, s);
@@ -219,7 +220,7 @@ __device__ __forceinline__ void tc_cluster_epilogue(const TcParams& p, cooperati
             case EPI_STORE: *yp = va[j]; break;
             case EPI_BIAS: *yp = va[j] + __bfloat162float(static_cast<const __nv_bfloat16*>(p.bias)[row]); break;
             case EPI_SILU: *yp = silu(va[j]); break;
-            case EPI_RESADD: *yp += va[j]; break;
+            case EPI_RESADD: *yp = (ypre ? ypre[j] : *yp) + va[j]; break;
             case EPI_ARGMAX:
                 if (p.dbg) p.dbg[(size_t)b * p.ld_dbg + row] = va[j];
                 atomicMax(p.am + b, argmax_key(va[j], row));
@@ -447,6 +448,10 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
     __shared__ float red_v[4][BH];
     __shared__ int red_r[4][BH];
     __shared__ float ss_s[BH], rstd_s[BH];
+    // EPI_RESADD: the residual values this thread's epilogue updates, loaded
+    // right after the dependency wait so that the epilogue does not wait for them
+    float ypre[BH];
+    constexpr int kPreItems = (kTcM / 2) * (BH / 4) / 128;  // cluster items per thread (splits >= 2)
     PIPO_TR(__shared__ unsigned long long tr_s[3], tr_e[3]; const TraceT0 tr0 = trace_begin();)
 
     pdl_launch();
@@ -536,6 +541,29 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
         // converter warps: raw fp32 tile -> bf16 hi | lo operand tile, sum(x^2)
         const int xt = threadIdx.x - 64;  // 0..127
         pdl_wait();
+        if (p.epi == EPI_RESADD) {
+            if (p.splits == 1) {
+                const int row = tile * kTcM + (warp & 3) * 32 + lane;
+#pragma unroll
+                for (int b = 0; b < BH; ++b)
+                    ypre[b] = (row < p.rows && b < p.B) ? __ldcg(p.y + (size_t)b * p.ldy + row) : 0.f;
+            } else {
+                const int R = (((kTcM + p.splits - 1) / p.splits) + 1) & ~1;
+                const int r0 = min(kTcM, split * R), r1 = min(kTcM, r0 + R);
+                const int items = (r1 - r0) * (BH / 4);  // RESADD: one row per item
+#pragma unroll
+                for (int k = 0; k < kPreItems; ++k) {
+                    const int it = xt + 128 * k;
+                    const int row = tile * kTcM + r0 + it / (BH / 4), c4 = it % (BH / 4);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int b = 4 * c4 + j;
+                        ypre[4 * k + j] = (it < items && row < p.rows && b < p.B)
+                                              ? __ldcg(p.y + (size_t)b * p.ldy + row) : 0.f;
+                    }
+                }
+            }
+        }
         PIPO_TR(if (xt == 0) tr_s[0] = trace_now();)
         if (in.zero_ptr && blockIdx.x == 0)
             for (int i = xt; i < in.zero_n; i += 128) in.zero_ptr[i] = 0ull;
@@ -623,14 +651,14 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
     };
     if (p.splits == 1) {
         if (epi_warp) {
-#pragma unroll 1
+#pragma unroll
             for (int c0 = 0; c0 < BH; c0 += 16) {
                 float v[16];
                 ld_cols(c0, v);
                 PIPO_TR(if (threadIdx.x == 64 && c0 == 0) tr_e[0] = trace_now();)
 #pragma unroll
                 for (int j = 0; j < 16; ++j) v[j] *= rstd_s[c0 + j];
-                tc_epilogue16<BH>(p, row, c0, v, red_v, red_r, quad);
+                tc_epilogue16<BH>(p, row, c0, v, red_v, red_r, quad, p.epi == EPI_RESADD ? ypre + c0 : nullptr);
             }
             PIPO_TR(if (threadIdx.x == 64) { tr_e[1] = trace_now(); tr_e[2] = tr_e[1]; })
             if (p.epi == EPI_ARGMAX) {
@@ -680,9 +708,13 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
             const int r0 = min(kTcM, split * R), r1 = min(kTcM, r0 + R);
             const int step = p.ru == 2 ? 2 : 1;
             const int items = (r1 - r0) / step * (BH / 4);
-            for (int it = xt; it < items; it += 128) {
+#pragma unroll
+            for (int k = 0; k < kPreItems; ++k) {
+                const int it = xt + 128 * k;
+                if (it >= items) break;
                 const int rr = r0 + (it / (BH / 4)) * step, c4 = it % (BH / 4);
-                tc_cluster_epilogue<BH>(p, cl, park, tile, rr, c4, rstd_s);
+                tc_cluster_epilogue<BH>(p, cl, park, tile, rr, c4, rstd_s,
+                                        p.epi == EPI_RESADD ? ypre + 4 * k : nullptr);
             }
             PIPO_TR(if (threadIdx.x == 64) tr_e[2] = trace_now();)
         }

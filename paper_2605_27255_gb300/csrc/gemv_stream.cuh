@@ -657,11 +657,6 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
         load_batch(bufA);
         load_batch(bufB);
         if (b0 == 0) {
-            if (p.l2_prefetch > 0 && lane == 0) {
-                // the chunks after the register batches, towards L2 while the kernel before finishes
-                const int n = min(p.l2_prefetch, c1 - (c0 + 2 * kU));
-                if (n > 0) prefetch_l2_bulk(wbase + (size_t)(c0 + 2 * kU) * 512, (uint32_t)n * 512u);
-            }
             pdl_wait();
             PIPO_TR(tr1 = trace_now();)
             if (p.zero_ptr && blockIdx.x == 0)

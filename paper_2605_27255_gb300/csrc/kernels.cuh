@@ -58,15 +58,7 @@ struct GemvParams {
     int zero_n;
     float* part;         // EPI_RESADD with splitk > 1: partials [splitk][B][N]
     unsigned* rowcnt;    // arrival counters per (batch group, row), [ceil(B/NB)][N] (zero between launches)
-    int l2_prefetch;     // streaming GEMV: 512-byte weight chunks per warp hinted into L2 before the
-                         // dependency wait, beyond the register prefetch (0: none)
 };
-
-// Hint a contiguous global range into L2 (16-byte aligned address, size a
-// multiple of 16); no completion, no effect on results.
-__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
 
 // ---------------------------------------------------------------- loads
 

@@ -149,7 +149,6 @@ struct pipo_ctx {
     int attn_flat = 1;                // register-ring decode attention without clusters (global merge):
                                       // 0 never, 1 from kFlatMinEntries cached entries, 2 always
     std::vector<CUtensorMap> kv_tm;   // tensor-core attention: K and V tensor map of every cache layer
-    int gemv_l2_prefetch = 0;         // streaming GEMV: weight chunks per warp hinted into L2 before the wait
     // per-launch timing (pipo_profile_step): events around every launch
     bool prof = false;
     int prof_kind = 2;
@@ -727,7 +726,6 @@ GemvParams gemv_base(pipo_ctx* ctx, const void* W, int N, int epi, float* y, int
     GemvParams p{};
     p.W = W; p.N = N; p.epi = epi; p.y = y; p.ldy = ldy;
     p.B = ctx->rows > 0 ? ctx->rows : ctx->B; p.splitk = 1; p.eps = ctx->cfg.rms_eps; p.nseg = 1;
-    p.l2_prefetch = ctx->gemv_l2_prefetch;
     return p;
 }
 
@@ -1540,7 +1538,6 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
                 ctx->attn_cs_force = v;
         }
         if (const char* ev = getenv("PIPO_ATTN_CS_TARGET")) ctx->attn_cs_target = std::max(1, atoi(ev));
-        if (const char* ev = getenv("PIPO_GEMV_L2_PREFETCH")) ctx->gemv_l2_prefetch = std::max(0, atoi(ev));
 
         // activations and state
         const int qd = c.n_q_heads * DH, kd = c.n_kv_heads * DH;

@@ -24,7 +24,8 @@ one launch over the same rows.
 
   python -m paper_2605_27255_gb300.kernel_bench --chain 32 --shape o_proj
 
-Shapes are the weight-streaming projections of the 4B-class model.  Weights
+Shapes are the weight-streaming projections of the 4B-class model (and, with
+the _9b suffix, of the 9B-class model).  Weights
 are random bf16; several copies are cycled so that every launch streams from
 HBM (more than twice the 129 MB L2 in total).  Prints one JSON line per shape
 with the CUDA-event time per launch and the achieved GB/s of algorithmic bytes.
@@ -46,10 +47,16 @@ SHAPES = {
     "down": (2560, 9728, 0),
     "w_fc": (2560, 5120, 0),
     "lm_head": (151936, 2560, 0),
+    # the 9B-class model
+    "qkv_9b": (6144, 4096, 0),
+    "o_proj_9b": (4096, 4096, 0),
+    "gate_up_9b": (12288, 4096, 1),
+    "down_9b": (4096, 12288, 0),
 }
 
 
-def run(name: str, batch: int, iters: int, min_bytes: float = 300e6, tc: bool = False, splits: int = 0) -> dict:
+def run(name: str, batch: int, iters: int, min_bytes: float = 300e6, tc: bool = False, splits: int = 0,
+        fused: bool = False) -> dict:
     N, K, mode = SHAPES[name]
     rows = 2 * N if mode else N
     nbytes = rows * K * 2
@@ -58,14 +65,19 @@ def run(name: str, batch: int, iters: int, min_bytes: float = 300e6, tc: bool = 
     x = torch.randn(batch, K, device="cuda")
     y = torch.empty(batch, N, device="cuda")
     st = torch.cuda.current_stream()
-    if tc:
+    if tc or fused:
         sb = capi.pipo_op_gemm_tc_scratch(mode, N, K, batch, splits)
         scratch = torch.empty(sb + 1024, dtype=torch.uint8, device="cuda")
         base = (scratch.data_ptr() + 1023) // 1024 * 1024
+        gamma = torch.ones(K, dtype=torch.bfloat16, device="cuda")
 
         def launch(i):
-            capi.pipo_op_gemm_tc(mode, Ws[i % copies].data_ptr(), N, K, x.data_ptr(), batch, y.data_ptr(), splits,
-                                 base, sb, st.cuda_stream)
+            if fused:  # normalised input: the converter warps inside the GEMM (batch 16 or 32)
+                capi.pipo_op_gemm_tc_norm(mode, Ws[i % copies].data_ptr(), N, x.data_ptr(), K, gamma.data_ptr(),
+                                          0, 0, 0, 0, 1e-6, batch, y.data_ptr(), splits, base, sb, st.cuda_stream)
+            else:
+                capi.pipo_op_gemm_tc(mode, Ws[i % copies].data_ptr(), N, K, x.data_ptr(), batch, y.data_ptr(),
+                                     splits, base, sb, st.cuda_stream)
     else:
         def launch(i):
             capi.pipo_op_gemv(1, mode, Ws[i % copies].data_ptr(), N, K, x.data_ptr(), batch, y.data_ptr(),
@@ -80,7 +92,7 @@ def run(name: str, batch: int, iters: int, min_bytes: float = 300e6, tc: bool = 
     e1.record(st)
     torch.cuda.synchronize()
     us = e0.elapsed_time(e1) * 1e3 / iters
-    return dict(kernel="gemm_tc" if tc else "gemv", shape=name, batch=batch, N=N, K=K, us_per_launch=us,
+    return dict(kernel="gemm_tcf" if fused else "gemm_tc" if tc else "gemv", shape=name, batch=batch, N=N, K=K, us_per_launch=us,
                 gbs=nbytes / us / 1e3, bytes_per_launch=nbytes, copies=copies)
 
 
@@ -195,6 +207,9 @@ def main() -> None:
     ap.add_argument("--iters", type=int, default=50)
     ap.add_argument("--tc", action="store_true", help="tensor-core projection (bf16 hi/lo activations)")
     ap.add_argument("--splits", type=int, default=0, help="K splits of the tensor-core GEMM (0: automatic)")
+    ap.add_argument("--fused", action="store_true",
+                    help="the tensor-core projection with the activation split inside the GEMM (the decode step's "
+                         "form at batch widths 16 and 32; --batch 16 or 32)")
     ap.add_argument("--step", action="store_true", help="one eager decode step of a small bf16 model")
     ap.add_argument("--ctx", type=int, default=512, help="--step: cached entries per sequence")
     ap.add_argument("--prefill", type=int, default=0, help="time a pair prefill of this many tokens per sequence")
@@ -216,7 +231,7 @@ def main() -> None:
         print(json.dumps(run_step(a.batch, a.ctx)), flush=True)
         return
     for name in (sorted(SHAPES) if a.shape == "all" else [a.shape]):
-        print(json.dumps(run(name, a.batch, a.iters, tc=a.tc, splits=a.splits)), flush=True)
+        print(json.dumps(run(name, a.batch, a.iters, tc=a.tc, splits=a.splits, fused=a.fused)), flush=True)
 
 
 if __name__ == "__main__":

@@ -61,7 +61,61 @@ static_assert(kMmaStages % kMmaWarps == 0, "every compute warp owns the same num
 // stage has phase k; the parity of group t is (t / kMmaStages) & 1.
 __device__ __forceinline__ int mma_stage(int t) { return (t % kMmaWarps) * kMmaSpw + (t / kMmaWarps) % kMmaSpw; }
 
-constexpr size_t mma_attn_smem() { return 1024 + (size_t)kMmaStages * kMmaStageBytes + 2 * kMmaStages * 8; }
+// dynamic shared memory: the stage ring, its barriers, and the receive
+// buffer of the cluster merge, one slot per CTA of the cluster (CS), each
+// [G][DH] partial output then [G] maxima and [G] sums (fp32; G <= 4)
+constexpr int kMmaRcvSlot = 4 * 128 + 8;  // floats per slot at G = 4 (smaller G use a prefix)
+constexpr size_t mma_attn_smem(int cs = 8) {
+    return 1024 + (size_t)kMmaStages * kMmaStageBytes + 2 * kMmaStages * 8 + (size_t)cs * kMmaRcvSlot * 4;
+}
+
+// The cluster merge pushes every CTA's partial softmax state into rank 0's
+// receive buffer (distributed shared memory stores), and each CTA then
+// arrives on rank 0's barrier with release semantics at cluster scope; rank
+// 0 waits (acquire, cluster scope, bounded), merges in rank order and writes
+// the output.  The other CTAs leave right after their arrival.
+__device__ __forceinline__ void cluster_arrive_release() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void fence_acq_rel_cluster() { asm volatile("fence.acq_rel.cluster;" ::: "memory"); }
+// arrive on the mbarrier at the same shared offset in the CTA of cluster rank `rank`
+__device__ __forceinline__ void mbar_arrive_remote(uint64_t* bar, int rank) {
+    asm volatile(
+        "{\n .reg .b32 ra;\n mapa.shared::cluster.u32 ra, %0, %1;\n"
+        " mbarrier.arrive.release.cluster.shared::cluster.b64 _, [ra];\n}" ::"r"(smem_u32(bar)),
+        "r"(rank)
+        : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// bounded wait (as mbar_wait) with cluster-scope acquire
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, unsigned site, unsigned iter) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    for (;;) {
+        for (int i = 0; i < 64; ++i)
+            if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (global_ns() - t0 > kWaitNs) break;
+    }
+    atomicOr(&g_pipo_error, kErrWaitTimeout);
+    if (atomicCAS(&g_pipo_error_info[0], 0u, site) == 0u) {
+        g_pipo_error_info[1] = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z);
+        g_pipo_error_info[2] = iter;
+        g_pipo_error_info[3] = parity;
+    }
+    return false;
+}
 
 // byte offset of 8-dim chunk c (0..15) of row `row` (0..15) of a K or V tile:
 // two 64-dim halves of 16 x 128 bytes, 16-byte chunks XOR-swizzled by row % 8
@@ -110,16 +164,19 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     extern __shared__ __align__(1024) unsigned char am_smem_raw[];
     __shared__ float qs[G][DH];       // rotated, pre-scaled queries (fp32)
     __shared__ float kn_s[DH], vn_s[DH];  // the new entry, rounded to bf16
-    __shared__ float sm_o[G][DH];
-    __shared__ float sm_m[G], sm_l[G];
     __shared__ float wm[NP][G], wl[NP][G];
-    __shared__ float wo[NP][G][DH];
+    __shared__ __align__(16) float wo_new[G][DH];  // the new entry's partial (partial NW); the compute
+                                     // warps' partials go to their own first stage
     __shared__ int abort_flag;
+    __shared__ __align__(8) uint64_t rcv_bar;  // rank 0: one arrival per CTA of the cluster
     PIPO_TR(__shared__ unsigned long long tr_s[3], tr_m[2]; const TraceT0 tr0 = trace_begin();)
 
     unsigned char* ring = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(am_smem_raw) + 1023) & ~(uintptr_t)1023);
     uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)kMmaStages * kMmaStageBytes);
     uint64_t* empty = full + kMmaStages;
+    float* rcv = reinterpret_cast<float*>(empty + kMmaStages);  // [CS][kMmaRcvSlot] (rank 0's is used)
+    // partial of compute warp w: [G][DH] floats at the start of its first stage
+    auto wpart = [&](int w) { return reinterpret_cast<float*>(ring + (size_t)(w * kMmaSpw) * kMmaStageBytes); };
 
     pdl_launch();
     cg::cluster_group cluster = cg::this_cluster();
@@ -146,9 +203,13 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             mbar_init(empty + i, 1);
         }
         abort_flag = 0;
+        mbar_init(&rcv_bar, (uint32_t)CS);
         mbar_init_fence();
     }
     __syncthreads();
+    // every thread: the first half of the cluster barrier that orders rank 0's
+    // barrier initialisation before the other CTAs' arrivals on it
+    if (CS > 1) cluster_arrive_release();
 
     if (warp == NW) {
         // ---- producer: whole 16-entry groups (earlier steps wrote them, so
@@ -224,7 +285,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
                 for (int d = lane; d < DH; d += 32) dsum += qs[h][d] * kn_s[d];
                 dsum = warp_sum(dsum);
             }
-            for (int d = lane; d < DH; d += 32) wo[NW][h][d] = owns_new ? vn_s[d] : 0.f;
+            for (int d = lane; d < DH; d += 32) wo_new[h][d] = owns_new ? vn_s[d] : 0.f;
             if (lane == 0) {
                 wm[NW][h] = owns_new ? dsum : -INFINITY;
                 wl[NW][h] = owns_new ? 1.f : 0.f;
@@ -337,13 +398,17 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         }
 
         PIPO_TR(if (ct == 0) tr_m[0] = trace_now();)
-        // warp partial: O of head r = bf16-part row r + remainder row r + G
+        // warp partial: O of head r = bf16-part row r + remainder row r + G,
+        // into this warp's first stage (its groups are all consumed: no copy
+        // lands in its stages any more)
+        __syncwarp();
+        float* wp = wpart(warp);
 #pragma unroll
         for (int nd = 0; nd < DH / 8; ++nd)
 #pragma unroll
             for (int j = 0; j < 2; ++j) {
                 const float v = o[nd][j] + __shfl_xor_sync(0xffffffffu, o[nd][j], 4 * G);
-                if (r < G) wo[warp][r][nd * 8 + 2 * tq + j] = v;
+                if (r < G) wp[r * DH + nd * 8 + 2 * tq + j] = v;
             }
         if (r < G && tq == 0) {
             wm[warp][r] = m_run;
@@ -351,33 +416,78 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         }
     }
     __syncthreads();
-    // merge the partials: CTA (m, l, o) in shared memory
-    for (int i = threadIdx.x; i < G * DH; i += blockDim.x) {
-        const int hh = i / DH, t = i % DH;
+    // merge the partials: this CTA's (m, l, o), then the cluster's at rank 0
+    float* slot = nullptr;
+    if (CS > 1) {
+        cluster_wait_acquire();  // rank 0's receive barrier is initialised
+        slot = cluster.map_shared_rank(rcv, 0) + (size_t)s * kMmaRcvSlot;
+    }
+    // four consecutive output dims per thread (16-byte stores, also into rank 0)
+    for (int i4 = threadIdx.x; i4 < G * DH / 4; i4 += blockDim.x) {
+        const int hh = (4 * i4) / DH, t = (4 * i4) % DH;
         float M = -INFINITY;
 #pragma unroll
         for (int w = 0; w < NP; ++w) M = fmaxf(M, wm[w][hh]);
-        float L = 0.f, Ov = 0.f;
+        float L = 0.f;
+        float4 Ov = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
         for (int w = 0; w < NP; ++w) {
             const float f = (wm[w][hh] == -INFINITY) ? 0.f : expf(wm[w][hh] - M);
             L += wl[w][hh] * f;
-            Ov += wo[w][hh][t] * f;
+            const float4 v = *reinterpret_cast<const float4*>(w < NW ? wpart(w) + hh * DH + t : &wo_new[hh][t]);
+            Ov.x += v.x * f; Ov.y += v.y * f; Ov.z += v.z * f; Ov.w += v.w * f;
         }
-        sm_o[hh][t] = Ov;
-        if (t == 0) { sm_m[hh] = M; sm_l[hh] = L; }
+        if (CS == 1) {
+            const float il = 1.0f / L;
+            *reinterpret_cast<float4*>(p.out + (size_t)row * n_q * DH + (size_t)(g * G + hh) * DH + t) =
+                make_float4(Ov.x * il, Ov.y * il, Ov.z * il, Ov.w * il);
+        } else {
+            *reinterpret_cast<float4*>(slot + hh * DH + t) = Ov;
+            if (t == 0) {
+                slot[G * DH + hh] = M;
+                slot[G * DH + G + hh] = L;
+            }
+        }
     }
     PIPO_TR(if (threadIdx.x == 0) tr_s[2] = trace_now();)
-    cluster.sync();
-    PIPO_TR(if (threadIdx.x == 0) tr_m[1] = trace_now();)
-    // cluster merge: CTA s finishes dims [s*G*DH/CS, (s+1)*G*DH/CS) of the G heads
-    const int PER = (G * DH + CS - 1) / CS;
-    for (int i = s * PER + threadIdx.x; i < min(G * DH, (s + 1) * PER); i += blockDim.x) {
-        const int hh = i / DH, t = i % DH;
-        p.out[(size_t)row * n_q * DH + (size_t)(g * G + hh) * DH + t] =
-            cluster_merge_elem(cluster, &sm_m[hh], &sm_l[hh], &sm_o[hh][t], CS);
+    if (CS == 1) {
+        PIPO_TR(if (threadIdx.x == 0) {
+            trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);
+            trace_put(TR_ATTN_MMA_EPI, tr0, tr_s[0], tr_s[1], tr_m[0], tr_s[2], tr_s[2]);
+        })
+        return;
     }
-    cluster.sync();  // keep every CTA's shared memory alive until all merges read it
+    fence_acq_rel_cluster();  // this thread's stores into rank 0, before the arrival below
+    __syncthreads();
+    if (threadIdx.x == 0) mbar_arrive_remote(&rcv_bar, 0);
+    if (s != 0) {
+        PIPO_TR(if (threadIdx.x == 0) {
+            trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);
+            trace_put(TR_ATTN_MMA_EPI, tr0, tr_s[0], tr_s[1], tr_m[0], tr_s[2], tr_s[2]);
+        })
+        return;  // rank 0 merges; nothing reads this CTA's shared memory
+    }
+    const bool got = mbar_wait_cluster(&rcv_bar, 0, 28, (unsigned)CS);
+    PIPO_TR(if (threadIdx.x == 0) tr_m[1] = trace_now();)
+    if (got) {
+        for (int i4 = threadIdx.x; i4 < G * DH / 4; i4 += blockDim.x) {
+            const int hh = (4 * i4) / DH, t = (4 * i4) % DH;
+            float M = -INFINITY;
+            for (int r2 = 0; r2 < CS; ++r2) M = fmaxf(M, rcv[r2 * kMmaRcvSlot + G * DH + hh]);
+            float L = 0.f;
+            float4 Ov = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int r2 = 0; r2 < CS; ++r2) {
+                const float* sl = rcv + r2 * kMmaRcvSlot;
+                const float f = (sl[G * DH + hh] == -INFINITY) ? 0.f : expf(sl[G * DH + hh] - M);
+                L += sl[G * DH + G + hh] * f;
+                const float4 v = *reinterpret_cast<const float4*>(sl + hh * DH + t);
+                Ov.x += v.x * f; Ov.y += v.y * f; Ov.z += v.z * f; Ov.w += v.w * f;
+            }
+            const float il = 1.0f / L;
+            *reinterpret_cast<float4*>(p.out + (size_t)row * n_q * DH + (size_t)(g * G + hh) * DH + t) =
+                make_float4(Ov.x * il, Ov.y * il, Ov.z * il, Ov.w * il);
+        }
+    }
     PIPO_TR(if (threadIdx.x == 0) {
         trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);
         trace_put(TR_ATTN_MMA_EPI, tr0, tr_s[0], tr_s[1], tr_m[0], tr_s[2], tr_m[1]);

@@ -978,7 +978,14 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
                           prefill_attn_smem(), pargs));
         } else if (attn_use_mma(ctx, R) && cs <= 8) {
             void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
-            TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, R), dim3(kMmaThreads), mma_attn_smem(),
+            static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
+            if (verbose) {
+                int per_sm = 0;
+                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attnm_pick(G), kMmaThreads, mma_attn_smem(cs));
+                fprintf(stderr, "[pipo] attention: tensor-core, cluster %d, %zu B shared memory, %d CTAs per SM\n", cs,
+                        mma_attn_smem(cs), per_sm);
+            }
+            TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, R), dim3(kMmaThreads), mma_attn_smem(cs),
                           margs, cs));
         }
         else if (attn_flat_now(ctx) && !chunk && !ctx->attn_cs_force) {

@@ -153,7 +153,12 @@ __device__ __forceinline__ void mma_rows8(float (&d)[4], uint32_t a0, uint32_t a
 
 // tmK, tmV: this layer's K and V cache as [blocks * n_kv * page][d_h] bf16,
 // boxes of 64 dims x 16 rows, 128-byte swizzle
-template <int G>
+// FLAT: no cluster; the grid's x dimension splits the entries (S = gridDim.x
+// CTAs per (row, kv head)), each CTA writes its partial to the global
+// scratch (AttnParams::part_o, part_ml) and the last of a (row, kv head) to
+// arrive (AttnParams::counters) merges the S partials in split order: any
+// split count, so that long caches fill the GPU evenly.
+template <int G, bool FLAT = false>
 __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, const __grid_constant__ CUtensorMap tmK,
                                                                const __grid_constant__ CUtensorMap tmV) {
     static_assert(G == 1 || G == 2 || G == 4, "2G query rows must fit the 8 live MMA rows");
@@ -180,8 +185,9 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
 
     pdl_launch();
     cg::cluster_group cluster = cg::this_cluster();
-    const int s = (int)cluster.block_rank();
-    const int CS = (int)cluster.num_blocks();
+    const int s = FLAT ? (int)blockIdx.x : (int)cluster.block_rank();
+    const int CS = FLAT ? (int)gridDim.x : (int)cluster.num_blocks();
+    __shared__ int last_cta;
     const int g = blockIdx.y, row = blockIdx.z;
     const int b = row % p.nseq;        // sequence: its block table and length
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -209,7 +215,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     __syncthreads();
     // every thread: the first half of the cluster barrier that orders rank 0's
     // barrier initialisation before the other CTAs' arrivals on it
-    if (CS > 1) cluster_arrive_release();
+    if (!FLAT && CS > 1) cluster_arrive_release();
 
     if (warp == NW) {
         // ---- producer: whole 16-entry groups (earlier steps wrote them, so
@@ -418,7 +424,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     __syncthreads();
     // merge the partials: this CTA's (m, l, o), then the cluster's at rank 0
     float* slot = nullptr;
-    if (CS > 1) {
+    if (!FLAT && CS > 1) {
         cluster_wait_acquire();  // rank 0's receive barrier is initialised
         slot = cluster.map_shared_rank(rcv, 0) + (size_t)s * kMmaRcvSlot;
     }
@@ -437,7 +443,14 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             const float4 v = *reinterpret_cast<const float4*>(w < NW ? wpart(w) + hh * DH + t : &wo_new[hh][t]);
             Ov.x += v.x * f; Ov.y += v.y * f; Ov.z += v.z * f; Ov.w += v.w * f;
         }
-        if (CS == 1) {
+        if (FLAT) {
+            const size_t pi = (size_t)(row * n_q + g * G + hh) * CS + s;
+            __stcg(reinterpret_cast<float4*>(p.part_o + pi * DH + t), Ov);
+            if (t == 0) {
+                p.part_ml[pi * 2] = M;
+                p.part_ml[pi * 2 + 1] = L;
+            }
+        } else if (CS == 1) {
             const float il = 1.0f / L;
             *reinterpret_cast<float4*>(p.out + (size_t)row * n_q * DH + (size_t)(g * G + hh) * DH + t) =
                 make_float4(Ov.x * il, Ov.y * il, Ov.z * il, Ov.w * il);
@@ -450,6 +463,62 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         }
     }
     PIPO_TR(if (threadIdx.x == 0) tr_s[2] = trace_now();)
+    if constexpr (FLAT) {
+        // the last CTA of (row, kv head) to arrive merges the CS partials in split order
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const unsigned prev = atomicAdd(p.counters + row * n_kv + g, 1u);
+            last_cta = prev == (unsigned)(CS - 1);
+            if (last_cta) p.counters[row * n_kv + g] = 0u;
+        }
+        __syncthreads();
+        if (!last_cta) return;
+        __threadfence();
+        // split weights per head in the (now idle) stage ring: ms [G][CS], fs [G][CS]
+        float* ms = reinterpret_cast<float*>(ring);
+        float* fs = ms + G * CS;
+        for (int i = threadIdx.x; i < G * CS; i += blockDim.x) {
+            const int hh = i / CS, r2 = i % CS;
+            const size_t pi = (size_t)(row * n_q + g * G + hh) * CS + r2;
+            ms[i] = __ldcg(p.part_ml + pi * 2);
+            fs[i] = __ldcg(p.part_ml + pi * 2 + 1);
+        }
+        __syncthreads();
+        if (threadIdx.x < G) {
+            const int hh = threadIdx.x;
+            float M = -INFINITY;
+            for (int r2 = 0; r2 < CS; ++r2) M = fmaxf(M, ms[hh * CS + r2]);
+            float L = 0.f;
+            for (int r2 = 0; r2 < CS; ++r2) {
+                const float f = (ms[hh * CS + r2] == -INFINITY) ? 0.f : expf(ms[hh * CS + r2] - M);
+                L += fs[hh * CS + r2] * f;
+                fs[hh * CS + r2] = f;  // weight of split r2
+            }
+            ms[hh * CS] = 1.0f / L;  // the maxima are no longer needed
+        }
+        __syncthreads();
+        for (int i4 = threadIdx.x; i4 < G * DH / 4; i4 += blockDim.x) {
+            const int hh = (4 * i4) / DH, t = (4 * i4) % DH;
+            const float* po = p.part_o + (size_t)(row * n_q + g * G + hh) * CS * DH + t;
+            float4 Ov = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int r0 = 0; r0 < CS; r0 += 4) {
+                float4 ov[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) ov[u] = __ldcg(reinterpret_cast<const float4*>(po + (size_t)min(r0 + u, CS - 1) * DH));
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (r0 + u < CS) {
+                        const float f = fs[hh * CS + r0 + u];
+                        Ov.x += ov[u].x * f; Ov.y += ov[u].y * f; Ov.z += ov[u].z * f; Ov.w += ov[u].w * f;
+                    }
+            }
+            const float il = ms[hh * CS];
+            *reinterpret_cast<float4*>(p.out + (size_t)row * n_q * DH + (size_t)(g * G + hh) * DH + t) =
+                make_float4(Ov.x * il, Ov.y * il, Ov.z * il, Ov.w * il);
+        }
+        return;
+    }
     if (CS == 1) {
         PIPO_TR(if (threadIdx.x == 0) {
             trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);

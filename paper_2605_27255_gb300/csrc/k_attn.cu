@@ -73,6 +73,16 @@ void* k_pick_attn_mma(int G) {
     }
 }
 
+// the same without clusters, split partials merged through global memory
+void* k_pick_attn_mma_flat(int G) {
+    switch (G) {
+        case 1: return reinterpret_cast<void*>(&attn_mma_kernel<1, true>);
+        case 2: return reinterpret_cast<void*>(&attn_mma_kernel<2, true>);
+        case 4: return reinterpret_cast<void*>(&attn_mma_kernel<4, true>);
+        default: return nullptr;
+    }
+}
+
 // causal tile attention of prefill chunks (same cache and head constraints)
 void* k_pick_attn_prefill(int G) {
     switch (G) {

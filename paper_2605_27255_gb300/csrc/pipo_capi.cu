@@ -409,11 +409,12 @@ cudaError_t set_smem_attrs(bool bf) {
                 if (e != cudaSuccess) return e;
             }
     if (bf)
-        for (int g : {1, 2, 4}) {
-            cudaError_t e = cudaFuncSetAttribute(attnm_pick(g), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)mma_attn_smem());
-            if (e != cudaSuccess) return e;
-        }
+        for (int g : {1, 2, 4})
+            for (void* f : {attnm_pick(g), k_pick_attn_mma_flat(g)}) {
+                cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                     (int)mma_attn_smem());
+                if (e != cudaSuccess) return e;
+            }
     if (bf)
         for (int bn : {16, 32, 64, 128})
             for (bool deep : {false, true})
@@ -879,6 +880,39 @@ bool attn_flat_now(const pipo_ctx* ctx) {
     return n > 0 && sum / n >= kFlatMinEntries;
 }
 
+// Split count of the unclustered tensor-core attention, or 0 for the
+// clustered one: when the (row, kv head) pairs times the largest cluster
+// (8) leave SMs without two CTAs and the cached slices stay long (mean
+// context at graph capture of kFlatMmaMinEntries and more), S splits fill
+// one wave of two CTAs per SM, at most kFlatMaxSplits.  Measured on 4b-lc
+// (B = 4, ~15.5 K cached pairs, ms per step): 8-CTA clusters (256 CTAs)
+// 4.32; unclustered one wave (S = 9, 288 CTAs) 4.09; two waves (S = 19)
+// 4.35; three 4.53 (more waves balance the SMs but leave no room for the
+// next kernel's CTAs to start early).  PIPO_ATTN_MMA_WAVES sets the waves,
+// PIPO_ATTN_MMA_FLAT=0 / 2: never / also for short caches.
+constexpr int kFlatMmaMinEntries = 4096;
+int attn_mma_flat_splits(const pipo_ctx* ctx, int R) {
+    static const int mode = [] {
+        const char* ev = getenv("PIPO_ATTN_MMA_FLAT");
+        return ev ? atoi(ev) : 1;
+    }();
+    if (mode <= 0) return 0;
+    const long long pairs = (long long)R * ctx->cfg.n_kv_heads;
+    if (pairs * 8 >= 2LL * ctx->sms) return 0;
+    double sum = 0.0;
+    int n = 0;
+    for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b, ++n) sum += ctx->h_len[b];
+    const double mean = n > 0 ? sum / n : 0.0;
+    if (mode == 1 && mean < kFlatMmaMinEntries) return 0;
+    static const int waves = [] {
+        const char* ev = getenv("PIPO_ATTN_MMA_WAVES");
+        return ev ? std::max(1, atoi(ev)) : 1;
+    }();
+    int S = (int)(2LL * waves * ctx->sms / pairs);
+    if (S > 0 && mean / S < 512.0) S = (int)(2LL * ctx->sms / pairs);
+    return std::max(1, std::min(S, kFlatMaxSplits));
+}
+
 // Long attention: the cached K/V bytes of a layer are at least six times the
 // QKV weight bytes (cached lengths at graph capture).  Then every projection
 // takes the two-per-SM ring, whose shared memory leaves room for a
@@ -976,6 +1010,15 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
             void* pargs[] = {&ap, &C, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
             TRY(launch_ex(ctx, fn, dim3((C + TP - 1) / TP, c.n_kv_heads, ctx->B), dim3(kPfThreads),
                           prefill_attn_smem(), pargs));
+        } else if (attn_use_mma(ctx, R) && !chunk && attn_mma_flat_splits(ctx, R) > 0) {
+            // long caches: unclustered splits, one wave of two CTAs per SM
+            ap.part_o = ctx->part_o;
+            ap.part_ml = ctx->part_ml;
+            ap.counters = ctx->counters;
+            const int S = attn_mma_flat_splits(ctx, R);
+            void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
+            TRY(launch_ex(ctx, k_pick_attn_mma_flat(G), dim3(S, c.n_kv_heads, R), dim3(kMmaThreads), mma_attn_smem(1),
+                          margs));
         } else if (attn_use_mma(ctx, R) && cs <= 8) {
             void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
             static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
@@ -1567,6 +1610,8 @@ pipo_status pipo_init(const pipo_config* cfg, const pipo_weights* w, pipo_ctx** 
         TRY(dalloc(ctx, &ctx->t, AR * H * 4));
         size_t parts = 0;
         for (int b = 1; b <= MB; ++b) parts = std::max(parts, (size_t)b * c.n_q_heads * attn_splits(ctx, b));
+        // the unclustered tensor-core attention: rows x n_kv < 2 sms / 8, at most kFlatMaxSplits splits
+        parts = std::max(parts, (size_t)(2 * ctx->sms / 8 + 1) * (c.n_q_heads / c.n_kv_heads) * kFlatMaxSplits);
         TRY(dalloc(ctx, &ctx->part_o, parts * DH * 4));
         TRY(dalloc(ctx, &ctx->part_ml, parts * 2 * 4));
         TRY(dalloc(ctx, &ctx->counters, (size_t)MB * c.n_kv_heads * 4));
@@ -2469,14 +2514,16 @@ pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {
                               cuda_core + ")";
     else proj = cuda_core;
     const int cs = attn_cluster_size(ctx, B);
-    const bool mma = attn_use_mma(ctx, B) && cs <= 8;
+    const int mma_flat = ctx->attn_v0 || !attn_use_mma(ctx, B) ? 0 : attn_mma_flat_splits(ctx, B);
+    const bool mma = attn_use_mma(ctx, B) && (cs <= 8 || mma_flat > 0);
     const bool flat = !ctx->attn_v0 && !mma && attn_flat_now(ctx) && !ctx->attn_cs_force;
     std::string d = "B=" + std::to_string(B) + " projections=" + proj + " attention=" +
                     (ctx->attn_v0 ? std::string("attn_decode_kernel") : mma ? "attn_mma_kernel" : "attn_cluster_kernel") +
-                    (flat ? " unclustered splits=" +
-                                std::to_string(std::max(1, std::min({ctx->sms / (B * c.n_kv_heads), (c.max_ctx + 15) / 16,
-                                                                     kFlatMaxSplits})))
-                          : " cluster=" + std::to_string(cs));
+                    (mma_flat > 0 ? " unclustered splits=" + std::to_string(mma_flat)
+                     : flat ? " unclustered splits=" +
+                                  std::to_string(std::max(1, std::min({ctx->sms / (B * c.n_kv_heads),
+                                                                       (c.max_ctx + 15) / 16, kFlatMaxSplits})))
+                            : " cluster=" + std::to_string(cs));
     // decoding mode, heads and prefill arrangement
     d += ctx->regular ? " mode=regular" : " mode=pair";
     d += ctx->samp_on ? " heads=sampled" : " heads=argmax";

@@ -124,7 +124,7 @@ struct pipo_ctx {
     int act_rows = 0;               // rows of the fp32 activation buffers (>= the batch width BH)
     bool tc_shallow = false;        // this step's projections: two-per-SM ring (room for a co-resident neighbour)
     int tc_min_b = 2;               // measured: a tie with the CUDA-core GEMV at B = 1, far ahead from B = 4
-    int attn_mma_min_b = 2;         // smallest batch on the tensor-core attention (PIPO_ATTN_MMA_MIN_BATCH)
+    int attn_mma_min_b = 1;         // smallest batch on the tensor-core attention (PIPO_ATTN_MMA_MIN_BATCH)
     int tc_splits = 0;              // forced K splits (0: automatic)
 
     int32_t *pending = nullptr, *n_pos = nullptr, *out_tokens = nullptr, *out_nacc = nullptr;
@@ -855,6 +855,9 @@ bool attn_use_mma(const pipo_ctx* ctx, int B) {
 // (sequence, kv head) pairs alone fill the GPU.
 int attn_cluster_size(const pipo_ctx* ctx, int B) {
     if (ctx->attn_cs_force) return ctx->attn_cs_force;
+    // one sequence on the tensor-core attention: 4-CTA clusters (4b-b1: 2.61
+    // against 2.63 ms per step with 8)
+    if (B == 1 && attn_use_mma(ctx, B)) return 4;
     const long long pairs = (long long)B * ctx->cfg.n_kv_heads;
     if (ctx->attn_cs16 && pairs * 16 <= 2 * ctx->sms) return 16;
     // measured best: about two tensor-core attention CTAs per SM (they are
@@ -888,9 +891,11 @@ bool attn_flat_now(const pipo_ctx* ctx) {
 // (B = 4, ~15.5 K cached pairs, ms per step): 8-CTA clusters (256 CTAs)
 // 4.32; unclustered one wave (S = 9, 288 CTAs) 4.09; two waves (S = 19)
 // 4.35; three 4.53 (more waves balance the SMs but leave no room for the
-// next kernel's CTAs to start early).  PIPO_ATTN_MMA_WAVES sets the waves,
-// PIPO_ATTN_MMA_FLAT=0 / 2: never / also for short caches.
-constexpr int kFlatMmaMinEntries = 4096;
+// next kernel's CTAs to start early).  One sequence at ~2180 pairs (9b-b1):
+// 3.83 against 3.89 ms with the register-ring attention (unclustered).
+// PIPO_ATTN_MMA_WAVES sets the waves, PIPO_ATTN_MMA_FLAT=0 / 2: never / also
+// for short caches.
+constexpr int kFlatMmaMinEntries = 2048;
 int attn_mma_flat_splits(const pipo_ctx* ctx, int R) {
     static const int mode = [] {
         const char* ev = getenv("PIPO_ATTN_MMA_FLAT");

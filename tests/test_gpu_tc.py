@@ -191,7 +191,9 @@ def test_mid_bf16_cuda_core_batches_over_8(monkeypatch):
 def test_decode_path_uses_tensor_core_kernels():
     """At B = 16 the block projections and the attention take the tcgen05 and
     mma.sync kernels (the down projection, K = 1376, stays on CUDA cores); a
-    single sequence stays on the CUDA-core GEMV and attention."""
+    single sequence keeps the CUDA-core GEMV (a matrix-vector product) and
+    takes the tensor-core attention in 4-CTA clusters (its 4 query heads per
+    kv head are the MMA rows)."""
     w = synth.gen_weights(MID, seed=23)
     g = capi.Pipo(MID, w, max_batch=16, max_ctx=40)
     try:
@@ -205,6 +207,6 @@ def test_decode_path_uses_tensor_core_kernels():
     try:
         g.prefill(synth.gen_prompts(1, 8, MID.V, seed=1).numpy())
         d = g.describe()
-        assert "projections=gemv_rows_kernel" in d and "attention=attn_cluster_kernel cluster=8" in d, d
+        assert "projections=gemv_rows_kernel" in d and "attention=attn_mma_kernel cluster=4" in d, d
     finally:
         g.close()

@@ -187,14 +187,24 @@ template <int BH>
 __device__ __forceinline__ void tc_cluster_epilogue(const TcParams& p, cooperative_groups::cluster_group& cl,
                                                     float* park, int tile, int rr, int c4,
                                                     const float* rstd = nullptr, const float* ypre = nullptr) {
+    // every split's distributed-shared-memory load is issued before any is
+    // used (a remote load takes several hundred cycles), then the splits are
+    // added in split order (deterministic)
+    float4 ta[kTcMaxSplits], tu[kTcMaxSplits];
+#pragma unroll
+    for (int s = 0; s < kTcMaxSplits; ++s) {
+        if (s < p.splits) {
+            const float* rem = cl.map_shared_rank(park, s);
+            ta[s] = *reinterpret_cast<const float4*>(rem + tc_park_idx<BH>(rr, c4));
+            if (p.ru == 2) tu[s] = *reinterpret_cast<const float4*>(rem + tc_park_idx<BH>(rr + 1, c4));
+        }
+    }
     float4 a = make_float4(0.f, 0.f, 0.f, 0.f), u = a;
-    for (int s = 0; s < p.splits; ++s) {
-        const float* rem = cl.map_shared_rank(park, s);
-        const float4 t = *reinterpret_cast<const float4*>(rem + tc_park_idx<BH>(rr, c4));
-        a.x += t.x; a.y += t.y; a.z += t.z; a.w += t.w;
-        if (p.ru == 2) {
-            const float4 t2 = *reinterpret_cast<const float4*>(rem + tc_park_idx<BH>(rr + 1, c4));
-            u.x += t2.x; u.y += t2.y; u.z += t2.z; u.w += t2.w;
+#pragma unroll
+    for (int s = 0; s < kTcMaxSplits; ++s) {
+        if (s < p.splits) {
+            a.x += ta[s].x; a.y += ta[s].y; a.z += ta[s].z; a.w += ta[s].w;
+            if (p.ru == 2) { u.x += tu[s].x; u.y += tu[s].y; u.z += tu[s].z; u.w += tu[s].w; }
         }
     }
     float va[4] = {a.x, a.y, a.z, a.w}, vu[4] = {u.x, u.y, u.z, u.w};
@@ -699,8 +709,14 @@ __global__ void __launch_bounds__(kTcfThreads, 1)
         if (epi_warp) {
             const int xt = threadIdx.x - 64;
             if (xt < BH) {
+                float ts[kTcMaxSplits];  // every remote load first, then the sum in split order
+#pragma unroll
+                for (int rk = 0; rk < kTcMaxSplits; ++rk)
+                    if (rk < p.splits) ts[rk] = *cl.map_shared_rank(&ss_s[xt], rk);
                 float t = 0.f;
-                for (int rk = 0; rk < p.splits; ++rk) t += *cl.map_shared_rank(&ss_s[xt], rk);
+#pragma unroll
+                for (int rk = 0; rk < kTcMaxSplits; ++rk)
+                    if (rk < p.splits) t += ts[rk];
                 rstd_s[xt] = in.norm ? 1.0f / sqrtf(t / (float)in.klen + in.eps) : 1.0f;
             }
             asm volatile("bar.sync 1, 128;" ::: "memory");

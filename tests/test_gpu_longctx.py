@@ -1,7 +1,8 @@
-"""Long-context parity: caches filled with 1500 seeded entries (many 64-entry
-pages per attention split) on both sides, then forced-replay decode steps;
-the split-KV attention with 8-CTA clusters (default) and 16-CTA clusters
-(opt-in) against the oracle."""
+"""Long-context parity: caches filled with seeded entries (many 64-entry
+pages per attention split) on both sides, then forced-replay decode steps
+against the oracle: at 1500 entries the split-KV attention with 8-CTA
+clusters (default) and 16-CTA clusters (opt-in); at 2500 entries the
+unclustered tensor-core attention."""
 import os
 
 import numpy as np
@@ -39,6 +40,41 @@ def test_long_context_forced_replay(cs16, monkeypatch):
             pend = [[orc.seq(b)["p0"], orc.seq(b)["p1"]] for b in range(B)]
             gpu.set_pending(pend)
             tok, nacc = gpu.step()
+            o = orc.step(tau=s.tau)
+            compare(s, s.tau, o, gpu.debug(), tok, nacc, 0, st, tol_for(s), f"step {i}")
+        n, _ = gpu.counters()
+        assert list(n) == [n_ctx + steps] * B
+    finally:
+        gpu.close()
+
+
+@pytest.mark.parametrize("B", [1, 2])
+def test_long_context_unclustered_tensor_core_attention(B):
+    """From 2048 cached pairs, when 8-CTA clusters would leave SMs idle, the
+    tensor-core attention splits each (sequence, kv head) over unclustered
+    CTAs whose partials the last arrival merges through global memory."""
+    s = MID
+    n_ctx, steps = 2500, 3
+    w = synth.gen_weights(s, seed=18)
+    K, V = synth.gen_kv_fill(s, n_ctx, seed=19)
+    K, V = K.numpy(), V.numpy()
+    prompts = synth.gen_prompts(B, 4, s.V, seed=14).numpy()
+    gpu = capi.Pipo(s, w, max_batch=B, max_ctx=n_ctx + steps + 2, debug=True, page_shuffle_seed=5)
+    orc = O.State(O.Model(s, w, max_ctx=n_ctx + steps + 2), B)
+    try:
+        gpu.prefill(prompts)
+        orc.prefill(prompts, tau=s.tau)
+        for b in range(B):
+            gpu.load_cache(b, K, V)
+            orc.set_cache(b, K, V)
+        st = Stats()
+        for i in range(steps):
+            pend = [[orc.seq(b)["p0"], orc.seq(b)["p1"]] for b in range(B)]
+            gpu.set_pending(pend)
+            tok, nacc = gpu.step()
+            if i == 0:
+                d = gpu.describe()
+                assert "attention=attn_mma_kernel unclustered splits=" in d, d
             o = orc.step(tau=s.tau)
             compare(s, s.tau, o, gpu.debug(), tok, nacc, 0, st, tol_for(s), f"step {i}")
         n, _ = gpu.counters()

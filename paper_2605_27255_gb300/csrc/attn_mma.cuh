@@ -11,8 +11,8 @@
 // distributed shared memory.
 //
 // Per CTA: a producer thread copies aligned 16-entry groups of the slice into
-// a ring of kMmaStages stages with TMA tensor copies (each compute warp owns
-// kMmaStages / kMmaWarps of the stages, see mma_stage): the cache layer is a 2-D
+// a ring of ST stages with TMA tensor copies (each compute warp owns
+// ST / kMmaWarps of the stages, see mma_stage): the cache layer is a 2-D
 // tensor of rows (block, kv head, slot) x d_h bf16, and a group is four boxes
 // of 16 rows x 64 dims (K and V, two halves each) stored with the 128-byte
 // swizzle, which keeps the ldmatrix reads free of bank conflicts.  Four
@@ -45,11 +45,19 @@ constexpr int kMmaStageBytes = 4 * kMmaHalf;        // K (2 halves) + V (2 halve
 #ifndef PIPO_MMA_WARPS
 #define PIPO_MMA_WARPS 5
 #endif
+#ifndef PIPO_MMA_DEEP_STAGES
+#define PIPO_MMA_DEEP_STAGES 20
+#endif
 constexpr int kMmaStages = PIPO_MMA_STAGES;
+// the deep ring, for launches whose CTAs each have an SM of their own: a CTA
+// whose slice has kMmaDeepStages groups of 16 entries or fewer issues every
+// copy at its entry (a shallow ring re-issues a stage only after its first
+// group is consumed, one more HBM round trip after the dependency wait)
+constexpr int kMmaDeepStages = PIPO_MMA_DEEP_STAGES;
 constexpr int kMmaWarps = PIPO_MMA_WARPS;           // compute warps (at least the G heads of a kv head)
 constexpr int kMmaThreads = (kMmaWarps + 1) * 32;   // + the producer warp
-constexpr int kMmaSpw = kMmaStages / kMmaWarps;     // stages of one compute warp
-static_assert(kMmaStages % kMmaWarps == 0, "every compute warp owns the same number of stages");
+static_assert(kMmaStages % kMmaWarps == 0 && kMmaDeepStages % kMmaWarps == 0,
+              "every compute warp owns the same number of stages");
 
 // Group t (16 cached entries) is consumed by compute warp t % kMmaWarps and
 // travels through that warp's own stages in turn.  Each stage then has one
@@ -58,15 +66,20 @@ static_assert(kMmaStages % kMmaWarps == 0, "every compute warp owns the same num
 // only the current and the preceding phase, and with one ring shared by all
 // warps a fast warp could otherwise meet the parity of a phase two behind
 // (copies need not land in the order they were issued).  The k-th group of a
-// stage has phase k; the parity of group t is (t / kMmaStages) & 1.
-__device__ __forceinline__ int mma_stage(int t) { return (t % kMmaWarps) * kMmaSpw + (t / kMmaWarps) % kMmaSpw; }
+// stage has phase k; the parity of group t is (t / ST) & 1 in a ring of ST
+// stages.
+template <int ST>
+__device__ __forceinline__ int mma_stage(int t) {
+    constexpr int spw = ST / kMmaWarps;  // stages of one compute warp
+    return (t % kMmaWarps) * spw + (t / kMmaWarps) % spw;
+}
 
 // dynamic shared memory: the stage ring, its barriers, and the receive
 // buffer of the cluster merge, one slot per CTA of the cluster (CS), each
 // [G][DH] partial output then [G] maxima and [G] sums (fp32; G <= 4)
 constexpr int kMmaRcvSlot = 4 * 128 + 8;  // floats per slot at G = 4 (smaller G use a prefix)
-constexpr size_t mma_attn_smem(int cs = 8) {
-    return 1024 + (size_t)kMmaStages * kMmaStageBytes + 2 * kMmaStages * 8 + (size_t)cs * kMmaRcvSlot * 4;
+constexpr size_t mma_attn_smem(int cs = 8, int st = kMmaStages) {
+    return 1024 + (size_t)st * kMmaStageBytes + 2 * st * 8 + (size_t)cs * kMmaRcvSlot * 4;
 }
 
 // The cluster merge pushes every CTA's partial softmax state into rank 0's
@@ -158,11 +171,12 @@ __device__ __forceinline__ void mma_rows8(float (&d)[4], uint32_t a0, uint32_t a
 // scratch (AttnParams::part_o, part_ml) and the last of a (row, kv head) to
 // arrive (AttnParams::counters) merges the S partials in split order: any
 // split count, so that long caches fill the GPU evenly.
-template <int G, bool FLAT = false>
+template <int G, bool FLAT = false, int ST = kMmaStages>
 __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, const __grid_constant__ CUtensorMap tmK,
                                                                const __grid_constant__ CUtensorMap tmV) {
     static_assert(G == 1 || G == 2 || G == 4, "2G query rows must fit the 8 live MMA rows");
-    static_assert(kMmaWarps >= G && kMmaWarps <= 16 && kMmaStages >= 2, "warps hold the new entry's heads");
+    static_assert(kMmaWarps >= G && kMmaWarps <= 16 && ST >= kMmaWarps && ST % kMmaWarps == 0,
+                  "warps hold the new entry's heads; every warp owns the same number of stages");
     constexpr int DH = kMmaDH;
     constexpr int NW = kMmaWarps;
     constexpr int NP = NW + 1;  // softmax partials: one per compute warp + the new entry
@@ -174,14 +188,14 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
                                      // warps' partials go to their own first stage
     __shared__ int abort_flag;
     __shared__ __align__(8) uint64_t rcv_bar;  // rank 0: one arrival per CTA of the cluster
-    PIPO_TR(__shared__ unsigned long long tr_s[3], tr_m[2]; const TraceT0 tr0 = trace_begin();)
+    PIPO_TR(__shared__ unsigned long long tr_s[3], tr_m[2], tr_f; const TraceT0 tr0 = trace_begin();)
 
     unsigned char* ring = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(am_smem_raw) + 1023) & ~(uintptr_t)1023);
-    uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)kMmaStages * kMmaStageBytes);
-    uint64_t* empty = full + kMmaStages;
-    float* rcv = reinterpret_cast<float*>(empty + kMmaStages);  // [CS][kMmaRcvSlot] (rank 0's is used)
+    uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)ST * kMmaStageBytes);
+    uint64_t* empty = full + ST;
+    float* rcv = reinterpret_cast<float*>(empty + ST);  // [CS][kMmaRcvSlot] (rank 0's is used)
     // partial of compute warp w: [G][DH] floats at the start of its first stage
-    auto wpart = [&](int w) { return reinterpret_cast<float*>(ring + (size_t)(w * kMmaSpw) * kMmaStageBytes); };
+    auto wpart = [&](int w) { return reinterpret_cast<float*>(ring + (size_t)(w * (ST / NW)) * kMmaStageBytes); };
 
     pdl_launch();
     cg::cluster_group cluster = cg::this_cluster();
@@ -204,7 +218,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     if (threadIdx.x == 0) {
         prefetch_tmap(&tmK);
         prefetch_tmap(&tmV);
-        for (int i = 0; i < kMmaStages; ++i) {
+        for (int i = 0; i < ST; ++i) {
             mbar_init(full + i, 1);
             mbar_init(empty + i, 1);
         }
@@ -225,9 +239,9 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
             if (p.no_append) pdl_wait();
             int t = 0;
             for (; t < ngrp; ++t) {
-                const int st = mma_stage(t);
-                if (t >= kMmaStages && (*(volatile int*)&abort_flag ||
-                                        !mbar_wait(empty + st, (uint32_t)(((t / kMmaStages) & 1) ^ 1), 21, t))) {
+                const int st = mma_stage<ST>(t);
+                if (t >= ST && (*(volatile int*)&abort_flag ||
+                                        !mbar_wait(empty + st, (uint32_t)(((t / ST) & 1) ^ 1), 21, t))) {
                     *(volatile int*)&abort_flag = 1;
                     break;
                 }
@@ -242,15 +256,15 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
                 tma_load_2d(stg + 3 * kMmaHalf, &tmV, 64, trow, full + st);
             }
             // no copy into this CTA's shared memory may still be in flight at exit
-            for (int i = max(0, t - kMmaStages); i < t; ++i)
-                mbar_wait(full + mma_stage(i), (uint32_t)((i / kMmaStages) & 1), 22, i);
+            for (int i = max(0, t - ST); i < t; ++i)
+                mbar_wait(full + mma_stage<ST>(i), (uint32_t)((i / ST) & 1), 22, i);
         }
         __syncwarp();
     } else {
         const int ct = threadIdx.x;  // 0 .. 32*NW-1
         // ---- prologue: rotated, pre-scaled q of the G heads; the new k, v
         pdl_wait();
-        PIPO_TR(if (ct == 0) tr_s[0] = trace_now();)
+        PIPO_TR(if (ct == 0) tr_s[0] = tr_f = trace_now();)
         const float* qrow = p.qkv + (size_t)row * p.ld_qkv;
         const float* rope = p.rope + (size_t)n * DH;  // [DH/2][2] cos, sin at position n
         for (int i = ct; i < (G + 1) * (DH / 2); i += 32 * NW) {
@@ -325,11 +339,12 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         const int lm = lane >> 3, lr = lane & 7;  // ldmatrix: matrix index, row within it
 
         for (int t = warp; t < ngrp; t += NW) {
-            const int st = mma_stage(t);
-            if (*(volatile int*)&abort_flag || !mbar_wait(full + st, (uint32_t)((t / kMmaStages) & 1), 23, t)) {
+            const int st = mma_stage<ST>(t);
+            if (*(volatile int*)&abort_flag || !mbar_wait(full + st, (uint32_t)((t / ST) & 1), 23, t)) {
                 *(volatile int*)&abort_flag = 1;
                 break;
             }
+            PIPO_TR(if (ct == 0 && t == warp) tr_f = trace_now();)
             const uint32_t kS = smem_u32(ring + (size_t)st * kMmaStageBytes);
             const uint32_t vS = kS + 2 * kMmaHalf;
             const int e0 = (grp0 + t) * kMmaRun;
@@ -521,7 +536,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     }
     if (CS == 1) {
         PIPO_TR(if (threadIdx.x == 0) {
-            trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);
+            trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_f, tr_s[2]);
             trace_put(TR_ATTN_MMA_EPI, tr0, tr_s[0], tr_s[1], tr_m[0], tr_s[2], tr_s[2]);
         })
         return;
@@ -531,7 +546,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
     if (threadIdx.x == 0) mbar_arrive_remote(&rcv_bar, 0);
     if (s != 0) {
         PIPO_TR(if (threadIdx.x == 0) {
-            trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);
+            trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_f, tr_s[2]);
             trace_put(TR_ATTN_MMA_EPI, tr0, tr_s[0], tr_s[1], tr_m[0], tr_s[2], tr_s[2]);
         })
         return;  // rank 0 merges; nothing reads this CTA's shared memory
@@ -558,7 +573,7 @@ __global__ void __launch_bounds__(kMmaThreads) attn_mma_kernel(AttnParams p, con
         }
     }
     PIPO_TR(if (threadIdx.x == 0) {
-        trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_s[1], tr_s[2]);
+        trace_put(TR_ATTN_MMA, tr0, tr0.clk, tr_s[0], tr_f, tr_s[2]);
         trace_put(TR_ATTN_MMA_EPI, tr0, tr_s[0], tr_s[1], tr_m[0], tr_s[2], tr_m[1]);
     })
 }

@@ -656,6 +656,8 @@ __global__ void __launch_bounds__(kStreamThreads) gemv_rows_kernel(GemvParams p)
         };
         load_batch(bufA);
         load_batch(bufB);
+        // with this warp's first weight loads in flight
+        if (b0 == 0 && p.pf_k && threadIdx.x == 0) l2_warm_pages(p);
         if (b0 == 0) {
             pdl_wait();
             PIPO_TR(tr1 = trace_now();)

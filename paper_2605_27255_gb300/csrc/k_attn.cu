@@ -63,12 +63,16 @@ void* k_pick_attn_flat(bool bf, int DH, int G) {
     return nullptr;
 }
 
-// tensor-core attention (bf16 cache, d_h = 128, 1, 2 or 4 query heads per kv head)
-void* k_pick_attn_mma(int G) {
+// tensor-core attention (bf16 cache, d_h = 128, 1, 2 or 4 query heads per
+// kv head); deep: the kMmaDeepStages ring
+void* k_pick_attn_mma(int G, bool deep) {
     switch (G) {
-        case 1: return reinterpret_cast<void*>(&attn_mma_kernel<1>);
-        case 2: return reinterpret_cast<void*>(&attn_mma_kernel<2>);
-        case 4: return reinterpret_cast<void*>(&attn_mma_kernel<4>);
+        case 1: return deep ? reinterpret_cast<void*>(&attn_mma_kernel<1, false, kMmaDeepStages>)
+                            : reinterpret_cast<void*>(&attn_mma_kernel<1>);
+        case 2: return deep ? reinterpret_cast<void*>(&attn_mma_kernel<2, false, kMmaDeepStages>)
+                            : reinterpret_cast<void*>(&attn_mma_kernel<2>);
+        case 4: return deep ? reinterpret_cast<void*>(&attn_mma_kernel<4, false, kMmaDeepStages>)
+                            : reinterpret_cast<void*>(&attn_mma_kernel<4>);
         default: return nullptr;
     }
 }

@@ -26,7 +26,7 @@ void* k_pick_wait_selftest();                       // wait_selftest_kernel (rep
 void* k_pick_attn_decode(bool bf, int DH, int G);   // attn_decode_kernel
 void* k_pick_attn_cluster(bool bf, int DH, int G);  // attn_cluster_kernel
 void* k_pick_attn_flat(bool bf, int DH, int G);     // attn_cluster_kernel, unclustered (global merge)
-void* k_pick_attn_mma(int G);                       // attn_mma_kernel
+void* k_pick_attn_mma(int G, bool deep);            // attn_mma_kernel (deep: the kMmaDeepStages ring)
 void* k_pick_attn_mma_flat(int G);                  // attn_mma_kernel, unclustered (global merge)
 void* k_pick_attn_prefill(int G);                   // attn_prefill_kernel
 void* k_pick_rope_append(bool bf, int DH);          // rope_append_kernel

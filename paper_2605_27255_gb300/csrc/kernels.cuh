@@ -58,6 +58,18 @@ struct GemvParams {
     int zero_n;
     float* part;         // EPI_RESADD with splitk > 1: partials [splitk][B][N]
     unsigned* rowcnt;    // arrival counters per (batch group, row), [ceil(B/NB)][N] (zero between launches)
+    // L2 warm-up of the next attention's cached pages (streaming GEMV, a
+    // decode step's QKV projection; pf_k == nullptr: none).  Before its
+    // dependency wait the kernel prefetches into L2 the key and value pages
+    // that hold entries 0 .. pf_npos[b] - 1 of sequences b < pf_nseq: page
+    // block blk of a layer is pf_bytes contiguous bytes at pf_k / pf_v +
+    // blk * pf_bytes (every kv head), blk = pf_table[b * pf_bps + page].
+    const void* pf_k;
+    const void* pf_v;
+    const int32_t* pf_table;
+    const int32_t* pf_npos;
+    int pf_bps, pf_page, pf_nseq;
+    unsigned pf_bytes;
 };
 
 // ---------------------------------------------------------------- loads
@@ -71,6 +83,30 @@ __device__ __forceinline__ uint4 ldg_stream(const void* p) {
         : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
         : "l"(p));
     return r;
+}
+
+// Bulk prefetch of [ptr, ptr + bytes) into L2 (16-byte aligned, bytes a
+// multiple of 16); no data reaches the SM.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* ptr, unsigned bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
+}
+
+// GemvParams::pf_*: the pages are spread over the CTAs of the grid, one bulk
+// prefetch per page of keys or values.  The cached lengths and page tables
+// change only between steps (graph launches), so they are read before the
+// dependency wait; the entries prefetched were written by earlier steps.
+__device__ __forceinline__ void l2_warm_pages(const GemvParams& p) {
+    int i0 = 0;  // items of the sequences before b
+    for (int b = 0; b < p.pf_nseq; ++b) {
+        const int items = 2 * ((p.pf_npos[b] + p.pf_page - 1) / p.pf_page);
+        for (int i = ((int)blockIdx.x - i0 % (int)gridDim.x + (int)gridDim.x) % (int)gridDim.x; i < items;
+             i += gridDim.x) {
+            const int blk = p.pf_table[(size_t)b * p.pf_bps + (i >> 1)];
+            const char* base = static_cast<const char*>((i & 1) ? p.pf_v : p.pf_k);
+            prefetch_l2_bulk(base + (size_t)blk * p.pf_bytes, p.pf_bytes);
+        }
+        i0 += items;
+    }
 }
 
 // 128-bit load of cache data written by earlier kernels (L1 bypassed).

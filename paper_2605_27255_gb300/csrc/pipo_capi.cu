@@ -379,7 +379,7 @@ size_t tcv_smem(int bh, bool deep, bool fused) {
 int tcv_threads(bool fused) { return fused ? kTcfThreads : kTcThreads; }
 
 bool tc_cluster_spread();
-void* attnm_pick(int G);
+void* attnm_pick(int G, bool deep = false);
 
 cudaError_t set_smem_attrs(bool bf) {
     int dev = 0, optin = 0;
@@ -410,9 +410,9 @@ cudaError_t set_smem_attrs(bool bf) {
             }
     if (bf)
         for (int g : {1, 2, 4})
-            for (void* f : {attnm_pick(g), k_pick_attn_mma_flat(g)}) {
-                cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                     (int)mma_attn_smem());
+            for (void* f : {attnm_pick(g), k_pick_attn_mma_flat(g), attnm_pick(g, true)}) {
+                const size_t smem = f == attnm_pick(g, true) ? mma_attn_smem(8, kMmaDeepStages) : mma_attn_smem();
+                cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
                 if (e != cudaSuccess) return e;
             }
     if (bf)
@@ -749,7 +749,7 @@ void* attn_pick(bool bf, int DH, int G) { return k_pick_attn_decode(bf, DH, G); 
 // one kernel for every cluster size (read from the cluster at run time)
 void* attnc_pick(bool bf, int DH, int G) { return k_pick_attn_cluster(bf, DH, G); }
 // tensor-core attention (bf16 cache, d_h = 128, 1, 2 or 4 query heads per kv head)
-void* attnm_pick(int G) { return k_pick_attn_mma(G); }
+void* attnm_pick(int G, bool deep) { return k_pick_attn_mma(G, deep); }
 
 // Can a 16-CTA cluster of this kernel be scheduled here?  (sets the
 // non-portable cluster attribute; any failure selects 8)
@@ -813,7 +813,8 @@ cudaError_t set_carveouts(bool bf) {
             for (bool deep : {false, true})
                 for (bool fused : {false, true}) fns.push_back(pick_tcv(bn, deep, fused));
         fns.push_back(reinterpret_cast<const void*>(k_pick_prep_bf16()));
-        for (int g : {1, 2, 4}) fns.push_back(attnm_pick(g));
+        for (int g : {1, 2, 4})
+            for (bool deep : {false, true}) fns.push_back(attnm_pick(g, deep));
     }
     for (int dh : {64, 128}) {
         for (int g : {1, 2, 4, 8}) {
@@ -850,14 +851,20 @@ bool attn_use_mma(const pipo_ctx* ctx, int B) {
            (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers;
 }
 
+bool attn_mma_deep_on();
+
 // CTAs per (sequence, kv head) of the clustered attention: 8 while the batch
 // leaves SMs idle (16 where allowed and still under two per SM), fewer as the
 // (sequence, kv head) pairs alone fill the GPU.
 int attn_cluster_size(const pipo_ctx* ctx, int B) {
     if (ctx->attn_cs_force) return ctx->attn_cs_force;
-    // one sequence on the tensor-core attention: 4-CTA clusters (4b-b1: 2.61
-    // against 2.63 ms per step with 8)
-    if (B == 1 && attn_use_mma(ctx, B)) return 4;
+    // one sequence on the tensor-core attention: 8-CTA clusters on the deep
+    // stage ring when every CTA has an SM of its own, else 4.  4b-b1 (ms per
+    // step): 8-CTA deep 2.463, 4-CTA deep 2.571, 4-CTA with 10 stages 2.615
+    // (an 8-CTA slice of ~1160 pairs spans 10 or 11 groups of 16: one more
+    // than 10 stages hold)
+    if (B == 1 && attn_use_mma(ctx, B))
+        return attn_mma_deep_on() && (long long)ctx->cfg.n_kv_heads * 8 <= ctx->sms ? 8 : 4;
     const long long pairs = (long long)B * ctx->cfg.n_kv_heads;
     if (ctx->attn_cs16 && pairs * 16 <= 2 * ctx->sms) return 16;
     // measured best: about two tensor-core attention CTAs per SM (they are
@@ -883,6 +890,37 @@ bool attn_flat_now(const pipo_ctx* ctx) {
     return n > 0 && sum / n >= kFlatMinEntries;
 }
 
+// The QKV projection of a decode step on the streaming GEMV prefetches the
+// layer's cached key and value pages into L2 before its dependency wait, so
+// that the attention's copies, issued when its CTAs find room (as the
+// projection's CTAs leave), are served from L2 rather than queued behind the
+// weight stream in HBM.  PIPO_ATTN_L2_WARM=0: never.
+bool attn_l2_warm() {
+    static const bool on = [] {
+        const char* ev = getenv("PIPO_ATTN_L2_WARM");
+        return ev ? atoi(ev) != 0 : true;
+    }();
+    return on;
+}
+
+// The deep stage ring for the clustered tensor-core attention when each of
+// its CTAs has an SM of its own (rows x kv heads x cluster size <= SMs): the
+// shared memory it takes then keeps no CTA of this launch from starting, and
+// a CTA's slice of up to kMmaDeepStages groups is in flight from its entry.
+// 4b-b1 (one sequence, ~1160 cached pairs, 4-CTA clusters, 32 CTAs):
+// 2.595 ms per step with 10 stages, 2.563 with 15, 2.551 with 20.
+// PIPO_ATTN_MMA_DEEP=0: never.
+bool attn_mma_deep_on() {
+    static const bool on = [] {
+        const char* ev = getenv("PIPO_ATTN_MMA_DEEP");
+        return ev ? atoi(ev) != 0 : true;
+    }();
+    return on;
+}
+bool attn_mma_deep(const pipo_ctx* ctx, int R, int cs) {
+    return attn_mma_deep_on() && (long long)R * ctx->cfg.n_kv_heads * cs <= ctx->sms;
+}
+
 // Split count of the unclustered tensor-core attention, or 0 for the
 // clustered one: when the (row, kv head) pairs times the largest cluster
 // (8) leave SMs without two CTAs and the cached slices stay long (mean
@@ -892,7 +930,9 @@ bool attn_flat_now(const pipo_ctx* ctx) {
 // 4.32; unclustered one wave (S = 9, 288 CTAs) 4.09; two waves (S = 19)
 // 4.35; three 4.53 (more waves balance the SMs but leave no room for the
 // next kernel's CTAs to start early).  One sequence at ~2180 pairs (9b-b1):
-// 3.83 against 3.89 ms with the register-ring attention (unclustered).
+// 3.83 against 3.89 ms with the register-ring attention (unclustered), but
+// 3.71 with 8-CTA clusters on the deep ring, which therefore stay while
+// that ring holds a CTA's slice.
 // PIPO_ATTN_MMA_WAVES sets the waves, PIPO_ATTN_MMA_FLAT=0 / 2: never / also
 // for short caches.
 constexpr int kFlatMmaMinEntries = 2048;
@@ -909,6 +949,9 @@ int attn_mma_flat_splits(const pipo_ctx* ctx, int R) {
     for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b, ++n) sum += ctx->h_len[b];
     const double mean = n > 0 ? sum / n : 0.0;
     if (mode == 1 && mean < kFlatMmaMinEntries) return 0;
+    // 8-CTA clusters on the deep ring while it holds a CTA's whole slice (a
+    // slice of c entries spans at most c / 16 + 2 groups)
+    if (mode == 1 && attn_mma_deep(ctx, R, 8) && mean <= 8.0 * kMmaRun * (kMmaDeepStages - 2)) return 0;
     static const int waves = [] {
         const char* ev = getenv("PIPO_ATTN_MMA_WAVES");
         return ev ? std::max(1, atoi(ev)) : 1;
@@ -972,8 +1015,19 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
     GemvParams p = gemv_base(ctx, bw.Wqkv, rows, EPI_STORE, ctx->qkv, rows);
     p.seg[0] = act_seg(xr, H, H, bw.attn_norm);
     p.K = H;
-    TRY(launch_gemv(ctx, p));
     KVView kv = kv_view(ctx, cache_layer);
+    if (attn_l2_warm() && (ctx->rows <= 0 || ctx->rows == ctx->B)) {
+        // a decode step: the streaming GEMV warms L2 with this layer's cached pages
+        p.pf_k = kv.K;
+        p.pf_v = kv.V;
+        p.pf_table = kv.table;
+        p.pf_npos = ctx->n_pos;
+        p.pf_bps = kv.blocks_per_seq;
+        p.pf_page = kv.page;
+        p.pf_nseq = ctx->B;
+        p.pf_bytes = (unsigned)((size_t)kv.n_kv * kv.page * DH * ctx->esz);
+    }
+    TRY(launch_gemv(ctx, p));
     if (!ctx->attn_v0) {
         // RoPE + KV append + split-KV attention, one cluster per (row, kv head).
         // A prefill chunk (several positions per sequence) appends all its
@@ -1026,15 +1080,16 @@ pipo_status enqueue_block(pipo_ctx* ctx, const BlockW& bw, int cache_layer, floa
                           margs));
         } else if (attn_use_mma(ctx, R) && cs <= 8) {
             void* margs[] = {&ap, &ctx->kv_tm[2 * cache_layer], &ctx->kv_tm[2 * cache_layer + 1]};
+            const bool deep = attn_mma_deep(ctx, R, cs);
+            const size_t smem = mma_attn_smem(cs, deep ? kMmaDeepStages : kMmaStages);
             static const bool verbose = getenv("PIPO_VERBOSE") != nullptr;
             if (verbose) {
                 int per_sm = 0;
-                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attnm_pick(G), kMmaThreads, mma_attn_smem(cs));
+                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attnm_pick(G, deep), kMmaThreads, smem);
                 fprintf(stderr, "[pipo] attention: tensor-core, cluster %d, %zu B shared memory, %d CTAs per SM\n", cs,
-                        mma_attn_smem(cs), per_sm);
+                        smem, per_sm);
             }
-            TRY(launch_ex(ctx, attnm_pick(G), dim3(cs, c.n_kv_heads, R), dim3(kMmaThreads), mma_attn_smem(cs),
-                          margs, cs));
+            TRY(launch_ex(ctx, attnm_pick(G, deep), dim3(cs, c.n_kv_heads, R), dim3(kMmaThreads), smem, margs, cs));
         }
         else if (attn_flat_now(ctx) && !chunk && !ctx->attn_cs_force) {
             // register-ring attention over about two CTAs per SM, no cluster:
@@ -2528,7 +2583,9 @@ pipo_status pipo_describe_step(const pipo_ctx* ctx, char* h_buf, size_t cap) {
                      : flat ? " unclustered splits=" +
                                   std::to_string(std::max(1, std::min({ctx->sms / (B * c.n_kv_heads),
                                                                        (c.max_ctx + 15) / 16, kFlatMaxSplits})))
-                            : " cluster=" + std::to_string(cs));
+                            : " cluster=" + std::to_string(cs) +
+                                  (mma && attn_mma_deep(ctx, B, cs) ? " stages=" + std::to_string(kMmaDeepStages)
+                                                                      : std::string()));
     // decoding mode, heads and prefill arrangement
     d += ctx->regular ? " mode=regular" : " mode=pair";
     d += ctx->samp_on ? " heads=sampled" : " heads=argmax";

@@ -1,8 +1,8 @@
 """Long-context parity: caches filled with seeded entries (many 64-entry
 pages per attention split) on both sides, then forced-replay decode steps
 against the oracle: at 1500 entries the split-KV attention with 8-CTA
-clusters (default) and 16-CTA clusters (opt-in); at 2500 entries the
-unclustered tensor-core attention."""
+clusters (default) and 16-CTA clusters (opt-in), and one sequence on the
+deep stage ring; at 2500 entries the unclustered tensor-core attention."""
 import os
 
 import numpy as np
@@ -79,5 +79,40 @@ def test_long_context_unclustered_tensor_core_attention(B):
             compare(s, s.tau, o, gpu.debug(), tok, nacc, 0, st, tol_for(s), f"step {i}")
         n, _ = gpu.counters()
         assert list(n) == [n_ctx + steps] * B
+    finally:
+        gpu.close()
+
+
+@pytest.mark.parametrize("cs", ["2", "8"])
+def test_long_context_deep_ring(cs, monkeypatch):
+    """One sequence with each cluster CTA on an SM of its own takes the deep
+    stage ring: with 2-CTA clusters a CTA's slice of 1500 entries spans about
+    47 groups of 16, so every stage is refilled while the warps compute; with
+    8 the whole slice is in flight from the CTA's entry."""
+    monkeypatch.setenv("PIPO_ATTN_CS", cs)
+    s = MID
+    n_ctx, B, steps = 1500, 1, 3
+    w = synth.gen_weights(s, seed=28)
+    K, V = synth.gen_kv_fill(s, n_ctx, seed=29)
+    K, V = K.numpy(), V.numpy()
+    prompts = synth.gen_prompts(B, 4, s.V, seed=24).numpy()
+    gpu = capi.Pipo(s, w, max_batch=B, max_ctx=n_ctx + steps + 2, debug=True, page_shuffle_seed=7)
+    orc = O.State(O.Model(s, w, max_ctx=n_ctx + steps + 2), B)
+    try:
+        gpu.prefill(prompts)
+        orc.prefill(prompts, tau=s.tau)
+        gpu.load_cache(0, K, V)
+        orc.set_cache(0, K, V)
+        st = Stats()
+        for i in range(steps):
+            gpu.set_pending([[orc.seq(0)["p0"], orc.seq(0)["p1"]]])
+            tok, nacc = gpu.step()
+            if i == 0:
+                d = gpu.describe()
+                assert f"attention=attn_mma_kernel cluster={cs} stages=20" in d, d
+            o = orc.step(tau=s.tau)
+            compare(s, s.tau, o, gpu.debug(), tok, nacc, 0, st, tol_for(s), f"step {i}")
+        n, _ = gpu.counters()
+        assert list(n) == [n_ctx + steps]
     finally:
         gpu.close()

@@ -192,8 +192,8 @@ def test_decode_path_uses_tensor_core_kernels():
     """At B = 16 the block projections and the attention take the tcgen05 and
     mma.sync kernels (the down projection, K = 1376, stays on CUDA cores); a
     single sequence keeps the CUDA-core GEMV (a matrix-vector product) and
-    takes the tensor-core attention in 4-CTA clusters (its 4 query heads per
-    kv head are the MMA rows)."""
+    takes the tensor-core attention (its 4 query heads per kv head are the
+    MMA rows) in 8-CTA clusters, one CTA per SM, on the deep stage ring."""
     w = synth.gen_weights(MID, seed=23)
     g = capi.Pipo(MID, w, max_batch=16, max_ctx=40)
     try:
@@ -207,6 +207,6 @@ def test_decode_path_uses_tensor_core_kernels():
     try:
         g.prefill(synth.gen_prompts(1, 8, MID.V, seed=1).numpy())
         d = g.describe()
-        assert "projections=gemv_rows_kernel" in d and "attention=attn_mma_kernel cluster=4" in d, d
+        assert "projections=gemv_rows_kernel" in d and "attention=attn_mma_kernel cluster=8 stages=20" in d, d
     finally:
         g.close()

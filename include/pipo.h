@@ -172,7 +172,11 @@ PIPO_API pipo_status pipo_decode_step(pipo_ctx *ctx, int32_t *h_tokens, int32_t 
 
 /* The same step, enqueued on the context stream without a host sync;
  * d_tokens[B,2] / d_n_accepted[B] are device buffers (may be NULL).  The
- * step is a captured CUDA graph replayed per call. */
+ * step is a captured CUDA graph replayed per call.  Its launch plan (kernel
+ * forms, attention splits) is made for the mean cached length at capture
+ * and kept while the caches grow; a prefill, a cache load or a change of
+ * batch, stream, threshold or sampler drops the graph, and the next step
+ * captures a new one. */
 PIPO_API pipo_status pipo_decode_step_async(pipo_ctx *ctx, int32_t *d_tokens, int32_t *d_n_accepted);
 
 /* n_steps pair-decode steps in one call (graph replays back to back, one
@@ -399,6 +403,7 @@ PIPO_API pipo_status pipo_profile_step(pipo_ctx *ctx, int32_t cap, int32_t *h_ki
  * (every projection of Eq. 1-6 and both LM-head passes, Eq. 3 and Eq. 5,
  * with the operand preparation some of them need); family 1: the attention
  * launches (Eq. 2).  Time the replays with events on the context stream.
+ * With a captured step graph the family takes that graph's launch plan.
  * The decoding state does not change: pending pairs, cache lengths,
  * counters and every live cache entry stay as they were (an attention
  * replay writes only the entry one past each sequence's cached length, which

@@ -189,6 +189,7 @@ struct pipo_ctx {
     std::vector<int32_t> h_len;
     cudaGraphExec_t graph = nullptr;
     int graph_B = -1;
+    double plan_len = -1.0;           // mean cached length the step graph's launch plan was made for
     bool graph_regular = false;       // the captured step is a regular-decoding step
     int launches = 0;
     std::map<long long, int> occ;
@@ -851,6 +852,19 @@ bool attn_use_mma(const pipo_ctx* ctx, int B) {
            (int)ctx->kv_tm.size() == 2 * ctx->n_cache_layers;
 }
 
+// Mean cached length (pairs per sequence) the launch plan is made for.  A
+// captured step graph keeps its launches while the caches grow, so the
+// length is frozen at its capture: later captures of kernel families and
+// pipo_describe_step then see the plan the graph runs.  Without a graph, the
+// current mean.
+double plan_mean_len(const pipo_ctx* ctx) {
+    if (ctx->graph && ctx->plan_len >= 0.0) return ctx->plan_len;
+    double sum = 0.0;
+    int n = 0;
+    for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b, ++n) sum += ctx->h_len[b];
+    return n > 0 ? sum / n : 0.0;
+}
+
 bool attn_mma_deep_on();
 
 // CTAs per (sequence, kv head) of the clustered attention: 8 while the batch
@@ -884,10 +898,7 @@ constexpr int kFlatMinEntries = 2048;
 bool attn_flat_now(const pipo_ctx* ctx) {
     if (ctx->attn_flat <= 0) return false;
     if (ctx->attn_flat >= 2) return true;
-    double sum = 0.0;
-    int n = 0;
-    for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b, ++n) sum += ctx->h_len[b];
-    return n > 0 && sum / n >= kFlatMinEntries;
+    return plan_mean_len(ctx) >= kFlatMinEntries;
 }
 
 // The QKV projection of a decode step on the streaming GEMV prefetches the
@@ -944,10 +955,7 @@ int attn_mma_flat_splits(const pipo_ctx* ctx, int R) {
     if (mode <= 0) return 0;
     const long long pairs = (long long)R * ctx->cfg.n_kv_heads;
     if (pairs * 8 >= 2LL * ctx->sms) return 0;
-    double sum = 0.0;
-    int n = 0;
-    for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b, ++n) sum += ctx->h_len[b];
-    const double mean = n > 0 ? sum / n : 0.0;
+    const double mean = plan_mean_len(ctx);
     if (mode == 1 && mean < kFlatMmaMinEntries) return 0;
     // 8-CTA clusters on the deep ring while it holds a CTA's whole slice (a
     // slice of c entries spans at most c / 16 + 2 groups)
@@ -978,8 +986,7 @@ bool attn_is_long(const pipo_ctx* ctx) {
     }();
     if (force >= 0) return force == 1;
     const pipo_config& c = ctx->cfg;
-    double ctx_sum = 0.0;
-    for (int b = 0; b < ctx->B && b < (int)ctx->h_len.size(); ++b) ctx_sum += ctx->h_len[b];
+    const double ctx_sum = plan_mean_len(ctx) * std::min(ctx->B, (int)ctx->h_len.size());
     const double kv_bytes = ctx_sum * c.n_kv_heads * c.head_dim * 2.0 * ctx->esz;
     const double qkv_bytes = (double)(c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim * c.hidden * ctx->esz;
     return kv_bytes >= 6.0 * qkv_bytes;
@@ -1430,6 +1437,7 @@ void drop_graph(pipo_ctx* ctx) {
     if (ctx->graph) cudaGraphExecDestroy(ctx->graph);
     ctx->graph = nullptr;
     ctx->graph_B = -1;
+    ctx->plan_len = -1.0;
     if (ctx->fam_graph) cudaGraphExecDestroy(ctx->fam_graph);
     ctx->fam_graph = nullptr;
     ctx->fam_graph_B = -1;
@@ -1438,6 +1446,7 @@ void drop_graph(pipo_ctx* ctx) {
 pipo_status ensure_graph(pipo_ctx* ctx) {
     if (ctx->graph && ctx->graph_B == ctx->B && ctx->graph_regular == ctx->regular) return PIPO_OK;
     drop_graph(ctx);
+    const double plan_len = plan_mean_len(ctx);
     cudaGraph_t g = nullptr;
     CK(cudaStreamBeginCapture(ctx->stream, cudaStreamCaptureModeThreadLocal));
     ctx->launches = 0;
@@ -1455,6 +1464,7 @@ pipo_status ensure_graph(pipo_ctx* ctx) {
     if (e != cudaSuccess) return fail(ctx, PIPO_ECUDA, "graph instantiate: %s", cudaGetErrorString(e));
     ctx->graph_B = ctx->B;
     ctx->graph_regular = ctx->regular;
+    ctx->plan_len = plan_len;
     return PIPO_OK;
 }
 
@@ -1843,6 +1853,7 @@ extern "C" {
 pipo_status pipo_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride, const int32_t* h_lens,
                          int32_t* h_tokens, int32_t* h_n_accepted) {
     if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    drop_graph(ctx);  // the next step's launch plan is made for the new lengths
     if (batch > 1 && batch <= ctx->cfg.max_batch && h_ids && h_lens && stride >= 1) {
         bool ragged = false;
         for (int b = 1; b < batch; ++b) ragged |= (h_lens[b] + 1) / 2 != (h_lens[0] + 1) / 2;
@@ -1966,6 +1977,7 @@ pipo_status pipo_prefill_slot(pipo_ctx* ctx, int32_t slot, const int32_t* h_ids,
         return fail(ctx, PIPO_EINVAL, "bad slot prefill arguments (slot %d of %d, length %d)", slot,
                     ctx->cfg.max_batch, len);
     if (ctx->prefilled && ctx->regular) return fail(ctx, PIPO_ESTATE, "slot prefill after a regular-decoding prefill");
+    drop_graph(ctx);  // the next step's launch plan is made for the new lengths
     const bool was = ctx->prefilled;
     const int B_old = was ? ctx->B : 0;
     const std::vector<int32_t> len_old = was ? ctx->h_len : std::vector<int32_t>();
@@ -1995,6 +2007,7 @@ pipo_status pipo_prefill_slot(pipo_ctx* ctx, int32_t slot, const int32_t* h_ids,
 pipo_status pipo_regular_prefill(pipo_ctx* ctx, int32_t batch, const int32_t* h_ids, int32_t stride,
                                  const int32_t* h_lens, int32_t* h_tokens, int32_t* h_n_accepted) {
     if (!ctx) return fail(nullptr, PIPO_EINVAL, "null context");
+    drop_graph(ctx);  // the next step's launch plan is made for the new lengths
     int N = 0;
     TRY(check_prompt(ctx, batch, h_ids, stride, h_lens, false, &N));
     CK(cudaSetDevice(ctx->dev));
@@ -2187,6 +2200,7 @@ pipo_status pipo_load_cache(pipo_ctx* ctx, int32_t b, int32_t n, const float* h_
     if (!ctx || !h_K || !h_V) return fail(ctx, PIPO_EINVAL, "null argument");
     if (!ctx->prefilled || b < 0 || b >= ctx->B) return fail(ctx, PIPO_ESTATE, "load_cache needs a prefilled sequence b");
     if (n < 1 || n > ctx->cfg.max_ctx) return fail(ctx, PIPO_ECAPACITY, "load_cache: %d entries", n);
+    drop_graph(ctx);  // the next step's launch plan is made for the new length
     CK(cudaSetDevice(ctx->dev));
     const size_t kd = (size_t)ctx->cfg.n_kv_heads * ctx->cfg.head_dim;
     TRY(ensure_cache_tmp(ctx, 2 * kd * n));

@@ -346,6 +346,15 @@ def make_line(m: dict) -> dict:
         "gpu_launches": m["launches"] * K,
         "clocks": m["clocks"],
     }
+    if m.get("prefill_s") and m.get("prefill_flops") and m.get("bf16_tflops"):
+        # the prefill is tensor-bound (positions x sequences through the projections)
+        tflops = m["prefill_flops"] / m["prefill_s"] / 1e12
+        line["prefill"] = {"seconds": m["prefill_s"], "pair_positions": (m["prompt_tokens"] + 1) // 2,
+                           "flops": m["prefill_flops"], "achieved_tflops": tflops,
+                           "peak_tflops": m["bf16_tflops"], "frac": tflops / m["bf16_tflops"],
+                           "bound": "tensor",
+                           "timing": "host clock around the first pipo_prefill call of the context (its one-time "
+                                     "set-up included), the time to first token"}
     regular = m.get("regular")
     if regular is not None:
         pipo_tpot = step_ms / (1.0 + acceptance)
@@ -506,7 +515,8 @@ def run_pipo(args):
         workload=args.workload, shape_name=wl["shape"], dtype=shape.dtype, n_gpus=ws, steps=K, warmup=W, batch=B,
         prompt_tokens=T, ms=ms, ms_all=ms_all, tokens=tokens, tokens_all=tokens_all, ctx_avg=ctx_avg, tau=tau,
         force=args.force, prefill_s=t_pf, prefill_rows=args.prefill_rows, sampler=args.sampler, desc=desc, fam=fam,
-        hbm=hbm, peak_source=src, step_bytes=roofline.step_bytes(shape, B, ctx_avg),
+        hbm=hbm, peak_source=src, step_bytes=roofline.step_bytes(shape, B, ctx_avg), bf16_tflops=tf,
+        prefill_flops=None if wl.get("kv_fill") else roofline.prefill_flops(shape, B, (T + 1) // 2),
         traffic=roofline.recorded_traffic(os.path.join(ROOT, "profiles"), args.workload),
         cpu=cpu, e2e_s=e2e_all, e2e_tokens=e2e_tok_all, launches=launches,
         clocks=clk.summary(), regular=regular))

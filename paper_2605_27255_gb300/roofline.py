@@ -56,6 +56,25 @@ def step_flops(s: ModelShape, batch: int, ctx_avg: float) -> float:
     return 2.0 * macs
 
 
+def prefill_flops(s: ModelShape, batch: int, n_pairs: int) -> float:
+    """Multiply-add flops (2 per MAC) of a pair prefill of n_pairs positions
+    per sequence: at every position the compressor, the L backbone blocks,
+    the teacher-forced MTP input projection and the MTP block; causal
+    attention of each position over itself and the positions before it
+    (q.k and p.v, every cached block); the heads once, at the last position
+    (two LM-head passes and the confidence head).  Norms and activations are
+    left out."""
+    H, qd, kd = s.H, s.n_q * s.d_h, s.n_kv * s.d_h
+    block = (qd + 2 * kd) * H + H * qd + 3 * s.F * H
+    comp = H * 2 * H + (H * H if s.compressor == "mlp" else 0)
+    mtp = H * 2 * H + (block if s.mtp_block else 0)
+    per_pos = comp + s.L * block + mtp
+    layers = s.L + (1 if s.mtp_block else 0)
+    attn = layers * s.n_q * s.d_h * 2 * (n_pairs * (n_pairs + 1) / 2.0)
+    heads = 2 * s.V * H + H * 2 * H + H
+    return 2.0 * batch * (n_pairs * per_pos + attn + heads)
+
+
 def regular_step_bytes(s: ModelShape, batch: int, ctx_avg: float) -> float:
     """Algorithmic HBM bytes of one step of regular decoding (the baseline of
     Sec. 4): the L backbone blocks and the final norm once, E once (one LM-head

@@ -64,6 +64,18 @@ def test_regular_ratios():
     assert line["regular"]["frac"] == pytest.approx(4000.0 / 6774.6)
 
 
+def test_prefill_tensor_fraction():
+    """The time to first token against the prefill's multiply-add flops and
+    the measured bf16 peak; absent when either is unknown."""
+    line = bench.make_line(_measured(prefill_flops=1.5e14, bf16_tflops=1934.6))
+    pf = line["prefill"]
+    assert pf["achieved_tflops"] == pytest.approx(1.5e14 / 3.0 / 1e12)
+    assert pf["frac"] == pytest.approx(50.0 / 1934.6) and pf["bound"] == "tensor"
+    assert pf["pair_positions"] == 1024 and pf["seconds"] == 3.0
+    assert "prefill" not in bench.make_line(_measured())
+    assert "prefill" not in bench.make_line(_measured(prefill_flops=1.5e14, bf16_tflops=None))
+
+
 def test_missing_family_time_gives_no_fraction():
     line = bench.make_line(_measured(fam={0: {"bytes": 0.0, "ms": 0.0, "launches": 0, "replays": 0},
                                           1: {"bytes": 0.0, "ms": 0.0, "launches": 0, "replays": 0}}))

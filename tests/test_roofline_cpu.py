@@ -61,3 +61,18 @@ def test_regular_step_bytes_are_the_backbone_part_of_the_pair_step(shape):
         w = (36 * 100_930_560 + 2560 + 151_936 * 2560) * 2
         assert w == 8_044_917_760
         assert roofline.regular_step_bytes(shape, 1, 0.0) == w + 2 * 36 * 2 * 8 * 128 * 2
+
+
+@pytest.mark.parametrize("shape", [synth.TINY, synth.B4, synth.B9])
+def test_prefill_flops_equal_the_tensor_list(shape):
+    """A pair prefill multiplies every matrix of the compressor, the backbone
+    blocks and the MTP head at each position, attends causally (q.k and p.v
+    per earlier-or-same position, every cached block), and runs the heads
+    (E twice, the confidence matrices) once."""
+    shapes = synth.tensor_shapes(shape)
+    per_pos = sum(math.prod(d) for n, d in shapes.items() if ".W" in n and not n.startswith("conf."))
+    heads = sum(math.prod(d) for n, d in shapes.items() if n.startswith("conf.W")) + 2 * math.prod(shapes["E"])
+    layers = shape.L + (1 if shape.mtp_block else 0)
+    for B, N in ((1, 1), (2, 7), (1, 8192)):
+        attn = sum(layers * shape.n_q * shape.d_h * 2 * (j + 1) for j in range(N))
+        assert roofline.prefill_flops(shape, B, N) == pytest.approx(2 * B * (N * per_pos + attn + heads), rel=1e-12)

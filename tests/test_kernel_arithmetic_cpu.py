@@ -9,7 +9,9 @@ numpy (no GPU):
   direct attention on one 16-entry group;
 * the sampler's selection (sample_kernel): per-thread sorted top lists,
   k warp-merge rounds with owner hand-off, the warp-0 merge of the warp
-  lists, against a sorted reference, with ties and small vocabularies.
+  lists, against a sorted reference, with ties and small vocabularies;
+* the decode attention's stage rings (attn_mma_kernel, 10 and 20 stages):
+  per-warp stage ownership and the mbarrier phase parities.
 """
 import numpy as np
 
@@ -243,3 +245,36 @@ def test_decode_attention_fragment_arithmetic_the_same_way():
             for j in range(2):
                 score = sacc[nt][lane][j] + sacc[nt][partner][j]
                 assert abs(score - ref[nt * 8 + 2 * t + j, r]) < 1e-4
+
+
+def _mma_stage(t, st, nw=5):
+    """Stage of group t in attn_mma_kernel's ring of st stages (nw compute
+    warps, st / nw stages each), restated."""
+    spw = st // nw
+    return (t % nw) * spw + (t // nw) % spw
+
+
+def test_decode_attention_stage_ring_phases():
+    """The tensor-core decode attention's stage rings (10 stages, and 20 for
+    the deep ring): group t goes to compute warp t % 5 and only through that
+    warp's own stages; the k-th group through a stage is its phase k, so the
+    consumer's parity (t / ST) & 1 and the producer's wait for the stage's
+    previous consumption (parity ((t / ST) & 1) ^ 1, from t >= ST) name the
+    right phases; and the first ST groups (issued before any wait) use ST
+    distinct stages."""
+    for st in (10, 20):
+        spw = st // 5
+        uses = {}
+        for t in range(12 * st):
+            s = _mma_stage(t, st)
+            assert 0 <= s < st and s // spw == t % 5  # the consuming warp's own stages
+            k = len(uses.setdefault(s, []))
+            assert (t // st) & 1 == k & 1  # consumer parity = phase k
+            if t >= st:
+                assert k >= 1 and ((t // st) & 1) ^ 1 == (k - 1) & 1  # previous consumption
+            uses[s].append(t)
+        assert sorted(_mma_stage(t, st) for t in range(st)) == list(range(st))
+        # a warp's consecutive groups cycle through its stages in order
+        for w in range(5):
+            seq = [_mma_stage(t, st) for t in range(w, 6 * st, 5)]
+            assert seq[:spw] == [w * spw + j for j in range(spw)] and seq[spw:2 * spw] == seq[:spw]
